@@ -1,0 +1,454 @@
+#!/usr/bin/env python3
+"""Throughput of the GB300 routing engine: requests routed/s and (request, peer) lookups/s.
+
+A step is one pass of the whole hot path over one batch: for the scale workload the anti-entropy delta on
+every replica (device INSERT/DELETE) followed by the route of the batch (longest-prefix match against all
+P trees + route decision); for the other workloads the route alone.  Inputs are seeded synthetic
+stand-ins for the paper's few-shot-prompt workloads (see workload/wl.h), resident in HBM when the timed
+region starts.  The JSON line also carries:
+  roofline      the route kernel's algorithmic bytes/s (per launch: the oracle's touched-byte accounting)
+                against the measured HBM copy bandwidth;
+  e2e           the same metric through the host-pointer C-ABI call (copies in the timed region);
+  cpu_baseline  the CPU oracle on the host cores over a bounded sample of the same workload.
+--impl reference times that oracle as the reference arm.
+
+Multi-GPU (torchrun): every rank holds all P trees and routes its own batch (requests [rank*B, (rank+1)*B)
+of the request stream); no data-path collective.  Timing is max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "requests routed/sec and (req,peer) lookups/sec at 1 GB300; % of HBM roofline"
+WORKLOADS = {
+    "cfg0": (0, "P=4 trees x 1,000 seqs (57 shared prefixes of 256-1,024 tokens), 4,096 requests/batch"),
+    "cfg1": (1, "P=16 trees x 20,000 seqs (512 prefixes of 128-2,048 tokens), 65,536 requests/batch"),
+    "cfg2": (2, "stale replicas: P=64 trees x 20,000 seqs (trees 1-63: -10%/+5%), 262,144 requests/batch"),
+    "cfg3": (3, "long context: P=32 trees x 5,000 seqs (prefixes 4,096-32,768), 16,384 requests/batch"),
+    "cfg4": (4, "scale + anti-entropy: P=256 trees x 100,000 seqs (10,000 prefixes of 128-4,096), "
+                "1,048,576 requests/batch, 5% DELETE + 5% INSERT per replica per batch"),
+}
+L2_BYTES = 126 * 2**20
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clock/throttle samples while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: int):
+        self.gpu = gpu
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_info():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ---- workload setup ---------------------------------------------------------------------------------
+
+def make_workload(cfg: int):
+    import workload as wl
+    return wl.Workload(cfg)
+
+
+def build_trees(W, router, with_oracle: bool, n_threads: int):
+    """Snapshots (and oracle trees) built on host threads, uploads in order on this thread."""
+    import paper_2606_17059_gb300 as g
+    import oracle as orc  # the oracle is used only by the CPU-baseline leg and the byte accounting
+    P = W.P
+    otrees = [None] * P
+
+    def make(p):
+        sl = W.tree(p)
+        snap = g.p2p_snapshot_build(sl)
+        if with_oracle:
+            t = orc.OTree()
+            t.insert_seqlist(sl)
+            otrees[p] = t
+        return snap
+
+    with ThreadPoolExecutor(max_workers=n_threads) as ex:
+        futs = [ex.submit(make, p) for p in range(P)]
+        for p, f in enumerate(futs):
+            snap = f.result()
+            flat = g.FlatTree()
+            g._load().p2p_snapshot_view(snap, flat)
+            g._check(g._load().p2p_tree_upload(router.handle, p, flat), router.handle)
+            g.p2p_snapshot_free(snap)
+    router.sync()
+    return otrees
+
+
+def delta_to_device(d):
+    import torch
+    import workload as wl
+    dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+    return (dev(d.op), wl.SeqList(dev(d.seqs.seg_begin), dev(d.seqs.seg_off), dev(d.seqs.seg_len), dev(d.seqs.pool)),
+            dev(d.peer_begin))
+
+
+def delta_bytes(d) -> int:
+    s = d.seqs
+    return d.op.nbytes + s.seg_begin.nbytes + s.seg_off.nbytes + s.seg_len.nbytes + s.pool.nbytes + d.peer_begin.nbytes
+
+
+# ---- the CPU oracle leg ------------------------------------------------------------------------------------
+
+def oracle_sample(W, otrees, tok, off, load, alpha, target_s: float, n_threads: int, delta=None, B_total=None):
+    """Times the oracle on a bounded prefix of the batch: n requests (and, with a delta, the matching share
+    of every tree's ops).  Returns (requests/s, seconds, n, counters, description)."""
+    import oracle as orc
+    B = len(off) - 1
+    pilot = min(B, 256)
+    t0 = time.perf_counter()
+    orc.route(otrees, tok, off[: pilot + 1], load, alpha, n_threads=n_threads)
+    per_req = (time.perf_counter() - t0) / pilot
+    n = int(min(B, max(pilot, target_s / max(per_req, 1e-9))))
+    frac = n / float(B_total or B)
+    t_delta = 0.0
+    n_ops = 0
+    if delta is not None:
+        pb = delta.peer_begin
+        t0 = time.perf_counter()
+
+        def apply(p):
+            lo = int(pb[p])
+            k = int(math.ceil(frac * (int(pb[p + 1]) - lo)))
+            otrees[p].apply_ops(delta.op, delta.seqs, lo, lo + k)
+            return k
+
+        with ThreadPoolExecutor(max_workers=n_threads) as ex:
+            n_ops = sum(ex.map(apply, range(len(otrees))))
+        t_delta = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    m, peer, ctr = orc.route(otrees, tok, off[: n + 1], load, alpha, n_threads=n_threads)
+    t_route = time.perf_counter() - t0
+    secs = t_delta + t_route
+    desc = f"first {n} of {B} requests of the batch x all {len(otrees)} trees"
+    if delta is not None:
+        desc += f", plus {n_ops} delta ops (the same {frac:.4%} share of every replica's delta)"
+    return n / secs, secs, n, ctr, desc, (m, peer)
+
+
+# ---- our arm --------------------------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    import paper_2606_17059_gb300 as g
+    import oracle as orc
+
+    ws, rank, local = dist_info()
+    torch.cuda.set_device(local)
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    cfg, wdesc = WORKLOADS[args.workload]
+    n_cpu = os.cpu_count() or 1
+    t_setup = time.perf_counter()
+    W = make_workload(cfg)
+    P, B, alpha = W.P, W.B, W.alpha
+    router = g.Router(P)
+    want_oracle = rank == 0 and not args.no_cpu_baseline
+    otrees = build_trees(W, router, want_oracle, n_cpu)
+    log(f"[rank {rank}] trees built in {time.perf_counter() - t_setup:.1f}s")
+    # Requests of this rank, pinned on the host (for the end-to-end leg) and resident on the device.
+    b0, b1 = rank * B, (rank + 1) * B
+    n_tok = W._lib.wl_requests_size(W._h, b0, b1, n_cpu)
+    h_tok = torch.empty(n_tok, dtype=torch.int32, pin_memory=True)
+    tok_np, off_np = W.requests(b0, b1, n_threads=n_cpu, out_tokens=h_tok.numpy())
+    h_off = torch.from_numpy(off_np).pin_memory()
+    d_tok = h_tok.cuda()
+    d_off = h_off.cuda()
+    load = W.load()
+    out_match = torch.empty((B, P), dtype=torch.int32, device="cuda")
+    out_peer = torch.empty(B, dtype=torch.int32, device="cuda")
+    has_delta = W.params["delta_frac"] > 0
+    n_steps = args.warmup + args.steps
+    deltas = []
+    if has_delta:
+        t0 = time.perf_counter()
+        for s in range(n_steps):
+            W.delta_make(s, W.params["delta_frac"], W.params["delta_frac"], n_threads=n_cpu)
+            d = W.delta(n_threads=n_cpu)
+            deltas.append(delta_to_device(d))
+            if s == 0:
+                host_delta0 = d
+        log(f"[rank {rank}] {n_steps} deltas staged in {time.perf_counter() - t0:.1f}s "
+            f"({len(host_delta0.op)} ops, {delta_bytes(host_delta0) / 1e6:.0f} MB each)")
+    flush = None
+    if (n_tok * 4 + B * P * 4) < 2 * L2_BYTES:
+        flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step(s, ev):
+        if has_delta:
+            op, sl, pb = deltas[s]
+            ev[0].record(stream)
+            router.apply_delta(-1, op, sl, pb, on_device=True)
+        ev[1].record(stream)
+        g.p2p_route_batch(router.handle, d_tok, n_tok, d_off, B, load, alpha, out_match, out_peer)
+        ev[2].record(stream)
+
+    mk = lambda: [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    for s in range(args.warmup):
+        step(s, mk())
+        if flush is not None:
+            flush.zero_()
+    router.sync()
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    launches0 = router.launch_count()
+    evs = []
+    t_begin = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_begin.record(stream)
+    for k in range(args.steps):
+        ev = mk()
+        step(args.warmup + k, ev)
+        evs.append(ev)
+        if flush is not None:
+            # L2 flush between steps, outside the per-step events below.
+            flush.zero_()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    launches = router.launch_count() - launches0
+    clk = clocks.stop()
+    if dist:
+        dist.barrier()
+    router.sync()
+    route_ms = [ev[1].elapsed_time(ev[2]) for ev in evs]
+    delta_ms = [ev[0].elapsed_time(ev[1]) for ev in evs] if has_delta else [0.0] * len(evs)
+    step_ms = [a + b for a, b in zip(route_ms, delta_ms)]
+    total_ms = sum(step_ms) if flush is not None else t_begin.elapsed_time(t_end)
+    if dist:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = ws * B / (ms_per_step / 1e3)
+    res = {}
+    if rank == 0:
+        gm = out_match.cpu().numpy()
+        gp = out_peer.cpu().numpy()
+        # ---- CPU oracle leg: baseline timing, touched-byte accounting and a parity spot check ----
+        # (For the delta workload the oracle trees are the initial replicas, before the GPU's deltas: they
+        # differ from the device trees by a few percent of their edges, so they give the byte accounting
+        # but no parity check; the tests check that workload's parity.)
+        ctr, n_acc, cpu = None, 0, None
+        if want_oracle:
+            rate, secs, n_acc, ctr, desc, (om, op) = oracle_sample(
+                W, otrees, tok_np, off_np, load, alpha, args.cpu_seconds, n_cpu,
+                delta=host_delta0 if has_delta else None, B_total=B)
+            cpu = {"value": rate, "unit": "requests/s", "cores": n_cpu, "kind": "oracle",
+                   "sample": desc + f" ({secs:.1f} s on {n_cpu} host threads)"}
+            if not has_delta:
+                same = bool(np.array_equal(gm[:n_acc], om) and np.array_equal(gp[:n_acc], op))
+                res["parity_spot_check"] = {"requests": n_acc, "bit_exact": same}
+        hbm, src = peaks()
+        route_avg_ms = statistics.mean(route_ms)
+        roof = None
+        if ctr is not None:
+            bytes_per_launch = orc.touched_bytes(ctr) / n_acc * B
+            achieved = bytes_per_launch / (route_avg_ms / 1e3) / 1e9
+            roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
+                    "traffic": None, "kernel": "route_kernel", "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
+                    "bytes_per_launch": bytes_per_launch, "route_ms": route_avg_ms,
+                    "bytes_basis": f"oracle touched-byte counters over {n_acc} requests x {P} trees, "
+                                   f"scaled to {B} requests per launch"}
+        # ---- end to end through the host-pointer C-ABI call ----
+        e2e = run_e2e(args, W, router, tok_np, off_np, load, alpha, has_delta, n_cpu)
+        res.update({
+            "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+            "config": {"workload": f"{args.workload}: {wdesc}", "P": P, "B_per_gpu": B, "alpha": alpha,
+                       "tokens_per_batch": int(n_tok), "l2": "L2 flushed between steps" if flush is not None
+                       else "inputs larger than L2 (request tokens stream from HBM each step)",
+                       "step": "delta on every replica + route" if has_delta else "route"},
+            "lookups_per_s": value * P, "route_ms": route_avg_ms,
+            "delta_ms": statistics.mean(delta_ms) if has_delta else None,
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+        })
+        print(json.dumps(res), flush=True)
+    router.close()
+    if dist:
+        dist.destroy_process_group()
+
+
+def run_e2e(args, W, router, tok_np, off_np, load, alpha, has_delta, n_cpu):
+    """The same metric through the host-pointer calls: request tokens/offsets copied in and match/peer
+    copied out every step (and, for the delta workload, each step's delta from host memory)."""
+    import torch
+    import paper_2606_17059_gb300 as g
+    B, P = len(off_np) - 1, W.P
+    h_match = torch.empty((B, P), dtype=torch.int32, pin_memory=True).numpy()
+    h_peer = torch.empty(B, dtype=torch.int32, pin_memory=True).numpy()
+    k = max(1, min(args.steps, args.e2e_steps))
+    hds = []
+    if has_delta:
+        base = args.warmup + args.steps
+        for s in range(k + 1):
+            W.delta_make(base + s, W.params["delta_frac"], W.params["delta_frac"], n_threads=n_cpu)
+            hds.append(W.delta(n_threads=n_cpu))
+
+    def one(i):
+        if has_delta:
+            d = hds[i]
+            router.apply_delta(-1, d.op, d.seqs, d.peer_begin)
+        g.p2p_route_batch_host(router.handle, tok_np, off_np, B, load, alpha, h_match, h_peer)
+
+    one(0)  # warm
+    t0 = time.perf_counter()
+    for i in range(1, k + 1):
+        one(i)
+    secs = time.perf_counter() - t0
+    h2d = tok_np.nbytes + off_np.nbytes + 4 * P
+    if has_delta:
+        h2d += delta_bytes(hds[1])
+    return {"value": k * B / secs, "unit": "requests/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(h_match.nbytes + h_peer.nbytes), "steps": k,
+            "call": "p2p_tree_apply_delta (host arrays) + p2p_route_batch_host" if has_delta else "p2p_route_batch_host"}
+
+
+# ---- reference arm: the CPU oracle as it stands -------------------------------------------------------------
+
+def run_reference(args):
+    ws, rank, _ = dist_info()
+    if rank != 0:
+        return
+    import oracle as orc
+    cfg, wdesc = WORKLOADS[args.workload]
+    n_cpu = os.cpu_count() or 1
+    W = make_workload(cfg)
+    P, B, alpha = W.P, W.B, W.alpha
+    otrees = orc.build_trees([W.tree(p) for p in range(P)], n_threads=n_cpu)
+    has_delta = W.params["delta_frac"] > 0
+    b_sample = min(B, args.ref_requests)
+    tok, off = W.requests(0, b_sample, n_threads=n_cpu)
+    load = W.load()
+    times = []
+    desc = ""
+    for s in range(args.warmup + args.steps):
+        d = None
+        if has_delta:
+            W.delta_make(s, W.params["delta_frac"], W.params["delta_frac"], n_threads=n_cpu)
+            d = W.delta(n_threads=n_cpu)
+        rate, secs, n, _, desc, _ = oracle_sample(W, otrees, tok, off, load, alpha, args.ref_seconds, n_cpu,
+                                                  delta=d, B_total=B)
+        if s >= args.warmup:
+            times.append((n, secs))
+    n_req = sum(n for n, _ in times)
+    secs = sum(t for _, t in times)
+    value = n_req / secs
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * secs / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": {"workload": f"{args.workload}: {wdesc}", "P": P, "B_per_gpu": B, "alpha": alpha},
+        "cpu_baseline": {"value": value, "unit": "requests/s", "cores": n_cpu, "kind": "oracle",
+                         "sample": "per step: " + desc},
+        "e2e": {"value": value, "unit": "requests/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="cfg4", choices=sorted(WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--ref-requests", type=int, default=65536)
+    ap.add_argument("--ref-seconds", type=float, default=4.0, help="oracle time per reference step")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        log("warmup < 3 is below the timing rules; using 3")
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,201 @@
+/*
+ * p2p_router.h -- C ABI of the GB300 batched routing engine for decentralized, prefix-cache-aware routing
+ * ("Towards Distributed Inference of LLMs on a P2P Network").
+ *
+ * A router holds P radix trees in GPU memory: by convention tree 0 is the node's own exact tree and trees
+ * 1..P-1 are its read-only estimates of the peers' trees (Section 2: one trie per node plus N-1 peer
+ * estimates).  Requests are routed in batches: every request is matched against every tree
+ * (PrefixMatch of Algorithm 1) and sent to the argmax (getBestNode), with a load term.  Trees are
+ * refreshed by anti-entropy: a full snapshot replaces a replica (Section 2, sendTrie; Section 3,
+ * "Trie-broadcast loss"), or an ordered INSERT/DELETE delta patches it on the device (updateTrie /
+ * updateTrieEstimate of Section 2 for INSERT; removal of a stored sequence for DELETE).
+ *
+ * Conventions
+ *   - Tokens are int32 (any value).  A tree stores a multiset S(T) of token sequences.
+ *   - match(r, T) = max over s in S(T) of LCP(r, s), 0 for an empty tree; this is the number of tokens
+ *     of r found along one path of T, a partially matched edge included.
+ *   - Route: score_p = match_p - alpha * load_p (exact, 64-bit); the chosen peer has the highest score,
+ *     ties go to the lower load, then to the lower tree index.  Requires alpha >= 0, 0 <= load <= 65535,
+ *     alpha * load <= 2^31 - 1 and P <= 65536.
+ *   - Every call returns P2P_OK (0) or a negative error code; p2p_last_error() gives a message.  A call
+ *     that fails leaves the router's trees unchanged.
+ *   - Device work is enqueued on the router's stream (p2p_router_set_stream); calls that take device
+ *     pointers return before the work finishes.  Asynchronous device-side errors are reported by the
+ *     next p2p_router_sync() as P2P_E_DEVICE.
+ *   - The caller owns every buffer it passes; the library never frees caller memory.  Objects the
+ *     library returns (routers, snapshots) are freed with their destroy/free call.
+ *   - One router is used by one host thread at a time (the single writer of Section 3, "Asynchrony").
+ */
+#ifndef P2P_ROUTER_H
+#define P2P_ROUTER_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+  P2P_OK = 0,
+  P2P_E_INVAL = -1,   /* bad argument */
+  P2P_E_NOMEM = -2,   /* allocation failed, or a tree outgrew the int32 flat format */
+  P2P_E_FORMAT = -3,  /* malformed snapshot */
+  P2P_E_CUDA = -4,    /* a CUDA runtime call failed */
+  P2P_E_DEVICE = -5   /* a kernel reported an error (bad request offsets, internal consistency) */
+};
+
+enum { P2P_OP_INSERT = 0, P2P_OP_DELETE = 1 };
+enum { P2P_MEM_HOST = 0, P2P_MEM_DEVICE = 1 };
+
+typedef struct p2p_router p2p_router;
+typedef struct p2p_snapshot p2p_snapshot;
+
+/*
+ * Flat radix tree: the full-snapshot wire format (Section 2, sendTrie).  n_nodes >= 1; node 0 is the root.
+ *   label_off[v], label_len[v]  edge label of node v = labels[label_off[v] .. +label_len[v]); root: len 0,
+ *                               every other node: len >= 1
+ *   child_begin[v], child_count[v]  v's children are entries child_begin[v] .. +child_count[v] of
+ *                               child_first_tok[] / child_idx[] (n_nodes - 1 entries in total)
+ *   term_count[v]               number of stored sequences ending at v (>= 0)
+ *   child_first_tok[e]          first label token of node child_idx[e]; strictly ascending within a node
+ * Valid: every non-root node is listed exactly once as a child and is reachable from the root, every
+ * non-root leaf and every non-root node with one child has term_count > 0, and every root-to-node path
+ * has at most 2^31 - 1 tokens.  Canonical (as built and downloaded by the library): nodes in preorder,
+ * children ascending, labels and child lists packed in node order.
+ */
+typedef struct p2p_flat_tree {
+  int32_t n_nodes;
+  int32_t n_labels;
+  const int32_t* label_off;
+  const int32_t* label_len;
+  const int32_t* child_begin;
+  const int32_t* child_count;
+  const int32_t* term_count;
+  const int32_t* child_first_tok;
+  const int32_t* child_idx;
+  const int32_t* labels;
+} p2p_flat_tree;
+
+/*
+ * Segmented sequence list: sequence i is the concatenation of the pool runs
+ * pool[seg_off[s] .. seg_off[s] + seg_len[s]) for s in [seg_begin[i], seg_begin[i+1]).  seg_begin has
+ * n + 1 entries, non-decreasing, starting at 0 and ending at n_segs; every run lies inside the pool.
+ * Runs may overlap, so a shared prefix is sent once and referenced by many sequences.
+ */
+typedef struct p2p_seqs {
+  int64_t n;
+  const int64_t* seg_begin;
+  const int64_t* seg_off;
+  const int32_t* seg_len;
+  const int32_t* pool;
+  int64_t n_segs;
+  int64_t n_pool;
+} p2p_seqs;
+
+/*
+ * Ordered anti-entropy delta: op[i] (P2P_OP_INSERT / P2P_OP_DELETE) applies to sequence i of seqs.
+ * With peer = -1, peer_begin[P+1] (non-decreasing, from 0 to seqs.n) gives tree p the ops
+ * peer_begin[p] .. peer_begin[p+1]-1; otherwise peer_begin is ignored and all ops go to one tree.
+ * mem = P2P_MEM_HOST: every array is in host memory; P2P_MEM_DEVICE: every array is in device memory.
+ */
+typedef struct p2p_delta {
+  const int32_t* op;
+  p2p_seqs seqs;
+  const int64_t* peer_begin;
+  int32_t mem;
+} p2p_delta;
+
+/* ---- router ---------------------------------------------------------------------------------------- */
+
+/* Creates a router with P >= 1 empty trees on the current CUDA device (Section 2: N-1 estimates plus the
+ * own tree; a restarted node starts with empty trees, Section 2 crash-recovery model).  *out receives the
+ * handle.  Errors: P2P_E_INVAL (P out of range, out NULL), P2P_E_CUDA, P2P_E_NOMEM. */
+int p2p_router_create(int32_t P, p2p_router** out);
+
+/* Frees the router and all device memory it owns (after finishing its queued work).  NULL is a no-op. */
+void p2p_router_destroy(p2p_router* r);
+
+/* Sets the CUDA stream (a cudaStream_t, NULL = legacy default stream) on which the router enqueues its
+ * work; the previous stream is synchronized first, so no router work is left on it. */
+int p2p_router_set_stream(p2p_router* r, void* stream);
+
+/* Waits for the router's queued work and reports device-side errors raised since the last sync
+ * (P2P_E_DEVICE, message in p2p_last_error; the error state is then cleared). */
+int p2p_router_sync(p2p_router* r);
+
+/* Message of the last failed call on r (or of the last failed p2p_router_create when r is NULL). */
+const char* p2p_last_error(const p2p_router* r);
+
+int32_t p2p_router_num_trees(const p2p_router* r);
+
+/* Number of CUDA kernels the router has launched since creation (route, delta, bookkeeping kernels);
+ * lets a caller count the device work a region of code issued.  Not part of the paper's method. */
+int64_t p2p_router_launch_count(const p2p_router* r);
+
+/* ---- snapshots (host only; no GPU needed) ---------------------------------------------------------- */
+
+/* Builds the canonical snapshot of the multiset `seqs` (host pointers), i.e. the radix tree a node would
+ * broadcast for these cached sequences (Section 2, sendTrie).  Errors: P2P_E_INVAL (malformed list),
+ * P2P_E_NOMEM (tree beyond the int32 flat format). */
+int p2p_snapshot_build(const p2p_seqs* seqs, p2p_snapshot** out);
+
+/* Read-only view of a snapshot's arrays (valid until p2p_snapshot_free). */
+void p2p_snapshot_view(const p2p_snapshot* s, p2p_flat_tree* out);
+
+void p2p_snapshot_free(p2p_snapshot* s);
+
+/* Checks a flat tree (host pointers) against the validity rules above: P2P_OK or P2P_E_FORMAT. */
+int p2p_flat_tree_validate(const p2p_flat_tree* t);
+
+/* ---- trees ----------------------------------------------------------------------------------------- */
+
+/* Replaces tree `peer` with the full snapshot t (host pointers, copied before return).  This is the
+ * receive side of the anti-entropy broadcast: delivering the same snapshot twice gives the same tree
+ * (Section 3, "Trie-broadcast loss").  Enqueued on the router stream after earlier routes.
+ * Errors: P2P_E_INVAL (peer), P2P_E_FORMAT (invalid tree; nothing changes), P2P_E_NOMEM, P2P_E_CUDA. */
+int p2p_tree_upload(p2p_router* r, int32_t peer, const p2p_flat_tree* t);
+
+/* Builds the canonical snapshot of `seqs` (host pointers) and uploads it as tree `peer`. */
+int p2p_tree_build(p2p_router* r, int32_t peer, const p2p_seqs* seqs);
+
+/* Exports tree `peer` as its canonical snapshot (waits for queued work).  Two trees holding the same
+ * multiset export identical arrays.  *out is freed with p2p_snapshot_free. */
+int p2p_tree_download(p2p_router* r, int32_t peer, p2p_snapshot** out);
+
+/* Applies the ordered delta d to tree `peer` (0 <= peer < P), or, with peer = -1, to every tree p its
+ * ops peer_begin[p] .. peer_begin[p+1]-1.  INSERT adds one occurrence of the sequence (Section 2,
+ * updateTrie / updateTrieEstimate); DELETE removes one occurrence, and is a counted no-op when the
+ * sequence is not stored.  Trees stay edge-compressed and canonical.  Runs on the device; the call
+ * returns when the delta is applied (device arrays are only read, host arrays are copied).
+ * *n_absent (nullable) receives the number of no-op DELETEs.
+ * Errors: P2P_E_INVAL (bad op code, peer, ranges or segments; nothing changes), P2P_E_NOMEM,
+ * P2P_E_CUDA, P2P_E_DEVICE. */
+int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent);
+
+/* Sizes of tree `peer`: out[0] live nodes (root included), out[1] node slots in use, out[2] child
+ * entries in use, out[3] label tokens in use, out[4] stale child entries, out[5] stale label tokens,
+ * out[6..8] node / child-entry / label capacities.  Waits for queued work. */
+int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]);
+
+/* ---- routing --------------------------------------------------------------------------------------- */
+
+/* Routes a batch of B requests (Algorithm 1: k = argmax_j PrefixMatch(r, T_j), with the load term).
+ *   tokens      DEVICE int32[n_tokens]; request b is tokens[offsets[b] .. offsets[b+1])
+ *   offsets     DEVICE int64[B+1]; a request with 0 <= offsets[b] <= offsets[b+1] <= n_tokens violated
+ *               gets match 0 and peer -1 and makes the next p2p_router_sync return P2P_E_DEVICE
+ *   load        HOST int32[P], copied before return; alpha >= 0 (see Conventions)
+ *   out_match   DEVICE int32[B*P], row-major: out_match[b*P + p] = match(r_b, T_p)
+ *   out_peer    DEVICE int32[B]: the chosen tree of request b
+ * Asynchronous on the router stream.  B = 0 is a no-op.  Errors: P2P_E_INVAL, P2P_E_CUDA. */
+int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
+                    const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
+
+/* As p2p_route_batch with every pointer in HOST memory (pinned memory makes the copies faster):
+ * copies the requests to the device, routes, copies both outputs back and waits.  Offsets are
+ * validated on the host (P2P_E_INVAL).  Requests are tokens[offsets[0] .. offsets[B]). */
+int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* offsets, int64_t B,
+                         const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* P2P_ROUTER_H */
