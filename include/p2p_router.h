@@ -171,6 +171,25 @@ int p2p_tree_download(p2p_router* r, int32_t peer, p2p_snapshot** out);
  * P2P_E_CUDA, P2P_E_DEVICE. */
 int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent);
 
+/* As p2p_tree_apply_delta, for callers that cannot allocate memory while they patch replicas: a serving
+ * loop whose device memory belongs to another allocator (it may not call cudaMalloc, cudaFree or a
+ * caching allocator on its hot path), or a process whose device footprint must stay fixed after start-up.
+ * The paper has no counterpart; this is a deployment variant of the delta call.
+ * It allocates nothing, host or device: d must be in device memory (d->mem = P2P_MEM_DEVICE, else
+ * P2P_E_INVAL); the delta is validated on the device; every op's sequence is gathered into one static
+ * device array of the library (8 MiB of tokens plus a 256-byte header, held by every GPU that loads the
+ * library until the process exits); trees are never grown or compacted.
+ * Limits: (number of trees the call touches) x (longest sequence in the delta) <= 2,097,152 tokens,
+ * else P2P_E_INVAL.  If a tree's arenas have no room for an op, that tree stops before it (its earlier
+ * ops stay applied, other trees finish) and the call returns P2P_E_NOMEM; p2p_tree_apply_delta, which
+ * may allocate, grows the tree.
+ * The first call on a device looks up the static array's device address (cudaGetSymbolAddress, with
+ * the router's device current) and caches it; make that first call before any stream capture.  Every
+ * call shares the array, so calls whose device work overlaps (for example two routers on different
+ * streams) race: order them.  The call returns when the delta is applied.  Other errors as
+ * p2p_tree_apply_delta. */
+int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent);
+
 /* Sizes of tree `peer`: out[0] live nodes (root included), out[1] node slots in use, out[2] child
  * entries in use, out[3] label tokens in use, out[4] stale child entries, out[5] stale label tokens,
  * out[6..8] node / child-entry / label capacities.  Waits for queued work. */

@@ -20,7 +20,7 @@ __all__ = [
     "p2p_router_create", "p2p_router_destroy", "p2p_router_set_stream", "p2p_router_sync", "p2p_last_error",
     "p2p_router_num_trees", "p2p_router_launch_count", "p2p_snapshot_build", "p2p_snapshot_view", "p2p_snapshot_free",
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
-    "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host",
+    "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -88,6 +88,7 @@ def _load():
             "p2p_tree_build": (ctypes.c_int, [_vp, _i32, P(Seqs)]),
             "p2p_tree_download": (ctypes.c_int, [_vp, _i32, P(_vp)]),
             "p2p_tree_apply_delta": (ctypes.c_int, [_vp, _i32, P(Delta), P(_i64)]),
+            "p2p_tree_apply_delta_static": (ctypes.c_int, [_vp, _i32, P(Delta), P(_i64)]),
             "p2p_tree_stats": (ctypes.c_int, [_vp, _i32, P(_i64 * 9)]),
             "p2p_route_batch": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, _i32, _vp, _vp]),
             "p2p_route_batch_host": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _i32, _vp, _vp]),
@@ -261,6 +262,16 @@ def p2p_tree_apply_delta(r, peer: int, op, seqlist, peer_begin=None, on_device: 
     d = Delta(_addr(op), _seqs_struct(seqlist, keep), _addr(peer_begin), P2P_MEM_DEVICE if on_device else P2P_MEM_HOST)
     absent = _i64()
     _check(_load().p2p_tree_apply_delta(r, peer, ctypes.byref(d), ctypes.byref(absent)), r)
+    return int(absent.value)
+
+
+def p2p_tree_apply_delta_static(r, peer: int, op, seqlist, peer_begin=None) -> int:
+    """The allocation-free delta call: op/segment/pool arrays (and peer_begin) must be CUDA tensors.
+    Returns the number of DELETEs of absent sequences."""
+    keep = [op, peer_begin]
+    d = Delta(_addr(op), _seqs_struct(seqlist, keep), _addr(peer_begin), P2P_MEM_DEVICE)
+    absent = _i64()
+    _check(_load().p2p_tree_apply_delta_static(r, peer, ctypes.byref(d), ctypes.byref(absent)), r)
     return int(absent.value)
 
 

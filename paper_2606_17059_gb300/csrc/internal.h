@@ -3,6 +3,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <algorithm>
+#include <cstring>
 #include <string>
 #include <vector>
 
@@ -67,6 +69,13 @@ cudaError_t launch_set_tree(TreeState* d_state, TreeView* d_view, TreeState valu
 
 // Rewrites views[0 .. n) from states[0 .. n) (after a delta moved some trees' arrays).
 cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, int32_t n, cudaStream_t st);
+
+// Static scratch of the allocation-free delta call (delta_static.cu).
+enum { STATIC_BAD_OP = 1, STATIC_BAD_SEGMENT = 2, STATIC_BAD_PEER_BEGIN = 4, STATIC_TOO_LONG = 8 };
+int64_t static_scratch_tokens();
+cudaError_t static_scratch(int device, int32_t** header, int32_t** tokens);
+cudaError_t launch_validate_static(int32_t* header, const p2p_delta* d, int32_t peer, int32_t P, cudaStream_t st);
+cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* peer_begin, int64_t n, cudaStream_t st);
 
 // Host-side helpers in snapshot.cpp.
 void set_global_error(const std::string& msg);

@@ -577,6 +577,68 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   return rc;
 }
 
+// The delta call for callers that cannot allocate (see the header and delta_static.cu): device-resident
+// delta, validation on the device, scratch in the library's static device array, no arena growth and no
+// compaction.
+int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (peer < -1 || peer >= r->P) return fail(r, P2P_E_INVAL, "peer out of range");
+  if (!d) return fail(r, P2P_E_INVAL, "delta is NULL");
+  if (d->mem != P2P_MEM_DEVICE) return fail(r, P2P_E_INVAL, "p2p_tree_apply_delta_static needs a delta in device memory");
+  const p2p_seqs& S = d->seqs;
+  if (S.n < 0 || S.n_segs < 0 || S.n_pool < 0) return fail(r, P2P_E_INVAL, "negative size in delta");
+  if (S.n > 0 && (!d->op || !S.seg_begin || (S.n_segs > 0 && (!S.seg_off || !S.seg_len)) || (S.n_pool > 0 && !S.pool)))
+    return fail(r, P2P_E_INVAL, "NULL array in delta");
+  if (peer == -1 && S.n > 0 && !d->peer_begin) return fail(r, P2P_E_INVAL, "peer = -1 needs peer_begin");
+  DeviceGuard g(r->device);
+  int32_t* header = nullptr;
+  int32_t* tokens = nullptr;
+  CK(p2p::static_scratch(r->device, &header, &tokens));
+  if (S.n == 0) {
+    if (n_absent) *n_absent = 0;
+    return P2P_OK;
+  }
+  CK(p2p::launch_validate_static(header, d, peer, r->P, r->stream));
+  r->launches += 1;
+  int32_t h[4] = {0, 0, 0, 0};
+  CK(cudaMemcpyAsync(h, header, sizeof(h), cudaMemcpyDeviceToHost, r->stream));
+  CK(cudaStreamSynchronize(r->stream));
+  unsigned long long max_len = 0;
+  std::memcpy(&max_len, h, sizeof(max_len));
+  const int32_t bits = h[2];
+  if (bits & p2p::STATIC_BAD_OP) return fail(r, P2P_E_INVAL, "bad op code in the delta");
+  if (bits & p2p::STATIC_BAD_SEGMENT) return fail(r, P2P_E_INVAL, "seg_begin or a segment is malformed or outside the pool");
+  if (bits & p2p::STATIC_TOO_LONG) return fail(r, P2P_E_INVAL, "a sequence is longer than 2^31-1 tokens");
+  if (bits & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
+  const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
+  const int32_t nt = p1 - p0;
+  const int64_t stride = max_len > 0 ? (int64_t)max_len : 1;
+  if ((int64_t)nt * stride > p2p::static_scratch_tokens())
+    return fail(r, P2P_E_INVAL, "trees x longest sequence = " + std::to_string((int64_t)nt * stride) +
+                                    " tokens exceeds the static scratch of " +
+                                    std::to_string(p2p::static_scratch_tokens()) + " tokens");
+  CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d->peer_begin : nullptr, S.n, r->stream));
+  CK(p2p::launch_delta(r->d_states + p0, nt, d->op, S.seg_begin, S.seg_off, S.seg_len, S.pool, tokens, stride, r->stream));
+  r->launches += 2;
+  CK(cudaMemcpyAsync(r->h_states, r->d_states + p0, (size_t)nt * sizeof(TreeState), cudaMemcpyDeviceToHost, r->stream));
+  CK(cudaStreamSynchronize(r->stream));
+  std::memcpy(r->hs.data() + p0, r->h_states, (size_t)nt * sizeof(TreeState));
+  int rc = P2P_OK;
+  int64_t absent = 0;
+  for (int32_t p = p0; p < p1; ++p) {
+    const TreeState& t = r->hs[(size_t)p];
+    absent += t.n_absent;
+    if (rc != P2P_OK) continue;
+    if (t.status == p2p::DELTA_CORRUPT)
+      rc = fail(r, P2P_E_DEVICE, "tree " + std::to_string(p) + " is inconsistent (delta stopped at op " + std::to_string(t.op_next) + ")");
+    else if (t.status == p2p::DELTA_NEED_SPACE)
+      rc = fail(r, P2P_E_NOMEM, "tree " + std::to_string(p) + " has no room for op " + std::to_string(t.op_next) +
+                                    "; its earlier ops were applied (p2p_tree_apply_delta grows trees)");
+  }
+  if (n_absent) *n_absent = absent;
+  return rc;
+}
+
 int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
                     const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
