@@ -119,9 +119,17 @@ def dist_info():
 
 # ---- workload setup ---------------------------------------------------------------------------------
 
-def make_workload(cfg: int):
+def make_workload(cfg: int, trees: int = 0, batch: int = 0):
+    """The preset workload; trees/batch > 0 scale P and B down (smaller variants for profiling only)."""
     import workload as wl
-    return wl.Workload(cfg)
+    if not trees and not batch:
+        return wl.Workload(cfg)
+    prm = wl.preset(cfg)
+    if trees:
+        prm["P"] = trees
+    if batch:
+        prm["B"] = batch
+    return wl.Workload(params=prm, seed=wl.default_seed(cfg))
 
 
 def build_trees(W, router, with_oracle: bool, n_threads: int):
@@ -227,8 +235,10 @@ def run_ours(args):
     cfg, wdesc = WORKLOADS[args.workload]
     n_cpu = os.cpu_count() or 1
     t_setup = time.perf_counter()
-    W = make_workload(cfg)
+    W = make_workload(cfg, args.trees, args.batch)
     P, B, alpha = W.P, W.B, W.alpha
+    if args.trees or args.batch:
+        wdesc += f" [scaled down: P={P}, B={B}]"
     router = g.Router(P)
     want_oracle = rank == 0 and not args.no_cpu_baseline
     otrees = build_trees(W, router, want_oracle, n_cpu)
@@ -404,7 +414,7 @@ def run_reference(args):
     import oracle as orc
     cfg, wdesc = WORKLOADS[args.workload]
     n_cpu = os.cpu_count() or 1
-    W = make_workload(cfg)
+    W = make_workload(cfg, args.trees, args.batch)
     P, B, alpha = W.P, W.B, W.alpha
     otrees = orc.build_trees([W.tree(p) for p in range(P)], n_threads=n_cpu)
     has_delta = W.params["delta_frac"] > 0
@@ -448,6 +458,8 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--ref-requests", type=int, default=65536)
     ap.add_argument("--ref-seconds", type=float, default=4.0, help="oracle time per reference step")
+    ap.add_argument("--trees", type=int, default=0, help="override P (a scaled-down variant, not a bench line)")
+    ap.add_argument("--batch", type=int, default=0, help="override B (a scaled-down variant, not a bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         log("warmup < 3 is below the timing rules; using 3")

@@ -176,13 +176,14 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
  * caching allocator on its hot path), or a process whose device footprint must stay fixed after start-up.
  * The paper has no counterpart; this is a deployment variant of the delta call.
  * It allocates nothing, host or device: d must be in device memory (d->mem = P2P_MEM_DEVICE, else
- * P2P_E_INVAL); the delta is validated on the device; every op's sequence is gathered into one static
- * device array of the library (8 MiB of tokens plus a 256-byte header, held by every GPU that loads the
- * library until the process exits); trees are never grown or compacted.
- * Limits: (number of trees the call touches) x (longest sequence in the delta) <= 2,097,152 tokens,
- * else P2P_E_INVAL.  If a tree's arenas have no room for an op, that tree stops before it (its earlier
- * ops stay applied, other trees finish) and the call returns P2P_E_NOMEM; p2p_tree_apply_delta, which
- * may allocate, grows the tree.
+ * P2P_E_INVAL); the delta is validated on the device; the call's scratch lives in one static device
+ * array of the library (8 MiB plus a 256-byte header, held by every GPU that loads the library until the
+ * process exits); trees are never grown or compacted.
+ * Limits: the scratch holds 256 bytes per tree the call touches, plus, only when some op's sequence is
+ * split into more than two pool runs, 128 bytes x (longest sequence in tokens) per tree; a delta that
+ * needs more gets P2P_E_INVAL.  If a tree's arenas run out of room, the call returns P2P_E_NOMEM and that
+ * tree holds only part of its ops (each op applied whole or not at all); p2p_tree_apply_delta, which may
+ * allocate, grows trees.
  * The first call on a device looks up the static array's device address (cudaGetSymbolAddress, with
  * the router's device current) and caches it; make that first call before any stream capture.  Every
  * call shares the array, so calls whose device work overlaps (for example two routers on different

@@ -6,232 +6,389 @@
 // that leaves an edge part-way splits it; a DELETE prunes a leaf that no longer stores anything and folds
 // a node left with one child and no sequence into that child.
 //
-// Mapping: one warp per tree; a tree's ops run in order, trees run in parallel.  Inside an op the warp
-// cooperates: the sequence is gathered into a per-warp scratch run, child searches probe 32 sorted first
-// tokens at a time, label compares and copies move 32 tokens per instruction, child-list shifts move 32
-// entries per step.  Lane 0 performs the scalar stores; __syncwarp() orders them before the next reads.
-// Before mutating, an op checks that the node, child-entry and label arenas have room for everything it
-// may allocate; if not, the tree stops at that op with DELTA_NEED_SPACE and the host grows the arenas and
-// relaunches, so every op is applied whole or not at all.  All loops are bounded by sequence lengths
-// and list sizes.
+// Parallel schedule.  Ops on sequences with different first tokens touch disjoint subtrees (the subtree
+// under the root child of that token) and, because every node's children live in a hash table with one
+// slot per first token, disjoint slots of the root's table.  So one CTA of kBuckets warps takes a tree; warp w applies,
+// in op order, exactly the ops whose first token hashes to bucket w.  Ops on the same sequence share a
+// bucket, so their relative order -- the only order that changes the result -- is kept.  The tree's op
+// list is scanned in chunks staged in shared memory; each warp walks a chunk's bucket ids with ballots.
+// Inside an op the warp cooperates: a child lookup probes 32 table slots at once, labels are compared 128
+// tokens per step and copied 32 per step; lane 0 performs scalar stores and __syncwarp() orders them before
+// later reads.  Adding or removing a child touches one slot (a table is doubled and rehashed when it
+// passes 3/4 occupancy), so the cost of an op does not grow with the fan-out of the nodes it passes.
+//
+// Space.  Node, child-entry and label arenas are bump-allocated with compare-and-swap on the tree's
+// counters; an op reserves everything it may need before it mutates anything.  If an arena is full the
+// warp stops at that op, records the op index in its bucket cursor and flags the tree; the host grows the
+// arenas and relaunches, and every bucket resumes at its cursor, so each op is applied whole or not at
+// all.  Every loop is bounded by a sequence length, a list size or an iteration cap.
 #include "internal.h"
 
 namespace p2p {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kChunk = 4096;  // ops whose bucket ids are staged in shared memory at a time
 enum { OP_DONE = 0, OP_NEED = 1, OP_CORRUPT = 2 };
 
-// Index of `tok` among child entries [b, b + cnt) (sorted by .x), or the slot where it would go.
-__device__ bool search(const int4* child, int32_t b, int32_t cnt, int32_t tok, int lane, int32_t& at) {
-  int32_t lo = b, hi = b + cnt;
-  while (hi - lo > 32) {
-    const int32_t step = (hi - lo + 31) >> 5;
-    const int32_t idx = lo + lane * step;
-    const bool le = idx < hi && child[idx].x <= tok;
-    const int c = __popc(__ballot_sync(kFull, le));
-    if (c == 0) {
-      at = lo;
-      return false;
+// Tokens [0, na) come from a, [na, n) from b (an op's sequence as at most two pool runs).
+struct Seq {
+  const int32_t* a;
+  const int32_t* b;
+  int64_t na, n;
+  __device__ int32_t at(int64_t i) const { return i < na ? a[i] : b[i - na]; }
+};
+
+// Per-warp view of one tree: array pointers and capacities (read-only during the kernel) and the
+// tree's shared counters in global memory (updated atomically by the tree's warps).
+struct Tree {
+  int4* node;
+  int4* child;
+  int32_t* label;
+  TreeState* g;
+};
+
+// Reserves k units of the counter (capacity cap); returns the first unit or -1.  Lane 0 does the CAS.
+__device__ int32_t bump(int32_t* ctr, int32_t cap, int64_t k, int lane) {
+  int32_t r = -1;
+  if (lane == 0) {
+    int32_t old = *(volatile int32_t*)ctr;
+    for (int it = 0; it < (1 << 20); ++it) {
+      if ((int64_t)old + k > cap) break;
+      const int32_t prev = atomicCAS(ctr, old, (int32_t)(old + k));
+      if (prev == old) {
+        r = old;
+        break;
+      }
+      old = prev;
     }
-    lo += (c - 1) * step;
-    hi = min(lo + step, hi);
   }
-  const bool valid = lo + lane < hi;
-  const int32_t key = valid ? child[lo + lane].x : 0;
-  const unsigned lt = __ballot_sync(kFull, valid && key < tok);
-  const unsigned eq = __ballot_sync(kFull, valid && key == tok);
-  at = lo + __popc(lt);
-  return eq != 0;
+  return __shfl_sync(kFull, r, 0);
 }
 
-// First j in [from, lim) with a[j] != b[j], or lim.
-__device__ int64_t first_diff(const int32_t* a, const int32_t* b, int64_t from, int64_t lim, int lane) {
+// Reserves the room an op may need.  On failure the op does nothing; the units it did get are counted as
+// stale (a later compaction reclaims them), and the request is recorded for the host to grow the arenas.
+__device__ bool reserve(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, int32_t& n0, int32_t& c0, int32_t& l0,
+                        int lane) {
+  n0 = c0 = l0 = 0;
+  if (nodes && (n0 = bump(&t.g->n_node, t.g->cap_node, nodes, lane)) < 0) {
+    nodes = 0;
+  } else if (entries && (c0 = bump(&t.g->n_child, t.g->cap_child, entries, lane)) < 0) {
+    entries = 0;
+  } else if (tokens && (l0 = bump(&t.g->n_label, t.g->cap_label, tokens, lane)) < 0) {
+    tokens = 0;
+  } else {
+    return true;
+  }
+  // Failed: nodes/entries/tokens now hold only what was obtained (the failed kind was zeroed).
+  if (lane == 0) {
+    if (nodes) atomicAdd((unsigned long long*)&t.g->dead_nodes, (unsigned long long)nodes);
+    if (entries) atomicAdd((unsigned long long*)&t.g->stale_child, (unsigned long long)entries);
+    atomicOr(&t.g->status, DELTA_NEED_SPACE);
+  }
+  return false;
+}
+
+// Reserves the room of one op; if it does not fit, records the request so that the host grows the arenas
+// by at least that much before the relaunch.
+__device__ bool take(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, int32_t& n0, int32_t& c0, int32_t& l0,
+                     int lane) {
+  if (reserve(t, nodes, entries, tokens, n0, c0, l0, lane)) return true;
+  if (lane == 0) {
+    atomicMax(&t.g->need_node, (int32_t)nodes);
+    atomicMax(&t.g->need_child, (int32_t)entries);
+    atomicMax(&t.g->need_label, (int32_t)(tokens > INT32_MAX ? INT32_MAX : tokens));
+  }
+  return false;
+}
+
+// Looks `tok` up in the children table of 2^bits slots at child[off]: returns 1 (live child), 2 (tombstone
+// of tok), or 0 (absent; *slot = the first empty slot of its probe run, or -1 if there is none).  Key and
+// state are read as one 64-bit word, so a slot another warp is claiming (root table only) is seen either
+// all zero or with its final key.  Only this warp ever looks up `tok` below this node.
+__device__ int probe(const Tree& t, int32_t off, int32_t bits, int32_t tok, int lane, int32_t& slot) {
+  slot = -1;
+  if (bits == 0) return 0;
+  const uint32_t mask = (1u << bits) - 1, h = slot_hash(tok, bits);
+  for (uint32_t base = 0; base <= mask; base += 32) {
+    const uint32_t s = (h + base + lane) & mask;
+    const unsigned long long kv = *(volatile unsigned long long*)&t.child[off + s];
+    const int32_t key = (int32_t)(kv & 0xffffffffull), state = (int32_t)(kv >> 32);
+    const unsigned mine = __ballot_sync(kFull, key == tok && (state >= 1 || state == -1));
+    const unsigned empty = __ballot_sync(kFull, state == 0);
+    const int fm = mine ? __ffs(mine) - 1 : 64;
+    const int fe = empty ? __ffs(empty) - 1 : 64;
+    if (fm < fe) {
+      slot = off + (int32_t)((h + base + fm) & mask);
+      return __shfl_sync(kFull, state, fm) >= 1 ? 1 : 2;
+    }
+    if (fe < 64) {
+      slot = off + (int32_t)((h + base + fe) & mask);
+      return 0;
+    }
+  }
+  return 0;
+}
+
+// Claims an empty slot for `tok` (64-bit compare-and-swap from all-zero, key written with the claim);
+// re-probes if another warp took the slot first.  Returns the slot or -1.
+__device__ int32_t claim(const Tree& t, int32_t off, int32_t bits, int32_t tok, int32_t slot, int lane) {
+  const unsigned long long want = (unsigned long long)(uint32_t)tok | ((unsigned long long)(uint32_t)-3 << 32);
+  for (int it = 0; it <= (1 << bits) && slot >= 0; ++it) {
+    int32_t got = 0;
+    if (lane == 0) got = atomicCAS((unsigned long long*)&t.child[slot], 0ull, want) == 0ull;
+    if (__shfl_sync(kFull, got, 0)) return slot;
+    if (probe(t, off, bits, tok, lane, slot) != 0) return -1;
+  }
+  return -1;
+}
+
+// Publishes a claimed slot: label position first, then the child (the slot becomes live).
+__device__ void publish(const Tree& t, int32_t slot, int32_t child_node, int32_t loff, int32_t llen, int lane) {
+  if (lane == 0) {
+    t.child[slot].z = loff;
+    t.child[slot].w = llen;
+    __threadfence();
+    atomicExch(&t.child[slot].y, child_node);
+  }
+  __syncwarp();
+}
+
+// Writes the live entries of a table into a fresh all-zero table of 2^bits slots at child[dst] (lanes
+// insert concurrently with compare-and-swap); returns false if an insertion found no slot.
+__device__ bool rehash(const Tree& t, int32_t src, int32_t src_bits, int32_t dst, int32_t bits, int lane) {
+  const uint32_t mask = (1u << bits) - 1;
+  bool ok = true;
+  for (int32_t j = lane; j < (1 << src_bits); j += 32) {
+    const int4 e = t.child[src + j];
+    if (e.y < 1) continue;
+    const unsigned long long kv = (unsigned long long)(uint32_t)e.x | ((unsigned long long)(uint32_t)e.y << 32);
+    uint32_t s = slot_hash(e.x, bits);
+    bool placed = false;
+    for (uint32_t it = 0; it <= mask && !placed; ++it, s = (s + 1) & mask) {
+      if (atomicCAS((unsigned long long*)&t.child[dst + s], 0ull, kv) == 0ull) {
+        t.child[dst + s].z = e.z;
+        t.child[dst + s].w = e.w;
+        placed = true;
+      }
+    }
+    ok = ok && placed;
+  }
+  return __all_sync(kFull, ok);
+}
+
+__device__ void zero_slots(const Tree& t, int32_t off, int32_t n, int lane) {
+  for (int32_t j = lane; j < n; j += 32) t.child[off + j] = make_int4(0, 0, 0, 0);
+  __syncwarp();
+}
+
+// The single live child slot of a node's table (the node has exactly one child), skipping `except`.
+__device__ int32_t only_child(const Tree& t, int32_t off, int32_t bits, int32_t except, int lane) {
+  for (int32_t base = 0; base < (1 << bits); base += 32) {
+    const int32_t j = base + lane;
+    const bool live = j < (1 << bits) && off + j != except && t.child[off + j].y >= 1;
+    const unsigned m = __ballot_sync(kFull, live);
+    if (m) return off + base + __ffs(m) - 1;
+  }
+  return -1;
+}
+
+__device__ void copy_seq(int32_t* dst, const Seq& q, int64_t from, int64_t n, int lane) {
+  for (int64_t j = lane; j < n; j += 32) dst[j] = q.at(from + j);
+}
+__device__ void copy_tokens(int32_t* dst, const int32_t* src, int64_t n, int lane) {
+  for (int64_t j = lane; j < n; j += 32) dst[j] = src[j];
+}
+
+// Label tokens are never overwritten once written (the label arena only grows) and the delta's pool is
+// read-only, so "label[a .. a+n) == pool[b .. b+n)" stays true for the whole kernel once verified.  Each
+// warp remembers the last such run; ops that walk the same shared prefix as the previous op (the common
+// case: a delta references one pool copy of each shared prefix) skip re-comparing it.
+struct Memo {
+  const int32_t* lab = nullptr;
+  const int32_t* seq = nullptr;
+  int64_t n = 0;
+};
+
+// First j in [from, lim) with lab[j] != q[pos + j], or lim.
+__device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int64_t from, int64_t lim, int lane,
+                              Memo& memo) {
+  const bool in_a = pos < q.na;  // q[pos ..] starts in the first pool run, which the memo can describe
+  if (in_a) {
+    const int64_t dl = lab - memo.lab, ds = (q.a + pos) - memo.seq;
+    if (memo.lab && dl == ds && dl >= 0 && dl < memo.n) from = max(from, min(lim, memo.n - dl));
+  }
+  int64_t k = lim;
   for (int64_t j0 = from; j0 < lim; j0 += 128) {
     int32_t x[4], y[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const int64_t j = j0 + u * 32 + lane;
-      x[u] = j < lim ? a[j] : 0;
-      y[u] = j < lim ? b[j] : 0;
+      x[u] = j < lim ? lab[j] : 0;
+      y[u] = j < lim ? q.at(pos + j) : 0;
     }
+    bool hit = false;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       const unsigned m = __ballot_sync(kFull, x[u] != y[u]);
-      if (m) return j0 + u * 32 + (__ffs(m) - 1);
+      if (m && !hit) {
+        k = j0 + u * 32 + (__ffs(m) - 1);
+        hit = true;
+      }
     }
+    if (hit) break;
   }
-  return lim;
-}
-
-__device__ void copy_tokens(int32_t* dst, const int32_t* src, int64_t n, int lane) {
-  for (int64_t j = lane; j < n; j += 32) dst[j] = src[j];
-}
-
-// Moves child entries [lo, hi) up by one slot (top chunk first, so nothing is overwritten unread).
-__device__ void shift_up(int4* child, int64_t lo, int64_t hi, int lane) {
-  for (int64_t top = hi; top > lo; top -= 32) {
-    const int64_t base = top - 32 > lo ? top - 32 : lo;
-    const int64_t j = base + lane;
-    int4 v = make_int4(0, 0, 0, 0);
-    if (j < top) v = child[j];
-    __syncwarp();
-    if (j < top) child[j + 1] = v;
-    __syncwarp();
+  if (in_a && k >= 64) {  // remember a long verified run (within the first pool run)
+    memo.lab = lab;
+    memo.seq = q.a + pos;
+    memo.n = min(k, q.na - pos);
   }
+  return k;
 }
 
-// Moves child entries [lo, hi) down by one slot (bottom chunk first).
-__device__ void shift_down(int4* child, int64_t lo, int64_t hi, int lane) {
-  for (int64_t base = lo; base < hi; base += 32) {
-    const int64_t j = base + lane;
-    int4 v = make_int4(0, 0, 0, 0);
-    if (j < hi) v = child[j];
-    __syncwarp();
-    if (j < hi) child[j - 1] = v;
-    __syncwarp();
-  }
+__device__ void add_stat(int64_t* p, int64_t v, int lane) {
+  if (lane == 0 && v) atomicAdd((unsigned long long*)p, (unsigned long long)v);
 }
 
-__device__ bool has_room(TreeState& s, int64_t nodes, int64_t entries, int64_t tokens) {
-  if ((int64_t)s.n_free + ((int64_t)s.cap_node - s.n_node) >= nodes && (int64_t)s.cap_child - s.n_child >= entries &&
-      (int64_t)s.cap_label - s.n_label >= tokens)
-    return true;
-  s.need_node = (int32_t)nodes;
-  s.need_child = (int32_t)entries;
-  s.need_label = (int32_t)(tokens > INT32_MAX ? INT32_MAX : tokens);
-  return false;
-}
-
-__device__ int32_t alloc_node(TreeState& s) {
-  if (s.free_head >= 0) {
-    const int32_t v = s.free_head;
-    s.free_head = s.node[v].x;
-    s.n_free -= 1;
-    return v;
-  }
-  return s.n_node++;
-}
-
-__device__ void free_node(TreeState& s, int32_t v, int lane) {
-  if (lane == 0) s.node[v] = make_int4(s.free_head, 0, 0, 0);
-  s.free_head = v;
-  s.n_free += 1;
-}
-
-// Node x (reached through parent entry ex) has one child and stores no sequence: fold the child into x.
-// The caller has checked that the label arena has room for the two labels.
-__device__ void merge_into_parent(TreeState& s, int32_t x, int32_t ex, int lane) {
-  const int4 xe = s.child[ex];
-  const int4 xn = s.node[x];
-  const int4 ye = s.child[xn.x];
-  const int4 yn = s.node[ye.y];
+// Node x (slot *ex in its parent's table) has one child and stores no sequence: fold the child's edge into
+// x's.  The joined label is written at l0 unless the two labels are adjacent in the arena.
+__device__ void fold_child(Tree& t, int32_t x, int4* ex, int32_t yslot, int32_t l0, int lane) {
+  const int4 xe = *ex;
+  const int4 xn = t.node[x];
+  const int4 ye = t.child[yslot];
+  const int4 yn = t.node[ye.y];
   int32_t off = xe.z;
-  if (xe.z + xe.w != ye.z) {  // labels not adjacent in the arena: write the joined label
-    off = s.n_label;
-    copy_tokens(s.label + off, s.label + xe.z, xe.w, lane);
-    copy_tokens(s.label + off + xe.w, s.label + ye.z, ye.w, lane);
-    s.n_label += xe.w + ye.w;
-    s.stale_label += xe.w + ye.w;
+  if (xe.z + xe.w != ye.z) {
+    off = l0;
+    copy_tokens(t.label + off, t.label + xe.z, xe.w, lane);
+    copy_tokens(t.label + off + xe.w, t.label + ye.z, ye.w, lane);
+    add_stat(&t.g->stale_label, (int64_t)xe.w + ye.w, lane);
   }
   __syncwarp();
   if (lane == 0) {
-    s.child[ex] = make_int4(xe.x, x, off, xe.w + ye.w);
-    s.node[x] = yn;
+    ex->z = off;
+    ex->w = xe.w + ye.w;
+    t.node[x] = yn;
   }
-  s.stale_child += xn.z;
-  free_node(s, ye.y, lane);
+  add_stat(&t.g->stale_child, tab_bits(xn.y) ? (int64_t)1 << tab_bits(xn.y) : 0, lane);
+  add_stat(&t.g->dead_nodes, 1, lane);
   __syncwarp();
 }
 
-__device__ bool adjacent_labels(const TreeState& s, int32_t ex, int32_t ey) {
-  const int4 a = s.child[ex], b = s.child[ey];
-  return a.z + a.w == b.z;
+__device__ bool adjacent(const int4& a, const int4& b) { return a.z + a.w == b.z; }
+
+// Room for one more child in node cur's table (cur != 0): grows the table (doubling, rehash into fresh
+// slots) when claimed slots would pass 3/4.  Returns false if the child arena is full.
+__device__ bool ensure_slot(Tree& t, int32_t cur, int4& nd, int lane) {
+  const int32_t bits = tab_bits(nd.y), used = tab_used(nd.y);
+  if (!tab_full(bits, (int64_t)used + 1)) return true;
+  int32_t nb = bits ? bits + 1 : kMinTabBits;
+  while (nb < kMaxTabBits && (int64_t)(nd.z + 1) * 2 > ((int64_t)1 << nb)) ++nb;
+  int32_t n0, c0, l0;
+  if (!take(t, 0, (int64_t)1 << nb, 0, n0, c0, l0, lane)) return false;
+  zero_slots(t, c0, 1 << nb, lane);
+  if (bits && !rehash(t, nd.x, bits, c0, nb, lane)) return false;
+  __syncwarp();
+  add_stat(&t.g->stale_child, bits ? (int64_t)1 << bits : 0, lane);
+  nd = make_int4(c0, make_meta(nb, nd.z), nd.z, nd.w);
+  if (lane == 0) t.node[cur] = nd;
+  __syncwarp();
+  return true;
 }
 
-__device__ int insert(TreeState& s, const int32_t* seq, int64_t n, int lane) {
+__device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
+  const int64_t n = q.n;
+  if (n == 0) {
+    if (lane == 0) atomicAdd(&t.node[0].w, 1);
+    __syncwarp();
+    return OP_DONE;
+  }
   int32_t cur = 0;
   int64_t pos = 0;
+  int32_t n0, c0, l0;
   for (int64_t guard = 0; guard <= n + 1; ++guard) {
-    const int4 nd = s.node[cur];
-    if (pos == n) {
-      if (lane == 0) s.node[cur].w = nd.w + 1;
+    if (pos == n) {  // the sequence ends exactly at node cur (never the root here: n > 0)
+      if (lane == 0) t.node[cur].w += 1;
       __syncwarp();
       return OP_DONE;
     }
-    const int32_t tok = seq[pos];
-    int32_t at;
-    if (!search(s.child, nd.x, nd.y, tok, lane, at)) {
-      // New leaf edge seq[pos, n) under cur, at slot `at` of cur's (sorted) child list.
+    const int32_t tok = q.at(pos);
+    int4 nd = t.node[cur];
+    int32_t slot;
+    int st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot);
+    if (st != 1) {
+      // New leaf edge q[pos, n) under cur: revive tok's tombstone, or claim an empty slot.
       const int64_t L = n - pos;
-      const bool grow = nd.y >= nd.z;
-      const int32_t newcap = grow ? max(2, 2 * nd.y) : 0;
-      if (!has_room(s, 1, newcap, L)) return OP_NEED;
-      const int32_t leaf = alloc_node(s);
-      const int32_t loff = s.n_label;
-      copy_tokens(s.label + loff, seq + pos, L, lane);
-      s.n_label += (int32_t)L;
-      const int4 ent = make_int4(tok, leaf, loff, (int32_t)L);
-      if (!grow) {
-        shift_up(s.child, at, (int64_t)nd.x + nd.y, lane);
-        if (lane == 0) {
-          s.child[at] = ent;
-          s.node[cur].y = nd.y + 1;
+      if (st == 0) {
+        if (cur == 0) {
+          // The root table is shared by all warps of the tree: count the claim atomically; if the table
+          // would pass 3/4 the host grows it between launches.
+          int32_t meta = 0;
+          if (lane == 0) meta = atomicAdd(&t.node[0].y, 1 << 5);
+          meta = __shfl_sync(kFull, meta, 0);
+          if (slot < 0 || tab_full(tab_bits(meta), (int64_t)tab_used(meta) + 1)) {
+            if (lane == 0) {
+              atomicSub(&t.node[0].y, 1 << 5);
+              atomicMax(&t.g->need_root, 1);
+              atomicOr(&t.g->status, DELTA_NEED_SPACE);
+            }
+            return OP_NEED;
+          }
+        } else {
+          if (!ensure_slot(t, cur, nd, lane)) return OP_NEED;
+          st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot);
+          if (st != 0 || slot < 0) return OP_CORRUPT;
+          if (lane == 0) t.node[cur].y = nd.y + (1 << 5);
         }
-      } else {
-        const int32_t nb = s.n_child;
-        s.n_child += newcap;
-        const int32_t before = at - nd.x;
-        for (int64_t j = lane; j < nd.y; j += 32) {
-          const int4 v = s.child[nd.x + j];
-          s.child[nb + j + (j >= before ? 1 : 0)] = v;
-        }
-        if (lane == 0) {
-          s.child[nb + before] = ent;
-          s.node[cur] = make_int4(nb, nd.y + 1, newcap, nd.w);
-        }
-        s.stale_child += nd.z;
       }
-      if (lane == 0) s.node[leaf] = make_int4(0, 0, 0, 1);
+      if (!take(t, 1, 0, L, n0, c0, l0, lane)) {
+        if (st == 0 && lane == 0) atomicSub(&t.node[cur].y, 1 << 5);
+        return OP_NEED;
+      }
+      copy_seq(t.label + l0, q, pos, L, lane);
+      if (lane == 0) t.node[n0] = make_int4(0, 0, 0, 1);
+      __syncwarp();
+      if (st == 0 && (slot = claim(t, nd.x, tab_bits(nd.y), tok, slot, lane)) < 0) return OP_CORRUPT;
+      publish(t, slot, n0, l0, (int32_t)L, lane);
+      if (lane == 0) atomicAdd(&t.node[cur].z, 1);
       __syncwarp();
       return OP_DONE;
     }
-    const int4 ce = s.child[at];
+    int4* ent = t.child + slot;
+    const int4 ce = *ent;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
     const int64_t lim = min((int64_t)ce.w, n - pos);
-    const int64_t k = first_diff(s.label + ce.z, seq + pos, 1, lim, lane);
+    const int64_t k = first_diff(t.label + ce.z, q, pos, 1, lim, lane, memo);
     if (k == ce.w) {
       cur = ce.y;
       pos += k;
       continue;
     }
-    // The sequence leaves (or ends inside) the edge after k tokens: split it there.
+    // The sequence leaves (or ends inside) the edge after k tokens: split it there.  The new node mid
+    // gets a 4-slot table holding the lower part of the edge (and the new leaf).
     const bool tail = pos + k < n;
     const int64_t L = n - pos - k;
-    if (!has_room(s, tail ? 2 : 1, 2, tail ? L : 0)) return OP_NEED;
-    const int32_t mid = alloc_node(s);
-    const int32_t leaf = tail ? alloc_node(s) : -1;
-    const int32_t nb = s.n_child;
-    s.n_child += 2;
-    const int4 lower = make_int4(s.label[ce.z + k], ce.y, ce.z + (int32_t)k, ce.w - (int32_t)k);
-    int4 leaf_ent = make_int4(0, 0, 0, 0);
-    if (tail) {
-      const int32_t loff = s.n_label;
-      copy_tokens(s.label + loff, seq + pos + k, L, lane);
-      s.n_label += (int32_t)L;
-      leaf_ent = make_int4(seq[pos + k], leaf, loff, (int32_t)L);
-    }
+    if (!take(t, tail ? 2 : 1, 1 << kMinTabBits, tail ? L : 0, n0, c0, l0, lane)) return OP_NEED;
+    const int32_t mid = n0, leaf = n0 + 1;
+    zero_slots(t, c0, 1 << kMinTabBits, lane);
+    const int4 lower = make_int4(t.label[ce.z + k], ce.y, ce.z + (int32_t)k, ce.w - (int32_t)k);
+    if (tail) copy_seq(t.label + l0, q, pos + k, L, lane);
+    const int32_t leaf_tok = tail ? q.at(pos + k) : 0;
+    __syncwarp();
     if (lane == 0) {
+      const uint32_t mask = (1u << kMinTabBits) - 1;
+      uint32_t s0 = slot_hash(lower.x, kMinTabBits);
+      t.child[c0 + s0] = lower;
       if (tail) {
-        const bool leaf_first = leaf_ent.x < lower.x;
-        s.child[nb] = leaf_first ? leaf_ent : lower;
-        s.child[nb + 1] = leaf_first ? lower : leaf_ent;
-        s.node[leaf] = make_int4(0, 0, 0, 1);
-      } else {
-        s.child[nb] = lower;
+        uint32_t s1 = slot_hash(leaf_tok, kMinTabBits);
+        while (s1 == s0) s1 = (s1 + 1) & mask;
+        t.child[c0 + s1] = make_int4(leaf_tok, leaf, l0, (int32_t)L);
+        t.node[leaf] = make_int4(0, 0, 0, 1);
       }
-      s.node[mid] = make_int4(nb, tail ? 2 : 1, 2, tail ? 0 : 1);
-      s.child[at] = make_int4(ce.x, mid, ce.z, (int32_t)k);
+      t.node[mid] = make_int4(c0, make_meta(kMinTabBits, tail ? 2 : 1), tail ? 2 : 1, tail ? 0 : 1);
+      __threadfence_block();
+      ent->w = (int32_t)k;  // the slot keeps its key; label_off is unchanged
+      atomicExch(&ent->y, mid);
     }
     __syncwarp();
     return OP_DONE;
@@ -239,103 +396,249 @@ __device__ int insert(TreeState& s, const int32_t* seq, int64_t n, int lane) {
   return OP_CORRUPT;
 }
 
-__device__ int remove(TreeState& s, const int32_t* seq, int64_t n, int lane) {
-  int32_t cur = 0, par = -1, e_cur = -1, e_par = -1;
+__device__ int remove(Tree& t, const Seq& q, int lane, Memo& memo) {
+  const int64_t n = q.n;
+  if (n == 0) {
+    int ok = 0;
+    if (lane == 0) {
+      const int32_t old = atomicAdd(&t.node[0].w, -1);
+      ok = old > 0;
+      if (!ok) atomicAdd(&t.node[0].w, 1);
+    }
+    if (!__shfl_sync(kFull, ok, 0)) add_stat(&t.g->n_absent, 1, lane);
+    __syncwarp();
+    return OP_DONE;
+  }
+  int32_t cur = 0, par = -1;
+  int4 *e_cur = nullptr, *e_par = nullptr;
   int64_t pos = 0;
   for (int64_t guard = 0; pos < n; ++guard) {
     if (guard > n) return OP_CORRUPT;
-    const int4 nd = s.node[cur];
-    int32_t at;
-    if (!search(s.child, nd.x, nd.y, seq[pos], lane, at)) {
-      s.n_absent += 1;
+    const int4 nd = t.node[cur];
+    int32_t slot;
+    if (probe(t, nd.x, tab_bits(nd.y), q.at(pos), lane, slot) != 1) {
+      add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
-    const int4 ce = s.child[at];
+    int4* ent = t.child + slot;
+    const int4 ce = *ent;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
-    if (pos + ce.w > n || first_diff(s.label + ce.z, seq + pos, 1, ce.w, lane) < ce.w) {
-      s.n_absent += 1;
+    if (pos + ce.w > n || first_diff(t.label + ce.z, q, pos, 1, ce.w, lane, memo) < ce.w) {
+      add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
     e_par = e_cur;
     par = cur;
-    e_cur = at;
+    e_cur = ent;
     cur = ce.y;
     pos += ce.w;
   }
-  const int4 nd = s.node[cur];
+  const int4 nd = t.node[cur];
   if (nd.w == 0) {
-    s.n_absent += 1;
+    add_stat(&t.g->n_absent, 1, lane);
     return OP_DONE;
   }
-  if (cur == 0 || nd.w > 1 || nd.y >= 2) {
-    if (lane == 0) s.node[cur].w = nd.w - 1;
+  if (nd.w > 1 || nd.z >= 2) {
+    if (lane == 0) t.node[cur].w = nd.w - 1;
     __syncwarp();
     return OP_DONE;
   }
-  if (nd.y == 1) {  // no sequence ends here any more and one child is left: fold the child in
-    const int64_t need = adjacent_labels(s, e_cur, nd.x) ? 0 : (int64_t)s.child[e_cur].w + s.child[nd.x].w;
-    if (!has_room(s, 0, 0, need)) return OP_NEED;
-    merge_into_parent(s, cur, e_cur, lane);
+  int32_t n0, c0, l0;
+  if (nd.z == 1) {  // no sequence ends here any more and one child is left: fold the child in
+    const int32_t ys = only_child(t, nd.x, tab_bits(nd.y), -1, lane);
+    if (ys < 0) return OP_CORRUPT;
+    const int4 ce = *e_cur, ye = t.child[ys];
+    const int64_t need = adjacent(ce, ye) ? 0 : (int64_t)ce.w + ye.w;
+    if (!take(t, 0, 0, need, n0, c0, l0, lane)) return OP_NEED;
+    fold_child(t, cur, e_cur, ys, l0, lane);
     return OP_DONE;
   }
-  // A leaf that stores nothing any more: unlink it from its parent.
-  const int4 pn = s.node[par];
-  const bool fold_parent = par != 0 && pn.w == 0 && pn.y == 2;
+  // A leaf that stores nothing any more: tombstone its slot in the parent's table.
+  const int4 pn = t.node[par];
+  const bool fold_parent = par != 0 && pn.w == 0 && pn.z == 2;
+  int32_t other = -1;
   if (fold_parent) {
-    const int32_t other = (e_cur == pn.x) ? pn.x + 1 : pn.x;
-    const int64_t need = adjacent_labels(s, e_par, other) ? 0 : (int64_t)s.child[e_par].w + s.child[other].w;
-    if (!has_room(s, 0, 0, need)) return OP_NEED;
+    other = only_child(t, pn.x, tab_bits(pn.y), (int32_t)(e_cur - t.child), lane);
+    if (other < 0) return OP_CORRUPT;
+    const int4 oe = t.child[other];
+    const int64_t need = adjacent(*e_par, oe) ? 0 : (int64_t)e_par->w + oe.w;
+    if (!take(t, 0, 0, need, n0, c0, l0, lane)) return OP_NEED;
   }
-  const int32_t leaf_label = s.child[e_cur].w;
-  shift_down(s.child, (int64_t)e_cur + 1, (int64_t)pn.x + pn.y, lane);
-  if (lane == 0) s.node[par].y = pn.y - 1;
-  s.stale_child += nd.z;
-  s.stale_label += leaf_label;
-  free_node(s, cur, lane);
+  const int32_t leaf_label = e_cur->w;
+  if (lane == 0) {
+    atomicExch(&e_cur->y, -1);  // the slot keeps its key
+    atomicAdd(&t.node[par].z, -1);
+  }
+  add_stat(&t.g->stale_label, leaf_label, lane);
+  add_stat(&t.g->dead_nodes, 1, lane);
+  add_stat(&t.g->stale_child, tab_bits(nd.y) ? (int64_t)1 << tab_bits(nd.y) : 0, lane);
   __syncwarp();
-  if (fold_parent) merge_into_parent(s, par, e_par, lane);
+  if (fold_parent) fold_child(t, par, e_par, other, l0, lane);
   return OP_DONE;
 }
 
-__global__ void __launch_bounds__(32) delta_kernel(TreeState* states, const int32_t* __restrict__ op,
-                                                   const int64_t* __restrict__ seg_begin,
-                                                   const int64_t* __restrict__ seg_off,
-                                                   const int32_t* __restrict__ seg_len,
-                                                   const int32_t* __restrict__ pool, int32_t* scratch,
-                                                   int64_t stride) {
-  const int lane = threadIdx.x;
-  TreeState s = states[blockIdx.x];
-  if (s.status != DELTA_OK || s.op_next >= s.op_end) return;
-  int32_t* buf = scratch + (int64_t)blockIdx.x * stride;
-  for (int64_t i = s.op_next; i < s.op_end; ++i) {
-    int64_t n = 0;
-    for (int64_t g = __ldg(seg_begin + i); g < __ldg(seg_begin + i + 1); ++g) {
-      const int32_t* src = pool + __ldg(seg_off + g);
-      const int32_t L = __ldg(seg_len + g);
-      for (int32_t j = lane; j < L; j += 32) buf[n + j] = __ldg(src + j);
-      n += L;
+// Bucket (warp) of an op: a hash of the sequence's first token.
+__device__ __forceinline__ int32_t bucket_of(int32_t tok) {
+  return (int32_t)(((uint32_t)tok * 0x85EBCA6Bu) >> (32 - kDeltaBucketBits));
+}
+
+__global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* states, int64_t* cursors,
+                                                                    const int32_t* __restrict__ op,
+                                                                    const int64_t* __restrict__ seg_begin,
+                                                                    const int64_t* __restrict__ seg_off,
+                                                                    const int32_t* __restrict__ seg_len,
+                                                                    const int32_t* __restrict__ pool,
+                                                                    int32_t* gather, int64_t stride) {
+  __shared__ int8_t s_bucket[kChunk];
+  __shared__ int s_any;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  TreeState* gs = states + blockIdx.x;
+  const int64_t op_begin = gs->op_begin, op_end = gs->op_end;
+  int64_t* my_cursor = cursors + (int64_t)blockIdx.x * kDeltaBuckets + warp;
+  int64_t next = *my_cursor;  // ops of this bucket before `next` are applied
+  if (threadIdx.x == 0) s_any = 0;
+  __syncthreads();
+  if (lane == 0 && next < op_end) atomicOr(&s_any, 1);
+  __syncthreads();
+  if (!s_any || gs->status & DELTA_CORRUPT) return;
+  Tree t;
+  t.node = gs->node;
+  t.child = gs->child;
+  t.label = gs->label;
+  t.g = gs;
+  int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaBuckets + warp) * stride : nullptr;
+  bool stopped = next >= op_end;
+  Memo memo;
+  for (int64_t c0 = op_begin; c0 < op_end; c0 += kChunk) {
+    const int64_t clen = min((int64_t)kChunk, op_end - c0);
+    for (int64_t j = threadIdx.x; j < clen; j += blockDim.x) {
+      const int64_t i = c0 + j;
+      int32_t b = 0;  // empty sequences: bucket 0
+      for (int64_t g = seg_begin[i]; g < seg_begin[i + 1]; ++g) {
+        if (seg_len[g] > 0) {
+          b = bucket_of(pool[seg_off[g]]);
+          break;
+        }
+      }
+      s_bucket[j] = (int8_t)b;
     }
-    __syncwarp();
-    const int r = __ldg(op + i) == 0 ? insert(s, buf, n, lane) : remove(s, buf, n, lane);
-    if (r != OP_DONE) {
-      s.status = r == OP_NEED ? DELTA_NEED_SPACE : DELTA_CORRUPT;
-      s.op_next = i;
-      break;
+    __syncthreads();
+    if (!stopped && next < c0 + clen) {
+      for (int64_t j0 = max((int64_t)0, next - c0); j0 < clen && !stopped; j0 += 32) {
+        const int64_t j = j0 + lane;
+        unsigned mine = __ballot_sync(kFull, j < clen && s_bucket[j] == warp);
+        while (mine && !stopped) {
+          const int64_t i = c0 + j0 + (__ffs(mine) - 1);
+          mine &= mine - 1;
+          // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
+          const int64_t g0 = seg_begin[i], g1 = seg_begin[i + 1];
+          Seq q;
+          if (g1 - g0 <= 2) {
+            q.a = pool + (g1 > g0 ? seg_off[g0] : 0);
+            q.na = g1 > g0 ? seg_len[g0] : 0;
+            q.b = g1 - g0 == 2 ? pool + seg_off[g0 + 1] : q.a;
+            q.n = q.na + (g1 - g0 == 2 ? seg_len[g0 + 1] : 0);
+          } else {
+            if (!buf) {  // the host gives gather scratch whenever an op has more than two runs
+              if (lane == 0) atomicOr(&gs->status, DELTA_CORRUPT);
+              stopped = true;
+              next = i;
+              break;
+            }
+            int64_t len = 0;
+            for (int64_t g = g0; g < g1; ++g) {
+              copy_tokens(buf + len, pool + seg_off[g], seg_len[g], lane);
+              len += seg_len[g];
+            }
+            __syncwarp();
+            q.a = q.b = buf;
+            q.na = q.n = len;
+          }
+          const int r = op[i] == P2P_OP_INSERT ? insert(t, q, lane, memo) : remove(t, q, lane, memo);
+          if (r != OP_DONE) {
+            stopped = true;
+            next = i;
+            if (r == OP_CORRUPT && lane == 0) atomicOr(&gs->status, DELTA_CORRUPT);
+          } else {
+            next = i + 1;
+          }
+        }
+      }
     }
-    s.op_next = i + 1;
+    __syncthreads();
   }
-  __syncwarp();
-  if (lane == 0) states[blockIdx.x] = s;
+  if (!stopped) next = op_end;
+  if (lane == 0) *my_cursor = next;
+}
+
+// Validates a device-resident delta into header (int32 words: [0..1] longest sequence as u64, [2] error
+// bits STATIC_*, [3] most pool runs of one op); the header must be zero on entry.
+__global__ void validate_kernel(int32_t* header, const int32_t* __restrict__ op, const int64_t* __restrict__ seg_begin,
+                                const int64_t* __restrict__ seg_off, const int32_t* __restrict__ seg_len, int64_t n,
+                                int64_t n_segs, int64_t n_pool, const int64_t* __restrict__ peer_begin, int32_t P) {
+  unsigned long long* max_len = reinterpret_cast<unsigned long long*>(header);
+  int32_t* err = header + 2;
+  int32_t* max_runs = header + 3;
+  const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+  for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+    int bits = 0;
+    if (op[i] != P2P_OP_INSERT && op[i] != P2P_OP_DELETE) bits |= STATIC_BAD_OP;
+    const int64_t a = seg_begin[i], b = seg_begin[i + 1];
+    if (a < 0 || b < a || b > n_segs || (i == 0 && a != 0) || (i == n - 1 && b != n_segs)) {
+      bits |= STATIC_BAD_SEGMENT;
+    } else {
+      int64_t len = 0;
+      for (int64_t g = a; g < b; ++g) {
+        const int64_t off = seg_off[g], l = seg_len[g];
+        if (l < 0 || off < 0 || off > n_pool - l) {
+          bits |= STATIC_BAD_SEGMENT;
+          break;
+        }
+        len += l;
+      }
+      if (len > INT32_MAX) bits |= STATIC_TOO_LONG;
+      atomicMax(max_len, (unsigned long long)len);
+      atomicMax(max_runs, (int32_t)min(b - a, (int64_t)INT32_MAX));
+    }
+    if (bits) atomicOr(err, bits);
+  }
+  if (peer_begin && blockIdx.x == 0) {
+    for (int32_t p = threadIdx.x; p <= P; p += blockDim.x) {
+      const int64_t v = peer_begin[p];
+      if ((p == 0 && v != 0) || (p == P && v != n) || (p > 0 && v < peer_begin[p - 1]))
+        atomicOr(err, STATIC_BAD_PEER_BEGIN);
+    }
+  }
+}
+
+// Sets each tree's op range for this call on the device (peer_begin stays in device memory).
+__global__ void init_ranges_kernel(TreeState* states, int32_t nt, const int64_t* __restrict__ peer_begin, int64_t n) {
+  const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= nt) return;
+  states[i].op_begin = peer_begin ? peer_begin[i] : 0;
+  states[i].op_end = peer_begin ? peer_begin[i + 1] : n;
+  states[i].status = DELTA_OK;
+  states[i].need_node = states[i].need_child = states[i].need_label = states[i].need_root = 0;
+  states[i].n_absent = 0;
+}
+
+__global__ void init_cursors_kernel(const TreeState* states, int64_t* cursors, int32_t nt) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < (int64_t)nt * kDeltaBuckets) cursors[i] = states[i / kDeltaBuckets].op_begin;
 }
 
 __global__ void set_tree_kernel(TreeState* st, TreeView* view, TreeState v) {
   *st = v;
-  *view = TreeView{v.node, v.child, v.label};
+  const int4 root = v.node[0];
+  *view = TreeView{v.node, v.child, v.label, root.x, tab_bits(root.y)};
 }
 
 __global__ void refresh_views_kernel(const TreeState* st, TreeView* view, int32_t n) {
   const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < n) view[i] = TreeView{st[i].node, st[i].child, st[i].label};
+  if (i < n) {
+    const int4 root = st[i].node[0];
+    view[i] = TreeView{st[i].node, st[i].child, st[i].label, root.x, tab_bits(root.y)};
+  }
 }
 
 }  // namespace
@@ -346,11 +649,35 @@ cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, i
   return cudaGetLastError();
 }
 
-cudaError_t launch_delta(TreeState* d_states, int32_t n_trees, const int32_t* op, const int64_t* seg_begin,
-                         const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool, int32_t* scratch,
-                         int64_t scratch_stride, cudaStream_t st) {
+cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int32_t n_trees, cudaStream_t st) {
   if (n_trees <= 0) return cudaSuccess;
-  delta_kernel<<<n_trees, 32, 0, st>>>(d_states, op, seg_begin, seg_off, seg_len, pool, scratch, scratch_stride);
+  const int64_t total = (int64_t)n_trees * kDeltaBuckets;
+  init_cursors_kernel<<<(int)((total + 255) / 256), 256, 0, st>>>(d_states, cursors, n_trees);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
+                         const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
+                         int32_t* gather, int64_t gather_stride, cudaStream_t st) {
+  if (n_trees <= 0) return cudaSuccess;
+  delta_kernel<<<n_trees, kDeltaBuckets * 32, 0, st>>>(d_states, cursors, op, seg_begin, seg_off, seg_len, pool, gather,
+                                                       gather_stride);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_validate(int32_t* header, const p2p_delta* d, int32_t peer, int32_t P, cudaStream_t st) {
+  cudaError_t e = cudaMemsetAsync(header, 0, kStaticHeaderInts * sizeof(int32_t), st);
+  if (e != cudaSuccess) return e;
+  const p2p_seqs& S = d->seqs;
+  const int64_t blocks = std::min<int64_t>((S.n + 255) / 256, 4096);
+  validate_kernel<<<(int)std::max<int64_t>(blocks, 1), 256, 0, st>>>(header, d->op, S.seg_begin, S.seg_off, S.seg_len,
+                                                                    S.n, S.n_segs, S.n_pool,
+                                                                    peer == -1 ? d->peer_begin : nullptr, P);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* peer_begin, int64_t n, cudaStream_t st) {
+  init_ranges_kernel<<<(nt + 127) / 128, 128, 0, st>>>(d_states, nt, peer_begin, n);
   return cudaGetLastError();
 }
 

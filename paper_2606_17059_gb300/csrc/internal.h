@@ -19,35 +19,56 @@ struct p2p_snapshot {
 namespace p2p {
 
 // Device layout of one tree (HBM, one allocation per array):
-//   node[v]  = {child_begin, child_count, child_cap, term_count}          (int4, 16 B)
-//   child[e] = {first_tok, node, label_off, label_len} of one child edge   (int4, 16 B)
-//   label[]  = int32 tokens; an edge's label is label[label_off .. +label_len)
-// Node 0 is the root.  A node's children occupy child[child_begin .. +child_count), ascending by
-// first_tok, inside a reserved range of child_cap entries.  Keeping the child's label position in the
-// parent's entry lets a walk start comparing the label as soon as the child search returns.
+//   node[v]  = {tab_off, meta, live, term_count}                          (int4, 16 B)
+//              v's children live in an open-addressing hash table of 2^(meta & 31) slots at
+//              child[tab_off ..] (no table when meta == 0); meta >> 5 counts the slots ever claimed
+//              (live children + tombstones); live = number of children; term_count = sequences ending at v.
+//   child[s] = {first_tok, node, label_off, label_len}: one slot of a children table (int4, 16 B).
+//              .node: 0 = empty slot (the slot is all zero), >= 1 = the child, -1 = removed (tombstone,
+//              key kept), -3 = being claimed during a delta.  Slots are probed linearly from a
+//              multiplicative hash of first_tok.
+//   label[]  = int32 tokens; an edge's label is label[label_off .. +label_len).
+// Node 0 is the root.  Keeping the child's label position in its slot lets a walk start comparing the
+// label as soon as the lookup returns; every lookup is one coalesced probe of 32 consecutive slots.
 struct TreeView {
   const int4* node;
   const int4* child;
   const int32_t* label;
+  int32_t root_off, root_bits;  // the root's children table (copied from node[0] when the view is set)
 };
 
-// Mutable state of one tree, owned by the delta kernel while it runs and mirrored on the host.
+// Mutable state of one tree, shared by the delta kernel's warps for that tree (counters updated with
+// atomics) and mirrored on the host between calls.
 struct TreeState {
   int4* node;
   int4* child;
   int32_t* label;
-  int32_t n_node, cap_node;    // node slots used (high-water mark) / capacity
-  int32_t n_child, cap_child;  // child entries used (bump arena) / capacity
+  int32_t n_node, cap_node;    // node slots used (bump arena) / capacity
+  int32_t n_child, cap_child;  // child-table slots used (bump arena) / capacity
   int32_t n_label, cap_label;  // label tokens used (bump arena) / capacity
-  int32_t free_head, n_free;   // free node slots, linked through node[v].x
-  int32_t status;              // DELTA_OK, DELTA_NEED_SPACE, DELTA_CORRUPT
-  int32_t need_node, need_child, need_label;  // room the first unapplied op needs
-  int64_t op_next, op_end;     // ops still to apply: [op_next, op_end)
+  int32_t status;              // DELTA_* bits
+  int32_t need_node, need_child, need_label, need_root;  // largest request that did not fit
+  int32_t pad_;
+  int64_t op_begin, op_end;    // this call's ops for the tree: [op_begin, op_end)
   int64_t n_absent;            // DELETEs of sequences that were not stored
-  int64_t stale_child, stale_label;  // unreachable child entries / label tokens
+  int64_t stale_child, stale_label, dead_nodes;  // unreachable arena space
 };
 
 enum { DELTA_OK = 0, DELTA_NEED_SPACE = 1, DELTA_CORRUPT = 2 };
+
+// Warps per tree in the delta kernel; ops are bucketed by a hash of their first token.
+constexpr int kDeltaBucketBits = 5;
+constexpr int kDeltaBuckets = 1 << kDeltaBucketBits;
+
+// Children tables: at least 4 slots; grown (doubled) when claimed slots would pass 3/4 of the table.
+constexpr int kMinTabBits = 2;
+inline __host__ __device__ int32_t tab_bits(int32_t meta) { return meta & 31; }
+inline __host__ __device__ int32_t tab_used(int32_t meta) { return (int32_t)((uint32_t)meta >> 5); }
+inline __host__ __device__ int32_t make_meta(int32_t bits, int32_t used) { return bits | (int32_t)((uint32_t)used << 5); }
+inline __host__ __device__ bool tab_full(int32_t bits, int64_t used_after) {
+  return bits == 0 || used_after * 4 > ((int64_t)3 << bits);
+}
+constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits of meta
 
 // Bits of the router's device error word.
 enum { ERR_BAD_OFFSETS = 1, ERR_CORRUPT_TREE = 2 };
@@ -57,11 +78,19 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
                          int32_t* out_match, int32_t* out_peer, int32_t* d_err, int num_sms, cudaStream_t st);
 
-// Delta kernel: applies the ops [op_next, op_end) of states[0 .. n_trees) (one warp per tree).
-// scratch holds n_trees * scratch_stride tokens (each op's sequence is gathered there).
-cudaError_t launch_delta(TreeState* d_states, int32_t n_trees, const int32_t* op, const int64_t* seg_begin,
-                         const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool, int32_t* scratch,
-                         int64_t scratch_stride, cudaStream_t st);
+// Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaBuckets warps
+// per tree.  cursors[n_trees * kDeltaBuckets] holds each bucket's next op (set by launch_init_cursors,
+// kept across relaunches).  gather (n_trees * kDeltaBuckets * gather_stride tokens) is needed only when an
+// op's sequence has more than two pool runs; otherwise it may be NULL.
+cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
+                         const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
+                         int32_t* gather, int64_t gather_stride, cudaStream_t st);
+cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int32_t n_trees, cudaStream_t st);
+
+// Home slot of a first token in a children table of 2^bits slots (host table builder and kernels).
+inline __host__ __device__ uint32_t slot_hash(int32_t tok, int32_t bits) {
+  return bits ? ((uint32_t)tok * 0x9E3779B1u) >> (32 - bits) : 0u;
+}
 
 // Writes a tree's state and view on the device (values passed as kernel parameters, so no host buffer
 // has to outlive the call).
@@ -74,8 +103,11 @@ cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, i
 enum { STATIC_BAD_OP = 1, STATIC_BAD_SEGMENT = 2, STATIC_BAD_PEER_BEGIN = 4, STATIC_TOO_LONG = 8 };
 int64_t static_scratch_tokens();
 cudaError_t static_scratch(int device, int32_t** header, int32_t** tokens);
-cudaError_t launch_validate_static(int32_t* header, const p2p_delta* d, int32_t peer, int32_t P, cudaStream_t st);
+// Validates a device-resident delta on the device into a kStaticHeaderInts-word header (zeroed first):
+// [0..1] longest sequence (u64), [2] STATIC_* error bits, [3] most pool runs of one op.
+cudaError_t launch_validate(int32_t* header, const p2p_delta* d, int32_t peer, int32_t P, cudaStream_t st);
 cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* peer_begin, int64_t n, cudaStream_t st);
+constexpr int kStaticHeaderInts = 64;
 
 // Host-side helpers in snapshot.cpp.
 void set_global_error(const std::string& msg);

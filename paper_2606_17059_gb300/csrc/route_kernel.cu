@@ -6,9 +6,9 @@
 //
 // Mapping: one CTA owns one request at a time (grid-stride over requests).  The request's tokens are
 // staged once into shared memory and shared by the CTA's warps; warp w walks trees w, w+W, ...  A walk
-// is warp-cooperative: a child search probes 32 sorted first tokens per step (32-ary narrowing for wide
-// nodes, then one ballot), and an edge label is compared 32 tokens per load with several loads in flight
-// per lane; the first mismatch comes from __ballot_sync + __ffs.  Each warp keeps the best packed route
+// is warp-cooperative: a child lookup probes 32 slots of the node's children hash table at once (one
+// coalesced load, whatever the fan-out), and an edge label is compared 32 tokens per load with several
+// loads in flight per lane; the first mismatch comes from __ballot_sync + __ffs.  Each warp keeps the best packed route
 // key of its trees; the CTA reduces the W keys in shared memory.  Integer work only: no tensor cores.
 #include "internal.h"
 
@@ -25,33 +25,29 @@ __device__ __forceinline__ int32_t req_at(const int32_t* s_req, int32_t n_s, con
   return i < n_s ? s_req[i] : __ldg(g_req + i);
 }
 
-// Child of the node whose entries are ent[0 .. cnt) with first token `tok`.  Returns false if none.
-__device__ __forceinline__ bool find_child(const int4* __restrict__ ent, int32_t cnt, int32_t tok, int lane,
+// Child with first token `tok` in the children table of 2^bits slots at tab: one coalesced probe of 32
+// consecutive slots (a table is at most 3/4 full, so the probe run almost always fits).  Returns false if
+// there is no such child.
+__device__ __forceinline__ bool find_child(const int4* __restrict__ tab, int32_t bits, int32_t tok, int lane,
                                            int4& out) {
-  int32_t lo = 0, hi = cnt;
-  while (hi - lo > 32) {
-    const int32_t step = (hi - lo + 31) >> 5;
-    const int32_t idx = lo + lane * step;
-    const bool le = idx < hi && __ldg(&ent[idx].x) <= tok;
-    const int c = __popc(__ballot_sync(kFull, le));
-    if (c == 0) return false;
-    lo += (c - 1) * step;
-    hi = min(lo + step, hi);
+  if (bits == 0) return false;
+  const uint32_t mask = (1u << bits) - 1, h = slot_hash(tok, bits);
+  for (uint32_t base = 0; base <= mask; base += 32) {
+    const int4 e = __ldg(tab + ((h + base + lane) & mask));
+    const unsigned live = __ballot_sync(kFull, e.y >= 1 && e.x == tok);
+    const unsigned empty = __ballot_sync(kFull, e.y == 0);
+    const int fl = live ? __ffs(live) - 1 : 64;
+    const int fe = empty ? __ffs(empty) - 1 : 64;
+    if (fl < fe) {
+      out.x = tok;
+      out.y = __shfl_sync(kFull, e.y, fl);
+      out.z = __shfl_sync(kFull, e.z, fl);
+      out.w = __shfl_sync(kFull, e.w, fl);
+      return true;
+    }
+    if (fe < 64) return false;
   }
-  int4 e = make_int4(0, 0, 0, 0);
-  bool hit = false;
-  if (lo + lane < hi) {
-    e = __ldg(ent + lo + lane);
-    hit = e.x == tok;
-  }
-  const unsigned m = __ballot_sync(kFull, hit);
-  if (!m) return false;
-  const int src = __ffs(m) - 1;
-  out.x = tok;
-  out.y = __shfl_sync(kFull, e.y, src);
-  out.z = __shfl_sync(kFull, e.z, src);
-  out.w = __shfl_sync(kFull, e.w, src);
-  return true;
+  return false;
 }
 
 // First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.
@@ -78,13 +74,12 @@ __device__ __forceinline__ int64_t first_mismatch(const int32_t* __restrict__ la
 // match(r, T) for one tree, computed by the whole warp (result uniform across lanes).
 __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int64_t len,
                         int lane, int32_t* err) {
+  if (len == 0) return 0;
+  int4 ce;
+  if (!find_child(t.child + t.root_off, t.root_bits, req_at(s_req, n_s, g_req, 0), lane, ce)) return 0;
   int64_t pos = 0;
-  int4 nd = __ldg(t.node);
-  while (pos < len && nd.y > 0) {
-    const int32_t tok = req_at(s_req, n_s, g_req, pos);
-    int4 ce;
-    if (!find_child(t.child + nd.x, nd.y, tok, lane, ce)) break;
-    if (ce.w <= 0) {  // cannot happen in a valid tree; keeps the loop finite if it does
+  for (;;) {
+    if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree; keeps the loop finite if it does
       if (lane == 0) atomicOr(err, ERR_CORRUPT_TREE);
       break;
     }
@@ -92,8 +87,8 @@ __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, co
     const int64_t lim = min((int64_t)ce.w, len - pos);
     const int64_t k = first_mismatch(t.label + ce.z, s_req, n_s, g_req, pos, lim, lane);
     pos += k;
-    if (k < ce.w) break;
-    nd = nn;
+    if (k < ce.w || pos >= len || nn.z <= 0) break;
+    if (!find_child(t.child + nn.x, tab_bits(nn.y), req_at(s_req, n_s, g_req, pos), lane, ce)) break;
   }
   return (int32_t)pos;
 }

@@ -24,6 +24,31 @@ struct DevBuf {
 
 int32_t clamp_i32(int64_t v) { return (int32_t)std::min<int64_t>(v, INT32_MAX); }
 
+int64_t next_pow2(int64_t v) {
+  int64_t p = 1;
+  while (p < v) p <<= 1;
+  return p;
+}
+int32_t log2_exact(int64_t p) {
+  int32_t b = 0;
+  while (((int64_t)1 << b) < p) ++b;
+  return b;
+}
+// Children-table sizes (log2 slots): load factor <= 1/2 at upload; the root's table gets extra room (at
+// least 64 slots) because only the host can grow it.
+int32_t table_bits_for(int64_t live, bool root) {
+  if (root) return log2_exact(next_pow2(std::max<int64_t>(64, 2 * live + 32)));
+  return live == 0 ? 0 : std::max<int32_t>(p2p::kMinTabBits, log2_exact(next_pow2(2 * live)));
+}
+
+// Inserts entry e into the table of 2^bits slots at tab (linear probing from its home slot).
+void table_put(int4* tab, int32_t bits, const int4& e) {
+  const uint32_t mask = (1u << bits) - 1;
+  uint32_t s = p2p::slot_hash(e.x, bits);
+  while (tab[s].y != 0) s = (s + 1) & mask;
+  tab[s] = e;
+}
+
 }  // namespace
 
 struct p2p_router {
@@ -37,13 +62,14 @@ struct p2p_router {
   TreeState* d_states = nullptr;
   int32_t* d_load = nullptr;
   int32_t* d_err = nullptr;
+  int32_t* d_hdr = nullptr;  // validation result of device-resident deltas
   int32_t* h_load = nullptr;  // pinned, kLoadRing slots of P values
   cudaEvent_t load_ev[kLoadRing] = {};
   int load_slot = 0;
-  int32_t* h_err = nullptr;        // pinned
-  TreeState* h_states = nullptr;   // pinned, P entries
+  int32_t* h_err = nullptr;       // pinned
+  TreeState* h_states = nullptr;  // pinned, P entries
   DevBuf req_tok, req_off, out_match, out_peer;
-  DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_scratch;
+  DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_cursors, d_gather;
   int64_t launches = 0;  // kernels this router has launched
   std::string err;
 };
@@ -74,9 +100,9 @@ int cuda_fail(p2p_router* r, cudaError_t e, const char* what) {
   return fail(r, P2P_E_CUDA, std::string(what) + ": " + cudaGetErrorString(e));
 }
 
-#define CK(call)                                         \
-  do {                                                   \
-    cudaError_t e_ = (call);                             \
+#define CK(call)                                           \
+  do {                                                     \
+    cudaError_t e_ = (call);                               \
     if (e_ != cudaSuccess) return cuda_fail(r, e_, #call); \
   } while (0)
 
@@ -127,16 +153,20 @@ cudaError_t alloc_tree_arrays(p2p_router* r, TreeState& t, int32_t cap_node, int
   t.cap_node = cap_node;
   t.cap_child = cap_child;
   t.cap_label = cap_label;
-  t.free_head = -1;
   return cudaSuccess;
 }
 
 int install_empty_tree(p2p_router* r, int32_t p) {
   TreeState t;
-  cudaError_t e = alloc_tree_arrays(r, t, 64, 64, 1024);
+  const int32_t rb = table_bits_for(0, true);
+  cudaError_t e = alloc_tree_arrays(r, t, 64, 4 << rb, 1024);
   if (e != cudaSuccess) return cuda_fail(r, e, "allocating an empty tree");
-  CK(cudaMemsetAsync(t.node, 0, sizeof(int4), r->stream));
+  const int4 root = make_int4(0, p2p::make_meta(rb, 0), 0, 0);
+  CK(cudaMemsetAsync(t.child, 0, ((size_t)1 << rb) * sizeof(int4), r->stream));
+  CK(cudaMemcpyAsync(t.node, &root, sizeof(int4), cudaMemcpyHostToDevice, r->stream));
+  CK(cudaStreamSynchronize(r->stream));  // `root` is a host temporary
   t.n_node = 1;
+  t.n_child = 1 << rb;
   r->hs[(size_t)p] = t;
   CK(p2p::launch_set_tree(r->d_states + p, r->d_views + p, t, r->stream));
   r->launches += 1;
@@ -191,23 +221,37 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   std::string err;
   if (!p2p::validate_flat(t, err)) return fail(r, P2P_E_FORMAT, err);
   const int64_t N = t->n_nodes, NL = t->n_labels;
-  std::vector<int4> node((size_t)N), child((size_t)std::max<int64_t>(N - 1, 0));
-  for (int64_t v = 0; v < N; ++v) node[(size_t)v] = make_int4(t->child_begin[v], t->child_count[v], t->child_count[v], t->term_count[v]);
-  for (int64_t e = 0; e < N - 1; ++e) {
-    const int32_t c = t->child_idx[e];
-    child[(size_t)e] = make_int4(t->child_first_tok[e], c, t->label_off[c], t->label_len[c]);
+  // Children tables, laid out in node order in the child arena.
+  std::vector<int32_t> bits((size_t)N), off((size_t)N, 0);
+  int64_t slots = 0;
+  for (int64_t v = 0; v < N; ++v) {
+    bits[(size_t)v] = table_bits_for(t->child_count[v], v == 0);
+    if (bits[(size_t)v] > p2p::kMaxTabBits) return fail(r, P2P_E_NOMEM, "a node has too many children");
+    off[(size_t)v] = (int32_t)slots;
+    slots += bits[(size_t)v] ? (int64_t)1 << bits[(size_t)v] : 0;
+    if (slots > INT32_MAX / 2) return fail(r, P2P_E_NOMEM, "children tables exceed the int32 arena");
   }
-  const int32_t cap_node = clamp_i32(N + std::max<int64_t>(N / 4, 64));
-  const int32_t cap_child = clamp_i32((N - 1) + std::max<int64_t>((N - 1) / 2, 64));
-  const int32_t cap_label = clamp_i32(NL + std::max<int64_t>(NL / 4, 1024));
+  std::vector<int4> node((size_t)N), child((size_t)slots, make_int4(0, 0, 0, 0));
+  for (int64_t v = 0; v < N; ++v) {
+    const int32_t cnt = t->child_count[v], b = bits[(size_t)v];
+    node[(size_t)v] = make_int4(b ? off[(size_t)v] : 0, p2p::make_meta(b, cnt), cnt, t->term_count[v]);
+    for (int64_t e = t->child_begin[v]; e < (int64_t)t->child_begin[v] + cnt; ++e) {
+      const int32_t c = t->child_idx[e];
+      table_put(child.data() + off[(size_t)v], b, make_int4(t->child_first_tok[e], c, t->label_off[c], t->label_len[c]));
+    }
+  }
+  // Headroom for device deltas (no regrowth for a few anti-entropy rounds of a few percent each).
+  const int32_t cap_node = clamp_i32(2 * N + 1024);
+  const int32_t cap_child = clamp_i32(2 * slots + 1024);
+  const int32_t cap_label = clamp_i32(NL + std::max<int64_t>(NL / 2, 4096));
   TreeState nt;
   cudaError_t e = alloc_tree_arrays(r, nt, cap_node, cap_child, cap_label);
   if (e != cudaSuccess) return fail(r, P2P_E_NOMEM, std::string("allocating the tree: ") + cudaGetErrorString(e));
   CK(cudaMemcpyAsync(nt.node, node.data(), (size_t)N * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
-  if (N > 1) CK(cudaMemcpyAsync(nt.child, child.data(), (size_t)(N - 1) * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
+  if (slots) CK(cudaMemcpyAsync(nt.child, child.data(), (size_t)slots * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   if (NL > 0) CK(cudaMemcpyAsync(nt.label, t->labels, (size_t)NL * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
   nt.n_node = (int32_t)N;
-  nt.n_child = (int32_t)(N - 1);
+  nt.n_child = (int32_t)slots;
   nt.n_label = (int32_t)NL;
   TreeState& old = r->hs[(size_t)peer];
   free_tree_arrays(r, old);
@@ -227,65 +271,102 @@ int download(p2p_router* r, int32_t peer, p2p_snapshot* out) {
   if (t.n_child) CK(d2h(r, child.data(), t.child, child.size() * sizeof(int4)));
   if (t.n_label) CK(d2h(r, label.data(), t.label, label.size() * sizeof(int32_t)));
   std::string err;
-  if (!p2p::snapshot_from_device_layout(node.data(), t.n_node, child.data(), t.n_child, label.data(), t.n_label, *out, err))
+  if (!p2p::snapshot_from_device_layout(node.data(), t.n_node, child.data(), t.n_child, label.data(), t.n_label, *out,
+                                        err))
     return fail(r, P2P_E_DEVICE, err);
   return P2P_OK;
 }
 
-// Grows the arenas of tree p so that the op that stopped with DELTA_NEED_SPACE fits.
+// Rebuilds tree p's root table (node 0's children) in fresh slots of the child arena, doubled and without
+// tombstones.  Only the host does this: during a delta every warp of the tree shares the root table.
+int regrow_root(p2p_router* r, int32_t p) {
+  TreeState& t = r->hs[(size_t)p];
+  int4 root;
+  CK(d2h(r, &root, t.node, sizeof(int4)));
+  const int32_t bits = p2p::tab_bits(root.y);
+  std::vector<int4> tab(bits ? (size_t)1 << bits : 0);
+  if (bits) CK(d2h(r, tab.data(), t.child + root.x, tab.size() * sizeof(int4)));
+  std::vector<int4> kids;
+  for (const int4& s : tab)
+    if (s.y >= 1) kids.push_back(s);
+  const int32_t nb = std::max(bits + 1, table_bits_for((int64_t)kids.size(), true));
+  if (nb > p2p::kMaxTabBits) return fail(r, P2P_E_NOMEM, "root table too large");
+  const int64_t n_slots = (int64_t)1 << nb;
+  if ((int64_t)t.cap_child - t.n_child < n_slots) {
+    t.need_child = (int32_t)n_slots;
+    t.need_root = 0;
+    return 1;  // the caller grows the child arena first, then comes back
+  }
+  std::vector<int4> nt((size_t)n_slots, make_int4(0, 0, 0, 0));
+  for (const int4& k : kids) table_put(nt.data(), nb, k);
+  const int4 nr = make_int4(t.n_child, p2p::make_meta(nb, (int32_t)kids.size()), (int32_t)kids.size(), root.w);
+  CK(cudaMemcpyAsync(t.child + t.n_child, nt.data(), (size_t)n_slots * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
+  CK(cudaMemcpyAsync(t.node, &nr, sizeof(int4), cudaMemcpyHostToDevice, r->stream));
+  CK(cudaStreamSynchronize(r->stream));  // nt and nr are host temporaries
+  t.stale_child += bits ? (int64_t)1 << bits : 0;
+  t.n_child += (int32_t)n_slots;
+  return P2P_OK;
+}
+
+// Grows the arenas of tree p so that the largest op that did not fit does.
 int grow_tree(p2p_router* r, int32_t p) {
   TreeState& t = r->hs[(size_t)p];
-  const int64_t nodes_short = (int64_t)t.need_node - t.n_free - ((int64_t)t.cap_node - t.n_node);
-  const int64_t child_short = (int64_t)t.need_child - ((int64_t)t.cap_child - t.n_child);
-  const int64_t label_short = (int64_t)t.need_label - ((int64_t)t.cap_label - t.n_label);
   auto newcap = [](int64_t cap, int64_t used, int64_t need) -> int64_t {
     return std::max<int64_t>(cap * 2, used + 2 * need + 1024);
   };
-  TreeState nt = t;
-  int64_t cn = t.cap_node, cc = t.cap_child, cl = t.cap_label;
-  if (nodes_short > 0) cn = newcap(t.cap_node, t.n_node, t.need_node);
-  if (child_short > 0) cc = newcap(t.cap_child, t.n_child, t.need_child);
-  if (label_short > 0) cl = newcap(t.cap_label, t.n_label, t.need_label);
-  if ((nodes_short > 0 && (int64_t)t.n_node + t.need_node > INT32_MAX) ||
-      (child_short > 0 && (int64_t)t.n_child + t.need_child > INT32_MAX) ||
-      (label_short > 0 && (int64_t)t.n_label + t.need_label > INT32_MAX))
+  bool grow_n = (int64_t)t.cap_node - t.n_node < t.need_node;
+  bool grow_c = (int64_t)t.cap_child - t.n_child < t.need_child;
+  bool grow_l = (int64_t)t.cap_label - t.n_label < t.need_label;
+  if (!grow_n && !grow_c && !grow_l && !t.need_root) grow_n = grow_c = grow_l = true;  // always make progress
+  if ((grow_n && (int64_t)t.n_node + t.need_node > INT32_MAX) ||
+      (grow_c && (int64_t)t.n_child + t.need_child > INT32_MAX) ||
+      (grow_l && (int64_t)t.n_label + t.need_label > INT32_MAX))
     return fail(r, P2P_E_NOMEM, "tree " + std::to_string(p) + " outgrows the int32 arena indices");
-  cn = std::min<int64_t>(cn, INT32_MAX);
-  cc = std::min<int64_t>(cc, INT32_MAX);
-  cl = std::min<int64_t>(cl, INT32_MAX);
+  const int64_t cn = grow_n ? std::min<int64_t>(newcap(t.cap_node, t.n_node, t.need_node), INT32_MAX) : t.cap_node;
+  const int64_t cc = grow_c ? std::min<int64_t>(newcap(t.cap_child, t.n_child, t.need_child), INT32_MAX) : t.cap_child;
+  const int64_t cl = grow_l ? std::min<int64_t>(newcap(t.cap_label, t.n_label, t.need_label), INT32_MAX) : t.cap_label;
   int4* nn = t.node;
   int4* nc = t.child;
   int32_t* nl = t.label;
   cudaError_t e = cudaSuccess;
-  if (cn != t.cap_node && e == cudaSuccess) e = dalloc(r, (void**)&nn, (size_t)cn * sizeof(int4));
-  if (cc != t.cap_child && e == cudaSuccess) e = dalloc(r, (void**)&nc, (size_t)cc * sizeof(int4));
-  if (cl != t.cap_label && e == cudaSuccess) e = dalloc(r, (void**)&nl, (size_t)cl * sizeof(int32_t));
+  if (grow_n && e == cudaSuccess) e = dalloc(r, (void**)&nn, (size_t)cn * sizeof(int4));
+  if (grow_c && e == cudaSuccess) e = dalloc(r, (void**)&nc, (size_t)cc * sizeof(int4));
+  if (grow_l && e == cudaSuccess) e = dalloc(r, (void**)&nl, (size_t)cl * sizeof(int32_t));
   if (e != cudaSuccess) {
     if (nn != t.node) dfree(r, nn);
     if (nc != t.child) dfree(r, nc);
     if (nl != t.label) dfree(r, nl);
     return fail(r, P2P_E_NOMEM, std::string("growing a tree: ") + cudaGetErrorString(e));
   }
-  if (nn != t.node) {
+  if (grow_n) {
     CK(cudaMemcpyAsync(nn, t.node, (size_t)t.n_node * sizeof(int4), cudaMemcpyDeviceToDevice, r->stream));
     dfree(r, t.node);
   }
-  if (nc != t.child) {
+  if (grow_c) {
     CK(cudaMemcpyAsync(nc, t.child, (size_t)t.n_child * sizeof(int4), cudaMemcpyDeviceToDevice, r->stream));
     dfree(r, t.child);
   }
-  if (nl != t.label) {
+  if (grow_l) {
     CK(cudaMemcpyAsync(nl, t.label, (size_t)t.n_label * sizeof(int32_t), cudaMemcpyDeviceToDevice, r->stream));
     dfree(r, t.label);
   }
-  nt.node = nn;
-  nt.child = nc;
-  nt.label = nl;
-  nt.cap_node = (int32_t)cn;
-  nt.cap_child = (int32_t)cc;
-  nt.cap_label = (int32_t)cl;
-  nt.status = p2p::DELTA_OK;
-  t = nt;
+  t.node = nn;
+  t.child = nc;
+  t.label = nl;
+  t.cap_node = (int32_t)cn;
+  t.cap_child = (int32_t)cc;
+  t.cap_label = (int32_t)cl;
+  if (t.need_root) {
+    int rc = regrow_root(r, p);
+    if (rc == 1) {  // the child arena had no room for the new root table: grow it, then retry
+      t.need_node = t.need_label = 0;
+      t.need_root = 1;
+      rc = grow_tree(r, p);
+    }
+    if (rc != P2P_OK) return rc;
+  }
+  t.status = p2p::DELTA_OK;
+  t.need_node = t.need_child = t.need_label = t.need_root = 0;
   return P2P_OK;
 }
 
@@ -297,6 +378,29 @@ int compact_tree(p2p_router* r, int32_t p) {
   p2p_flat_tree v;
   p2p_snapshot_view(&snap, &v);
   return upload_flat(r, p, &v);
+}
+
+bool needs_compaction(const TreeState& t) {
+  return (t.stale_label > 65536 && 2 * t.stale_label > t.n_label) ||
+         (t.stale_child > 65536 && 2 * t.stale_child > t.n_child) ||
+         (t.dead_nodes > 16384 && 2 * t.dead_nodes > t.n_node);
+}
+
+// Resets the per-call fields of trees [p0, p1) and copies their states to the device.
+int push_states(p2p_router* r, int32_t p0, int32_t p1) {
+  std::memcpy(r->h_states, r->hs.data() + p0, (size_t)(p1 - p0) * sizeof(TreeState));
+  CK(cudaMemcpyAsync(r->d_states + p0, r->h_states, (size_t)(p1 - p0) * sizeof(TreeState), cudaMemcpyHostToDevice,
+                     r->stream));
+  CK(cudaStreamSynchronize(r->stream));  // h_states is reused right after
+  return P2P_OK;
+}
+
+int pull_states(p2p_router* r, int32_t p0, int32_t p1) {
+  CK(cudaMemcpyAsync(r->h_states, r->d_states + p0, (size_t)(p1 - p0) * sizeof(TreeState), cudaMemcpyDeviceToHost,
+                     r->stream));
+  CK(cudaStreamSynchronize(r->stream));
+  std::memcpy(r->hs.data() + p0, r->h_states, (size_t)(p1 - p0) * sizeof(TreeState));
+  return P2P_OK;
 }
 
 }  // namespace
@@ -338,6 +442,7 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_states, (size_t)P * sizeof(TreeState));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_load, (size_t)P * sizeof(int32_t));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_err, sizeof(int32_t));
+  if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_hdr, p2p::kStaticHeaderInts * sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_load, (size_t)kLoadRing * P * sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_err, sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_states, (size_t)P * sizeof(TreeState));
@@ -367,12 +472,13 @@ void p2p_router_destroy(p2p_router* r) {
   if (r->pool) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
-                      &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_scratch})
+                      &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_cursors, &r->d_gather})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
     dfree(r, r->d_load);
     dfree(r, r->d_err);
+    dfree(r, r->d_hdr);
     cudaStreamSynchronize(r->stream);
     cudaMemPoolDestroy(r->pool);
   }
@@ -443,7 +549,7 @@ int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]) {
   DeviceGuard g(r->device);
   CK(cudaStreamSynchronize(r->stream));
   const TreeState& t = r->hs[(size_t)peer];
-  const int64_t v[9] = {(int64_t)t.n_node - t.n_free, t.n_node, t.n_child, t.n_label, t.stale_child,
+  const int64_t v[9] = {(int64_t)t.n_node - t.dead_nodes, t.n_node, t.n_child, t.n_label, t.stale_child,
                         t.stale_label, t.cap_node, t.cap_child, t.cap_label};
   std::memcpy(out, v, sizeof(v));
   return P2P_OK;
@@ -458,55 +564,48 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   const p2p_seqs& S = d->seqs;
   const int64_t n = S.n;
   if (n < 0 || S.n_segs < 0 || S.n_pool < 0) return fail(r, P2P_E_INVAL, "negative size in delta");
-  if (n > 0 && (!d->op || !S.seg_begin)) return fail(r, P2P_E_INVAL, "NULL op or seg_begin");
-  // Host view of the op metadata (device deltas: copy it out to validate it; the pool stays on the device).
-  std::vector<int32_t> h_op, h_seg_len;
-  std::vector<int64_t> h_seg_begin, h_seg_off, h_peer_begin;
-  const int32_t* op = d->op;
-  const int64_t* peer_begin = d->peer_begin;
-  p2p_seqs hv = S;
-  if (d->mem == P2P_MEM_DEVICE) {
-    CK(cudaStreamSynchronize(r->stream));
-    h_op.resize((size_t)n);
-    h_seg_begin.resize((size_t)n + 1);
-    h_seg_off.resize((size_t)S.n_segs);
-    h_seg_len.resize((size_t)S.n_segs);
-    if (n) CK(d2h(r, h_op.data(), d->op, (size_t)n * sizeof(int32_t)));
-    if (S.seg_begin) CK(d2h(r, h_seg_begin.data(), S.seg_begin, (size_t)(n + 1) * sizeof(int64_t)));
-    if (S.n_segs && S.seg_off && S.seg_len) {
-      CK(d2h(r, h_seg_off.data(), S.seg_off, (size_t)S.n_segs * sizeof(int64_t)));
-      CK(d2h(r, h_seg_len.data(), S.seg_len, (size_t)S.n_segs * sizeof(int32_t)));
-    }
-    if (peer == -1 && d->peer_begin) {
-      h_peer_begin.resize((size_t)r->P + 1);
-      CK(d2h(r, h_peer_begin.data(), d->peer_begin, (size_t)(r->P + 1) * sizeof(int64_t)));
-      peer_begin = h_peer_begin.data();
-    }
-    op = h_op.data();
-    hv.seg_begin = S.seg_begin ? h_seg_begin.data() : nullptr;
-    hv.seg_off = S.seg_off ? h_seg_off.data() : nullptr;
-    hv.seg_len = S.seg_len ? h_seg_len.data() : nullptr;
-  }
+  if (n > 0 && (!d->op || !S.seg_begin || (S.n_segs > 0 && (!S.seg_off || !S.seg_len)) || (S.n_pool > 0 && !S.pool)))
+    return fail(r, P2P_E_INVAL, "NULL array in delta");
+  if (peer == -1 && n > 0 && !d->peer_begin) return fail(r, P2P_E_INVAL, "peer = -1 needs peer_begin");
   if (n == 0) {
     if (n_absent) *n_absent = 0;
     return P2P_OK;
   }
-  std::string err;
-  int64_t max_len = 0;
-  if (!p2p::check_seqs(&hv, err, &max_len, nullptr)) return fail(r, P2P_E_INVAL, err);
-  for (int64_t i = 0; i < n; ++i)
-    if (op[i] != P2P_OP_INSERT && op[i] != P2P_OP_DELETE) return fail(r, P2P_E_INVAL, "bad op code at " + std::to_string(i));
-  if (peer == -1) {
-    if (!peer_begin) return fail(r, P2P_E_INVAL, "peer = -1 needs peer_begin");
-    if (peer_begin[0] != 0 || peer_begin[r->P] != n) return fail(r, P2P_E_INVAL, "peer_begin must run from 0 to n");
-    for (int32_t p = 0; p < r->P; ++p)
-      if (peer_begin[p + 1] < peer_begin[p]) return fail(r, P2P_E_INVAL, "peer_begin not non-decreasing");
-  }
-  // Device copies of the delta.
+  const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
+  const int32_t nt = p1 - p0;
+  int64_t max_len = 0, max_runs = 0;
   const int32_t* d_op = d->op;
-  const int64_t *d_sb = S.seg_begin, *d_so = S.seg_off;
+  const int64_t *d_sb = S.seg_begin, *d_so = S.seg_off, *d_pb = d->peer_begin;
   const int32_t *d_sl = S.seg_len, *d_pool = S.pool;
-  if (d->mem == P2P_MEM_HOST) {
+  if (d->mem == P2P_MEM_DEVICE) {
+    // Validate on the device; only the 16-byte result comes back.
+    CK(p2p::launch_validate(r->d_hdr, d, peer, r->P, r->stream));
+    r->launches += 1;
+    int32_t h[4] = {0, 0, 0, 0};
+    CK(d2h(r, h, r->d_hdr, sizeof(h)));
+    unsigned long long ml = 0;
+    std::memcpy(&ml, h, sizeof(ml));
+    max_len = (int64_t)ml;
+    max_runs = h[3];
+    if (h[2] & p2p::STATIC_BAD_OP) return fail(r, P2P_E_INVAL, "bad op code in the delta");
+    if (h[2] & p2p::STATIC_BAD_SEGMENT) return fail(r, P2P_E_INVAL, "seg_begin or a segment is malformed or outside the pool");
+    if (h[2] & p2p::STATIC_TOO_LONG) return fail(r, P2P_E_INVAL, "a sequence is longer than 2^31-1 tokens");
+    if (h[2] & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
+  } else {
+    std::string err;
+    if (!p2p::check_seqs(&S, err, &max_len, nullptr)) return fail(r, P2P_E_INVAL, err);
+    for (int64_t i = 0; i < n; ++i) {
+      if (d->op[i] != P2P_OP_INSERT && d->op[i] != P2P_OP_DELETE)
+        return fail(r, P2P_E_INVAL, "bad op code at " + std::to_string(i));
+      max_runs = std::max(max_runs, S.seg_begin[i + 1] - S.seg_begin[i]);
+    }
+    if (peer == -1) {
+      const int64_t* pb = d->peer_begin;
+      if (pb[0] != 0 || pb[r->P] != n) return fail(r, P2P_E_INVAL, "peer_begin must run from 0 to n");
+      for (int32_t p = 0; p < r->P; ++p)
+        if (pb[p + 1] < pb[p]) return fail(r, P2P_E_INVAL, "peer_begin not non-decreasing");
+    }
+    // Device copies of the delta.
     CK(ensure(r, r->d_op, (size_t)n * sizeof(int32_t)));
     CK(ensure(r, r->d_seg_begin, (size_t)(n + 1) * sizeof(int64_t)));
     CK(ensure(r, r->d_seg_off, (size_t)std::max<int64_t>(S.n_segs, 1) * sizeof(int64_t)));
@@ -519,60 +618,63 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
       CK(cudaMemcpyAsync(r->d_seg_len.p, S.seg_len, (size_t)S.n_segs * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
     }
     if (S.n_pool) CK(cudaMemcpyAsync(r->d_pool.p, S.pool, (size_t)S.n_pool * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
+    if (peer == -1) {
+      CK(ensure(r, r->d_peer_begin, (size_t)(r->P + 1) * sizeof(int64_t)));
+      CK(cudaMemcpyAsync(r->d_peer_begin.p, d->peer_begin, (size_t)(r->P + 1) * sizeof(int64_t), cudaMemcpyHostToDevice,
+                         r->stream));
+      d_pb = (const int64_t*)r->d_peer_begin.p;
+    }
     d_op = (const int32_t*)r->d_op.p;
     d_sb = (const int64_t*)r->d_seg_begin.p;
     d_so = (const int64_t*)r->d_seg_off.p;
     d_sl = (const int32_t*)r->d_seg_len.p;
     d_pool = (const int32_t*)r->d_pool.p;
   }
-  // Trees touched by this call and their op ranges.
-  const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
-  for (int32_t p = p0; p < p1; ++p) {
-    TreeState& t = r->hs[(size_t)p];
-    t.op_next = peer == -1 ? peer_begin[p] : 0;
-    t.op_end = peer == -1 ? peer_begin[p + 1] : n;
-    t.status = p2p::DELTA_OK;
-    t.n_absent = 0;
-  }
-  const int32_t nt = p1 - p0;
+  CK(ensure(r, r->d_cursors, (size_t)nt * p2p::kDeltaBuckets * sizeof(int64_t)));
+  int32_t* gather = nullptr;
   const int64_t stride = std::max<int64_t>(max_len, 1);
-  CK(ensure(r, r->d_scratch, (size_t)nt * stride * sizeof(int32_t)));
+  if (max_runs > 2) {
+    CK(ensure(r, r->d_gather, (size_t)nt * p2p::kDeltaBuckets * stride * sizeof(int32_t)));
+    gather = (int32_t*)r->d_gather.p;
+  }
+  int64_t* cursors = (int64_t*)r->d_cursors.p;
+  // Device states = host mirror, then this call's op ranges and bucket cursors (set on the device).
+  if (int rc = push_states(r, p0, p1)) return rc;
+  CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d_pb : nullptr, n, r->stream));
+  CK(p2p::launch_init_cursors(r->d_states + p0, cursors, nt, r->stream));
+  r->launches += 2;
   int rc = P2P_OK;
   for (int round = 0;; ++round) {
-    std::memcpy(r->h_states, r->hs.data() + p0, (size_t)nt * sizeof(TreeState));
-    CK(cudaMemcpyAsync(r->d_states + p0, r->h_states, (size_t)nt * sizeof(TreeState), cudaMemcpyHostToDevice, r->stream));
-    CK(p2p::launch_delta(r->d_states + p0, nt, d_op, d_sb, d_so, d_sl, d_pool, (int32_t*)r->d_scratch.p, stride, r->stream));
+    if (round == 64) {
+      rc = fail(r, P2P_E_NOMEM, "delta did not fit after 64 arena growths");
+      break;
+    }
+    CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->stream));
     r->launches += 1;
-    CK(cudaMemcpyAsync(r->h_states, r->d_states + p0, (size_t)nt * sizeof(TreeState), cudaMemcpyDeviceToHost, r->stream));
-    CK(cudaStreamSynchronize(r->stream));
-    std::memcpy(r->hs.data() + p0, r->h_states, (size_t)nt * sizeof(TreeState));
+    if (int e = pull_states(r, p0, p1)) return e;
     bool again = false;
     for (int32_t p = p0; p < p1 && rc == P2P_OK; ++p) {
       TreeState& t = r->hs[(size_t)p];
-      if (t.status == p2p::DELTA_CORRUPT) {
-        rc = fail(r, P2P_E_DEVICE, "tree " + std::to_string(p) + " is inconsistent (delta stopped at op " + std::to_string(t.op_next) + ")");
-      } else if (t.status == p2p::DELTA_NEED_SPACE) {
+      if (t.status & p2p::DELTA_CORRUPT) {
+        rc = fail(r, P2P_E_DEVICE, "tree " + std::to_string(p) + " is inconsistent");
+      } else if (t.status & p2p::DELTA_NEED_SPACE) {
         rc = grow_tree(r, p);
         again = true;
       }
     }
     if (rc != P2P_OK || !again) break;
+    if (int e = push_states(r, p0, p1)) return e;
   }
   // Publish the (possibly moved) arrays to the route kernel's view table; compact very stale trees.
-  std::memcpy(r->h_states, r->hs.data() + p0, (size_t)nt * sizeof(TreeState));
-  CK(cudaMemcpyAsync(r->d_states + p0, r->h_states, (size_t)nt * sizeof(TreeState), cudaMemcpyHostToDevice, r->stream));
+  if (int e = push_states(r, p0, p1)) return e;
   CK(p2p::launch_refresh_views(r->d_states + p0, r->d_views + p0, nt, r->stream));
   r->launches += 1;
   int64_t absent = 0;
   for (int32_t p = p0; p < p1; ++p) {
-    TreeState& t = r->hs[(size_t)p];
+    const TreeState& t = r->hs[(size_t)p];
     absent += t.n_absent;
-    const int64_t used = (int64_t)t.n_child + t.n_label;
-    const int64_t stale = t.stale_child + t.stale_label;
-    if (rc == P2P_OK && stale > 65536 && 2 * stale > used) rc = compact_tree(r, p);
+    if (rc == P2P_OK && needs_compaction(t)) rc = compact_tree(r, p);
   }
-  // h_states is reused by the next call only after this copy has run.
-  CK(cudaStreamSynchronize(r->stream));
   if (n_absent) *n_absent = absent;
   return rc;
 }
@@ -598,28 +700,36 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
     if (n_absent) *n_absent = 0;
     return P2P_OK;
   }
-  CK(p2p::launch_validate_static(header, d, peer, r->P, r->stream));
+  CK(p2p::launch_validate(header, d, peer, r->P, r->stream));
   r->launches += 1;
   int32_t h[4] = {0, 0, 0, 0};
   CK(cudaMemcpyAsync(h, header, sizeof(h), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaStreamSynchronize(r->stream));
   unsigned long long max_len = 0;
   std::memcpy(&max_len, h, sizeof(max_len));
-  const int32_t bits = h[2];
+  const int32_t bits = h[2], max_runs = h[3];
   if (bits & p2p::STATIC_BAD_OP) return fail(r, P2P_E_INVAL, "bad op code in the delta");
   if (bits & p2p::STATIC_BAD_SEGMENT) return fail(r, P2P_E_INVAL, "seg_begin or a segment is malformed or outside the pool");
   if (bits & p2p::STATIC_TOO_LONG) return fail(r, P2P_E_INVAL, "a sequence is longer than 2^31-1 tokens");
   if (bits & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
   const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
   const int32_t nt = p1 - p0;
+  // Scratch: one int64 cursor per (tree, bucket); gathered sequences only when an op has > 2 pool runs.
+  const int64_t cursor_ints = (int64_t)nt * p2p::kDeltaBuckets * 2;
   const int64_t stride = max_len > 0 ? (int64_t)max_len : 1;
-  if ((int64_t)nt * stride > p2p::static_scratch_tokens())
-    return fail(r, P2P_E_INVAL, "trees x longest sequence = " + std::to_string((int64_t)nt * stride) +
-                                    " tokens exceeds the static scratch of " +
-                                    std::to_string(p2p::static_scratch_tokens()) + " tokens");
+  const int64_t gather_ints = max_runs > 2 ? (int64_t)nt * p2p::kDeltaBuckets * stride : 0;
+  if (cursor_ints + gather_ints > p2p::static_scratch_tokens())
+    return fail(r, P2P_E_INVAL, "the delta needs " + std::to_string(cursor_ints + gather_ints) +
+                                    " words of scratch, more than the static scratch of " +
+                                    std::to_string(p2p::static_scratch_tokens()) +
+                                    " (exceeds the static scratch: split the delta or its sequences' runs)");
+  int64_t* cursors = reinterpret_cast<int64_t*>(tokens);
+  int32_t* gather = gather_ints ? tokens + cursor_ints : nullptr;
   CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d->peer_begin : nullptr, S.n, r->stream));
-  CK(p2p::launch_delta(r->d_states + p0, nt, d->op, S.seg_begin, S.seg_off, S.seg_len, S.pool, tokens, stride, r->stream));
-  r->launches += 2;
+  CK(p2p::launch_init_cursors(r->d_states + p0, cursors, nt, r->stream));
+  CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d->op, S.seg_begin, S.seg_off, S.seg_len, S.pool, gather, stride,
+                       r->stream));
+  r->launches += 3;
   CK(cudaMemcpyAsync(r->h_states, r->d_states + p0, (size_t)nt * sizeof(TreeState), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaStreamSynchronize(r->stream));
   std::memcpy(r->hs.data() + p0, r->h_states, (size_t)nt * sizeof(TreeState));
@@ -629,11 +739,11 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
     const TreeState& t = r->hs[(size_t)p];
     absent += t.n_absent;
     if (rc != P2P_OK) continue;
-    if (t.status == p2p::DELTA_CORRUPT)
-      rc = fail(r, P2P_E_DEVICE, "tree " + std::to_string(p) + " is inconsistent (delta stopped at op " + std::to_string(t.op_next) + ")");
-    else if (t.status == p2p::DELTA_NEED_SPACE)
-      rc = fail(r, P2P_E_NOMEM, "tree " + std::to_string(p) + " has no room for op " + std::to_string(t.op_next) +
-                                    "; its earlier ops were applied (p2p_tree_apply_delta grows trees)");
+    if (t.status & p2p::DELTA_CORRUPT)
+      rc = fail(r, P2P_E_DEVICE, "tree " + std::to_string(p) + " is inconsistent");
+    else if (t.status & p2p::DELTA_NEED_SPACE)
+      rc = fail(r, P2P_E_NOMEM, "tree " + std::to_string(p) +
+                                    " ran out of arena room: some of its ops were not applied (p2p_tree_apply_delta grows trees)");
   }
   if (n_absent) *n_absent = absent;
   return rc;

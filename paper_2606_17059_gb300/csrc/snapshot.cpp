@@ -258,24 +258,44 @@ bool validate_flat(const p2p_flat_tree* t, std::string& err) {
   return true;
 }
 
-// Canonical snapshot of a device tree copied to the host (node, child and label arrays as laid out on
-// the device, see internal.h).
+// Canonical snapshot of a device tree copied to the host (node, child and label arrays as laid out on the
+// device, see internal.h): every node's children are the live slots of its table, sorted by first token.
 bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* child, int64_t n_child,
                                  const int32_t* label, int64_t n_label, p2p_snapshot& out, std::string& err) {
+  if (n_node < 1) return err = "corrupt device tree (no root)", false;
+  auto kids = [&](int64_t v, std::vector<int4>& k) -> bool {
+    k.clear();
+    const int4 nd = node[v];
+    const int32_t bits = tab_bits(nd.y);
+    if (bits == 0) return nd.z == 0;
+    if (bits > kMaxTabBits || nd.x < 0 || (int64_t)nd.x + ((int64_t)1 << bits) > n_child) return false;
+    for (int64_t s = 0; s < ((int64_t)1 << bits); ++s)
+      if (child[nd.x + s].y >= 1) k.push_back(child[nd.x + s]);
+    std::sort(k.begin(), k.end(), [](const int4& a, const int4& b) { return a.x < b.x; });
+    for (size_t i = 1; i < k.size(); ++i)
+      if (k[i - 1].x == k[i].x) return false;
+    return (int64_t)k.size() == nd.z;
+  };
+  // Preorder DFS; each stacked item carries the slot through which the node was reached.
   std::vector<int64_t> order;
-  std::vector<int64_t> via;  // entry index through which each ordered node was reached (-1 root)
-  std::vector<std::pair<int64_t, int64_t>> st{{0, -1}};
+  std::vector<int4> via;
+  std::vector<std::vector<int4>> children;
+  std::vector<std::pair<int64_t, int4>> st{{0, make_int4(0, 0, 0, 0)}};
+  std::vector<int4> k;
   int64_t total_label = 0;
   while (!st.empty()) {
     auto [v, e] = st.back();
     st.pop_back();
     if (v < 0 || v >= n_node || (int64_t)order.size() >= n_node) return err = "corrupt device tree (node index)", false;
+    if (v != 0) {
+      if (e.z < 0 || e.w < 1 || (int64_t)e.z + e.w > n_label) return err = "corrupt device tree (label)", false;
+      total_label += e.w;
+    }
+    if (!kids(v, k)) return err = "corrupt device tree (children table)", false;
     order.push_back(v);
     via.push_back(e);
-    if (e >= 0) total_label += child[e].w;
-    const int4 nd = node[v];
-    if (nd.y < 0 || nd.x < 0 || (int64_t)nd.x + nd.y > n_child) return err = "corrupt device tree (child range)", false;
-    for (int64_t k = (int64_t)nd.x + nd.y - 1; k >= nd.x; --k) st.push_back({child[k].y, k});
+    children.push_back(k);
+    for (auto it = k.rbegin(); it != k.rend(); ++it) st.push_back({it->y, *it});
   }
   if (total_label > INT32_MAX) return err = "tree has more than 2^31-1 label tokens", false;
   const size_t N = order.size();
@@ -294,21 +314,20 @@ bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* c
   int64_t lab = 0, ch = 0;
   for (size_t j = 0; j < N; ++j) {
     const int64_t v = order[j];
-    const int4 nd = node[v];
     out.label_off[j] = (int32_t)lab;
-    if (via[j] >= 0) {
-      const int4 ce = child[via[j]];
-      if (ce.z < 0 || ce.w < 1 || (int64_t)ce.z + ce.w > n_label) return err = "corrupt device tree (label)", false;
+    if (v != 0) {
+      const int4 ce = via[j];
       std::memcpy(out.labels.data() + lab, label + ce.z, (size_t)ce.w * sizeof(int32_t));
       out.label_len[j] = ce.w;
       lab += ce.w;
     }
+    const std::vector<int4>& kk = children[j];
     out.child_begin[j] = (int32_t)ch;
-    out.child_count[j] = nd.y;
-    out.term_count[j] = nd.w;
-    for (int64_t k = nd.x; k < (int64_t)nd.x + nd.y; ++k) {
-      out.child_first_tok[(size_t)ch] = child[k].x;
-      out.child_idx[(size_t)ch] = id[(size_t)child[k].y];
+    out.child_count[j] = (int32_t)kk.size();
+    out.term_count[j] = node[v].w;
+    for (const int4& c : kk) {
+      out.child_first_tok[(size_t)ch] = c.x;
+      out.child_idx[(size_t)ch] = id[(size_t)c.y];
       ++ch;
     }
   }

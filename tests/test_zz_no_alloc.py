@@ -92,14 +92,18 @@ def test_static_delta_rejects_host_memory_sizes_beyond_its_scratch_and_full_tree
     d = g.Delta(h_op.ctypes.data, g._seqs_struct(h, keep), None, g.P2P_MEM_HOST)
     rc = g._load().p2p_tree_apply_delta_static(r.handle, 0, ctypes.byref(d), None)
     assert rc == g.P2P_E_INVAL and "device memory" in g.p2p_last_error(r.handle)
-    # 4 trees x a 600,000-token sequence exceeds the 2,097,152-token scratch.
+    # An op whose sequence is split into more than two pool runs is gathered into the scratch: 32 buckets x
+    # a 600,000-token sequence per tree cannot fit in the 8 MiB array.
     n = 600_000
-    big = wl.SeqList(_dev(np.array([0, 1], np.int64)), _dev(np.array([0], np.int64)),
-                     _dev(np.array([n], np.int32)), _dev(np.arange(n, dtype=np.int32)))
+    pool = _dev(np.arange(n, dtype=np.int32))
+    three = wl.SeqList(_dev(np.array([0, 3], np.int64)), _dev(np.array([0, 200_000, 400_000], np.int64)),
+                       _dev(np.array([200_000] * 3, np.int32)), pool)
     ins = _dev(np.zeros(1, np.int32))
     with pytest.raises(g.P2PError) as e:
-        g.p2p_tree_apply_delta_static(r.handle, -1, ins, big, _dev(np.array([0, 1, 1, 1, 1], np.int64)))
+        g.p2p_tree_apply_delta_static(r.handle, 0, ins, three, None)
     assert e.value.code == g.P2P_E_INVAL and "exceeds the static scratch" in str(e.value)
+    big = wl.SeqList(_dev(np.array([0, 1], np.int64)), _dev(np.array([0], np.int64)),
+                     _dev(np.array([n], np.int32)), pool)
     # On one tree the scratch suffices, but an empty tree's label arena cannot hold 600,000 tokens and the
     # static variant never grows a tree: P2P_E_NOMEM, nothing applied.
     with pytest.raises(g.P2PError) as e:
