@@ -71,7 +71,7 @@ inline __host__ __device__ bool tab_full(int32_t bits, int64_t used_after) {
 constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits of meta
 
 // Bits of the router's device error word.
-enum { ERR_BAD_OFFSETS = 1, ERR_CORRUPT_TREE = 2 };
+enum { ERR_BAD_OFFSETS = 1, ERR_CORRUPT_TREE = 2, ERR_STALL = 4 };
 
 // Route kernel (lookup + route decision), see route_kernel.cu.
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens,

@@ -4,24 +4,43 @@
 // number of leading request tokens found along one path of T_p, a partial edge included), and the
 // chosen peer argmax_p (match - alpha*load_p, -load_p, -p) (Algorithm 1's argmax with a load term).
 //
-// Mapping: one CTA owns one request at a time (grid-stride over requests).  The request's tokens are
-// staged once into shared memory and shared by the CTA's warps; warp w walks trees w, w+W, ...  A walk
-// is warp-cooperative: a child lookup probes 32 slots of the node's children hash table at once (one
-// coalesced load, whatever the fan-out), and an edge label is compared 32 tokens per load with several
-// loads in flight per lane; the first mismatch comes from __ballot_sync + __ffs.  Each warp keeps the best packed route
-// key of its trees; the CTA reduces the W keys in shared memory.  Integer work only: no tensor cores.
+// Schedule.  A CTA takes requests b = blockIdx.x, blockIdx.x + gridDim.x, ...; its work items are the
+// (request, tree) pairs in that order, handed to warps from a shared counter, so a warp that finishes a
+// short walk immediately takes the next item instead of waiting for the slowest walk of the request.
+// Requests are staged in shared memory in kSlots slots: the warp that takes a request's first item copies
+// its tokens in (up to kSlotTokens; longer requests read the rest through the read-only path); warps
+// with later items of that request wait until it is staged; the last warp to finish one of its items
+// writes the route and frees the slot for the request kSlots later.  Every wait is bounded.
+//
+// A walk is warp-cooperative: a child lookup probes 32 slots of the node's children hash table at once
+// (one coalesced load, whatever the fan-out), and an edge label is compared with 6 (long labels) or 4
+// loads of 32 tokens in flight per lane; the first mismatch comes from __ballot_sync + __ffs.  The route
+// decision keeps the max of a packed 64-bit key per request.  Integer work only: no tensor cores.
 #include "internal.h"
 
 namespace p2p {
 namespace {
 
-constexpr int kWarps = 8;                 // warps per CTA
+constexpr int kWarps = 16;              // warps per CTA
 constexpr int kThreads = kWarps * 32;
-constexpr int kUnroll = 4;                // label loads in flight per lane (128 tokens per warp step)
-constexpr int kSmemTokens = 4096;         // request tokens staged in shared memory (16 KB)
+constexpr int kSlots = 4;               // requests staged at a time per CTA
+constexpr int kSlotTokens = 4096;       // tokens of a request kept in shared memory (16 KB per slot)
+constexpr int kCtasPerSm = 3;           // 48 warps per SM: 64 KB of slots and <= 40 registers per thread
+constexpr int kWide = 6;                // label loads in flight per lane on long labels (256 tokens per step)
 constexpr unsigned kFull = 0xffffffffu;
+constexpr int kSpinLimit = 1 << 24;     // bounded waits (~1 s): the kernel flags ERR_STALL and stops
 
-__device__ __forceinline__ int32_t req_at(const int32_t* s_req, int32_t n_s, const int32_t* g_req, int64_t i) {
+struct Slot {
+  int ready;        // request (CTA-local index k) whose tokens are staged here
+  int free_for;     // the request allowed to stage here next
+  int len_s;        // tokens held in shared memory
+  int done;         // items of the request finished
+  long long len;    // request length; -1 = the request's offsets are invalid
+  long long start;  // index of the request's first token in `tokens`
+  unsigned long long best;  // max packed route key so far
+};
+
+__device__ __forceinline__ int32_t req_at(const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t i) {
   return i < n_s ? s_req[i] : __ldg(g_req + i);
 }
 
@@ -50,96 +69,169 @@ __device__ __forceinline__ bool find_child(const int4* __restrict__ tab, int32_t
   return false;
 }
 
+// U loads of 32 label tokens in flight per lane, compared with the request; returns the first mismatch
+// in [j0, j0 + 32U) below lim, or -1 if there is none.  Positions are 32-bit: a walk never passes more
+// tokens than one tree path holds (< 2^31).
+template <int U>
+__device__ __forceinline__ int32_t compare_block(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
+                                                 const int32_t* g_req, int32_t pos, int32_t j0, int32_t lim,
+                                                 int lane) {
+  int32_t v[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const int32_t j = j0 + u * 32 + lane;
+    v[u] = j < lim ? __ldg(lab + j) : 0;
+  }
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const int32_t j = j0 + u * 32 + lane;
+    const unsigned m = __ballot_sync(kFull, j < lim && v[u] != req_at(s_req, n_s, g_req, pos + j));
+    if (m) return j0 + u * 32 + (__ffs(m) - 1);
+  }
+  return -1;
+}
+
 // First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.
-__device__ __forceinline__ int64_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
-                                                  const int32_t* g_req, int64_t pos, int64_t lim, int lane) {
-  for (int64_t j0 = 1; j0 < lim; j0 += kUnroll * 32) {
-    int32_t v[kUnroll];
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t j = j0 + u * 32 + lane;
-      v[u] = j < lim ? __ldg(lab + j) : 0;
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t j = j0 + u * 32 + lane;
-      const bool ne = j < lim && v[u] != req_at(s_req, n_s, g_req, pos + j);
-      const unsigned m = __ballot_sync(kFull, ne);
-      if (m) return j0 + u * 32 + (__ffs(m) - 1);
-    }
+__device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
+                                                  const int32_t* g_req, int32_t pos, int32_t lim, int lane) {
+  int32_t j0 = 1;
+  for (; lim - j0 >= kWide * 32; j0 += kWide * 32) {
+    const int32_t k = compare_block<kWide>(lab, s_req, n_s, g_req, pos, j0, lim, lane);
+    if (k >= 0) return k;
+  }
+  for (; j0 < lim; j0 += 128) {
+    const int32_t k = compare_block<4>(lab, s_req, n_s, g_req, pos, j0, lim, lane);
+    if (k >= 0) return k;
   }
   return lim;
 }
 
-// match(r, T) for one tree, computed by the whole warp (result uniform across lanes).
-__device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int64_t len,
+// match(r, T) for one tree, computed by the whole warp (result uniform across lanes).  len is the request
+// length clamped to 2^31 - 1 (no match can be longer than a tree path).
+__device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t len,
                         int lane, int32_t* err) {
   if (len == 0) return 0;
   int4 ce;
   if (!find_child(t.child + t.root_off, t.root_bits, req_at(s_req, n_s, g_req, 0), lane, ce)) return 0;
-  int64_t pos = 0;
+  int32_t pos = 0;
   for (;;) {
     if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree; keeps the loop finite if it does
       if (lane == 0) atomicOr(err, ERR_CORRUPT_TREE);
       break;
     }
     const int4 nn = __ldg(t.node + ce.y);  // the child's record, fetched while its label is compared
-    const int64_t lim = min((int64_t)ce.w, len - pos);
-    const int64_t k = first_mismatch(t.label + ce.z, s_req, n_s, g_req, pos, lim, lane);
+    const int32_t lim = min(ce.w, len - pos);
+    const int32_t k = first_mismatch(t.label + ce.z, s_req, n_s, g_req, pos, lim, lane);
     pos += k;
     if (k < ce.w || pos >= len || nn.z <= 0) break;
     if (!find_child(t.child + nn.x, tab_bits(nn.y), req_at(s_req, n_s, g_req, pos), lane, ce)) break;
   }
-  return (int32_t)pos;
+  return pos;
 }
 
-__global__ void __launch_bounds__(kThreads) route_kernel(const TreeView* __restrict__ trees, int32_t P,
-                                                         const int32_t* __restrict__ tokens, int64_t n_tokens,
-                                                         int64_t tok_base, const int64_t* __restrict__ offsets,
-                                                         int64_t B, const int32_t* __restrict__ load, int32_t alpha,
-                                                         int32_t* __restrict__ out_match,
-                                                         int32_t* __restrict__ out_peer, int32_t* err) {
-  extern __shared__ int32_t s_req[];
-  __shared__ unsigned long long s_best[kWarps];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int64_t b = blockIdx.x; b < B; b += gridDim.x) {
-    const int64_t start = __ldg(offsets + b) - tok_base, end = __ldg(offsets + b + 1) - tok_base;
-    if (!(start >= 0 && start <= end && end <= n_tokens)) {  // same for every thread of the CTA
-      for (int32_t p = threadIdx.x; p < P; p += kThreads) out_match[b * P + p] = 0;
-      if (threadIdx.x == 0) {
-        out_peer[b] = -1;
-        atomicOr(err, ERR_BAD_OFFSETS);
+// Lane 0 waits (bounded) until *flag == v; the outcome is broadcast to the warp.
+__device__ __forceinline__ bool wait_for(const int* flag, int v, int lane) {
+  int ok = 1;
+  if (lane == 0) {
+    int it = 0;
+    while (*(const volatile int*)flag != v && ++it < kSpinLimit) __nanosleep(64);
+    ok = it < kSpinLimit;
+  }
+  return __shfl_sync(kFull, ok, 0) != 0;
+}
+
+__global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
+    const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
+    int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ load, int32_t alpha,
+    int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
+  extern __shared__ int32_t s_tok[];  // kSlots x kSlotTokens
+  __shared__ Slot s_slot[kSlots];
+  __shared__ unsigned long long s_next;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x < kSlots) {
+    Slot& sl = s_slot[threadIdx.x];
+    sl.ready = -1;
+    sl.free_for = threadIdx.x;
+    sl.done = 0;
+    sl.best = 0;
+  }
+  if (threadIdx.x == 0) s_next = 0;
+  __syncthreads();
+  const int64_t n_req = B > blockIdx.x ? (B - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+  const unsigned long long total = (unsigned long long)n_req * (unsigned long long)P;
+  for (;;) {
+    unsigned long long i = 0;
+    if (lane == 0) i = atomicAdd(&s_next, 1ull);
+    i = __shfl_sync(kFull, i, 0);
+    if (i >= total) break;
+    const int64_t k = (int64_t)(i / (unsigned long long)P);
+    const int32_t p = (int32_t)(i - (unsigned long long)k * P);
+    const int s = (int)(k % kSlots);
+    const int64_t b = blockIdx.x + k * gridDim.x;
+    Slot& sl = s_slot[s];
+    int32_t* st = s_tok + s * kSlotTokens;
+    if (p == 0) {
+      // Stage request k once the request kSlots earlier has released the slot.
+      if (!wait_for(&sl.free_for, (int)k, lane)) {
+        if (lane == 0) atomicOr(err, ERR_STALL);
+        return;
       }
-      continue;
+      const int64_t start = __ldg(offsets + b) - tok_base, end = __ldg(offsets + b + 1) - tok_base;
+      const bool valid = start >= 0 && start <= end && end <= n_tokens;
+      const int32_t n_s = valid ? (int32_t)min(end - start, (int64_t)kSlotTokens) : 0;
+      const int32_t* g = tokens + (valid ? start : 0);
+      for (int32_t j = lane; j < n_s; j += 128) {
+        int32_t v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) v[u] = j + u * 32 < n_s ? __ldg(g + j + u * 32) : 0;
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+          if (j + u * 32 < n_s) st[j + u * 32] = v[u];
+      }
+      __syncwarp();
+      if (lane == 0) {
+        sl.len = valid ? end - start : -1;
+        sl.start = valid ? start : 0;
+        sl.len_s = n_s;
+        sl.best = 0;
+        sl.done = 0;
+        __threadfence_block();
+        *(volatile int*)&sl.ready = (int)k;
+      }
+      __syncwarp();
+    } else if (!wait_for(&sl.ready, (int)k, lane)) {
+      if (lane == 0) atomicOr(err, ERR_STALL);
+      return;
     }
-    const int64_t len = end - start;
-    const int32_t* g_req = tokens + start;
-    const int32_t n_s = (int32_t)min(len, (int64_t)kSmemTokens);
-    for (int32_t i = threadIdx.x; i < n_s; i += kThreads) s_req[i] = __ldg(g_req + i);
-    __syncthreads();
-    unsigned long long best = 0;
-    for (int32_t p = warp; p < P; p += kWarps) {
-      const TreeView t = trees[p];
-      const int32_t m = walk(t, s_req, n_s, g_req, len, lane, err);
-      const int32_t ld = __ldg(load + p);
-      if (lane == 0) out_match[b * P + p] = m;
+    const int64_t len = *(volatile long long*)&sl.len;
+    const int64_t start = *(volatile long long*)&sl.start;
+    const int32_t n_s = *(volatile int*)&sl.len_s;
+    const int32_t m = len > 0 ? walk(trees[p], st, n_s, tokens + start, (int32_t)min(len, (int64_t)INT32_MAX), lane, err) : 0;
+    if (lane == 0) {
+      out_match[b * P + p] = m;
       // Packed key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a
       // better route (higher score, then lower load, then lower index).  The host guarantees
       // alpha * load <= 2^31 - 1, load <= 65535 and P <= 65536, so every field fits.
+      const int32_t ld = __ldg(load + p);
       const long long score = (long long)m - (long long)alpha * ld;
       const unsigned long long key = ((unsigned long long)(score + 2147483648LL) << 32) |
                                      ((unsigned long long)(0xFFFF - ld) << 16) | (unsigned long long)(0xFFFF - p);
-      best = key > best ? key : best;
+      atomicMax(&sl.best, key);
+      __threadfence_block();
+      if (atomicAdd(&sl.done, 1) == P - 1) {  // last item of request k: route it, free the slot
+        __threadfence_block();
+        const unsigned long long bk = *(volatile unsigned long long*)&sl.best;
+        if (len < 0) {
+          out_peer[b] = -1;
+          atomicOr(err, ERR_BAD_OFFSETS);
+        } else {
+          out_peer[b] = 0xFFFF - (int32_t)(bk & 0xFFFFull);
+        }
+        __threadfence_block();
+        *(volatile int*)&sl.free_for = (int)(k + kSlots);
+      }
     }
-    if (lane == 0) s_best[warp] = best;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      unsigned long long k = s_best[0];
-#pragma unroll
-      for (int w = 1; w < kWarps; ++w) k = s_best[w] > k ? s_best[w] : k;
-      out_peer[b] = 0xFFFF - (int32_t)(k & 0xFFFFull);
-    }
-    __syncthreads();
+    __syncwarp();
   }
 }
 
@@ -149,10 +241,13 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
                          int32_t* out_peer, int32_t* d_err, int num_sms, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  const int64_t max_ctas = (int64_t)num_sms * 8;
+  const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
+  cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
   const int grid = (int)(B < max_ctas ? B : max_ctas);
-  route_kernel<<<grid, kThreads, kSmemTokens * sizeof(int32_t), st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
-                                                                      B, d_load, alpha, out_match, out_peer, d_err);
+  route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, d_load, alpha,
+                                             out_match, out_peer, d_err);
   return cudaGetLastError();
 }
 

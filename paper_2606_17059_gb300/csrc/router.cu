@@ -212,6 +212,7 @@ int do_sync(p2p_router* r) {
     std::string m = "device reported:";
     if (bits & p2p::ERR_BAD_OFFSETS) m += " request offsets outside [0, n_tokens] or decreasing;";
     if (bits & p2p::ERR_CORRUPT_TREE) m += " an inconsistent tree;";
+    if (bits & p2p::ERR_STALL) m += " a route kernel wait timed out (outputs incomplete);";
     return fail(r, P2P_E_DEVICE, m);
   }
   return P2P_OK;
