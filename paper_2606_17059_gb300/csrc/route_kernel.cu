@@ -26,7 +26,7 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kSlots = 4;               // requests staged at a time per CTA
 constexpr int kSlotTokens = 4096;       // tokens of a request kept in shared memory (16 KB per slot)
 constexpr int kCtasPerSm = 3;           // 48 warps per SM: 64 KB of slots and <= 40 registers per thread
-constexpr int kWide = 6;                // label loads in flight per lane on long labels (256 tokens per step)
+constexpr int kWide = 6;                // label loads in flight per lane on long labels (192 tokens per step)
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kSpinLimit = 1 << 24;     // bounded waits (~1 s): the kernel flags ERR_STALL and stops
 
