@@ -91,12 +91,32 @@ __device__ __forceinline__ int32_t compare_block(const int32_t* __restrict__ lab
   return -1;
 }
 
+// U loads of 32 label tokens in flight per lane when the whole block lies inside the label and inside the
+// request's shared-memory window: no per-element bounds checks.
+template <int U>
+__device__ __forceinline__ int32_t compare_full(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t j0,
+                                                int lane) {
+  int32_t v[U], r[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) v[u] = __ldg(lab + j0 + u * 32 + lane);
+#pragma unroll
+  for (int u = 0; u < U; ++u) r[u] = sreq[j0 + u * 32 + lane];
+  unsigned m[U];
+#pragma unroll
+  for (int u = 0; u < U; ++u) m[u] = __ballot_sync(kFull, v[u] != r[u]);
+#pragma unroll
+  for (int u = 0; u < U; ++u)
+    if (m[u]) return j0 + u * 32 + (__ffs(m[u]) - 1);
+  return -1;
+}
+
 // First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.
 __device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
                                                   const int32_t* g_req, int32_t pos, int32_t lim, int lane) {
   int32_t j0 = 1;
-  for (; lim - j0 >= kWide * 32; j0 += kWide * 32) {
-    const int32_t k = compare_block<kWide>(lab, s_req, n_s, g_req, pos, j0, lim, lane);
+  const int32_t fast_end = min(lim, n_s - pos);  // blocks below this need no checks
+  for (; j0 + kWide * 32 <= fast_end; j0 += kWide * 32) {
+    const int32_t k = compare_full<kWide>(lab, s_req + pos, j0, lane);
     if (k >= 0) return k;
   }
   for (; j0 < lim; j0 += 128) {
@@ -159,13 +179,22 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
   __syncthreads();
   const int64_t n_req = B > blockIdx.x ? (B - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
   const unsigned long long total = (unsigned long long)n_req * (unsigned long long)P;
+  const bool small = total <= 0xffffffffull;  // 32-bit item arithmetic (the usual case) is much cheaper
   for (;;) {
     unsigned long long i = 0;
     if (lane == 0) i = atomicAdd(&s_next, 1ull);
     i = __shfl_sync(kFull, i, 0);
     if (i >= total) break;
-    const int64_t k = (int64_t)(i / (unsigned long long)P);
-    const int32_t p = (int32_t)(i - (unsigned long long)k * P);
+    int64_t k;
+    int32_t p;
+    if (small) {
+      const uint32_t k32 = (uint32_t)i / (uint32_t)P;
+      k = k32;
+      p = (int32_t)((uint32_t)i - k32 * (uint32_t)P);
+    } else {
+      k = (int64_t)(i / (unsigned long long)P);
+      p = (int32_t)(i - (unsigned long long)k * P);
+    }
     const int s = (int)(k % kSlots);
     const int64_t b = blockIdx.x + k * gridDim.x;
     Slot& sl = s_slot[s];
