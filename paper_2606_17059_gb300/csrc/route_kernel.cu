@@ -8,13 +8,14 @@
 // (request, tree) pairs in that order, handed to warps from a shared counter, so a warp that finishes a
 // short walk immediately takes the next item instead of waiting for the slowest walk of the request.
 // Requests are staged in shared memory in kSlots slots: the warp that takes a request's first item copies
-// its tokens in (up to kSlotTokens; longer requests read the rest through the read-only path); warps
+// its tokens in with one bulk (TMA) copy (up to kSlotTokens; longer requests read the rest through the
+// read-only path); warps
 // with later items of that request wait until it is staged; the last warp to finish one of its items
 // writes the route and frees the slot for the request kSlots later.  Every wait is bounded.
 //
 // A walk is warp-cooperative: a child lookup probes 32 slots of the node's children hash table at once
-// (one coalesced load, whatever the fan-out), and an edge label is compared with 6 (long labels) or 4
-// loads of 32 tokens in flight per lane; the first mismatch comes from __ballot_sync + __ffs.  The route
+// (one coalesced load, whatever the fan-out), and an edge label is compared with 2 16-byte loads (long labels) or 4 4-byte loads
+// loads in flight per lane; the first mismatch comes from a warp min-reduction.  The route
 // decision keeps the max of a packed 64-bit key per request.  Integer work only: no tensor cores.
 #include "internal.h"
 
@@ -26,19 +27,38 @@ constexpr int kThreads = kWarps * 32;
 constexpr int kSlots = 4;               // requests staged at a time per CTA
 constexpr int kSlotTokens = 4096;       // tokens of a request kept in shared memory (16 KB per slot)
 constexpr int kCtasPerSm = 3;           // 48 warps per SM: 64 KB of slots and <= 40 registers per thread
-constexpr int kWide = 6;                // label loads in flight per lane on long labels (192 tokens per step)
+constexpr int kVec = 2;                 // 16-byte label loads in flight per lane on long labels (256 tokens per step)
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kSpinLimit = 1 << 24;     // bounded waits (~1 s): the kernel flags ERR_STALL and stops
 
 struct Slot {
+  unsigned long long bar;   // mbarrier of the slot's bulk copy (one phase per staged request)
+  unsigned long long best;  // max packed route key so far
+  long long len;    // request length; -1 = the request's offsets are invalid
+  long long start;  // index of the request's first token in `tokens`
   int ready;        // request (CTA-local index k) whose tokens are staged here
   int free_for;     // the request allowed to stage here next
   int len_s;        // tokens held in shared memory
+  int shift;        // token j of the request sits at slot token shift + j (keeps bulk copies 16-byte aligned)
   int done;         // items of the request finished
-  long long len;    // request length; -1 = the request's offsets are invalid
-  long long start;  // index of the request's first token in `tokens`
-  unsigned long long best;  // max packed route key so far
 };
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// Bulk copy global -> shared (untiled TMA), completing on the slot's mbarrier.
+__device__ __forceinline__ void bulk_copy(void* dst, const void* src, uint32_t bytes, unsigned long long* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               :: "r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect(unsigned long long* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" :: "r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(unsigned long long* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+               : "=r"(ok) : "r"(smem_u32(bar)), "r"(parity) : "memory");
+  return ok != 0;
+}
 
 __device__ __forceinline__ int32_t req_at(const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t i) {
   return i < n_s ? s_req[i] : __ldg(g_req + i);
@@ -92,7 +112,7 @@ __device__ __forceinline__ int32_t compare_block(const int32_t* __restrict__ lab
 }
 
 // U loads of 32 label tokens in flight per lane when the whole block lies inside the label and inside the
-// request's shared-memory window: no per-element bounds checks.
+// request's shared-memory window: no per-element checks, one reduction for the first mismatch.
 template <int U>
 __device__ __forceinline__ int32_t compare_full(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t j0,
                                                 int lane) {
@@ -101,13 +121,55 @@ __device__ __forceinline__ int32_t compare_full(const int32_t* __restrict__ lab,
   for (int u = 0; u < U; ++u) v[u] = __ldg(lab + j0 + u * 32 + lane);
 #pragma unroll
   for (int u = 0; u < U; ++u) r[u] = sreq[j0 + u * 32 + lane];
-  unsigned m[U];
+  int32_t first = INT32_MAX;
 #pragma unroll
-  for (int u = 0; u < U; ++u) m[u] = __ballot_sync(kFull, v[u] != r[u]);
+  for (int u = U - 1; u >= 0; --u)
+    if (v[u] != r[u]) first = u * 32 + lane;
+  first = __reduce_min_sync(kFull, first);
+  return first == INT32_MAX ? -1 : j0 + first;
+}
+
+// As compare_full for a block that may run past the label end (tokens at or after lim are ignored) but
+// stays inside the shared-memory window.
+__device__ __forceinline__ int32_t compare_tail(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t j0,
+                                                int32_t lim, int lane) {
+  int32_t v[4], r[4];
 #pragma unroll
-  for (int u = 0; u < U; ++u)
-    if (m[u]) return j0 + u * 32 + (__ffs(m[u]) - 1);
-  return -1;
+  for (int u = 0; u < 4; ++u) {
+    const int32_t j = j0 + u * 32 + lane;
+    v[u] = j < lim ? __ldg(lab + j) : 0;
+    r[u] = j < lim ? sreq[j] : 0;
+  }
+  int32_t first = INT32_MAX;
+#pragma unroll
+  for (int u = 3; u >= 0; --u)
+    if (v[u] != r[u]) first = u * 32 + lane;
+  first = __reduce_min_sync(kFull, first);
+  return first == INT32_MAX ? -1 : j0 + first;
+}
+
+// V 16-byte label loads per lane (4 tokens each, 128V tokens per warp step) compared with the staged
+// request; lab + jb must be 16-byte aligned and [jb, jb + 128V) inside the label and the shared-memory
+// window.  Each lane keeps its first mismatching token; one reduction gives the warp's first.
+template <int V>
+__device__ __forceinline__ int32_t compare_vec(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t jb,
+                                               int lane) {
+  const int4* l4 = reinterpret_cast<const int4*>(lab + jb);
+  int4 v[V];
+#pragma unroll
+  for (int q = 0; q < V; ++q) v[q] = __ldg(l4 + q * 32 + lane);
+  int32_t first = INT32_MAX;
+#pragma unroll
+  for (int q = V - 1; q >= 0; --q) {
+    const int32_t base = q * 128 + 4 * lane;
+    const int32_t* rr = sreq + jb + base;
+    if (v[q].w != rr[3]) first = base + 3;
+    if (v[q].z != rr[2]) first = base + 2;
+    if (v[q].y != rr[1]) first = base + 1;
+    if (v[q].x != rr[0]) first = base;
+  }
+  first = __reduce_min_sync(kFull, first);
+  return first == INT32_MAX ? -1 : jb + first;
 }
 
 // First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.
@@ -115,12 +177,20 @@ __device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ la
                                                   const int32_t* g_req, int32_t pos, int32_t lim, int lane) {
   int32_t j0 = 1;
   const int32_t fast_end = min(lim, n_s - pos);  // blocks below this need no checks
-  for (; j0 + kWide * 32 <= fast_end; j0 += kWide * 32) {
-    const int32_t k = compare_full<kWide>(lab, s_req + pos, j0, lane);
+  if (j0 + 32 <= fast_end) {
+    const int32_t k = compare_full<1>(lab, s_req + pos, j0, lane);
     if (k >= 0) return k;
+    // Continue at the first 16-byte-aligned label position at or below j0 + 32 (re-comparing <= 3 tokens).
+    j0 += 32;
+    j0 -= (int32_t)(((uintptr_t)(lab + j0) >> 2) & 3);
+    for (; j0 + kVec * 128 <= fast_end; j0 += kVec * 128) {
+      const int32_t k2 = compare_vec<kVec>(lab, s_req + pos, j0, lane);
+      if (k2 >= 0) return k2;
+    }
   }
   for (; j0 < lim; j0 += 128) {
-    const int32_t k = compare_block<4>(lab, s_req, n_s, g_req, pos, j0, lim, lane);
+    const int32_t k = pos + j0 + 128 <= n_s ? compare_tail(lab, s_req + pos, j0, lim, lane)
+                                            : compare_block<4>(lab, s_req, n_s, g_req, pos, j0, lim, lane);
     if (k >= 0) return k;
   }
   return lim;
@@ -164,7 +234,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ load, int32_t alpha,
     int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
-  extern __shared__ int32_t s_tok[];  // kSlots x kSlotTokens
+  extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
   __shared__ unsigned long long s_next;
   const int lane = threadIdx.x & 31;
@@ -174,6 +244,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     sl.free_for = threadIdx.x;
     sl.done = 0;
     sl.best = 0;
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" :: "r"(smem_u32(&sl.bar)) : "memory");
   }
   if (threadIdx.x == 0) s_next = 0;
   __syncthreads();
@@ -207,35 +278,65 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
       }
       const int64_t start = __ldg(offsets + b) - tok_base, end = __ldg(offsets + b + 1) - tok_base;
       const bool valid = start >= 0 && start <= end && end <= n_tokens;
-      const int32_t n_s = valid ? (int32_t)min(end - start, (int64_t)kSlotTokens) : 0;
       const int32_t* g = tokens + (valid ? start : 0);
-      for (int32_t j = lane; j < n_s; j += 128) {
-        int32_t v[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) v[u] = j + u * 32 < n_s ? __ldg(g + j + u * 32) : 0;
-#pragma unroll
-        for (int u = 0; u < 4; ++u)
-          if (j + u * 32 < n_s) st[j + u * 32] = v[u];
+      // Token j goes to slot token shift + j, so that 16-byte-aligned global addresses land on 16-byte-aligned
+      // shared addresses: the aligned middle of the request moves with one bulk copy, the <= 3 tokens on
+      // each side with plain loads.
+      const int32_t shift = (int32_t)(((uintptr_t)g >> 2) & 3);
+      const int32_t n_s = valid ? (int32_t)min(end - start, (int64_t)(kSlotTokens - shift)) : 0;
+      const int32_t j_lo = min((4 - shift) & 3, n_s);
+      const int32_t j_hi = max(j_lo, n_s - (int32_t)(((uintptr_t)(g + n_s) >> 2) & 3));
+      const uint32_t bytes = (uint32_t)(j_hi - j_lo) * 4u;
+      if (lane == 0) {
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // earlier reads of the slot come first
+        mbar_arrive_expect(&sl.bar, bytes);
+        if (bytes) bulk_copy(st + shift + j_lo, g + j_lo, bytes, &sl.bar);
+      }
+      if (lane < j_lo) st[shift + lane] = __ldg(g + lane);
+      if (lane < n_s - j_hi) st[shift + j_hi + lane] = __ldg(g + j_hi + lane);
+      // Bounded wait for the bulk copy (this slot's phase parity alternates with each staged request).
+      const uint32_t parity = (uint32_t)((k / kSlots) & 1);
+      int ok = 1;
+      if (lane == 0) {
+        int it = 0;
+        while (!mbar_test(&sl.bar, parity) && ++it < kSpinLimit) __nanosleep(32);
+        ok = it < kSpinLimit;
+      }
+      if (!__shfl_sync(kFull, ok, 0)) {
+        if (lane == 0) atomicOr(err, ERR_STALL);
+        return;
       }
       __syncwarp();
       if (lane == 0) {
         sl.len = valid ? end - start : -1;
         sl.start = valid ? start : 0;
         sl.len_s = n_s;
+        sl.shift = shift;
         sl.best = 0;
         sl.done = 0;
         __threadfence_block();
         *(volatile int*)&sl.ready = (int)k;
       }
       __syncwarp();
-    } else if (!wait_for(&sl.ready, (int)k, lane)) {
-      if (lane == 0) atomicOr(err, ERR_STALL);
-      return;
+    } else {
+      // Wait until request k is staged: its slot fields (ready flag), then its bulk copy (mbarrier phase).
+      bool ok = wait_for(&sl.ready, (int)k, lane);
+      if (ok && lane == 0) {
+        int it = 0;
+        while (!mbar_test(&sl.bar, (uint32_t)((k / kSlots) & 1)) && ++it < kSpinLimit) __nanosleep(32);
+        ok = it < kSpinLimit;
+      }
+      if (!__shfl_sync(kFull, (int)ok, 0)) {
+        if (lane == 0) atomicOr(err, ERR_STALL);
+        return;
+      }
+      __threadfence_block();
     }
     const int64_t len = *(volatile long long*)&sl.len;
     const int64_t start = *(volatile long long*)&sl.start;
     const int32_t n_s = *(volatile int*)&sl.len_s;
-    const int32_t m = len > 0 ? walk(trees[p], st, n_s, tokens + start, (int32_t)min(len, (int64_t)INT32_MAX), lane, err) : 0;
+    const int32_t* req = st + *(volatile int*)&sl.shift;
+    const int32_t m = len > 0 ? walk(trees[p], req, n_s, tokens + start, (int32_t)min(len, (int64_t)INT32_MAX), lane, err) : 0;
     if (lane == 0) {
       out_match[b * P + p] = m;
       // Packed key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a
