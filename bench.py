@@ -117,6 +117,22 @@ def dist_info():
     return ws, rank, local
 
 
+def rank_requests(rank: int, B: int) -> tuple[int, int]:
+    """Weak scaling: rank r routes requests [r*B, (r+1)*B) of the request stream (every rank holds all P
+    trees and applies every delta; no data-path collective)."""
+    return rank * B, (rank + 1) * B
+
+
+def max_over_ranks(ms: float, dist, device=None) -> float:
+    """Slowest rank's time: the job is done when every rank is."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 # ---- workload setup ---------------------------------------------------------------------------------
 
 def make_workload(cfg: int, trees: int = 0, batch: int = 0):
@@ -244,7 +260,7 @@ def run_ours(args):
     otrees = build_trees(W, router, want_oracle, n_cpu)
     log(f"[rank {rank}] trees built in {time.perf_counter() - t_setup:.1f}s")
     # Requests of this rank, pinned on the host (for the end-to-end leg) and resident on the device.
-    b0, b1 = rank * B, (rank + 1) * B
+    b0, b1 = rank_requests(rank, B)
     n_tok = W._lib.wl_requests_size(W._h, b0, b1, n_cpu)
     h_tok = torch.empty(n_tok, dtype=torch.int32, pin_memory=True)
     tok_np, off_np = W.requests(b0, b1, n_threads=n_cpu, out_tokens=h_tok.numpy())
@@ -315,10 +331,7 @@ def run_ours(args):
     delta_ms = [ev[0].elapsed_time(ev[1]) for ev in evs] if has_delta else [0.0] * len(evs)
     step_ms = [a + b for a, b in zip(route_ms, delta_ms)]
     total_ms = sum(step_ms) if flush is not None else t_begin.elapsed_time(t_end)
-    if dist:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, dist, device="cuda")
     ms_per_step = total_ms / args.steps
     value = ws * B / (ms_per_step / 1e3)
     res = {}

@@ -1,0 +1,88 @@
+"""GPU parity at the full sizes of the stale-replica workload (P=64, 262,144 requests) and the scale workload
+(P=256 trees of 100,000 sequences, 1,048,576 requests, a 5% + 5% delta per replica), in the launch
+configuration the bench times.  The stale-replica workload is compared in full; for the scale workload the
+oracle cannot hold all 256 trees in a test, so outputs are sampled: match columns of sampled trees for
+sampled requests, the route of every sampled request recomputed from its GPU match row, and the patched
+trees of sampled replicas byte for byte."""
+import numpy as np
+import pytest
+
+import oracle
+import paper_2606_17059_gb300 as g
+import workload as wl
+from gpu_util import assert_same_route, oracle_route, same_snapshot
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    g.build()
+
+
+def _route_full(router, tok, off, load, alpha):
+    import torch
+    t = torch.from_numpy(tok).cuda()
+    o = torch.from_numpy(off).cuda()
+    m, p = router.route(t, o, load, alpha)
+    router.sync()
+    return m.cpu().numpy(), p.cpu().numpy()
+
+
+def test_stale_replica_workload_full_size():
+    W = wl.Workload(2)
+    r = g.Router(W.P)
+    for p in range(W.P):
+        r.build(p, W.tree(p, 1))  # the exact trees
+    d = W.delta()  # exact -> replica for trees 1..63
+    assert r.apply_delta(-1, d.op, d.seqs, d.peer_begin) == 0
+    replicas = [W.tree(p, 0) for p in range(W.P)]
+    trees = oracle.build_trees(replicas, n_threads=16)
+    for p in (0, 1, 17, 63):
+        assert same_snapshot(r.download(p), trees[p].export()), p
+    tok, off = W.requests()
+    gm, gp = _route_full(r, tok, off, W.load(), W.alpha)
+    om, op, _ = oracle.route(trees, tok, off, W.load(), W.alpha, n_threads=16)
+    assert_same_route(gm, gp, om, op, "stale replicas, full size")
+
+
+def test_scale_workload_sampled_outputs():
+    W = wl.Workload(4)
+    P, B = W.P, W.B
+    r = g.Router(P)
+    for p in range(P):
+        r.build(p, W.tree(p))
+    rng = np.random.default_rng(4)
+    sample_trees = sorted(rng.choice(P, size=6, replace=False).tolist())
+    otrees = {p: t for p, t in zip(sample_trees, oracle.build_trees([W.tree(p) for p in sample_trees], n_threads=16))}
+    # One anti-entropy round on every replica (device), the same ops on the sampled oracle trees.
+    W.delta_make(0, W.params["delta_frac"], W.params["delta_frac"], n_threads=16)
+    d = W.delta(n_threads=16)
+    assert r.apply_delta(-1, d.op, d.seqs, d.peer_begin) == 0
+    for p in sample_trees:
+        assert otrees[p].apply_ops(d.op, d.seqs, int(d.peer_begin[p]), int(d.peer_begin[p + 1])) == 0
+    for p in sample_trees[:3]:
+        assert same_snapshot(r.download(p), otrees[p].export()), p
+    # The full batch on the device.
+    tok, off = W.requests(n_threads=16)
+    load = W.load()
+    gm, gp = _route_full(r, tok, off, load, W.alpha)
+    assert gm.shape == (B, P) and gp.min() >= 0 and gp.max() < P
+    lens = np.diff(off)
+    assert np.all(gm <= lens[:, None]) and gm.max() > 1000
+    # Sampled requests: match columns of the sampled trees, and the route from each full GPU match row.
+    reqs = np.sort(rng.choice(B, size=20000, replace=False))
+    sub_tok = np.concatenate([tok[off[b]:off[b + 1]] for b in reqs])
+    sub_off = np.zeros(len(reqs) + 1, np.int64)
+    np.cumsum(lens[reqs], out=sub_off[1:])
+    om, _, _ = oracle.route([otrees[p] for p in sample_trees], sub_tok, sub_off, load[sample_trees], W.alpha,
+                            n_threads=16)
+    got = gm[reqs][:, sample_trees]
+    bad = np.argwhere(got != om)
+    assert len(bad) == 0, f"{len(bad)} sampled match mismatches, first {bad[:3].tolist()}"
+    for i in range(0, len(reqs), 7):
+        b = reqs[i]
+        assert oracle.argmax_peer(gm[b], load, W.alpha) == gp[b], b
