@@ -45,7 +45,9 @@ struct Tree {
   int4* node;
   int4* child;
   int32_t* label;
+  const int32_t* shared;  // router-wide pool of interned labels (read-only here)
   TreeState* g;
+  __device__ const int32_t* lab(int32_t off) const { return label_ptr(label, shared, off); }
 };
 
 // Reserves k units of the counter (capacity cap); returns the first unit or -1.  Lane 0 does the CAS.
@@ -250,6 +252,13 @@ __device__ void add_stat(int64_t* p, int64_t v, int lane) {
   if (lane == 0 && v) atomicAdd((unsigned long long*)p, (unsigned long long)v);
 }
 
+// Labels a then b are one contiguous run (same label space, b starting where a ends): folding needs no copy.
+__device__ bool adjacent(const int4& a, const int4& b) {
+  if (a.z >= 0 && b.z >= 0) return (int64_t)a.z + a.w == b.z;
+  if (a.z < 0 && b.z < 0) return (int64_t)~a.z + a.w == (int64_t)~b.z;
+  return false;
+}
+
 // Node x (slot *ex in its parent's table) has one child and stores no sequence: fold the child's edge into
 // x's.  The joined label is written at l0 unless the two labels are adjacent in the arena.
 __device__ void fold_child(Tree& t, int32_t x, int4* ex, int32_t yslot, int32_t l0, int lane) {
@@ -258,10 +267,10 @@ __device__ void fold_child(Tree& t, int32_t x, int4* ex, int32_t yslot, int32_t 
   const int4 ye = t.child[yslot];
   const int4 yn = t.node[ye.y];
   int32_t off = xe.z;
-  if (xe.z + xe.w != ye.z) {
+  if (!adjacent(xe, ye)) {
     off = l0;
-    copy_tokens(t.label + off, t.label + xe.z, xe.w, lane);
-    copy_tokens(t.label + off + xe.w, t.label + ye.z, ye.w, lane);
+    copy_tokens(t.label + off, t.lab(xe.z), xe.w, lane);
+    copy_tokens(t.label + off + xe.w, t.lab(ye.z), ye.w, lane);
     add_stat(&t.g->stale_label, (int64_t)xe.w + ye.w, lane);
   }
   __syncwarp();
@@ -274,8 +283,6 @@ __device__ void fold_child(Tree& t, int32_t x, int4* ex, int32_t yslot, int32_t 
   add_stat(&t.g->dead_nodes, 1, lane);
   __syncwarp();
 }
-
-__device__ bool adjacent(const int4& a, const int4& b) { return a.z + a.w == b.z; }
 
 // Room for one more child in node cur's table (cur != 0): grows the table (doubling, rehash into fresh
 // slots) when claimed slots would pass 3/4.  Returns false if the child arena is full.
@@ -358,7 +365,7 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
     const int4 ce = *ent;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
     const int64_t lim = min((int64_t)ce.w, n - pos);
-    const int64_t k = first_diff(t.label + ce.z, q, pos, 1, lim, lane, memo);
+    const int64_t k = first_diff(t.lab(ce.z), q, pos, 1, lim, lane, memo);
     if (k == ce.w) {
       cur = ce.y;
       pos += k;
@@ -371,7 +378,7 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
     if (!take(t, tail ? 2 : 1, 1 << kMinTabBits, tail ? L : 0, n0, c0, l0, lane)) return OP_NEED;
     const int32_t mid = n0, leaf = n0 + 1;
     zero_slots(t, c0, 1 << kMinTabBits, lane);
-    const int4 lower = make_int4(t.label[ce.z + k], ce.y, ce.z + (int32_t)k, ce.w - (int32_t)k);
+    const int4 lower = make_int4(t.lab(ce.z)[k], ce.y, label_adv(ce.z, (int32_t)k), ce.w - (int32_t)k);
     if (tail) copy_seq(t.label + l0, q, pos + k, L, lane);
     const int32_t leaf_tok = tail ? q.at(pos + k) : 0;
     __syncwarp();
@@ -423,7 +430,7 @@ __device__ int remove(Tree& t, const Seq& q, int lane, Memo& memo) {
     int4* ent = t.child + slot;
     const int4 ce = *ent;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
-    if (pos + ce.w > n || first_diff(t.label + ce.z, q, pos, 1, ce.w, lane, memo) < ce.w) {
+    if (pos + ce.w > n || first_diff(t.lab(ce.z), q, pos, 1, ce.w, lane, memo) < ce.w) {
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
@@ -488,7 +495,8 @@ __global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* st
                                                                     const int64_t* __restrict__ seg_off,
                                                                     const int32_t* __restrict__ seg_len,
                                                                     const int32_t* __restrict__ pool,
-                                                                    int32_t* gather, int64_t stride) {
+                                                                    int32_t* gather, int64_t stride,
+                                                                    const int32_t* shared) {
   __shared__ int8_t s_bucket[kChunk];
   __shared__ int s_any;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -505,6 +513,7 @@ __global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* st
   t.node = gs->node;
   t.child = gs->child;
   t.label = gs->label;
+  t.shared = shared;
   t.g = gs;
   int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaBuckets + warp) * stride : nullptr;
   bool stopped = next >= op_end;
@@ -627,25 +636,26 @@ __global__ void init_cursors_kernel(const TreeState* states, int64_t* cursors, i
   if (i < (int64_t)nt * kDeltaBuckets) cursors[i] = states[i / kDeltaBuckets].op_begin;
 }
 
-__global__ void set_tree_kernel(TreeState* st, TreeView* view, TreeState v) {
+__global__ void set_tree_kernel(TreeState* st, TreeView* view, TreeState v, const int32_t* shared) {
   *st = v;
   const int4 root = v.node[0];
-  *view = TreeView{v.node, v.child, v.label, root.x, tab_bits(root.y)};
+  *view = TreeView{v.node, v.child, v.label, shared, root.x, tab_bits(root.y)};
 }
 
-__global__ void refresh_views_kernel(const TreeState* st, TreeView* view, int32_t n) {
+__global__ void refresh_views_kernel(const TreeState* st, TreeView* view, int32_t n, const int32_t* shared) {
   const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) {
     const int4 root = st[i].node[0];
-    view[i] = TreeView{st[i].node, st[i].child, st[i].label, root.x, tab_bits(root.y)};
+    view[i] = TreeView{st[i].node, st[i].child, st[i].label, shared, root.x, tab_bits(root.y)};
   }
 }
 
 }  // namespace
 
-cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, int32_t n, cudaStream_t st) {
+cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, int32_t n, const int32_t* shared,
+                                 cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
-  refresh_views_kernel<<<(n + 127) / 128, 128, 0, st>>>(d_states, d_views, n);
+  refresh_views_kernel<<<(n + 127) / 128, 128, 0, st>>>(d_states, d_views, n, shared);
   return cudaGetLastError();
 }
 
@@ -658,10 +668,10 @@ cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int
 
 cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
-                         int32_t* gather, int64_t gather_stride, cudaStream_t st) {
+                         int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st) {
   if (n_trees <= 0) return cudaSuccess;
   delta_kernel<<<n_trees, kDeltaBuckets * 32, 0, st>>>(d_states, cursors, op, seg_begin, seg_off, seg_len, pool, gather,
-                                                       gather_stride);
+                                                       gather_stride, shared);
   return cudaGetLastError();
 }
 
@@ -681,8 +691,9 @@ cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* p
   return cudaGetLastError();
 }
 
-cudaError_t launch_set_tree(TreeState* d_state, TreeView* d_view, TreeState value, cudaStream_t st) {
-  set_tree_kernel<<<1, 1, 0, st>>>(d_state, d_view, value);
+cudaError_t launch_set_tree(TreeState* d_state, TreeView* d_view, TreeState value, const int32_t* shared,
+                            cudaStream_t st) {
+  set_tree_kernel<<<1, 1, 0, st>>>(d_state, d_view, value, shared);
   return cudaGetLastError();
 }
 

@@ -27,15 +27,26 @@ namespace p2p {
 //              .node: 0 = empty slot (the slot is all zero), >= 1 = the child, -1 = removed (tombstone,
 //              key kept), -3 = being claimed during a delta.  Slots are probed linearly from a
 //              multiplicative hash of first_tok.
-//   label[]  = int32 tokens; an edge's label is label[label_off .. +label_len).
+//   label[]  = int32 tokens of the tree's own label arena.  An edge's label is label[label_off ..
+//              +label_len) when label_off >= 0, and shared[~label_off ..] when label_off < 0: long labels
+//              are interned in a router-wide pool (the same few-shot prefixes are cached by many peers, so
+//              one copy serves every replica that holds it).
 // Node 0 is the root.  Keeping the child's label position in its slot lets a walk start comparing the
 // label as soon as the lookup returns; every lookup is one coalesced probe of 32 consecutive slots.
 struct TreeView {
   const int4* node;
   const int4* child;
   const int32_t* label;
+  const int32_t* shared;        // the router's shared label pool
   int32_t root_off, root_bits;  // the root's children table (copied from node[0] when the view is set)
 };
+
+// Start of the label of an edge whose label_off is `off` (see the layout above).
+inline __host__ __device__ const int32_t* label_ptr(const int32_t* label, const int32_t* shared, int32_t off) {
+  return off >= 0 ? label + off : shared + ~off;
+}
+// label_off of the same label advanced by k tokens.
+inline __host__ __device__ int32_t label_adv(int32_t off, int32_t k) { return off >= 0 ? off + k : off - k; }
 
 // Mutable state of one tree, shared by the delta kernel's warps for that tree (counters updated with
 // atomics) and mirrored on the host between calls.
@@ -84,7 +95,7 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
 // op's sequence has more than two pool runs; otherwise it may be NULL.
 cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
-                         int32_t* gather, int64_t gather_stride, cudaStream_t st);
+                         int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st);
 cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int32_t n_trees, cudaStream_t st);
 
 // Home slot of a first token in a children table of 2^bits slots (host table builder and kernels).
@@ -94,10 +105,12 @@ inline __host__ __device__ uint32_t slot_hash(int32_t tok, int32_t bits) {
 
 // Writes a tree's state and view on the device (values passed as kernel parameters, so no host buffer
 // has to outlive the call).
-cudaError_t launch_set_tree(TreeState* d_state, TreeView* d_view, TreeState value, cudaStream_t st);
+cudaError_t launch_set_tree(TreeState* d_state, TreeView* d_view, TreeState value, const int32_t* shared,
+                            cudaStream_t st);
 
 // Rewrites views[0 .. n) from states[0 .. n) (after a delta moved some trees' arrays).
-cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, int32_t n, cudaStream_t st);
+cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, int32_t n, const int32_t* shared,
+                                 cudaStream_t st);
 
 // Static scratch of the allocation-free delta call (delta_static.cu).
 enum { STATIC_BAD_OP = 1, STATIC_BAD_SEGMENT = 2, STATIC_BAD_PEER_BEGIN = 4, STATIC_TOO_LONG = 8 };
@@ -117,6 +130,7 @@ bool check_seqs(const p2p_seqs* s, std::string& err, int64_t* max_len, std::vect
 bool build_snapshot(const p2p_seqs& S, p2p_snapshot& out, std::string& err);
 bool validate_flat(const p2p_flat_tree* t, std::string& err);
 bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* child, int64_t n_child,
-                                 const int32_t* label, int64_t n_label, p2p_snapshot& out, std::string& err);
+                                 const int32_t* label, int64_t n_label, const int32_t* shared, int64_t n_shared,
+                                 p2p_snapshot& out, std::string& err);
 
 }  // namespace p2p

@@ -211,7 +211,7 @@ __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, co
     }
     const int4 nn = __ldg(t.node + ce.y);  // the child's record, fetched while its label is compared
     const int32_t lim = min(ce.w, len - pos);
-    const int32_t k = first_mismatch(t.label + ce.z, s_req, n_s, g_req, pos, lim, lane);
+    const int32_t k = first_mismatch(label_ptr(t.label, t.shared, ce.z), s_req, n_s, g_req, pos, lim, lane);
     pos += k;
     if (k < ce.w || pos >= len || nn.z <= 0) break;
     if (!find_child(t.child + nn.x, tab_bits(nn.y), req_at(s_req, n_s, g_req, pos), lane, ce)) break;

@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <cstring>
 #include <string>
+#include <unordered_map>
 #include <vector>
 
 #include "internal.h"
@@ -34,6 +35,20 @@ int32_t log2_exact(int64_t p) {
   while (((int64_t)1 << b) < p) ++b;
   return b;
 }
+// Labels at least this long are interned in the router's shared pool (shorter ones stay in the tree's
+// own arena): the long runs are the shared prompt prefixes that many replicas hold.
+constexpr int32_t kInternMin = 128;
+
+// 64-bit content hash of a token run (FNV-1a over the 32-bit tokens, then a final avalanche); interning
+// always verifies the content, so a collision only means a run is not shared.
+uint64_t run_hash(const int32_t* p, int64_t n) {
+  uint64_t h = 0xcbf29ce484222325ull ^ (uint64_t)n;
+  for (int64_t i = 0; i < n; ++i) h = (h ^ (uint32_t)p[i]) * 0x100000001b3ull;
+  h ^= h >> 33;
+  h *= 0xff51afd7ed558ccdull;
+  return h ^ (h >> 33);
+}
+
 // Children-table sizes (log2 slots): load factor <= 1/2 at upload; the root's table gets extra room (at
 // least 64 slots) because only the host can grow it.
 int32_t table_bits_for(int64_t live, bool root) {
@@ -71,6 +86,11 @@ struct p2p_router {
   DevBuf req_tok, req_off, out_match, out_peer;
   DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_cursors, d_gather;
   int64_t launches = 0;  // kernels this router has launched
+  // Shared label pool: long labels interned across trees (device array, host mirror, content index).
+  int32_t* d_shared = nullptr;
+  int64_t shared_cap = 0;
+  std::vector<int32_t> h_shared;
+  std::unordered_map<uint64_t, int32_t> intern;
   std::string err;
 };
 
@@ -168,7 +188,7 @@ int install_empty_tree(p2p_router* r, int32_t p) {
   t.n_node = 1;
   t.n_child = 1 << rb;
   r->hs[(size_t)p] = t;
-  CK(p2p::launch_set_tree(r->d_states + p, r->d_views + p, t, r->stream));
+  CK(p2p::launch_set_tree(r->d_states + p, r->d_views + p, t, r->d_shared, r->stream));
   r->launches += 1;
   return P2P_OK;
 }
@@ -218,10 +238,66 @@ int do_sync(p2p_router* r) {
   return P2P_OK;
 }
 
+int push_states(p2p_router* r, int32_t p0, int32_t p1);
+
+// Makes the device shared pool hold the host mirror's tokens [from, end): grows it (stream-ordered copy)
+// if needed, in which case every tree's view is refreshed with the new pool address.
+int sync_shared_pool(p2p_router* r, int64_t from) {
+  const int64_t n = (int64_t)r->h_shared.size();
+  if (n == from) return P2P_OK;
+  if (n > r->shared_cap) {
+    const int64_t cap = std::min<int64_t>(std::max<int64_t>(2 * r->shared_cap, n + (1 << 20)), INT32_MAX);
+    int32_t* np = nullptr;
+    cudaError_t e = dalloc(r, (void**)&np, (size_t)cap * sizeof(int32_t));
+    if (e != cudaSuccess) return fail(r, P2P_E_NOMEM, std::string("growing the shared label pool: ") + cudaGetErrorString(e));
+    if (from > 0) CK(cudaMemcpyAsync(np, r->d_shared, (size_t)from * sizeof(int32_t), cudaMemcpyDeviceToDevice, r->stream));
+    dfree(r, r->d_shared);
+    r->d_shared = np;
+    r->shared_cap = cap;
+    if (int rc = push_states(r, 0, r->P)) return rc;
+    CK(p2p::launch_refresh_views(r->d_states, r->d_views, r->P, r->d_shared, r->stream));
+    r->launches += 1;
+  }
+  CK(cudaMemcpyAsync(r->d_shared + from, r->h_shared.data() + from, (size_t)(n - from) * sizeof(int32_t),
+                     cudaMemcpyHostToDevice, r->stream));
+  CK(cudaStreamSynchronize(r->stream));  // the mirror may reallocate on the next append
+  return P2P_OK;
+}
+
 int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   std::string err;
   if (!p2p::validate_flat(t, err)) return fail(r, P2P_E_FORMAT, err);
   const int64_t N = t->n_nodes, NL = t->n_labels;
+  // Labels: long runs are interned in the shared pool (label_off < 0 encodes pool offset ~off), the rest
+  // go to the tree's own arena.
+  const int64_t shared_before = (int64_t)r->h_shared.size();
+  std::vector<int32_t> enc((size_t)N, 0), own;
+  own.reserve((size_t)NL);
+  for (int64_t v = 1; v < N; ++v) {
+    const int32_t* src = t->labels + t->label_off[v];
+    const int32_t len = t->label_len[v];
+    bool interned = false;
+    if (len >= kInternMin && (int64_t)r->h_shared.size() + len < INT32_MAX) {
+      const uint64_t h = run_hash(src, len);
+      auto it = r->intern.find(h);
+      if (it == r->intern.end()) {
+        const int32_t at = (int32_t)r->h_shared.size();
+        r->h_shared.insert(r->h_shared.end(), src, src + len);
+        r->intern.emplace(h, at);
+        enc[(size_t)v] = ~at;
+        interned = true;
+      } else if ((int64_t)it->second + len <= (int64_t)r->h_shared.size() &&
+                 std::memcmp(r->h_shared.data() + it->second, src, (size_t)len * sizeof(int32_t)) == 0) {
+        enc[(size_t)v] = ~it->second;
+        interned = true;
+      }
+    }
+    if (!interned) {
+      enc[(size_t)v] = (int32_t)own.size();
+      own.insert(own.end(), src, src + len);
+    }
+  }
+  if (int rc = sync_shared_pool(r, shared_before)) return rc;
   // Children tables, laid out in node order in the child arena.
   std::vector<int32_t> bits((size_t)N), off((size_t)N, 0);
   int64_t slots = 0;
@@ -238,26 +314,27 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
     node[(size_t)v] = make_int4(b ? off[(size_t)v] : 0, p2p::make_meta(b, cnt), cnt, t->term_count[v]);
     for (int64_t e = t->child_begin[v]; e < (int64_t)t->child_begin[v] + cnt; ++e) {
       const int32_t c = t->child_idx[e];
-      table_put(child.data() + off[(size_t)v], b, make_int4(t->child_first_tok[e], c, t->label_off[c], t->label_len[c]));
+      table_put(child.data() + off[(size_t)v], b, make_int4(t->child_first_tok[e], c, enc[(size_t)c], t->label_len[c]));
     }
   }
+  const int64_t n_own = (int64_t)own.size();
   // Headroom for device deltas (no regrowth for a few anti-entropy rounds of a few percent each).
   const int32_t cap_node = clamp_i32(2 * N + 1024);
   const int32_t cap_child = clamp_i32(2 * slots + 1024);
-  const int32_t cap_label = clamp_i32(NL + std::max<int64_t>(NL / 2, 4096));
+  const int32_t cap_label = clamp_i32(n_own + std::max<int64_t>(NL / 2, 4096));
   TreeState nt;
   cudaError_t e = alloc_tree_arrays(r, nt, cap_node, cap_child, cap_label);
   if (e != cudaSuccess) return fail(r, P2P_E_NOMEM, std::string("allocating the tree: ") + cudaGetErrorString(e));
   CK(cudaMemcpyAsync(nt.node, node.data(), (size_t)N * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   if (slots) CK(cudaMemcpyAsync(nt.child, child.data(), (size_t)slots * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
-  if (NL > 0) CK(cudaMemcpyAsync(nt.label, t->labels, (size_t)NL * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
+  if (n_own) CK(cudaMemcpyAsync(nt.label, own.data(), (size_t)n_own * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
   nt.n_node = (int32_t)N;
   nt.n_child = (int32_t)slots;
-  nt.n_label = (int32_t)NL;
+  nt.n_label = (int32_t)n_own;
   TreeState& old = r->hs[(size_t)peer];
   free_tree_arrays(r, old);
   old = nt;
-  CK(p2p::launch_set_tree(r->d_states + peer, r->d_views + peer, nt, r->stream));
+  CK(p2p::launch_set_tree(r->d_states + peer, r->d_views + peer, nt, r->d_shared, r->stream));
   r->launches += 1;
   // The host vectors above are released on return; pageable copies have consumed them by now.
   return P2P_OK;
@@ -272,8 +349,8 @@ int download(p2p_router* r, int32_t peer, p2p_snapshot* out) {
   if (t.n_child) CK(d2h(r, child.data(), t.child, child.size() * sizeof(int4)));
   if (t.n_label) CK(d2h(r, label.data(), t.label, label.size() * sizeof(int32_t)));
   std::string err;
-  if (!p2p::snapshot_from_device_layout(node.data(), t.n_node, child.data(), t.n_child, label.data(), t.n_label, *out,
-                                        err))
+  if (!p2p::snapshot_from_device_layout(node.data(), t.n_node, child.data(), t.n_child, label.data(), t.n_label,
+                                        r->h_shared.data(), (int64_t)r->h_shared.size(), *out, err))
     return fail(r, P2P_E_DEVICE, err);
   return P2P_OK;
 }
@@ -480,6 +557,7 @@ void p2p_router_destroy(p2p_router* r) {
     dfree(r, r->d_load);
     dfree(r, r->d_err);
     dfree(r, r->d_hdr);
+    dfree(r, r->d_shared);
     cudaStreamSynchronize(r->stream);
     cudaMemPoolDestroy(r->pool);
   }
@@ -650,7 +728,8 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
       rc = fail(r, P2P_E_NOMEM, "delta did not fit after 64 arena growths");
       break;
     }
-    CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->stream));
+    CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->d_shared,
+                         r->stream));
     r->launches += 1;
     if (int e = pull_states(r, p0, p1)) return e;
     bool again = false;
@@ -668,7 +747,7 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   }
   // Publish the (possibly moved) arrays to the route kernel's view table; compact very stale trees.
   if (int e = push_states(r, p0, p1)) return e;
-  CK(p2p::launch_refresh_views(r->d_states + p0, r->d_views + p0, nt, r->stream));
+  CK(p2p::launch_refresh_views(r->d_states + p0, r->d_views + p0, nt, r->d_shared, r->stream));
   r->launches += 1;
   int64_t absent = 0;
   for (int32_t p = p0; p < p1; ++p) {
@@ -729,7 +808,7 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
   CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d->peer_begin : nullptr, S.n, r->stream));
   CK(p2p::launch_init_cursors(r->d_states + p0, cursors, nt, r->stream));
   CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d->op, S.seg_begin, S.seg_off, S.seg_len, S.pool, gather, stride,
-                       r->stream));
+                       r->d_shared, r->stream));
   r->launches += 3;
   CK(cudaMemcpyAsync(r->h_states, r->d_states + p0, (size_t)nt * sizeof(TreeState), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaStreamSynchronize(r->stream));

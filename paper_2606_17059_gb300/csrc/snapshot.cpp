@@ -261,7 +261,8 @@ bool validate_flat(const p2p_flat_tree* t, std::string& err) {
 // Canonical snapshot of a device tree copied to the host (node, child and label arrays as laid out on the
 // device, see internal.h): every node's children are the live slots of its table, sorted by first token.
 bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* child, int64_t n_child,
-                                 const int32_t* label, int64_t n_label, p2p_snapshot& out, std::string& err) {
+                                 const int32_t* label, int64_t n_label, const int32_t* shared, int64_t n_shared,
+                                 p2p_snapshot& out, std::string& err) {
   if (n_node < 1) return err = "corrupt device tree (no root)", false;
   auto kids = [&](int64_t v, std::vector<int4>& k) -> bool {
     k.clear();
@@ -288,7 +289,9 @@ bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* c
     st.pop_back();
     if (v < 0 || v >= n_node || (int64_t)order.size() >= n_node) return err = "corrupt device tree (node index)", false;
     if (v != 0) {
-      if (e.z < 0 || e.w < 1 || (int64_t)e.z + e.w > n_label) return err = "corrupt device tree (label)", false;
+      const bool own = e.z >= 0;
+      const int64_t start = own ? e.z : ~(int64_t)e.z;
+      if (e.w < 1 || start + e.w > (own ? n_label : n_shared)) return err = "corrupt device tree (label)", false;
       total_label += e.w;
     }
     if (!kids(v, k)) return err = "corrupt device tree (children table)", false;
@@ -317,7 +320,7 @@ bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* c
     out.label_off[j] = (int32_t)lab;
     if (v != 0) {
       const int4 ce = via[j];
-      std::memcpy(out.labels.data() + lab, label + ce.z, (size_t)ce.w * sizeof(int32_t));
+      std::memcpy(out.labels.data() + lab, label_ptr(label, shared, ce.z), (size_t)ce.w * sizeof(int32_t));
       out.label_len[j] = ce.w;
       lab += ce.w;
     }
