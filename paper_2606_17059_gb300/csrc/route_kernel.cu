@@ -4,19 +4,20 @@
 // number of leading request tokens found along one path of T_p, a partial edge included), and the
 // chosen peer argmax_p (match - alpha*load_p, -load_p, -p) (Algorithm 1's argmax with a load term).
 //
-// Schedule.  A CTA takes requests b = blockIdx.x, blockIdx.x + gridDim.x, ...; its work items are the
-// (request, tree) pairs in that order, handed to warps from a shared counter, so a warp that finishes a
-// short walk immediately takes the next item instead of waiting for the slowest walk of the request.
-// Requests are staged in shared memory in kSlots slots: the warp that takes a request's first item copies
-// its tokens in with one bulk (TMA) copy (up to kSlotTokens; longer requests read the rest through the
-// read-only path); warps
-// with later items of that request wait until it is staged; the last warp to finish one of its items
-// writes the route and frees the slot for the request kSlots later.  Every wait is bounded.
+// Schedule.  A CTA takes requests b = blockIdx.x, blockIdx.x + gridDim.x, ...; its work items are
+// (request, group of G consecutive trees) in that order, handed to warps from a shared counter, so a warp
+// that finishes short walks immediately takes the next item instead of waiting for the slowest walk of the
+// request.  Requests are staged in shared memory in kSlots slots: the warp that takes a request's first item
+// copies its tokens in with one bulk (TMA) copy (up to kSlotTokens; longer requests read the rest through
+// the read-only path); warps with later items of that request wait until it is staged; the last warp to
+// finish one of its items writes the route and frees the slot for the request kSlots later.  Every wait is
+// bounded.
 //
 // A walk is warp-cooperative: a child lookup probes 32 slots of the node's children hash table at once
-// (one coalesced load, whatever the fan-out), and an edge label is compared with 2 16-byte loads (long labels) or 4 4-byte loads
-// loads in flight per lane; the first mismatch comes from a warp min-reduction.  The route
-// decision keeps the max of a packed 64-bit key per request.  Integer work only: no tensor cores.
+// (one coalesced load, whatever the fan-out), and an edge label is compared 32 consecutive tokens per warp
+// load, up to kUnroll loads in flight per lane, folded into one vote per block; the first mismatch is
+// searched only inside the block that holds it.  The route decision keeps the max of a packed 64-bit key
+// per request.  Integer work only: no tensor cores.
 #include "internal.h"
 
 namespace p2p {
@@ -26,8 +27,9 @@ constexpr int kWarps = 16;              // warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kSlots = 4;               // requests staged at a time per CTA
 constexpr int kSlotTokens = 4096;       // tokens of a request kept in shared memory (16 KB per slot)
-constexpr int kCtasPerSm = 3;           // 48 warps per SM: 64 KB of slots and <= 40 registers per thread
-constexpr int kVec = 2;                 // 16-byte label loads in flight per lane on long labels (256 tokens per step)
+constexpr int kCtasPerSm = 2;           // 32 warps per SM: 64 KB of slots and <= 64 registers per thread
+constexpr int kUnroll = 16;             // label loads in flight per lane on long labels (512 tokens per step)
+constexpr int kMaxGroup = 8;            // trees per work item, at most
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kSpinLimit = 1 << 24;     // bounded waits (~1 s): the kernel flags ERR_STALL and stops
 
@@ -89,111 +91,93 @@ __device__ __forceinline__ bool find_child(const int4* __restrict__ tab, int32_t
   return false;
 }
 
-// U loads of 32 label tokens in flight per lane, compared with the request; returns the first mismatch
-// in [j0, j0 + 32U) below lim, or -1 if there is none.  Positions are 32-bit: a walk never passes more
-// tokens than one tree path holds (< 2^31).
-template <int U>
-__device__ __forceinline__ int32_t compare_block(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
-                                                 const int32_t* g_req, int32_t pos, int32_t j0, int32_t lim,
-                                                 int lane) {
+// Request token j: from the shared-memory window, or past it through the read-only path.
+template <bool kGlobal>
+__device__ __forceinline__ int32_t rq(const int32_t* req, int32_t j) {
+  if constexpr (kGlobal) return __ldg(req + j);
+  else return req[j];
+}
+
+// U label loads of 32 tokens in flight per lane over [j0, j0 + 32U), a block inside both the label and the
+// request.  The block is folded into one OR of XORs per lane and one warp vote; only a block that holds a
+// mismatch is searched again for the first one.  Returns it, or -1.  Positions are 32-bit: a walk never
+// passes more tokens than one tree path holds (< 2^31).
+template <int U, bool kGlobal>
+__device__ __forceinline__ int32_t compare_full(const int32_t* __restrict__ lab, const int32_t* req, int32_t j0,
+                                                int lane) {
   int32_t v[U];
 #pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const int32_t j = j0 + u * 32 + lane;
-    v[u] = j < lim ? __ldg(lab + j) : 0;
-  }
+  for (int u = 0; u < U; ++u) v[u] = __ldg(lab + j0 + u * 32 + lane);
+  int32_t diff = 0;
+#pragma unroll
+  for (int u = 0; u < U; ++u) diff |= v[u] ^ rq<kGlobal>(req, j0 + u * 32 + lane);
+  if (!__any_sync(kFull, diff != 0)) return -1;
 #pragma unroll
   for (int u = 0; u < U; ++u) {
-    const int32_t j = j0 + u * 32 + lane;
-    const unsigned m = __ballot_sync(kFull, j < lim && v[u] != req_at(s_req, n_s, g_req, pos + j));
+    const unsigned m = __ballot_sync(kFull, v[u] != rq<kGlobal>(req, j0 + u * 32 + lane));
     if (m) return j0 + u * 32 + (__ffs(m) - 1);
   }
   return -1;
 }
 
-// U loads of 32 label tokens in flight per lane when the whole block lies inside the label and inside the
-// request's shared-memory window: no per-element checks, one reduction for the first mismatch.
-template <int U>
-__device__ __forceinline__ int32_t compare_full(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t j0,
-                                                int lane) {
-  int32_t v[U], r[U];
-#pragma unroll
-  for (int u = 0; u < U; ++u) v[u] = __ldg(lab + j0 + u * 32 + lane);
-#pragma unroll
-  for (int u = 0; u < U; ++u) r[u] = sreq[j0 + u * 32 + lane];
-  int32_t first = INT32_MAX;
-#pragma unroll
-  for (int u = U - 1; u >= 0; --u)
-    if (v[u] != r[u]) first = u * 32 + lane;
-  first = __reduce_min_sync(kFull, first);
-  return first == INT32_MAX ? -1 : j0 + first;
-}
-
-// As compare_full for a block that may run past the label end (tokens at or after lim are ignored) but
-// stays inside the shared-memory window.
-__device__ __forceinline__ int32_t compare_tail(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t j0,
-                                                int32_t lim, int lane) {
-  int32_t v[4], r[4];
+// As compare_full<4> for a block that may run past end (tokens at or after end are ignored).
+template <bool kGlobal>
+__device__ __forceinline__ int32_t compare_tail(const int32_t* __restrict__ lab, const int32_t* req, int32_t j0,
+                                                int32_t end, int lane) {
+  int32_t v[4];
 #pragma unroll
   for (int u = 0; u < 4; ++u) {
     const int32_t j = j0 + u * 32 + lane;
-    v[u] = j < lim ? __ldg(lab + j) : 0;
-    r[u] = j < lim ? sreq[j] : 0;
+    v[u] = j < end ? __ldg(lab + j) : 0;
   }
-  int32_t first = INT32_MAX;
+  int32_t diff = 0;
 #pragma unroll
-  for (int u = 3; u >= 0; --u)
-    if (v[u] != r[u]) first = u * 32 + lane;
-  first = __reduce_min_sync(kFull, first);
-  return first == INT32_MAX ? -1 : j0 + first;
+  for (int u = 0; u < 4; ++u) {
+    const int32_t j = j0 + u * 32 + lane;
+    if (j < end) diff |= v[u] ^ rq<kGlobal>(req, j);
+  }
+  if (!__any_sync(kFull, diff != 0)) return -1;
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int32_t j = j0 + u * 32 + lane;
+    const unsigned m = __ballot_sync(kFull, j < end && v[u] != rq<kGlobal>(req, j));
+    if (m) return j0 + u * 32 + (__ffs(m) - 1);
+  }
+  return -1;
 }
 
-// V 16-byte label loads per lane (4 tokens each, 128V tokens per warp step) compared with the staged
-// request; lab + jb must be 16-byte aligned and [jb, jb + 128V) inside the label and the shared-memory
-// window.  Each lane keeps its first mismatching token; one reduction gives the warp's first.
-template <int V>
-__device__ __forceinline__ int32_t compare_vec(const int32_t* __restrict__ lab, const int32_t* sreq, int32_t jb,
-                                               int lane) {
-  const int4* l4 = reinterpret_cast<const int4*>(lab + jb);
-  int4 v[V];
-#pragma unroll
-  for (int q = 0; q < V; ++q) v[q] = __ldg(l4 + q * 32 + lane);
-  int32_t first = INT32_MAX;
-#pragma unroll
-  for (int q = V - 1; q >= 0; --q) {
-    const int32_t base = q * 128 + 4 * lane;
-    const int32_t* rr = sreq + jb + base;
-    if (v[q].w != rr[3]) first = base + 3;
-    if (v[q].z != rr[2]) first = base + 2;
-    if (v[q].y != rr[1]) first = base + 1;
-    if (v[q].x != rr[0]) first = base;
-  }
-  first = __reduce_min_sync(kFull, first);
-  return first == INT32_MAX ? -1 : jb + first;
-}
-
-// First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.
-__device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
-                                                  const int32_t* g_req, int32_t pos, int32_t lim, int lane) {
-  int32_t j0 = 1;
-  const int32_t fast_end = min(lim, n_s - pos);  // blocks below this need no checks
-  if (j0 + 32 <= fast_end) {
-    const int32_t k = compare_full<1>(lab, s_req + pos, j0, lane);
+// First j in [j0, end) with lab[j] != req[j], or -1.  After one block at j0 the label side continues at a
+// 128-byte-aligned position at or below j0 + 32 (re-comparing <= 31 tokens): a warp's 32 consecutive label
+// tokens are then one cache line, and its 32 request tokens in shared memory fall in 32 distinct banks at
+// any alignment, so each load is a single wavefront on both sides.
+template <bool kGlobal>
+__device__ __forceinline__ int32_t compare_range(const int32_t* __restrict__ lab, const int32_t* req, int32_t j0,
+                                                 int32_t end, int lane) {
+  if (j0 + 32 <= end) {
+    const int32_t k = compare_full<1, kGlobal>(lab, req, j0, lane);
     if (k >= 0) return k;
-    // Continue at the first 16-byte-aligned label position at or below j0 + 32 (re-comparing <= 3 tokens).
     j0 += 32;
-    j0 -= (int32_t)(((uintptr_t)(lab + j0) >> 2) & 3);
-    for (; j0 + kVec * 128 <= fast_end; j0 += kVec * 128) {
-      const int32_t k2 = compare_vec<kVec>(lab, s_req + pos, j0, lane);
+    j0 -= (int32_t)(((uintptr_t)(lab + j0) >> 2) & 31);
+    for (; j0 + kUnroll * 32 <= end; j0 += kUnroll * 32) {
+      const int32_t k2 = compare_full<kUnroll, kGlobal>(lab, req, j0, lane);
       if (k2 >= 0) return k2;
     }
   }
-  for (; j0 < lim; j0 += 128) {
-    const int32_t k = pos + j0 + 128 <= n_s ? compare_tail(lab, s_req + pos, j0, lim, lane)
-                                            : compare_block<4>(lab, s_req, n_s, g_req, pos, j0, lim, lane);
+  for (; j0 < end; j0 += 128) {
+    const int32_t k = compare_tail<kGlobal>(lab, req, j0, end, lane);
     if (k >= 0) return k;
   }
-  return lim;
+  return -1;
+}
+
+// First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.  Request
+// tokens inside the shared-memory window (the first n_s) come from it, later ones from global memory.
+__device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
+                                                  const int32_t* g_req, int32_t pos, int32_t lim, int lane) {
+  const int32_t split = max(1, min(lim, n_s - pos));
+  int32_t k = compare_range<false>(lab, s_req + pos, 1, split, lane);
+  if (k < 0 && split < lim) k = compare_range<true>(lab, g_req + pos, split, lim, lane);
+  return k < 0 ? lim : k;
 }
 
 // match(r, T) for one tree, computed by the whole warp (result uniform across lanes).  len is the request
@@ -249,7 +233,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
   if (threadIdx.x == 0) s_next = 0;
   __syncthreads();
   const int64_t n_req = B > blockIdx.x ? (B - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
-  const unsigned long long total = (unsigned long long)n_req * (unsigned long long)P;
+  // A work item is (request k, trees p0 .. p0 + G - 1): G grows with P so that the per-item costs (the
+  // shared counter, the staging waits, the route-key merge) are shared by several walks while every warp of
+  // the CTA still finds items of the same request.
+  const int32_t G = min(kMaxGroup, max(1, P / kWarps));
+  const int32_t C = (P + G - 1) / G;  // work items per request
+  const unsigned long long total = (unsigned long long)n_req * (unsigned long long)C;
   const bool small = total <= 0xffffffffull;  // 32-bit item arithmetic (the usual case) is much cheaper
   for (;;) {
     unsigned long long i = 0;
@@ -257,20 +246,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     i = __shfl_sync(kFull, i, 0);
     if (i >= total) break;
     int64_t k;
-    int32_t p;
+    int32_t c;
     if (small) {
-      const uint32_t k32 = (uint32_t)i / (uint32_t)P;
+      const uint32_t k32 = (uint32_t)i / (uint32_t)C;
       k = k32;
-      p = (int32_t)((uint32_t)i - k32 * (uint32_t)P);
+      c = (int32_t)((uint32_t)i - k32 * (uint32_t)C);
     } else {
-      k = (int64_t)(i / (unsigned long long)P);
-      p = (int32_t)(i - (unsigned long long)k * P);
+      k = (int64_t)(i / (unsigned long long)C);
+      c = (int32_t)(i - (unsigned long long)k * C);
     }
     const int s = (int)(k % kSlots);
     const int64_t b = blockIdx.x + k * gridDim.x;
     Slot& sl = s_slot[s];
     int32_t* st = s_tok + s * kSlotTokens;
-    if (p == 0) {
+    if (c == 0) {
       // Stage request k once the request kSlots earlier has released the slot.
       if (!wait_for(&sl.free_for, (int)k, lane)) {
         if (lane == 0) atomicOr(err, ERR_STALL);
@@ -336,19 +325,27 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const int64_t start = *(volatile long long*)&sl.start;
     const int32_t n_s = *(volatile int*)&sl.len_s;
     const int32_t* req = st + *(volatile int*)&sl.shift;
-    const int32_t m = len > 0 ? walk(trees[p], req, n_s, tokens + start, (int32_t)min(len, (int64_t)INT32_MAX), lane, err) : 0;
+    const int32_t len32 = (int32_t)min(len, (int64_t)INT32_MAX);
+    const int32_t p1 = min(P, (c + 1) * G);
+    unsigned long long best = 0;
+    for (int32_t p = c * G; p < p1; ++p) {
+      const int32_t m = len > 0 ? walk(trees[p], req, n_s, tokens + start, len32, lane, err) : 0;
+      if (lane == 0) {
+        out_match[b * P + p] = m;
+        // Packed key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a
+        // better route (higher score, then lower load, then lower index).  The host guarantees
+        // alpha * load <= 2^31 - 1, load <= 65535 and P <= 65536, so every field fits.
+        const int32_t ld = __ldg(load + p);
+        const long long score = (long long)m - (long long)alpha * ld;
+        const unsigned long long key = ((unsigned long long)(score + 2147483648LL) << 32) |
+                                       ((unsigned long long)(0xFFFF - ld) << 16) | (unsigned long long)(0xFFFF - p);
+        best = key > best ? key : best;
+      }
+    }
     if (lane == 0) {
-      out_match[b * P + p] = m;
-      // Packed key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a
-      // better route (higher score, then lower load, then lower index).  The host guarantees
-      // alpha * load <= 2^31 - 1, load <= 65535 and P <= 65536, so every field fits.
-      const int32_t ld = __ldg(load + p);
-      const long long score = (long long)m - (long long)alpha * ld;
-      const unsigned long long key = ((unsigned long long)(score + 2147483648LL) << 32) |
-                                     ((unsigned long long)(0xFFFF - ld) << 16) | (unsigned long long)(0xFFFF - p);
-      atomicMax(&sl.best, key);
+      atomicMax(&sl.best, best);
       __threadfence_block();
-      if (atomicAdd(&sl.done, 1) == P - 1) {  // last item of request k: route it, free the slot
+      if (atomicAdd(&sl.done, 1) == C - 1) {  // last item of request k: route it, free the slot
         __threadfence_block();
         const unsigned long long bk = *(volatile unsigned long long*)&sl.best;
         if (len < 0) {
