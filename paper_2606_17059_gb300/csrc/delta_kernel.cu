@@ -489,24 +489,30 @@ __device__ __forceinline__ int32_t bucket_of(int32_t tok) {
   return (int32_t)(((uint32_t)tok * 0x85EBCA6Bu) >> (32 - kDeltaBucketBits));
 }
 
-__global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* states, int64_t* cursors,
-                                                                    const int32_t* __restrict__ op,
-                                                                    const int64_t* __restrict__ seg_begin,
-                                                                    const int64_t* __restrict__ seg_off,
-                                                                    const int32_t* __restrict__ seg_len,
-                                                                    const int32_t* __restrict__ pool,
-                                                                    int32_t* gather, int64_t stride,
-                                                                    const int32_t* shared) {
+__global__ void __launch_bounds__(kDeltaWarps * 32) delta_kernel(TreeState* states, int64_t* cursors,
+                                                                  const int32_t* __restrict__ op,
+                                                                  const int64_t* __restrict__ seg_begin,
+                                                                  const int64_t* __restrict__ seg_off,
+                                                                  const int32_t* __restrict__ seg_len,
+                                                                  const int32_t* __restrict__ pool,
+                                                                  int32_t* gather, int64_t stride,
+                                                                  const int32_t* shared) {
   __shared__ int8_t s_bucket[kChunk];
+  __shared__ int s_count[kDeltaBuckets];  // ops of each bucket in the chunk
+  __shared__ int s_order[kDeltaBuckets];  // buckets, heaviest first
+  __shared__ int s_stopped[kDeltaBuckets];
+  __shared__ int s_take;
   __shared__ int s_any;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   TreeState* gs = states + blockIdx.x;
   const int64_t op_begin = gs->op_begin, op_end = gs->op_end;
-  int64_t* my_cursor = cursors + (int64_t)blockIdx.x * kDeltaBuckets + warp;
-  int64_t next = *my_cursor;  // ops of this bucket before `next` are applied
+  int64_t* my_cursors = cursors + (int64_t)blockIdx.x * kDeltaBuckets;  // ops of a bucket before it are applied
   if (threadIdx.x == 0) s_any = 0;
   __syncthreads();
-  if (lane == 0 && next < op_end) atomicOr(&s_any, 1);
+  if (threadIdx.x < kDeltaBuckets) {
+    s_stopped[threadIdx.x] = 0;
+    if (my_cursors[threadIdx.x] < op_end) atomicOr(&s_any, 1);
+  }
   __syncthreads();
   if (!s_any || gs->status & DELTA_CORRUPT) return;
   Tree t;
@@ -515,11 +521,13 @@ __global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* st
   t.label = gs->label;
   t.shared = shared;
   t.g = gs;
-  int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaBuckets + warp) * stride : nullptr;
-  bool stopped = next >= op_end;
-  Memo memo;
+  int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaWarps + warp) * stride : nullptr;
+  Memo memo;  // facts about immutable labels: valid whichever bucket the warp works on
   for (int64_t c0 = op_begin; c0 < op_end; c0 += kChunk) {
     const int64_t clen = min((int64_t)kChunk, op_end - c0);
+    if (threadIdx.x < kDeltaBuckets) s_count[threadIdx.x] = 0;
+    if (threadIdx.x == 0) s_take = 0;
+    __syncthreads();
     for (int64_t j = threadIdx.x; j < clen; j += blockDim.x) {
       const int64_t i = c0 + j;
       int32_t b = 0;  // empty sequences: bucket 0
@@ -530,12 +538,32 @@ __global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* st
         }
       }
       s_bucket[j] = (int8_t)b;
+      atomicAdd(&s_count[b], 1);
     }
     __syncthreads();
-    if (!stopped && next < c0 + clen) {
+    if (warp == 0) {  // rank the buckets by op count (ties: lower bucket first)
+      const int mine = s_count[lane];
+      int rank = 0;
+      for (int o = 0; o < kDeltaBuckets; ++o) {
+        const int other = s_count[o];
+        rank += other > mine || (other == mine && o < lane);
+      }
+      s_order[rank] = lane;
+    }
+    __syncthreads();
+    for (;;) {
+      int idx = 0;
+      if (lane == 0) idx = atomicAdd(&s_take, 1);
+      idx = __shfl_sync(kFull, idx, 0);
+      if (idx >= kDeltaBuckets) break;
+      const int bk = s_order[idx];
+      if (s_count[bk] == 0 || s_stopped[bk]) continue;
+      int64_t next = my_cursors[bk];
+      if (next >= c0 + clen) continue;
+      bool stopped = false;
       for (int64_t j0 = max((int64_t)0, next - c0); j0 < clen && !stopped; j0 += 32) {
         const int64_t j = j0 + lane;
-        unsigned mine = __ballot_sync(kFull, j < clen && s_bucket[j] == warp);
+        unsigned mine = __ballot_sync(kFull, j < clen && s_bucket[j] == bk);
         while (mine && !stopped) {
           const int64_t i = c0 + j0 + (__ffs(mine) - 1);
           mine &= mine - 1;
@@ -568,16 +596,19 @@ __global__ void __launch_bounds__(kDeltaBuckets * 32) delta_kernel(TreeState* st
             stopped = true;
             next = i;
             if (r == OP_CORRUPT && lane == 0) atomicOr(&gs->status, DELTA_CORRUPT);
-          } else {
-            next = i + 1;
           }
         }
       }
+      if (lane == 0) {
+        my_cursors[bk] = stopped ? next : c0 + clen;
+        if (stopped) s_stopped[bk] = 1;
+      }
+      __syncwarp();
     }
     __syncthreads();
   }
-  if (!stopped) next = op_end;
-  if (lane == 0) *my_cursor = next;
+  // Buckets that never stopped have applied all their ops.
+  if (threadIdx.x < kDeltaBuckets && !s_stopped[threadIdx.x]) my_cursors[threadIdx.x] = op_end;
 }
 
 // Validates a device-resident delta into header (int32 words: [0..1] longest sequence as u64, [2] error
@@ -670,8 +701,8 @@ cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st) {
   if (n_trees <= 0) return cudaSuccess;
-  delta_kernel<<<n_trees, kDeltaBuckets * 32, 0, st>>>(d_states, cursors, op, seg_begin, seg_off, seg_len, pool, gather,
-                                                       gather_stride, shared);
+  delta_kernel<<<n_trees, kDeltaWarps * 32, 0, st>>>(d_states, cursors, op, seg_begin, seg_off, seg_len, pool, gather,
+                                                     gather_stride, shared);
   return cudaGetLastError();
 }
 

@@ -67,9 +67,11 @@ struct TreeState {
 
 enum { DELTA_OK = 0, DELTA_NEED_SPACE = 1, DELTA_CORRUPT = 2 };
 
-// Warps per tree in the delta kernel; ops are bucketed by a hash of their first token.
+// Delta kernel: ops are bucketed by a hash of their first token (kDeltaBuckets per tree); one CTA of
+// kDeltaWarps warps per tree takes the buckets heaviest first.
 constexpr int kDeltaBucketBits = 5;
 constexpr int kDeltaBuckets = 1 << kDeltaBucketBits;
+constexpr int kDeltaWarps = 8;
 
 // Children tables: at least 4 slots; grown (doubled) when claimed slots would pass 3/4 of the table.
 constexpr int kMinTabBits = 2;
@@ -89,9 +91,9 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
                          int32_t* out_match, int32_t* out_peer, int32_t* d_err, int num_sms, cudaStream_t st);
 
-// Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaBuckets warps
+// Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaWarps warps
 // per tree.  cursors[n_trees * kDeltaBuckets] holds each bucket's next op (set by launch_init_cursors,
-// kept across relaunches).  gather (n_trees * kDeltaBuckets * gather_stride tokens) is needed only when an
+// kept across relaunches).  gather (n_trees * kDeltaWarps * gather_stride tokens) is needed only when an
 // op's sequence has more than two pool runs; otherwise it may be NULL.
 cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,

@@ -713,7 +713,7 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   int32_t* gather = nullptr;
   const int64_t stride = std::max<int64_t>(max_len, 1);
   if (max_runs > 2) {
-    CK(ensure(r, r->d_gather, (size_t)nt * p2p::kDeltaBuckets * stride * sizeof(int32_t)));
+    CK(ensure(r, r->d_gather, (size_t)nt * p2p::kDeltaWarps * stride * sizeof(int32_t)));
     gather = (int32_t*)r->d_gather.p;
   }
   int64_t* cursors = (int64_t*)r->d_cursors.p;
@@ -797,7 +797,7 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
   // Scratch: one int64 cursor per (tree, bucket); gathered sequences only when an op has > 2 pool runs.
   const int64_t cursor_ints = (int64_t)nt * p2p::kDeltaBuckets * 2;
   const int64_t stride = max_len > 0 ? (int64_t)max_len : 1;
-  const int64_t gather_ints = max_runs > 2 ? (int64_t)nt * p2p::kDeltaBuckets * stride : 0;
+  const int64_t gather_ints = max_runs > 2 ? (int64_t)nt * p2p::kDeltaWarps * stride : 0;
   if (cursor_ints + gather_ints > p2p::static_scratch_tokens())
     return fail(r, P2P_E_INVAL, "the delta needs " + std::to_string(cursor_ints + gather_ints) +
                                     " words of scratch, more than the static scratch of " +
