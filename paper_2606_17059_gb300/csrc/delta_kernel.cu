@@ -50,42 +50,38 @@ struct Tree {
   __device__ const int32_t* lab(int32_t off) const { return label_ptr(label, shared, off); }
 };
 
-// Reserves k units of the counter (capacity cap); returns the first unit or -1.  Lane 0 does the CAS.
-__device__ int32_t bump(int32_t* ctr, int32_t cap, int64_t k, int lane) {
-  int32_t r = -1;
-  if (lane == 0) {
-    int32_t old = *(volatile int32_t*)ctr;
-    for (int it = 0; it < (1 << 20); ++it) {
-      if ((int64_t)old + k > cap) break;
-      const int32_t prev = atomicCAS(ctr, old, (int32_t)(old + k));
-      if (prev == old) {
-        r = old;
-        break;
-      }
-      old = prev;
-    }
-  }
-  return __shfl_sync(kFull, r, 0);
-}
-
-// Reserves the room an op may need.  On failure the op does nothing; the units it did get are counted as
-// stale (a later compaction reclaims them), and the request is recorded for the host to grow the arenas.
+// Reserves the room an op may need: lanes 0, 1 and 2 bump the node, child-entry and label counters at the
+// same time.  On failure the op does nothing; the units it did get are counted as stale (a later compaction
+// reclaims them), and the request is recorded for the host to grow the arenas.
 __device__ bool reserve(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, int32_t& n0, int32_t& c0, int32_t& l0,
                         int lane) {
-  n0 = c0 = l0 = 0;
-  if (nodes && (n0 = bump(&t.g->n_node, t.g->cap_node, nodes, lane)) < 0) {
-    nodes = 0;
-  } else if (entries && (c0 = bump(&t.g->n_child, t.g->cap_child, entries, lane)) < 0) {
-    entries = 0;
-  } else if (tokens && (l0 = bump(&t.g->n_label, t.g->cap_label, tokens, lane)) < 0) {
-    tokens = 0;
-  } else {
-    return true;
+  int32_t r = 0;
+  if (lane < 3) {
+    const int64_t k = lane == 0 ? nodes : lane == 1 ? entries : tokens;
+    if (k) {
+      int32_t* ctr = lane == 0 ? &t.g->n_node : lane == 1 ? &t.g->n_child : &t.g->n_label;
+      const int32_t cap = lane == 0 ? t.g->cap_node : lane == 1 ? t.g->cap_child : t.g->cap_label;
+      r = -1;
+      int32_t old = *(volatile int32_t*)ctr;
+      for (int it = 0; it < (1 << 20); ++it) {
+        if ((int64_t)old + k > cap) break;
+        const int32_t prev = atomicCAS(ctr, old, (int32_t)(old + k));
+        if (prev == old) {
+          r = old;
+          break;
+        }
+        old = prev;
+      }
+    }
   }
-  // Failed: nodes/entries/tokens now hold only what was obtained (the failed kind was zeroed).
+  n0 = __shfl_sync(kFull, r, 0);
+  c0 = __shfl_sync(kFull, r, 1);
+  l0 = __shfl_sync(kFull, r, 2);
+  if (n0 >= 0 && c0 >= 0 && l0 >= 0) return true;
   if (lane == 0) {
-    if (nodes) atomicAdd((unsigned long long*)&t.g->dead_nodes, (unsigned long long)nodes);
-    if (entries) atomicAdd((unsigned long long*)&t.g->stale_child, (unsigned long long)entries);
+    if (nodes && n0 >= 0) atomicAdd((unsigned long long*)&t.g->dead_nodes, (unsigned long long)nodes);
+    if (entries && c0 >= 0) atomicAdd((unsigned long long*)&t.g->stale_child, (unsigned long long)entries);
+    if (tokens && l0 >= 0) atomicAdd((unsigned long long*)&t.g->stale_label, (unsigned long long)tokens);
     atomicOr(&t.g->status, DELTA_NEED_SPACE);
   }
   return false;
@@ -104,25 +100,29 @@ __device__ bool take(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, in
   return false;
 }
 
-// Looks `tok` up in the children table of 2^bits slots at child[off]: returns 1 (live child), 2 (tombstone
-// of tok), or 0 (absent; *slot = the first empty slot of its probe run, or -1 if there is none).  Key and
-// state are read as one 64-bit word, so a slot another warp is claiming (root table only) is seen either
-// all zero or with its final key.  Only this warp ever looks up `tok` below this node.
-__device__ int probe(const Tree& t, int32_t off, int32_t bits, int32_t tok, int lane, int32_t& slot) {
+// Looks `tok` up in the children table of 2^bits slots at child[off]: returns 1 (live child; e = its slot's
+// entry), 2 (tombstone of tok), or 0 (absent; *slot = the first empty slot of its probe run, or -1 if there is
+// none).  A slot is read as two 64-bit words (each single-copy atomic, the first holding key and state), so
+// a slot another warp is claiming (root table only) is seen either all zero or with its final key.  Only
+// this warp ever writes the slot of `tok` below this node, so the entry of a live `tok` is current.
+__device__ int probe(const Tree& t, int32_t off, int32_t bits, int32_t tok, int lane, int32_t& slot, int4& e) {
   slot = -1;
   if (bits == 0) return 0;
   const uint32_t mask = (1u << bits) - 1, h = slot_hash(tok, bits);
   for (uint32_t base = 0; base <= mask; base += 32) {
     const uint32_t s = (h + base + lane) & mask;
-    const unsigned long long kv = *(volatile unsigned long long*)&t.child[off + s];
-    const int32_t key = (int32_t)(kv & 0xffffffffull), state = (int32_t)(kv >> 32);
+    const longlong2 kv = __ldcv(reinterpret_cast<const longlong2*>(&t.child[off + s]));
+    const int32_t key = (int32_t)(kv.x & 0xffffffffll), state = (int32_t)((unsigned long long)kv.x >> 32);
     const unsigned mine = __ballot_sync(kFull, key == tok && (state >= 1 || state == -1));
     const unsigned empty = __ballot_sync(kFull, state == 0);
     const int fm = mine ? __ffs(mine) - 1 : 64;
     const int fe = empty ? __ffs(empty) - 1 : 64;
     if (fm < fe) {
       slot = off + (int32_t)((h + base + fm) & mask);
-      return __shfl_sync(kFull, state, fm) >= 1 ? 1 : 2;
+      const long long a = __shfl_sync(kFull, kv.x, fm), b = __shfl_sync(kFull, kv.y, fm);
+      e = make_int4((int32_t)(a & 0xffffffffll), (int32_t)((unsigned long long)a >> 32),
+                    (int32_t)(b & 0xffffffffll), (int32_t)((unsigned long long)b >> 32));
+      return e.y >= 1 ? 1 : 2;
     }
     if (fe < 64) {
       slot = off + (int32_t)((h + base + fe) & mask);
@@ -140,7 +140,8 @@ __device__ int32_t claim(const Tree& t, int32_t off, int32_t bits, int32_t tok, 
     int32_t got = 0;
     if (lane == 0) got = atomicCAS((unsigned long long*)&t.child[slot], 0ull, want) == 0ull;
     if (__shfl_sync(kFull, got, 0)) return slot;
-    if (probe(t, off, bits, tok, lane, slot) != 0) return -1;
+    int4 e;
+    if (probe(t, off, bits, tok, lane, slot, e) != 0) return -1;
   }
   return -1;
 }
@@ -303,7 +304,8 @@ __device__ bool ensure_slot(Tree& t, int32_t cur, int4& nd, int lane) {
   return true;
 }
 
-__device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
+// root: the root's node record as of the launch (its table moves only between launches).
+__device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& memo) {
   const int64_t n = q.n;
   if (n == 0) {
     if (lane == 0) atomicAdd(&t.node[0].w, 1);
@@ -313,6 +315,7 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
   int32_t cur = 0;
   int64_t pos = 0;
   int32_t n0, c0, l0;
+  int4 nd = root;  // record of node cur: below the root only this warp writes it
   for (int64_t guard = 0; guard <= n + 1; ++guard) {
     if (pos == n) {  // the sequence ends exactly at node cur (never the root here: n > 0)
       if (lane == 0) t.node[cur].w += 1;
@@ -320,9 +323,9 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
       return OP_DONE;
     }
     const int32_t tok = q.at(pos);
-    int4 nd = t.node[cur];
     int32_t slot;
-    int st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot);
+    int4 ce;
+    int st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot, ce);
     if (st != 1) {
       // New leaf edge q[pos, n) under cur: revive tok's tombstone, or claim an empty slot.
       const int64_t L = n - pos;
@@ -343,7 +346,7 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
           }
         } else {
           if (!ensure_slot(t, cur, nd, lane)) return OP_NEED;
-          st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot);
+          st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot, ce);
           if (st != 0 || slot < 0) return OP_CORRUPT;
           if (lane == 0) t.node[cur].y = nd.y + (1 << 5);
         }
@@ -362,13 +365,14 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
       return OP_DONE;
     }
     int4* ent = t.child + slot;
-    const int4 ce = *ent;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
+    const int4 nn = t.node[ce.y];  // the child's record, fetched while the label is compared
     const int64_t lim = min((int64_t)ce.w, n - pos);
     const int64_t k = first_diff(t.lab(ce.z), q, pos, 1, lim, lane, memo);
     if (k == ce.w) {
       cur = ce.y;
       pos += k;
+      nd = nn;
       continue;
     }
     // The sequence leaves (or ends inside) the edge after k tokens: split it there.  The new node mid
@@ -403,7 +407,7 @@ __device__ int insert(Tree& t, const Seq& q, int lane, Memo& memo) {
   return OP_CORRUPT;
 }
 
-__device__ int remove(Tree& t, const Seq& q, int lane, Memo& memo) {
+__device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& memo) {
   const int64_t n = q.n;
   if (n == 0) {
     int ok = 0;
@@ -419,28 +423,30 @@ __device__ int remove(Tree& t, const Seq& q, int lane, Memo& memo) {
   int32_t cur = 0, par = -1;
   int4 *e_cur = nullptr, *e_par = nullptr;
   int64_t pos = 0;
+  int4 nd = root, pn = root;  // records of cur and par (below the root only this warp writes them)
   for (int64_t guard = 0; pos < n; ++guard) {
     if (guard > n) return OP_CORRUPT;
-    const int4 nd = t.node[cur];
     int32_t slot;
-    if (probe(t, nd.x, tab_bits(nd.y), q.at(pos), lane, slot) != 1) {
+    int4 ce;
+    if (probe(t, nd.x, tab_bits(nd.y), q.at(pos), lane, slot, ce) != 1) {
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
     int4* ent = t.child + slot;
-    const int4 ce = *ent;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
+    const int4 nn = t.node[ce.y];  // the child's record, fetched while the label is compared
     if (pos + ce.w > n || first_diff(t.lab(ce.z), q, pos, 1, ce.w, lane, memo) < ce.w) {
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
     e_par = e_cur;
     par = cur;
+    pn = nd;
     e_cur = ent;
     cur = ce.y;
     pos += ce.w;
+    nd = nn;
   }
-  const int4 nd = t.node[cur];
   if (nd.w == 0) {
     add_stat(&t.g->n_absent, 1, lane);
     return OP_DONE;
@@ -460,8 +466,8 @@ __device__ int remove(Tree& t, const Seq& q, int lane, Memo& memo) {
     fold_child(t, cur, e_cur, ys, l0, lane);
     return OP_DONE;
   }
-  // A leaf that stores nothing any more: tombstone its slot in the parent's table.
-  const int4 pn = t.node[par];
+  // A leaf that stores nothing any more: tombstone its slot in the parent's table.  (pn is only read when
+  // par is not the root.)
   const bool fold_parent = par != 0 && pn.w == 0 && pn.z == 2;
   int32_t other = -1;
   if (fold_parent) {
@@ -489,15 +495,13 @@ __device__ __forceinline__ int32_t bucket_of(int32_t tok) {
   return (int32_t)(((uint32_t)tok * 0x85EBCA6Bu) >> (32 - kDeltaBucketBits));
 }
 
-__global__ void __launch_bounds__(kDeltaWarps * 32) delta_kernel(TreeState* states, int64_t* cursors,
-                                                                  const int32_t* __restrict__ op,
-                                                                  const int64_t* __restrict__ seg_begin,
-                                                                  const int64_t* __restrict__ seg_off,
-                                                                  const int32_t* __restrict__ seg_len,
-                                                                  const int32_t* __restrict__ pool,
-                                                                  int32_t* gather, int64_t stride,
-                                                                  const int32_t* shared) {
+__global__ void __launch_bounds__(kDeltaWarps * 32, 3)
+    delta_kernel(TreeState* states, int64_t* cursors, const int32_t* __restrict__ op,
+                 const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
+                 const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int32_t* gather,
+                 int64_t stride, const int32_t* shared) {
   __shared__ int8_t s_bucket[kChunk];
+  __shared__ int64_t s_run[kChunk + 1];   // seg_begin of the chunk's ops (and of the op after it)
   __shared__ int s_count[kDeltaBuckets];  // ops of each bucket in the chunk
   __shared__ int s_order[kDeltaBuckets];  // buckets, heaviest first
   __shared__ int s_stopped[kDeltaBuckets];
@@ -521,6 +525,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32) delta_kernel(TreeState* stat
   t.label = gs->label;
   t.shared = shared;
   t.g = gs;
+  const int4 root = t.node[0];  // its table offset and size hold for the whole launch
   int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaWarps + warp) * stride : nullptr;
   Memo memo;  // facts about immutable labels: valid whichever bucket the warp works on
   for (int64_t c0 = op_begin; c0 < op_end; c0 += kChunk) {
@@ -528,10 +533,13 @@ __global__ void __launch_bounds__(kDeltaWarps * 32) delta_kernel(TreeState* stat
     if (threadIdx.x < kDeltaBuckets) s_count[threadIdx.x] = 0;
     if (threadIdx.x == 0) s_take = 0;
     __syncthreads();
+    if (threadIdx.x == 0) s_run[clen] = seg_begin[c0 + clen];
     for (int64_t j = threadIdx.x; j < clen; j += blockDim.x) {
       const int64_t i = c0 + j;
       int32_t b = 0;  // empty sequences: bucket 0
-      for (int64_t g = seg_begin[i]; g < seg_begin[i + 1]; ++g) {
+      const int64_t g0 = seg_begin[i];
+      s_run[j] = g0;
+      for (int64_t g = g0; g < seg_begin[i + 1]; ++g) {
         if (seg_len[g] > 0) {
           b = bucket_of(pool[seg_off[g]]);
           break;
@@ -565,10 +573,10 @@ __global__ void __launch_bounds__(kDeltaWarps * 32) delta_kernel(TreeState* stat
         const int64_t j = j0 + lane;
         unsigned mine = __ballot_sync(kFull, j < clen && s_bucket[j] == bk);
         while (mine && !stopped) {
-          const int64_t i = c0 + j0 + (__ffs(mine) - 1);
+          const int64_t jj = j0 + (__ffs(mine) - 1), i = c0 + jj;
           mine &= mine - 1;
           // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
-          const int64_t g0 = seg_begin[i], g1 = seg_begin[i + 1];
+          const int64_t g0 = s_run[jj], g1 = s_run[jj + 1];
           Seq q;
           if (g1 - g0 <= 2) {
             q.a = pool + (g1 > g0 ? seg_off[g0] : 0);
@@ -591,7 +599,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32) delta_kernel(TreeState* stat
             q.a = q.b = buf;
             q.na = q.n = len;
           }
-          const int r = op[i] == P2P_OP_INSERT ? insert(t, q, lane, memo) : remove(t, q, lane, memo);
+          const int r = op[i] == P2P_OP_INSERT ? insert(t, q, root, lane, memo) : remove(t, q, root, lane, memo);
           if (r != OP_DONE) {
             stopped = true;
             next = i;
