@@ -1,0 +1,158 @@
+// group_kernel.cu -- shared-prefix groups of a request batch, ahead of the route kernel.
+//
+// Requests of one batch often share long prefixes (a few-shot or system prompt in front of each query).
+// Their walks in a tree coincide along the shared part, so a batch is routed in two passes: group leaders
+// walk every tree as usual, and every other request of a group (a follower) starts from its leader's result.
+// For a follower f of leader l with c = LCP(r_f, r_l) (exact, computed here):
+//   - if match(r_l, T) < c, then match(r_f, T) = match(r_l, T): both walks stop at the same token;
+//   - otherwise match(r_f, T) >= c, and the follower's walk need not compare its first c tokens.
+// Both facts hold for the PrefixMatch of Algorithm 1 because a walk depends only on the request tokens it
+// has consumed.  Results are therefore identical to independent walks; grouping changes only the work.
+//
+// Grouping: a request of at least kGroupHead tokens is keyed by a 64-bit hash of its first kGroupHead tokens
+// and inserted into an open-addressing table; the smallest request index with that key leads the group.
+// A follower whose exact common prefix with its leader is shorter than kGroupHead (a hash collision) routes
+// as a leader instead.  The leader choice is deterministic (smallest index); the order of the two request
+// lists is not, and only affects scheduling.
+#include "internal.h"
+
+namespace p2p {
+namespace {
+
+constexpr unsigned kFull = 0xffffffffu;
+constexpr int kGroupThreads = 256;
+
+// SplitMix64 output function (Steele, Lea & Flood 2014; constants published by Vigna).
+__device__ __forceinline__ unsigned long long mix64(unsigned long long z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ bool request_range(const int64_t* offsets, int64_t b, int64_t tok_base, int64_t n_tokens,
+                                              int64_t& start, int64_t& len) {
+  start = offsets[b] - tok_base;
+  const int64_t end = offsets[b + 1] - tok_base;
+  len = end - start;
+  return start >= 0 && start <= end && end <= n_tokens;
+}
+
+// One warp per request: hash of the first kGroupHead tokens (one token per lane and position, each mixed
+// with its position, summed), then lane 0 finds or claims the key's slot and lowers its leader index.
+__global__ void __launch_bounds__(kGroupThreads) group_hash_kernel(
+    const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
+    int64_t B, unsigned long long* keys, int32_t* vals, int32_t bits, int32_t* slot_of) {
+  static_assert(kGroupHead == 64, "two tokens per lane");
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
+  const uint32_t mask = (1u << bits) - 1;
+  for (int64_t b = ((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5; b < B; b += warps) {
+    int64_t start, len;
+    if (!request_range(offsets, b, tok_base, n_tokens, start, len) || len < kGroupHead) {
+      if (lane == 0) slot_of[b] = -1;
+      continue;
+    }
+    const int32_t* g = tokens + start;
+    unsigned long long h = mix64((unsigned long long)(uint32_t)__ldg(g + lane) | ((unsigned long long)lane << 32)) +
+                           mix64((unsigned long long)(uint32_t)__ldg(g + lane + 32) |
+                                 ((unsigned long long)(lane + 32) << 32));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) h += __shfl_xor_sync(kFull, h, o);
+    h |= 1ull;  // 0 marks an empty slot
+    if (lane == 0) {
+      int32_t slot = -1;
+      uint32_t s = (uint32_t)h & mask;
+      for (uint32_t it = 0; it <= mask; ++it, s = (s + 1) & mask) {
+        const unsigned long long prev = atomicCAS(&keys[s], 0ull, h);
+        if (prev == 0ull || prev == h) {
+          slot = (int32_t)s;
+          break;
+        }
+      }
+      if (slot >= 0) atomicMin(&vals[slot], (int32_t)b);
+      slot_of[b] = slot;
+    }
+  }
+}
+
+// First position in [0, n) where a and b differ, or n (one warp, both in global memory).
+__device__ int64_t lcp_warp(const int32_t* __restrict__ a, const int32_t* __restrict__ b, int64_t n, int lane) {
+  constexpr int U = 8;
+  int64_t j0 = 0;
+  for (; j0 + 32 * U <= n; j0 += 32 * U) {
+    int32_t x[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) x[u] = __ldg(a + j0 + u * 32 + lane);
+    int32_t diff = 0;
+#pragma unroll
+    for (int u = 0; u < U; ++u) diff |= x[u] ^ __ldg(b + j0 + u * 32 + lane);
+    if (__any_sync(kFull, diff != 0)) {
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const unsigned m = __ballot_sync(kFull, x[u] != __ldg(b + j0 + u * 32 + lane));
+        if (m) return j0 + u * 32 + (__ffs(m) - 1);
+      }
+    }
+  }
+  for (; j0 < n; j0 += 32) {
+    const int64_t j = j0 + lane;
+    const unsigned m = __ballot_sync(kFull, j < n && __ldg(a + j) != __ldg(b + j));
+    if (m) return j0 + (__ffs(m) - 1);
+  }
+  return n;
+}
+
+// One warp per request: its leader, the exact common prefix with it, and the request appended to the leader
+// list (lists[0 ..)) or the follower list (lists[B ..)); counts[0] and counts[1] must start at zero.
+__global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
+    const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
+    int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
+    int32_t* lists, int32_t* counts) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
+  for (int64_t b = ((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5; b < B; b += warps) {
+    const int32_t s = slot_of[b];
+    const int32_t l = s >= 0 ? vals[s] : (int32_t)b;
+    int64_t c = -1;
+    if (l != (int32_t)b) {  // both requests are valid and hold at least kGroupHead tokens
+      int64_t sb, nb, sl, nl;
+      request_range(offsets, b, tok_base, n_tokens, sb, nb);
+      request_range(offsets, l, tok_base, n_tokens, sl, nl);
+      c = lcp_warp(tokens + sb, tokens + sl, min(nb, nl), lane);
+      if (c < kGroupHead || c > INT32_MAX) c = -1;
+    }
+    if (lane == 0) {
+      if (c < 0) {
+        lead[b] = (int32_t)b;
+        lists[atomicAdd(&counts[0], 1)] = (int32_t)b;
+      } else {
+        lead[b] = l;
+        cpre[b] = (int32_t)c;
+        lists[B + atomicAdd(&counts[1], 1)] = (int32_t)b;
+      }
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
+                         const GroupScratch& g, int num_sms, cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  const size_t slots = (size_t)1 << g.bits;
+  cudaError_t e = cudaMemsetAsync(g.keys, 0, slots * sizeof(unsigned long long), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.vals, 0x7f, slots * sizeof(int32_t), st);  // 0x7f7f7f7f > any index
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 2 * sizeof(int32_t), st);
+  if (e != cudaSuccess) return e;
+  const int64_t want = (B + kGroupThreads / 32 - 1) / (kGroupThreads / 32);
+  const int grid = (int)std::min<int64_t>(want, (int64_t)num_sms * 8);
+  group_hash_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.keys, g.vals, g.bits,
+                                                    g.slot_of);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  group_resolve_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
+                                                       g.lead, g.cpre, g.lists, g.counts);
+  return cudaGetLastError();
+}
+
+}  // namespace p2p

@@ -86,10 +86,29 @@ constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits 
 // Bits of the router's device error word.
 enum { ERR_BAD_OFFSETS = 1, ERR_CORRUPT_TREE = 2, ERR_STALL = 4 };
 
-// Route kernel (lookup + route decision), see route_kernel.cu.
+// Shared-prefix groups of a batch (group_kernel.cu): requests of at least kGroupHead tokens are grouped by
+// their first kGroupHead tokens; lead[b] is b's group leader, cpre[b] its exact common prefix with the
+// leader (followers only); lists[0 .. counts[0]) are the leaders, lists[B .. B + counts[1]) the followers.
+constexpr int kGroupHead = 64;
+struct GroupScratch {
+  unsigned long long* keys;  // 2^bits slots
+  int32_t* vals;             // 2^bits slots
+  int32_t bits;
+  int32_t* slot_of;  // [B]
+  int32_t* lead;     // [B]
+  int32_t* cpre;     // [B]
+  int32_t* lists;    // [2B]
+  int32_t* counts;   // [2]
+};
+cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
+                         const GroupScratch& g, int num_sms, cudaStream_t st);
+
+// Route kernel (lookup + route decision), see route_kernel.cu.  Without groups (g == nullptr) one launch
+// routes every request; with groups, one launch routes the leaders and a second the followers.
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens,
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
-                         int32_t* out_match, int32_t* out_peer, int32_t* d_err, int num_sms, cudaStream_t st);
+                         int32_t* out_match, int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms,
+                         cudaStream_t st);
 
 // Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaWarps warps
 // per tree.  cursors[n_trees * kDeltaBuckets] holds each bucket's next op (set by launch_init_cursors,

@@ -43,6 +43,8 @@ struct Slot {
   int len_s;        // tokens held in shared memory
   int shift;        // token j of the request sits at slot token shift + j (keeps bulk copies 16-byte aligned)
   int done;         // items of the request finished
+  int lead;         // follower pass: the request's group leader
+  int cpre;         // follower pass: its exact common prefix with the leader
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -170,20 +172,24 @@ __device__ __forceinline__ int32_t compare_range(const int32_t* __restrict__ lab
   return -1;
 }
 
-// First j in [1, lim) with lab[j] != request[pos + j], or lim.  lab[0] == request[pos] is known.  Request
-// tokens inside the shared-memory window (the first n_s) come from it, later ones from global memory.
+// First j in [from, lim) with lab[j] != request[pos + j], or lim; the tokens before `from` are known to
+// match (from >= 1: lab[0] == request[pos] is known).  Request tokens inside the shared-memory window (the
+// first n_s) come from it, later ones from global memory.
 __device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
-                                                  const int32_t* g_req, int32_t pos, int32_t lim, int lane) {
-  const int32_t split = max(1, min(lim, n_s - pos));
-  int32_t k = compare_range<false>(lab, s_req + pos, 1, split, lane);
+                                                  const int32_t* g_req, int32_t pos, int32_t lim, int32_t from,
+                                                  int lane) {
+  if (from >= lim) return lim;
+  const int32_t split = max(from, min(lim, n_s - pos));
+  int32_t k = compare_range<false>(lab, s_req + pos, from, split, lane);
   if (k < 0 && split < lim) k = compare_range<true>(lab, g_req + pos, split, lim, lane);
   return k < 0 ? lim : k;
 }
 
 // match(r, T) for one tree, computed by the whole warp (result uniform across lanes).  len is the request
-// length clamped to 2^31 - 1 (no match can be longer than a tree path).
+// length clamped to 2^31 - 1 (no match can be longer than a tree path).  The first `known` tokens are known
+// to be matched (known <= match(r, T)): the walk still follows their path but does not compare them.
 __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t len,
-                        int lane, int32_t* err) {
+                        int32_t known, int lane, int32_t* err) {
   if (len == 0) return 0;
   int4 ce;
   if (!find_child(t.child + t.root_off, t.root_bits, req_at(s_req, n_s, g_req, 0), lane, ce)) return 0;
@@ -195,7 +201,8 @@ __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, co
     }
     const int4 nn = __ldg(t.node + ce.y);  // the child's record, fetched while its label is compared
     const int32_t lim = min(ce.w, len - pos);
-    const int32_t k = first_mismatch(label_ptr(t.label, t.shared, ce.z), s_req, n_s, g_req, pos, lim, lane);
+    const int32_t k = first_mismatch(label_ptr(t.label, t.shared, ce.z), s_req, n_s, g_req, pos, lim,
+                                     max(1, known - pos), lane);
     pos += k;
     if (k < ce.w || pos >= len || nn.z <= 0) break;
     if (!find_child(t.child + nn.x, tab_bits(nn.y), req_at(s_req, n_s, g_req, pos), lane, ce)) break;
@@ -214,10 +221,17 @@ __device__ __forceinline__ bool wait_for(const int* flag, int v, int lane) {
   return __shfl_sync(kFull, ok, 0) != 0;
 }
 
+// kFollow = false: routes requests list[0 .. *count) (every request b < B if list is NULL) with full walks.
+// kFollow = true: routes the followers list[0 .. *count) of a grouped batch, after the leaders' pass; a
+// follower's match in tree p is its leader's when that is below their common prefix c, else a walk that
+// skips comparing the first c tokens.  Followers are not staged: their walks compare only tokens past c.
+template <bool kFollow>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
-    int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ load, int32_t alpha,
-    int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
+    int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ list,
+    const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
+    const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
+    int32_t* err) {
   extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
   __shared__ unsigned long long s_next;
@@ -232,7 +246,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
   }
   if (threadIdx.x == 0) s_next = 0;
   __syncthreads();
-  const int64_t n_req = B > blockIdx.x ? (B - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
+  const int64_t n_all = count ? (int64_t)*count : B;  // requests of this launch
+  const int64_t n_req = n_all > blockIdx.x ? (n_all - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
   // A work item is (request k, trees p0 .. p0 + G - 1): G grows with P so that the per-item costs (the
   // shared counter, the staging waits, the route-key merge) are shared by several walks while every warp of
   // the CTA still finds items of the same request.
@@ -256,7 +271,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
       c = (int32_t)(i - (unsigned long long)k * C);
     }
     const int s = (int)(k % kSlots);
-    const int64_t b = blockIdx.x + k * gridDim.x;
+    const int64_t kb = blockIdx.x + k * gridDim.x;
+    const int64_t b = list ? (int64_t)__ldg(list + kb) : kb;
     Slot& sl = s_slot[s];
     int32_t* st = s_tok + s * kSlotTokens;
     if (c == 0) {
@@ -272,7 +288,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
       // shared addresses: the aligned middle of the request moves with one bulk copy, the <= 3 tokens on
       // each side with plain loads.
       const int32_t shift = (int32_t)(((uintptr_t)g >> 2) & 3);
-      const int32_t n_s = valid ? (int32_t)min(end - start, (int64_t)(kSlotTokens - shift)) : 0;
+      const int32_t n_s = valid && !kFollow ? (int32_t)min(end - start, (int64_t)(kSlotTokens - shift)) : 0;
       const int32_t j_lo = min((4 - shift) & 3, n_s);
       const int32_t j_hi = max(j_lo, n_s - (int32_t)(((uintptr_t)(g + n_s) >> 2) & 3));
       const uint32_t bytes = (uint32_t)(j_hi - j_lo) * 4u;
@@ -303,6 +319,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
         sl.shift = shift;
         sl.best = 0;
         sl.done = 0;
+        if (kFollow) {
+          sl.lead = __ldg(lead + b);
+          sl.cpre = __ldg(cpre + b);
+        }
         __threadfence_block();
         *(volatile int*)&sl.ready = (int)k;
       }
@@ -327,9 +347,22 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const int32_t* req = st + *(volatile int*)&sl.shift;
     const int32_t len32 = (int32_t)min(len, (int64_t)INT32_MAX);
     const int32_t p1 = min(P, (c + 1) * G);
+    int64_t lrow = 0;
+    int32_t cp = 0;
+    if (kFollow) {
+      lrow = (int64_t)*(volatile int*)&sl.lead * P;
+      cp = *(volatile int*)&sl.cpre;
+    }
     unsigned long long best = 0;
     for (int32_t p = c * G; p < p1; ++p) {
-      const int32_t m = len > 0 ? walk(trees[p], req, n_s, tokens + start, len32, lane, err) : 0;
+      int32_t m;
+      if (kFollow) {
+        // The leader's match (its pass has finished) decides, or bounds, the follower's.
+        const int32_t ml = __ldg(out_match + lrow + p);
+        m = ml < cp ? ml : cp >= len32 ? len32 : walk(trees[p], req, 0, tokens + start, len32, cp, lane, err);
+      } else {
+        m = len > 0 ? walk(trees[p], req, n_s, tokens + start, len32, 0, lane, err) : 0;
+      }
       if (lane == 0) {
         out_match[b * P + p] = m;
         // Packed key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a
@@ -366,15 +399,29 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
 
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
                          const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
-                         int32_t* out_peer, int32_t* d_err, int num_sms, cudaStream_t st) {
+                         int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
   const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
-  cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(route_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
   const int grid = (int)(B < max_ctas ? B : max_ctas);
-  route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, d_load, alpha,
-                                             out_match, out_peer, d_err);
+  if (!g) {
+    route_kernel<false><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, nullptr,
+                                                      nullptr, nullptr, nullptr, d_load, alpha, out_match, out_peer,
+                                                      d_err);
+    return cudaGetLastError();
+  }
+  route_kernel<false><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists,
+                                                    g->counts, nullptr, nullptr, d_load, alpha, out_match, out_peer,
+                                                    d_err);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  route_kernel<true><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists + B,
+                                                   g->counts + 1, g->lead, g->cpre, d_load, alpha, out_match,
+                                                   out_peer, d_err);
   return cudaGetLastError();
 }
 

@@ -85,6 +85,7 @@ struct p2p_router {
   TreeState* h_states = nullptr;  // pinned, P entries
   DevBuf req_tok, req_off, out_match, out_peer;
   DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_cursors, d_gather;
+  DevBuf grp_keys, grp_vals, grp_req;  // shared-prefix grouping of a batch
   int64_t launches = 0;  // kernels this router has launched
   // Shared label pool: long labels interned across trees (device array, host mirror, content index).
   int32_t* d_shared = nullptr;
@@ -143,6 +144,45 @@ cudaError_t ensure(p2p_router* r, DevBuf& b, size_t bytes) {
   cudaError_t e = dalloc(r, &b.p, cap);
   if (e == cudaSuccess) b.cap = cap;
   return e;
+}
+
+// Scratch of the shared-prefix grouping for a batch of B requests (B <= 2^30): a key table of at least 2B
+// slots, then slot_of, lead, cpre (B each), the two request lists (2B) and their two counts.
+cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
+  const int64_t slots = std::max<int64_t>(next_pow2(2 * B), 1024);
+  cudaError_t e = ensure(r, r->grp_keys, (size_t)slots * sizeof(unsigned long long));
+  if (e == cudaSuccess) e = ensure(r, r->grp_vals, (size_t)slots * sizeof(int32_t));
+  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(5 * B + 2) * sizeof(int32_t));
+  if (e != cudaSuccess) return e;
+  int32_t* q = static_cast<int32_t*>(r->grp_req.p);
+  g.keys = static_cast<unsigned long long*>(r->grp_keys.p);
+  g.vals = static_cast<int32_t*>(r->grp_vals.p);
+  g.bits = log2_exact(slots);
+  g.slot_of = q;
+  g.lead = q + B;
+  g.cpre = q + 2 * B;
+  g.lists = q + 3 * B;
+  g.counts = q + 5 * B;
+  return cudaSuccess;
+}
+
+// Groups the batch by shared prefix and routes it (leaders, then followers); batches too large for 32-bit
+// request indices are routed in one ungrouped pass.
+int route(p2p_router* r, const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
+          int32_t alpha, int32_t* out_match, int32_t* out_peer) {
+  if (B > ((int64_t)1 << 30)) {
+    CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
+                         r->d_err, nullptr, r->num_sms, r->stream));
+    r->launches += 1;
+    return P2P_OK;
+  }
+  p2p::GroupScratch g;
+  CK(group_scratch(r, B, g));
+  CK(p2p::launch_group(tokens, n_tokens, tok_base, offsets, B, g, r->num_sms, r->stream));
+  CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
+                       r->d_err, &g, r->num_sms, r->stream));
+  r->launches += 4;
+  return P2P_OK;
 }
 
 // Device-to-host copy ordered on the router stream (waits for it).
@@ -550,7 +590,8 @@ void p2p_router_destroy(p2p_router* r) {
   if (r->pool) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
-                      &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_cursors, &r->d_gather})
+                      &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_cursors, &r->d_gather,
+                      &r->grp_keys, &r->grp_vals, &r->grp_req})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -838,10 +879,7 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
   if (!offsets || !out_match || !out_peer || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
   DeviceGuard g(r->device);
   if (int rc = stage_load(r, load)) return rc;
-  CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, 0, offsets, B, r->d_load, alpha, out_match, out_peer,
-                       r->d_err, r->num_sms, r->stream));
-  r->launches += 1;
-  return P2P_OK;
+  return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer);
 }
 
 int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* offsets, int64_t B, const int32_t* load,
@@ -864,10 +902,9 @@ int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* of
   if (n_tok) CK(cudaMemcpyAsync(r->req_tok.p, tokens + offsets[0], (size_t)n_tok * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
   CK(cudaMemcpyAsync(r->req_off.p, offsets, (size_t)(B + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, r->stream));
   if (int rc = stage_load(r, load)) return rc;
-  CK(p2p::launch_route(r->d_views, r->P, (const int32_t*)r->req_tok.p, n_tok, offsets[0], (const int64_t*)r->req_off.p, B,
-                       r->d_load, alpha, (int32_t*)r->out_match.p, (int32_t*)r->out_peer.p, r->d_err, r->num_sms,
-                       r->stream));
-  r->launches += 1;
+  if (int rc = route(r, (const int32_t*)r->req_tok.p, n_tok, offsets[0], (const int64_t*)r->req_off.p, B, alpha,
+                     (int32_t*)r->out_match.p, (int32_t*)r->out_peer.p))
+    return rc;
   CK(cudaMemcpyAsync(out_match, r->out_match.p, (size_t)B * r->P * sizeof(int32_t), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaMemcpyAsync(out_peer, r->out_peer.p, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, r->stream));
   return do_sync(r);
