@@ -43,8 +43,6 @@ struct Slot {
   int len_s;        // tokens held in shared memory
   int shift;        // token j of the request sits at slot token shift + j (keeps bulk copies 16-byte aligned)
   int done;         // items of the request finished
-  int lead;         // follower pass: the request's group leader
-  int cpre;         // follower pass: its exact common prefix with the leader
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -152,7 +150,7 @@ __device__ __forceinline__ int32_t compare_tail(const int32_t* __restrict__ lab,
 // 128-byte-aligned position at or below j0 + 32 (re-comparing <= 31 tokens): a warp's 32 consecutive label
 // tokens are then one cache line, and its 32 request tokens in shared memory fall in 32 distinct banks at
 // any alignment, so each load is a single wavefront on both sides.
-template <bool kGlobal>
+template <int U, bool kGlobal>
 __device__ __forceinline__ int32_t compare_range(const int32_t* __restrict__ lab, const int32_t* req, int32_t j0,
                                                  int32_t end, int lane) {
   if (j0 + 32 <= end) {
@@ -160,8 +158,8 @@ __device__ __forceinline__ int32_t compare_range(const int32_t* __restrict__ lab
     if (k >= 0) return k;
     j0 += 32;
     j0 -= (int32_t)(((uintptr_t)(lab + j0) >> 2) & 31);
-    for (; j0 + kUnroll * 32 <= end; j0 += kUnroll * 32) {
-      const int32_t k2 = compare_full<kUnroll, kGlobal>(lab, req, j0, lane);
+    for (; j0 + U * 32 <= end; j0 += U * 32) {
+      const int32_t k2 = compare_full<U, kGlobal>(lab, req, j0, lane);
       if (k2 >= 0) return k2;
     }
   }
@@ -175,19 +173,21 @@ __device__ __forceinline__ int32_t compare_range(const int32_t* __restrict__ lab
 // First j in [from, lim) with lab[j] != request[pos + j], or lim; the tokens before `from` are known to
 // match (from >= 1: lab[0] == request[pos] is known).  Request tokens inside the shared-memory window (the
 // first n_s) come from it, later ones from global memory.
+template <int U>
 __device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ lab, const int32_t* s_req, int32_t n_s,
                                                   const int32_t* g_req, int32_t pos, int32_t lim, int32_t from,
                                                   int lane) {
   if (from >= lim) return lim;
   const int32_t split = max(from, min(lim, n_s - pos));
-  int32_t k = compare_range<false>(lab, s_req + pos, from, split, lane);
-  if (k < 0 && split < lim) k = compare_range<true>(lab, g_req + pos, split, lim, lane);
+  int32_t k = compare_range<U, false>(lab, s_req + pos, from, split, lane);
+  if (k < 0 && split < lim) k = compare_range<U, true>(lab, g_req + pos, split, lim, lane);
   return k < 0 ? lim : k;
 }
 
 // match(r, T) for one tree, computed by the whole warp (result uniform across lanes).  len is the request
 // length clamped to 2^31 - 1 (no match can be longer than a tree path).  The first `known` tokens are known
 // to be matched (known <= match(r, T)): the walk still follows their path but does not compare them.
+template <int U>
 __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t len,
                         int32_t known, int lane, int32_t* err) {
   if (len == 0) return 0;
@@ -201,8 +201,8 @@ __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, co
     }
     const int4 nn = __ldg(t.node + ce.y);  // the child's record, fetched while its label is compared
     const int32_t lim = min(ce.w, len - pos);
-    const int32_t k = first_mismatch(label_ptr(t.label, t.shared, ce.z), s_req, n_s, g_req, pos, lim,
-                                     max(1, known - pos), lane);
+    const int32_t k = first_mismatch<U>(label_ptr(t.label, t.shared, ce.z), s_req, n_s, g_req, pos, lim,
+                                        max(1, known - pos), lane);
     pos += k;
     if (k < ce.w || pos >= len || nn.z <= 0) break;
     if (!find_child(t.child + nn.x, tab_bits(nn.y), req_at(s_req, n_s, g_req, pos), lane, ce)) break;
@@ -221,17 +221,21 @@ __device__ __forceinline__ bool wait_for(const int* flag, int v, int lane) {
   return __shfl_sync(kFull, ok, 0) != 0;
 }
 
-// kFollow = false: routes requests list[0 .. *count) (every request b < B if list is NULL) with full walks.
-// kFollow = true: routes the followers list[0 .. *count) of a grouped batch, after the leaders' pass; a
-// follower's match in tree p is its leader's when that is below their common prefix c, else a walk that
-// skips comparing the first c tokens.  Followers are not staged: their walks compare only tokens past c.
-template <bool kFollow>
+// Packed route key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a better
+// route (higher score, then lower load, then lower index).  The host guarantees alpha * load <= 2^31 - 1,
+// load <= 65535 and P <= 65536, so every field fits.
+__device__ __forceinline__ unsigned long long route_key(int32_t m, int32_t ld, int32_t p, int32_t alpha) {
+  const long long score = (long long)m - (long long)alpha * ld;
+  return ((unsigned long long)(score + 2147483648LL) << 32) | ((unsigned long long)(0xFFFF - ld) << 16) |
+         (unsigned long long)(0xFFFF - p);
+}
+
+// Routes requests list[0 .. *count) (every request b < B if list is NULL) with full walks.
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ list,
-    const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
-    const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int32_t* err) {
+    const int32_t* __restrict__ count, const int32_t* __restrict__ load, int32_t alpha,
+    int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
   extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
   __shared__ unsigned long long s_next;
@@ -288,7 +292,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
       // shared addresses: the aligned middle of the request moves with one bulk copy, the <= 3 tokens on
       // each side with plain loads.
       const int32_t shift = (int32_t)(((uintptr_t)g >> 2) & 3);
-      const int32_t n_s = valid && !kFollow ? (int32_t)min(end - start, (int64_t)(kSlotTokens - shift)) : 0;
+      const int32_t n_s = valid ? (int32_t)min(end - start, (int64_t)(kSlotTokens - shift)) : 0;
       const int32_t j_lo = min((4 - shift) & 3, n_s);
       const int32_t j_hi = max(j_lo, n_s - (int32_t)(((uintptr_t)(g + n_s) >> 2) & 3));
       const uint32_t bytes = (uint32_t)(j_hi - j_lo) * 4u;
@@ -319,10 +323,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
         sl.shift = shift;
         sl.best = 0;
         sl.done = 0;
-        if (kFollow) {
-          sl.lead = __ldg(lead + b);
-          sl.cpre = __ldg(cpre + b);
-        }
         __threadfence_block();
         *(volatile int*)&sl.ready = (int)k;
       }
@@ -347,31 +347,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const int32_t* req = st + *(volatile int*)&sl.shift;
     const int32_t len32 = (int32_t)min(len, (int64_t)INT32_MAX);
     const int32_t p1 = min(P, (c + 1) * G);
-    int64_t lrow = 0;
-    int32_t cp = 0;
-    if (kFollow) {
-      lrow = (int64_t)*(volatile int*)&sl.lead * P;
-      cp = *(volatile int*)&sl.cpre;
-    }
     unsigned long long best = 0;
     for (int32_t p = c * G; p < p1; ++p) {
-      int32_t m;
-      if (kFollow) {
-        // The leader's match (its pass has finished) decides, or bounds, the follower's.
-        const int32_t ml = __ldg(out_match + lrow + p);
-        m = ml < cp ? ml : cp >= len32 ? len32 : walk(trees[p], req, 0, tokens + start, len32, cp, lane, err);
-      } else {
-        m = len > 0 ? walk(trees[p], req, n_s, tokens + start, len32, 0, lane, err) : 0;
-      }
+      const int32_t m = len > 0 ? walk<kUnroll>(trees[p], req, n_s, tokens + start, len32, 0, lane, err) : 0;
       if (lane == 0) {
         out_match[b * P + p] = m;
-        // Packed key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a
-        // better route (higher score, then lower load, then lower index).  The host guarantees
-        // alpha * load <= 2^31 - 1, load <= 65535 and P <= 65536, so every field fits.
-        const int32_t ld = __ldg(load + p);
-        const long long score = (long long)m - (long long)alpha * ld;
-        const unsigned long long key = ((unsigned long long)(score + 2147483648LL) << 32) |
-                                       ((unsigned long long)(0xFFFF - ld) << 16) | (unsigned long long)(0xFFFF - p);
+        const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
         best = key > best ? key : best;
       }
     }
@@ -395,6 +376,142 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
   }
 }
 
+// ---- Follower pass of a grouped batch -------------------------------------------------------------------
+//
+// A follower f with leader l and exact common prefix c: in tree p, match(f) = match(l) if match(l) < c, else
+// a walk that does not compare f's first c tokens.  Such a walk is short (a child lookup at each node on
+// the known part, then the compare past c), so each lane walks its own (follower, tree) pair: a warp keeps
+// 32 independent chains of dependent loads in flight.  A lane whose remaining compare is longer than
+// kThreadSpan tokens hands that pair to the whole warp (the cooperative walk above).
+
+constexpr int kFollowThreads = 256;
+constexpr int kFollowCtasPerSm = 4;
+constexpr int kThreadSpan = 64;
+
+// One thread: the child with first token tok in a table of 2^bits (>= 4, even) slots, two slots per step of
+// the linear probe.  Returns false if there is none.
+__device__ __forceinline__ bool find_child_1(const int4* __restrict__ tab, int32_t bits, int32_t tok, int4& out) {
+  if (bits == 0) return false;
+  const uint32_t mask = (1u << bits) - 1, h = slot_hash(tok, bits);
+  for (uint32_t i = 0; i <= mask; i += 2) {
+    const int4 a = __ldg(tab + ((h + i) & mask));
+    const int4 b = __ldg(tab + ((h + i + 1) & mask));
+    if (a.y >= 1 && a.x == tok) {
+      out = a;
+      return true;
+    }
+    if (a.y == 0) return false;
+    if (b.y >= 1 && b.x == tok) {
+      out = b;
+      return true;
+    }
+    if (b.y == 0) return false;
+  }
+  return false;
+}
+
+// One thread: first j in [from, lim) with lab[j] != req[j], or lim; 8 token pairs in flight per step.
+__device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab, const int32_t* __restrict__ req,
+                                                int32_t from, int32_t lim) {
+  for (int32_t j0 = from; j0 < lim; j0 += 8) {
+    int32_t x[8], y[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int32_t j = j0 + u;
+      x[u] = j < lim ? __ldg(lab + j) : 0;
+      y[u] = j < lim ? __ldg(req + j) : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (j0 + u < lim && x[u] != y[u]) return j0 + u;
+  }
+  return lim;
+}
+
+// One thread: match(r, T) with the first `known` tokens known to match (1 <= known < len).  state = 1 when
+// a compare longer than kThreadSpan remains (the result is then left to the warp), 2 on a corrupt entry.
+__device__ int32_t walk_1(const TreeView& t, const int32_t* __restrict__ req, int32_t len, int32_t known,
+                          int& state) {
+  state = 0;
+  int4 ce;
+  if (!find_child_1(t.child + t.root_off, t.root_bits, __ldg(req), ce)) return 0;
+  int32_t pos = 0;
+  for (;;) {  // pos grows by >= 1 per step (the child's first token matched), so at most len steps
+    if (ce.w <= 0 || ce.y <= 0) {
+      state = 2;
+      return pos;
+    }
+    const int4 nn = __ldg(t.node + ce.y);  // the child's record, fetched while the label is compared
+    const int32_t lim = min(ce.w, len - pos);
+    const int32_t from = max(1, known - pos);
+    int32_t k = lim;
+    if (from < lim) {
+      if (lim - from > kThreadSpan) {
+        state = 1;
+        return 0;
+      }
+      k = first_diff_1(label_ptr(t.label, t.shared, ce.z), req + pos, from, lim);
+    }
+    pos += k;
+    if (k < ce.w || pos >= len || nn.z <= 0) return pos;
+    if (!find_child_1(t.child + nn.x, tab_bits(nn.y), __ldg(req + pos), ce)) return pos;
+  }
+}
+
+// One warp per follower list[i], i < *count; lane j takes trees j, j + 32, ...
+__global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kernel(
+    const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
+    int64_t tok_base, const int64_t* __restrict__ offsets, const int32_t* __restrict__ list,
+    const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
+    const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
+    int32_t* err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
+  const int64_t n = *count;
+  for (int64_t i = ((int64_t)blockIdx.x * kFollowThreads + threadIdx.x) >> 5; i < n; i += warps) {
+    const int64_t f = __ldg(list + i);
+    const int64_t start = __ldg(offsets + f) - tok_base, end = __ldg(offsets + f + 1) - tok_base;
+    if (!(start >= 0 && start <= end && end <= n_tokens)) {  // cannot happen: only valid requests are grouped
+      if (lane == 0) {
+        out_peer[f] = -1;
+        atomicOr(err, ERR_BAD_OFFSETS);
+      }
+      continue;
+    }
+    const int32_t* req = tokens + start;
+    const int32_t len = (int32_t)min(end - start, (int64_t)INT32_MAX);
+    const int32_t c = __ldg(cpre + f);
+    const int64_t lrow = (int64_t)__ldg(lead + f) * P, frow = f * P;
+    unsigned long long best = 0;
+    for (int32_t p0 = 0; p0 < P; p0 += 32) {
+      const int32_t p = p0 + lane;
+      int32_t m = 0;
+      int state = 0;
+      if (p < P) {
+        const int32_t ml = out_match[lrow + p];  // the leaders' pass has finished
+        m = ml < c ? ml : c >= len ? len : walk_1(trees[p], req, len, c, state);
+      }
+      if (state == 2) atomicOr(err, ERR_CORRUPT_TREE);
+      for (unsigned need = __ballot_sync(kFull, state == 1); need; need &= need - 1) {
+        const int j = __ffs(need) - 1;
+        const int32_t mm = walk<4>(trees[p0 + j], req, 0, req, len, c, lane, err);
+        if (lane == j) m = mm;
+      }
+      if (p < P) {
+        out_match[frow + p] = m;
+        const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
+        best = key > best ? key : best;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(kFull, best, o);
+      best = other > best ? other : best;
+    }
+    if (lane == 0) out_peer[f] = 0xFFFF - (int32_t)(best & 0xFFFFull);
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
@@ -402,26 +519,20 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
   const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
-  cudaError_t e = cudaFuncSetAttribute(route_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e == cudaSuccess)
-    e = cudaFuncSetAttribute(route_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
   const int grid = (int)(B < max_ctas ? B : max_ctas);
-  if (!g) {
-    route_kernel<false><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, nullptr,
-                                                      nullptr, nullptr, nullptr, d_load, alpha, out_match, out_peer,
-                                                      d_err);
-    return cudaGetLastError();
-  }
-  route_kernel<false><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists,
-                                                    g->counts, nullptr, nullptr, d_load, alpha, out_match, out_peer,
-                                                    d_err);
+  route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B,
+                                             g ? g->lists : nullptr, g ? g->counts : nullptr, d_load, alpha, out_match,
+                                             out_peer, d_err);
   e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  route_kernel<true><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists + B,
-                                                   g->counts + 1, g->lead, g->cpre, d_load, alpha, out_match,
-                                                   out_peer, d_err);
+  if (e != cudaSuccess || !g) return e;
+  const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
+  const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
+  follow_kernel<<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
+                                                  g->counts + 1, g->lead, g->cpre, d_load, alpha, out_match, out_peer,
+                                                  d_err);
   return cudaGetLastError();
 }
 
