@@ -494,7 +494,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kerne
       if (state == 2) atomicOr(err, ERR_CORRUPT_TREE);
       for (unsigned need = __ballot_sync(kFull, state == 1); need; need &= need - 1) {
         const int j = __ffs(need) - 1;
-        const int32_t mm = walk<4>(trees[p0 + j], req, 0, req, len, c, lane, err);
+        const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err);
         if (lane == j) m = mm;
       }
       if (p < P) {
