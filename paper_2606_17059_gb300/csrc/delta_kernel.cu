@@ -196,11 +196,36 @@ __device__ int32_t only_child(const Tree& t, int32_t off, int32_t bits, int32_t 
   return -1;
 }
 
+// Warp copies: 4 loads per lane in flight before their stores (128 tokens per step).
 __device__ void copy_seq(int32_t* dst, const Seq& q, int64_t from, int64_t n, int lane) {
-  for (int64_t j = lane; j < n; j += 32) dst[j] = q.at(from + j);
+  for (int64_t j0 = 0; j0 < n; j0 += 128) {
+    int32_t x[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t j = j0 + u * 32 + lane;
+      x[u] = j < n ? q.at(from + j) : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t j = j0 + u * 32 + lane;
+      if (j < n) dst[j] = x[u];
+    }
+  }
 }
 __device__ void copy_tokens(int32_t* dst, const int32_t* src, int64_t n, int lane) {
-  for (int64_t j = lane; j < n; j += 32) dst[j] = src[j];
+  for (int64_t j0 = 0; j0 < n; j0 += 128) {
+    int32_t x[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t j = j0 + u * 32 + lane;
+      x[u] = j < n ? src[j] : 0;
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int64_t j = j0 + u * 32 + lane;
+      if (j < n) dst[j] = x[u];
+    }
+  }
 }
 
 // Label tokens are never overwritten once written (the label arena only grows) and the delta's pool is
@@ -675,6 +700,198 @@ __global__ void init_cursors_kernel(const TreeState* states, int64_t* cursors, i
   if (i < (int64_t)nt * kDeltaBuckets) cursors[i] = states[i / kDeltaBuckets].op_begin;
 }
 
+constexpr int kCompactThreads = 512;   // two CTAs per SM: every tree of a 256-tree router at once
+constexpr int kSmallBits = 4;   // tables of at most 16 slots are copied by one thread
+constexpr int kBigCap = 2048;   // big tables queued per level for the warps (more are copied by threads)
+
+// One thread copies n tokens, 8 loads in flight before their stores.
+__device__ __forceinline__ void copy_run(int32_t* __restrict__ dst, const int32_t* __restrict__ src, int32_t n) {
+  int32_t t = 0;
+  for (; t + 8 <= n; t += 8) {
+    int32_t x[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) x[u] = src[t + u];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) dst[t + u] = x[u];
+  }
+  for (; t < n; ++t) dst[t] = src[t];
+}
+
+struct CompactShared {
+  int node, child, label, tail, fail, nbig;
+  int big[kBigCap];
+};
+
+// Copies queued node q (old id, new id) and its table, one thread.
+__device__ void compact_node_thread(CompactJob& J, CompactShared& S, int2 q, const int4& rec) {
+  const int32_t bits = tab_bits(rec.y);
+  int32_t noff = 0, live = 0;
+  if (bits) {
+    const int32_t size = 1 << bits;
+    const uint32_t mask = (uint32_t)size - 1;
+    noff = atomicAdd(&S.child, size);
+    if ((int64_t)noff + size > J.cap_child) {
+      atomicOr(&S.fail, 1);
+      return;
+    }
+    for (int32_t j = 0; j < size; ++j) J.nchild[noff + j] = make_int4(0, 0, 0, 0);
+    for (int32_t j = 0; j < size; ++j) {
+      const int4 e = J.child[rec.x + j];
+      if (e.y < 1) continue;
+      const int32_t cid = atomicAdd(&S.node, 1);
+      int32_t nz = e.z;
+      if (e.z >= 0) nz = atomicAdd(&S.label, e.w);
+      if (cid >= J.cap_node || (e.z >= 0 && (int64_t)nz + e.w > J.cap_label)) {
+        atomicOr(&S.fail, 1);
+        return;
+      }
+      if (e.z >= 0) copy_run(J.nlabel + nz, J.label + e.z, e.w);
+      J.queue[atomicAdd(&S.tail, 1)] = make_int2(e.y, cid);
+      uint32_t sl = slot_hash(e.x, bits);
+      for (uint32_t it = 0; it < mask && J.nchild[noff + sl].y != 0; ++it) sl = (sl + 1) & mask;
+      J.nchild[noff + sl] = make_int4(e.x, cid, nz, e.w);
+      ++live;
+    }
+  }
+  J.nnode[q.y] = make_int4(noff, make_meta(bits, live), rec.z, rec.w);
+}
+
+// Copies queued node q and its (large) table, one warp: lane j takes slot base + j, and new ids, queue
+// entries and label offsets of the live slots come from one reservation per 32 slots (ranks and a prefix
+// sum of label lengths); entries go into the new table with a 64-bit compare-and-swap.
+__device__ void compact_node_warp(CompactJob& J, CompactShared& S, int2 q, const int4& rec, int lane) {
+  const int32_t bits = tab_bits(rec.y);
+  const int32_t size = 1 << bits;
+  const uint32_t mask = (uint32_t)size - 1;
+  int32_t noff = 0, live = 0;
+  if (lane == 0) {
+    noff = atomicAdd(&S.child, size);
+    if ((int64_t)noff + size > J.cap_child) atomicOr(&S.fail, 1);
+  }
+  noff = __shfl_sync(kFull, noff, 0);
+  if (__shfl_sync(kFull, *(volatile int*)&S.fail, 0)) return;  // one decision for the whole warp
+  for (int32_t j = lane; j < size; j += 32) J.nchild[noff + j] = make_int4(0, 0, 0, 0);
+  __syncwarp();
+  for (int32_t base = 0; base < size; base += 32) {
+    const int32_t j = base + lane;
+    const int4 e = j < size ? J.child[rec.x + j] : make_int4(0, 0, 0, 0);
+    const bool is_live = j < size && e.y >= 1;
+    const unsigned m = __ballot_sync(kFull, is_live);
+    if (!m) continue;
+    const int32_t cnt = __popc(m), rank = __popc(m & ((1u << lane) - 1));
+    const int32_t w = is_live && e.z >= 0 ? e.w : 0;
+    int32_t incl = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const int32_t total = __shfl_sync(kFull, incl, 31);
+    int32_t lbase = 0, nbase = 0, qbase = 0, bad = 0;
+    if (lane == 0) {
+      lbase = atomicAdd(&S.label, total);
+      nbase = atomicAdd(&S.node, cnt);
+      qbase = atomicAdd(&S.tail, cnt);
+      bad = (int64_t)lbase + total > J.cap_label || (int64_t)nbase + cnt > J.cap_node;
+      if (bad) atomicOr(&S.fail, 1);
+    }
+    if (__shfl_sync(kFull, bad, 0)) return;
+    lbase = __shfl_sync(kFull, lbase, 0);
+    nbase = __shfl_sync(kFull, nbase, 0);
+    qbase = __shfl_sync(kFull, qbase, 0);
+    // The 32 slots' own-arena labels as one run of `total` tokens: token i of the run belongs to the first
+    // lane whose inclusive prefix sum exceeds i (a binary search over the lanes, every lane taking part in
+    // the shuffles); lanes move 8 tokens each per step, loads before stores.
+    for (int32_t i0 = 0; i0 < total; i0 += 256) {
+      int32_t x[8], dst[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int32_t i = i0 + u * 32 + lane;
+        int lo = 0;
+#pragma unroll
+        for (int step = 16; step > 0; step >>= 1)
+          if (__shfl_sync(kFull, incl, lo + step - 1) <= i) lo += step;
+        const int32_t k_end = __shfl_sync(kFull, incl, lo & 31), k_w = __shfl_sync(kFull, w, lo & 31);
+        const int32_t k_src = __shfl_sync(kFull, e.z, lo & 31);
+        const bool ok = i < total;
+        x[u] = ok ? J.label[k_src + (i - (k_end - k_w))] : 0;
+        dst[u] = ok ? lbase + i : -1;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (dst[u] >= 0) J.nlabel[dst[u]] = x[u];
+    }
+    if (is_live) {
+      const int32_t cid = nbase + rank;
+      const int32_t nz = e.z >= 0 ? lbase + incl - w : e.z;
+      J.queue[qbase + rank] = make_int2(e.y, cid);
+      const unsigned long long kv = (unsigned long long)(uint32_t)e.x | ((unsigned long long)(uint32_t)cid << 32);
+      uint32_t sl = slot_hash(e.x, bits);
+      for (uint32_t it = 0; it <= mask; ++it, sl = (sl + 1) & mask) {
+        if (atomicCAS((unsigned long long*)&J.nchild[noff + sl], 0ull, kv) == 0ull) {
+          J.nchild[noff + sl].z = nz;
+          J.nchild[noff + sl].w = e.w;
+          break;
+        }
+      }
+    }
+    live += cnt;
+  }
+  __syncwarp();
+  if (lane == 0) J.nnode[q.y] = make_int4(noff, make_meta(bits, live), rec.z, rec.w);
+}
+
+// One CTA per tree: level-synchronous breadth-first copy from the root.  A thread takes each queued node;
+// nodes whose table has more than 2^kSmallBits slots are listed and then copied by whole warps.  Every node
+// is queued with a new id below cap_node (checked before the append), so the queue needs cap_node entries.
+__global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jobs) {
+  CompactJob& J = jobs[blockIdx.x];
+  __shared__ CompactShared S;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (threadIdx.x == 0) {
+    S.node = 1;
+    S.child = 0;
+    S.label = 0;
+    S.tail = 1;
+    S.fail = 0;
+    S.nbig = 0;
+    J.queue[0] = make_int2(0, 0);
+  }
+  __syncthreads();
+  int begin = 0, end = 1;
+  while (begin < end) {
+    for (int i = begin + threadIdx.x; i < end; i += kCompactThreads) {
+      const int2 q = J.queue[i];
+      const int4 rec = J.node[q.x];
+      if (tab_bits(rec.y) > kSmallBits) {
+        const int k = atomicAdd(&S.nbig, 1);
+        if (k < kBigCap) {
+          S.big[k] = i;
+          continue;
+        }
+      }
+      compact_node_thread(J, S, q, rec);
+    }
+    __syncthreads();
+    const int nbig = min(S.nbig, kBigCap);
+    for (int k = warp; k < nbig; k += kCompactThreads / 32) {
+      const int2 q = J.queue[S.big[k]];
+      compact_node_warp(J, S, q, J.node[q.x], lane);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) S.nbig = 0;
+    begin = end;
+    end = *(volatile int*)&S.fail ? end : *(volatile int*)&S.tail;
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    J.n_node = S.node;
+    J.n_child = S.child;
+    J.n_label = S.label;
+    J.status = S.fail;
+  }
+}
+
 __global__ void set_tree_kernel(TreeState* st, TreeView* view, TreeState v, const int32_t* shared) {
   *st = v;
   const int4 root = v.node[0];
@@ -695,6 +912,12 @@ cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, i
                                  cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   refresh_views_kernel<<<(n + 127) / 128, 128, 0, st>>>(d_states, d_views, n, shared);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, cudaStream_t st) {
+  if (n_jobs <= 0) return cudaSuccess;
+  compact_kernel<<<n_jobs, kCompactThreads, 0, st>>>(d_jobs);
   return cudaGetLastError();
 }
 

@@ -119,6 +119,24 @@ cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st);
 cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int32_t n_trees, cudaStream_t st);
 
+// Compaction: copies the live part of a tree (everything reachable from the root) into fresh arrays, with
+// nodes renumbered in breadth-first order, every live table rehashed at its size without tombstones, and
+// own-arena labels packed (shared-pool labels stay where they are).  One CTA per job.
+struct CompactJob {
+  const int4* node;  // old arrays
+  const int4* child;
+  const int32_t* label;
+  int4* nnode;  // new arrays and their capacities
+  int4* nchild;
+  int32_t* nlabel;
+  int2* queue;  // cap_node entries of scratch (a node is queued only with a new id below cap_node)
+  int32_t cap_node, cap_child, cap_label;
+  int32_t n_node, n_child, n_label;  // out: the new counts
+  int32_t status;                    // out: 0, or 1 if a new array was too small (the job is then void)
+  int32_t pad_;
+};
+cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, cudaStream_t st);
+
 // Home slot of a first token in a children table of 2^bits slots (host table builder and kernels).
 inline __host__ __device__ uint32_t slot_hash(int32_t tok, int32_t bits) {
   return bits ? ((uint32_t)tok * 0x9E3779B1u) >> (32 - bits) : 0u;

@@ -86,6 +86,7 @@ struct p2p_router {
   DevBuf req_tok, req_off, out_match, out_peer;
   DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_cursors, d_gather;
   DevBuf grp_keys, grp_vals, grp_req;  // shared-prefix grouping of a batch
+  DevBuf cmp_jobs, cmp_queue;          // device compaction
   int64_t launches = 0;  // kernels this router has launched
   // Shared label pool: long labels interned across trees (device array, host mirror, content index).
   int32_t* d_shared = nullptr;
@@ -498,6 +499,62 @@ int compact_tree(p2p_router* r, int32_t p) {
   return upload_flat(r, p, &v);
 }
 
+// Compacts trees ps on the device (compact_kernel): fresh arrays sized from the live counts with the same
+// headroom as an upload, one CTA per tree, then the states and views of [p0, p1) are republished.  A tree
+// whose fresh arrays turn out too small keeps its old arrays and is compacted through the host instead.
+int compact_trees(p2p_router* r, const std::vector<int32_t>& ps, int32_t p0, int32_t p1) {
+  if (ps.empty()) return P2P_OK;
+  const size_t n = ps.size();
+  std::vector<p2p::CompactJob> jobs(n);
+  std::vector<TreeState> fresh(n);
+  std::vector<int64_t> qoff(n);
+  int64_t qtotal = 0;
+  for (size_t i = 0; i < n; ++i) {
+    const TreeState& t = r->hs[(size_t)ps[i]];
+    const int64_t nodes = std::max<int64_t>((int64_t)t.n_node - t.dead_nodes, 1);
+    const int64_t slots = std::max<int64_t>((int64_t)t.n_child - t.stale_child, 0);
+    const int64_t own = std::max<int64_t>((int64_t)t.n_label - t.stale_label, 0);
+    cudaError_t e = alloc_tree_arrays(r, fresh[i], clamp_i32(2 * nodes + 1024), clamp_i32(2 * slots + 1024),
+                                      clamp_i32(own + std::max<int64_t>(own, 65536)));
+    if (e != cudaSuccess) {
+      for (size_t j = 0; j < i; ++j) free_tree_arrays(r, fresh[j]);
+      return fail(r, P2P_E_NOMEM, std::string("allocating a compacted tree: ") + cudaGetErrorString(e));
+    }
+    const TreeState& f = fresh[i];
+    jobs[i] = p2p::CompactJob{t.node, t.child, t.label, f.node, f.child, f.label, nullptr,
+                              f.cap_node, f.cap_child, f.cap_label, 0, 0, 0, 0, 0};
+    qoff[i] = qtotal;
+    qtotal += f.cap_node;
+  }
+  CK(ensure(r, r->cmp_queue, (size_t)qtotal * sizeof(int2)));
+  CK(ensure(r, r->cmp_jobs, n * sizeof(p2p::CompactJob)));
+  for (size_t i = 0; i < n; ++i) jobs[i].queue = static_cast<int2*>(r->cmp_queue.p) + qoff[i];
+  CK(cudaMemcpyAsync(r->cmp_jobs.p, jobs.data(), n * sizeof(p2p::CompactJob), cudaMemcpyHostToDevice, r->stream));
+  CK(p2p::launch_compact(static_cast<p2p::CompactJob*>(r->cmp_jobs.p), (int32_t)n, r->stream));
+  r->launches += 1;
+  CK(d2h(r, jobs.data(), r->cmp_jobs.p, n * sizeof(p2p::CompactJob)));
+  std::vector<int32_t> retry;
+  for (size_t i = 0; i < n; ++i) {
+    TreeState& t = r->hs[(size_t)ps[i]];
+    if (jobs[i].status != 0) {
+      free_tree_arrays(r, fresh[i]);
+      retry.push_back(ps[i]);
+      continue;
+    }
+    free_tree_arrays(r, t);
+    t = fresh[i];
+    t.n_node = jobs[i].n_node;
+    t.n_child = jobs[i].n_child;
+    t.n_label = jobs[i].n_label;
+  }
+  if (int rc = push_states(r, p0, p1)) return rc;
+  CK(p2p::launch_refresh_views(r->d_states + p0, r->d_views + p0, p1 - p0, r->d_shared, r->stream));
+  r->launches += 1;
+  for (int32_t p : retry)
+    if (int rc = compact_tree(r, p)) return rc;
+  return P2P_OK;
+}
+
 bool needs_compaction(const TreeState& t) {
   return (t.stale_label > 65536 && 2 * t.stale_label > t.n_label) ||
          (t.stale_child > 65536 && 2 * t.stale_child > t.n_child) ||
@@ -591,7 +648,7 @@ void p2p_router_destroy(p2p_router* r) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_cursors, &r->d_gather,
-                      &r->grp_keys, &r->grp_vals, &r->grp_req})
+                      &r->grp_keys, &r->grp_vals, &r->grp_req, &r->cmp_jobs, &r->cmp_queue})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -791,11 +848,13 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   CK(p2p::launch_refresh_views(r->d_states + p0, r->d_views + p0, nt, r->d_shared, r->stream));
   r->launches += 1;
   int64_t absent = 0;
+  std::vector<int32_t> stale;
   for (int32_t p = p0; p < p1; ++p) {
     const TreeState& t = r->hs[(size_t)p];
     absent += t.n_absent;
-    if (rc == P2P_OK && needs_compaction(t)) rc = compact_tree(r, p);
+    if (needs_compaction(t)) stale.push_back(p);
   }
+  if (rc == P2P_OK) rc = compact_trees(r, stale, p0, p1);
   if (n_absent) *n_absent = absent;
   return rc;
 }

@@ -202,3 +202,32 @@ def test_repeated_generator_deltas_and_compaction():
     assert_same_route(gm, gp, om, op, "after 30 rounds")
     st = r.stats(0)
     assert st["stale_label"] + st["stale_child"] <= st["label_tokens"] + st["child_entries"]
+
+
+def test_device_compaction_keeps_every_tree_canonical():
+    """Deletes of a third of each replica per round make stale own-arena labels pass half of the arena, so
+    apply_delta compacts the trees on the device (breadth-first copy, tables rehashed without tombstones).
+    After every round the downloads and the routes must equal the oracle's, and the stale counters of a
+    compacted tree start again from zero."""
+    prm = wl.preset(4)
+    prm.update(P=4, n_seq=4000, n_prefix=60, pre_lo=16, pre_hi=100, B=2000)
+    W = wl.Workload(params=prm, seed=5)
+    r = router_from_seqlists([W.tree(p) for p in range(W.P)])
+    trees = oracle.build_trees([W.tree(p) for p in range(W.P)])
+    compacted = 0
+    for step in range(4):
+        W.delta_make(step, 0.33, 0.05)
+        d = W.delta()
+        before = [r.stats(p)["stale_label"] for p in range(W.P)]
+        assert r.apply_delta(-1, d.op, d.seqs, d.peer_begin, on_device=step % 2 == 1) == 0
+        for p in range(W.P):
+            trees[p].apply_ops(d.op, d.seqs, int(d.peer_begin[p]), int(d.peer_begin[p + 1]))
+            st = r.stats(p)
+            if st["stale_label"] == 0 and st["stale_child"] == 0 and before[p] > 0:
+                compacted += 1
+            assert same_snapshot(r.download(p), trees[p].export()), (step, p)
+        tok, off = W.requests()
+        gm, gp = route_device(r, tok, off, W.load(), W.alpha)
+        om, op, _ = oracle.route(trees, tok, off, W.load(), W.alpha)
+        assert_same_route(gm, gp, om, op, f"round {step}")
+    assert compacted >= W.P
