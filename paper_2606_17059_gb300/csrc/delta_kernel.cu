@@ -6,30 +6,50 @@
 // that leaves an edge part-way splits it; a DELETE prunes a leaf that no longer stores anything and folds
 // a node left with one child and no sequence into that child.
 //
-// Parallel schedule.  Ops on sequences with different first tokens touch disjoint subtrees (the subtree
-// under the root child of that token) and, because every node's children live in a hash table with one
-// slot per first token, disjoint slots of the root's table.  So one CTA of kBuckets warps takes a tree; warp w applies,
-// in op order, exactly the ops whose first token hashes to bucket w.  Ops on the same sequence share a
-// bucket, so their relative order -- the only order that changes the result -- is kept.  The tree's op
-// list is scanned in chunks staged in shared memory; each warp walks a chunk's bucket ids with ballots.
-// Inside an op the warp cooperates: a child lookup probes 32 table slots at once, labels are compared 128
-// tokens per step and copied 32 per step; lane 0 performs scalar stores and __syncwarp() orders them before
-// later reads.  Adding or removing a child touches one slot (a table is doubled and rehashed when it
-// passes 3/4 occupancy), so the cost of an op does not grow with the fan-out of the nodes it passes.
+// Parallel schedule.  One CTA of kDeltaWarps warps takes a tree; the tree's ops are taken in chunks.
+// Two facts make ops independent:
+//   - ops on different sequences commute (the canonical tree depends only on the multiset), so only ops
+//     on the same sequence must keep their order;
+//   - two ops touch disjoint nodes when their paths part at some node and neither changes that node or
+//     anything above it.
+// Each chunk runs in two phases.
+//   Parallel phase.  A read-only pre-walk finds, for every op, the first node with at least kWide
+//   children on its path (its anchor, at most kAnchorDepth levels down).  Ops anchored at a node that
+//   qualifies -- its table already fits the chunk's inserts under it (grown first if not) and it keeps at
+//   least 3 children whatever the chunk's deletes under it do -- are bucketed by (anchor, next token) and
+//   the warps take these sub-buckets concurrently.  They change only the anchor's table (slots claimed by
+//   compare-and-swap, counters atomically) and the subtree of their own next token; nothing above the
+//   anchor changes in this phase.  An op whose real walk does not pass through its anchor (the pre-walk
+//   compares no labels) is deferred, untouched.
+//   Serial phase.  The remaining ops, deferred ones included, are bucketed by a hash of their first token
+//   (ops with different first tokens touch disjoint subtrees under the root and disjoint slots of the
+//   root's table) and the warps take these buckets, heaviest first.
+// Ops on the same sequence share an anchor and a next token, or a first token, so every bucket applies
+// them in op order.  Inside an op the warp cooperates: a child lookup probes 32 table slots at once, labels
+// are compared 128 tokens per step and copied 128 per step; lane 0 performs scalar stores and __syncwarp()
+// orders them before later reads.  Adding or removing a child touches one slot (a table is doubled and
+// rehashed when it passes 3/4 occupancy), so the cost of an op does not grow with the fan-out of the nodes
+// it passes.
 //
 // Space.  Node, child-entry and label arenas are bump-allocated with compare-and-swap on the tree's
-// counters; an op reserves everything it may need before it mutates anything.  If an arena is full the
-// warp stops at that op, records the op index in its bucket cursor and flags the tree; the host grows the
-// arenas and relaunches, and every bucket resumes at its cursor, so each op is applied whole or not at
-// all.  Every loop is bounded by a sequence length, a list size or an iteration cap.
+// counters; an op reserves everything it may need before it mutates anything.  If an arena is full the op
+// is left undone, its bucket stops (as do, for the rest of the launch, the first-token buckets of every op
+// it holds back, so no later op on the same sequence overtakes it) and the tree is flagged; the host grows
+// the arenas and relaunches.  A per-op done flag records what is applied, so every op is applied whole,
+// once.  Every loop is bounded by a sequence length, a list size or an iteration cap.
 #include "internal.h"
 
 namespace p2p {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 4096;  // ops whose bucket ids are staged in shared memory at a time
-enum { OP_DONE = 0, OP_NEED = 1, OP_CORRUPT = 2 };
+constexpr int kChunk = 2048;        // ops staged in shared memory at a time
+constexpr int kWide = 64;           // children that make a node an anchor of parallel sub-buckets
+constexpr int kAnchorDepth = 3;     // tree levels the pre-walk descends looking for an anchor
+constexpr int kAnchorSlots = 256;   // distinct anchors per chunk (ops beyond stay in the serial phase)
+constexpr int kSplitOps = 32;       // an anchor with this many ops in a chunk is split by next token
+enum { OP_DONE = 0, OP_NEED = 1, OP_CORRUPT = 2, OP_DEFER = 3 };
+enum { F_DONE = 1, F_ANCHORED = 2, F_DEFERRED = 4 };
 
 // Tokens [0, na) come from a, [na, n) from b (an op's sequence as at most two pool runs).
 struct Seq {
@@ -232,19 +252,32 @@ __device__ void copy_tokens(int32_t* dst, const int32_t* src, int64_t n, int lan
 // read-only, so "label[a .. a+n) == pool[b .. b+n)" stays true for the whole kernel once verified.  Each
 // warp remembers the last such run; ops that walk the same shared prefix as the previous op (the common
 // case: a delta references one pool copy of each shared prefix) skip re-comparing it.
+constexpr int kMemoSlots = 16;  // verified runs each warp remembers
+
+struct MemoEntry {
+  const int32_t* lab;
+  const int32_t* seq;
+  int64_t n;
+};
+// A warp's memo: kMemoSlots entries in shared memory, so that the shared prefixes of the several anchors a
+// warp serves all stay remembered.
 struct Memo {
-  const int32_t* lab = nullptr;
-  const int32_t* seq = nullptr;
-  int64_t n = 0;
+  MemoEntry* e;
 };
 
-// First j in [from, lim) with lab[j] != q[pos + j], or lim.
+// First j in [from, lim) with lab[j] != q[pos + j], or lim.  Lane k looks at memo entry k, so a lookup is
+// one step.
 __device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int64_t from, int64_t lim, int lane,
                               Memo& memo) {
   const bool in_a = pos < q.na;  // q[pos ..] starts in the first pool run, which the memo can describe
   if (in_a) {
-    const int64_t dl = lab - memo.lab, ds = (q.a + pos) - memo.seq;
-    if (memo.lab && dl == ds && dl >= 0 && dl < memo.n) from = max(from, min(lim, memo.n - dl));
+    int32_t skip = 0;
+    if (lane < kMemoSlots) {
+      const MemoEntry m = memo.e[lane];
+      const int64_t dl = lab - m.lab, ds = (q.a + pos) - m.seq;
+      if (m.lab && dl == ds && dl >= 0 && dl < m.n) skip = (int32_t)min(lim, m.n - dl);
+    }
+    from = max(from, (int64_t)__reduce_max_sync(kFull, (unsigned)skip));
   }
   int64_t k = lim;
   for (int64_t j0 = from; j0 < lim; j0 += 128) {
@@ -266,10 +299,12 @@ __device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int
     }
     if (hit) break;
   }
-  if (in_a && k >= 64) {  // remember a long verified run (within the first pool run)
-    memo.lab = lab;
-    memo.seq = q.a + pos;
-    memo.n = min(k, q.na - pos);
+  if (in_a && k >= 64) {  // remember a long verified run (within the first pool run), slot by label address
+    if (lane == 0) {
+      const uint32_t h = (uint32_t)(((uintptr_t)lab >> 2) * 0x9E3779B97F4A7C15ull >> 32) & (kMemoSlots - 1);
+      memo.e[h] = MemoEntry{lab, q.a + pos, min(k, q.na - pos)};
+    }
+    __syncwarp();
   }
   return k;
 }
@@ -310,13 +345,13 @@ __device__ void fold_child(Tree& t, int32_t x, int4* ex, int32_t yslot, int32_t 
   __syncwarp();
 }
 
-// Room for one more child in node cur's table (cur != 0): grows the table (doubling, rehash into fresh
-// slots) when claimed slots would pass 3/4.  Returns false if the child arena is full.
-__device__ bool ensure_slot(Tree& t, int32_t cur, int4& nd, int lane) {
+// Room for `extra` more children in node cur's table (cur != 0): grows the table (doubling, rehash into
+// fresh slots) when claimed slots would pass 3/4.  Returns false if the child arena is full.
+__device__ bool ensure_room(Tree& t, int32_t cur, int4& nd, int32_t extra, int lane) {
   const int32_t bits = tab_bits(nd.y), used = tab_used(nd.y);
-  if (!tab_full(bits, (int64_t)used + 1)) return true;
+  if (!tab_full(bits, (int64_t)used + extra)) return true;
   int32_t nb = bits ? bits + 1 : kMinTabBits;
-  while (nb < kMaxTabBits && (int64_t)(nd.z + 1) * 2 > ((int64_t)1 << nb)) ++nb;
+  while (nb < kMaxTabBits && ((int64_t)nd.z + extra) * 2 > ((int64_t)1 << nb)) ++nb;
   int32_t n0, c0, l0;
   if (!take(t, 0, (int64_t)1 << nb, 0, n0, c0, l0, lane)) return false;
   zero_slots(t, c0, 1 << nb, lane);
@@ -329,8 +364,10 @@ __device__ bool ensure_slot(Tree& t, int32_t cur, int4& nd, int lane) {
   return true;
 }
 
-// root: the root's node record as of the launch (its table moves only between launches).
-__device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& memo) {
+// root: the root's node record as of the launch (its table moves only between launches).  anchor: in the
+// parallel phase, the op's anchor node (else -1): the op changes nothing until its walk has passed through
+// the anchor (OP_DEFER otherwise), and claims in the anchor's table are counted atomically.
+__device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo) {
   const int64_t n = q.n;
   if (n == 0) {
     if (lane == 0) atomicAdd(&t.node[0].w, 1);
@@ -340,9 +377,11 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
   int32_t cur = 0;
   int64_t pos = 0;
   int32_t n0, c0, l0;
-  int4 nd = root;  // record of node cur: below the root only this warp writes it
+  int4 nd = root;  // record of node cur: below the root (and the anchor) only this warp writes it
+  bool passed = anchor < 0;
   for (int64_t guard = 0; guard <= n + 1; ++guard) {
     if (pos == n) {  // the sequence ends exactly at node cur (never the root here: n > 0)
+      if (!passed || cur == anchor) return OP_DEFER;
       if (lane == 0) t.node[cur].w += 1;
       __syncwarp();
       return OP_DONE;
@@ -353,9 +392,20 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
     int st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot, ce);
     if (st != 1) {
       // New leaf edge q[pos, n) under cur: revive tok's tombstone, or claim an empty slot.
+      if (!passed) return OP_DEFER;
       const int64_t L = n - pos;
       if (st == 0) {
-        if (cur == 0) {
+        if (cur == anchor) {
+          // The anchor's table is shared by the parallel phase's warps and was sized for the chunk's
+          // inserts under it: count the claim atomically; a table that would pass 3/4 defers the op.
+          int32_t meta = 0;
+          if (lane == 0) meta = atomicAdd(&t.node[cur].y, 1 << 5);
+          meta = __shfl_sync(kFull, meta, 0);
+          if (slot < 0 || tab_full(tab_bits(meta), (int64_t)tab_used(meta) + 1)) {
+            if (lane == 0) atomicSub(&t.node[cur].y, 1 << 5);
+            return OP_DEFER;
+          }
+        } else if (cur == 0) {
           // The root table is shared by all warps of the tree: count the claim atomically; if the table
           // would pass 3/4 the host grows it between launches.
           int32_t meta = 0;
@@ -370,7 +420,7 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
             return OP_NEED;
           }
         } else {
-          if (!ensure_slot(t, cur, nd, lane)) return OP_NEED;
+          if (!ensure_room(t, cur, nd, 1, lane)) return OP_NEED;
           st = probe(t, nd.x, tab_bits(nd.y), tok, lane, slot, ce);
           if (st != 0 || slot < 0) return OP_CORRUPT;
           if (lane == 0) t.node[cur].y = nd.y + (1 << 5);
@@ -398,10 +448,12 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
       cur = ce.y;
       pos += k;
       nd = nn;
+      passed = passed || cur == anchor;
       continue;
     }
     // The sequence leaves (or ends inside) the edge after k tokens: split it there.  The new node mid
     // gets a 4-slot table holding the lower part of the edge (and the new leaf).
+    if (!passed) return OP_DEFER;
     const bool tail = pos + k < n;
     const int64_t L = n - pos - k;
     if (!take(t, tail ? 2 : 1, 1 << kMinTabBits, tail ? L : 0, n0, c0, l0, lane)) return OP_NEED;
@@ -432,7 +484,9 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
   return OP_CORRUPT;
 }
 
-__device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& memo) {
+// anchor as for insert: nothing changes (OP_DEFER) unless the walk passed through it, and the anchor is
+// never folded here.
+__device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo) {
   const int64_t n = q.n;
   if (n == 0) {
     int ok = 0;
@@ -448,12 +502,14 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
   int32_t cur = 0, par = -1;
   int4 *e_cur = nullptr, *e_par = nullptr;
   int64_t pos = 0;
-  int4 nd = root, pn = root;  // records of cur and par (below the root only this warp writes them)
+  int4 nd = root, pn = root;  // records of cur and par (below the root and the anchor only this warp writes them)
+  bool passed = anchor < 0;
   for (int64_t guard = 0; pos < n; ++guard) {
     if (guard > n) return OP_CORRUPT;
     int32_t slot;
     int4 ce;
     if (probe(t, nd.x, tab_bits(nd.y), q.at(pos), lane, slot, ce) != 1) {
+      if (!passed) return OP_DEFER;
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
@@ -461,6 +517,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
     const int4 nn = t.node[ce.y];  // the child's record, fetched while the label is compared
     if (pos + ce.w > n || first_diff(t.lab(ce.z), q, pos, 1, ce.w, lane, memo) < ce.w) {
+      if (!passed) return OP_DEFER;
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
@@ -471,7 +528,9 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
     cur = ce.y;
     pos += ce.w;
     nd = nn;
+    passed = passed || cur == anchor;
   }
+  if (!passed || cur == anchor) return OP_DEFER;
   if (nd.w == 0) {
     add_stat(&t.g->n_absent, 1, lane);
     return OP_DONE;
@@ -494,6 +553,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
   // A leaf that stores nothing any more: tombstone its slot in the parent's table.  (pn is only read when
   // par is not the root.)
   const bool fold_parent = par != 0 && pn.w == 0 && pn.z == 2;
+  if (fold_parent && par == anchor) return OP_DEFER;  // (cannot happen: an anchor keeps >= 3 children)
   int32_t other = -1;
   if (fold_parent) {
     other = only_child(t, pn.x, tab_bits(pn.y), (int32_t)(e_cur - t.child), lane);
@@ -515,33 +575,133 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int lane, Memo& m
   return OP_DONE;
 }
 
-// Bucket (warp) of an op: a hash of the sequence's first token.
+// Bucket of an op in the serial phase: a hash of the sequence's first token.
 __device__ __forceinline__ int32_t bucket_of(int32_t tok) {
   return (int32_t)(((uint32_t)tok * 0x85EBCA6Bu) >> (32 - kDeltaBucketBits));
 }
+// Sub-bucket of an anchored op in the parallel phase: a hash of (anchor, next token) for an anchor with
+// many ops in the chunk, else of the anchor alone (one warp then serves all of that anchor's ops, and its
+// memo keeps their shared prefix).
+__device__ __forceinline__ int32_t sub_bucket_of(int32_t anchor, int32_t tok, bool split) {
+  const uint32_t h = ((uint32_t)anchor * 0x9E3779B1u) ^ (split ? (uint32_t)tok * 0x85EBCA6Bu : 0u);
+  return (int32_t)((h * 0xC2B2AE35u) >> (32 - kDeltaBucketBits));
+}
+
+// Token pos of an op's sequence given by pool runs [g0, g1) (one thread); -1 past the end.
+__device__ int32_t run_token(const int64_t* __restrict__ seg_off, const int32_t* __restrict__ seg_len,
+                             const int32_t* __restrict__ pool, int64_t g0, int64_t g1, int64_t pos) {
+  for (int64_t g = g0; g < g1; ++g) {
+    const int32_t l = seg_len[g];
+    if (pos < l) return pool[seg_off[g] + pos];
+    pos -= l;
+  }
+  return -1;
+}
+
+// Read-only pre-walk of one op (one thread, no label compares): the first node with at least kWide
+// children on the path that the sequence's tokens select, within kAnchorDepth levels, provided the sequence
+// continues past it; anchor = -1 if there is none.  next_tok is the sequence's token just past the anchor.
+__device__ void find_anchor(const Tree& t, const int4& root, const int64_t* __restrict__ seg_off,
+                            const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int64_t g0,
+                            int64_t g1, int64_t n, int32_t& anchor, int32_t& next_tok) {
+  anchor = -1;
+  next_tok = 0;
+  int4 nd = root;
+  int64_t pos = 0;
+  for (int depth = 0; depth < kAnchorDepth && pos < n; ++depth) {
+    const int32_t bits = tab_bits(nd.y);
+    if (bits == 0) return;
+    const int32_t tok = run_token(seg_off, seg_len, pool, g0, g1, pos);
+    const uint32_t mask = (1u << bits) - 1;
+    uint32_t sl = slot_hash(tok, bits);
+    int4 ce = make_int4(0, 0, 0, 0);
+    for (uint32_t it = 0; it <= mask; ++it, sl = (sl + 1) & mask) {
+      const int4 e = __ldcg(t.child + nd.x + sl);
+      if (e.y == 0) return;
+      if (e.y >= 1 && e.x == tok) {
+        ce = e;
+        break;
+      }
+    }
+    if (ce.y < 1 || ce.w <= 0) return;
+    pos += ce.w;
+    if (pos >= n) return;
+    const int4 cn = __ldcg(t.node + ce.y);
+    if (cn.z >= kWide) {
+      anchor = ce.y;
+      next_tok = run_token(seg_off, seg_len, pool, g0, g1, pos);
+      return;
+    }
+    nd = cn;
+  }
+}
+
+// Applies op i (one warp); anchor as for insert/remove.
+__device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcode, int64_t g0, int64_t g1,
+                        const int64_t* __restrict__ seg_off, const int32_t* __restrict__ seg_len,
+                        const int32_t* __restrict__ pool, int32_t* buf, int lane, Memo& memo) {
+  // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
+  Seq q;
+  if (g1 - g0 <= 2) {
+    q.a = pool + (g1 > g0 ? seg_off[g0] : 0);
+    q.na = g1 > g0 ? seg_len[g0] : 0;
+    q.b = g1 - g0 == 2 ? pool + seg_off[g0 + 1] : q.a;
+    q.n = q.na + (g1 - g0 == 2 ? seg_len[g0 + 1] : 0);
+  } else {
+    if (!buf) return OP_CORRUPT;  // the host gives gather scratch whenever an op has more than two runs
+    int64_t len = 0;
+    for (int64_t g = g0; g < g1; ++g) {
+      copy_tokens(buf + len, pool + seg_off[g], seg_len[g], lane);
+      len += seg_len[g];
+    }
+    __syncwarp();
+    q.a = q.b = buf;
+    q.na = q.n = len;
+  }
+  return opcode == P2P_OP_INSERT ? insert(t, q, root, anchor, lane, memo) : remove(t, q, root, anchor, lane, memo);
+}
+
+// Ranks kDeltaBuckets buckets by count (heaviest first, ties to the lower bucket) into order; one warp.
+__device__ void rank_buckets(const int* count, int* order, int lane) {
+  const int mine = count[lane];
+  int rank = 0;
+  for (int o = 0; o < kDeltaBuckets; ++o) {
+    const int other = count[o];
+    rank += other > mine || (other == mine && o < lane);
+  }
+  order[rank] = lane;
+}
 
 __global__ void __launch_bounds__(kDeltaWarps * 32, 3)
-    delta_kernel(TreeState* states, int64_t* cursors, const int32_t* __restrict__ op,
+    delta_kernel(TreeState* states, uint8_t* done, const int32_t* __restrict__ op,
                  const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
                  const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int32_t* gather,
                  int64_t stride, const int32_t* shared) {
-  __shared__ int8_t s_bucket[kChunk];
-  __shared__ int64_t s_run[kChunk + 1];   // seg_begin of the chunk's ops (and of the op after it)
-  __shared__ int s_count[kDeltaBuckets];  // ops of each bucket in the chunk
-  __shared__ int s_order[kDeltaBuckets];  // buckets, heaviest first
-  __shared__ int s_stopped[kDeltaBuckets];
+  __shared__ int64_t s_run[kChunk + 1];  // seg_begin of the chunk's ops (and of the op after them)
+  __shared__ int32_t s_anchor[kChunk];   // anchor of an anchored op
+  __shared__ int16_t s_aslot[kChunk];    // its entry in the anchor table
+  __shared__ int8_t s_bucket[kChunk];    // first-token bucket
+  __shared__ int32_t s_next[kChunk];     // an anchored op's token just past its anchor
+  __shared__ uint8_t s_flag[kChunk];     // F_* bits
+  __shared__ int s_akey[kAnchorSlots], s_ains[kAnchorSlots], s_adel[kAnchorSlots], s_aok[kAnchorSlots];
+  __shared__ int s_count[kDeltaBuckets];
+  __shared__ int s_order[kDeltaBuckets];
+  __shared__ int s_stop[kDeltaBuckets];  // first-token buckets held back for the rest of the launch
   __shared__ int s_take;
   __shared__ int s_any;
+  __shared__ MemoEntry s_memo[kDeltaWarps][kMemoSlots];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   TreeState* gs = states + blockIdx.x;
+  if (lane < kMemoSlots) s_memo[warp][lane] = MemoEntry{nullptr, nullptr, 0};
   const int64_t op_begin = gs->op_begin, op_end = gs->op_end;
-  int64_t* my_cursors = cursors + (int64_t)blockIdx.x * kDeltaBuckets;  // ops of a bucket before it are applied
   if (threadIdx.x == 0) s_any = 0;
+  if (threadIdx.x < kDeltaBuckets) s_stop[threadIdx.x] = 0;
   __syncthreads();
-  if (threadIdx.x < kDeltaBuckets) {
-    s_stopped[threadIdx.x] = 0;
-    if (my_cursors[threadIdx.x] < op_end) atomicOr(&s_any, 1);
-  }
+  for (int64_t i = op_begin + threadIdx.x; i < op_end; i += blockDim.x)
+    if (!done[i]) {
+      s_any = 1;
+      break;
+    }
   __syncthreads();
   if (!s_any || gs->status & DELTA_CORRUPT) return;
   Tree t;
@@ -552,37 +712,132 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 3)
   t.g = gs;
   const int4 root = t.node[0];  // its table offset and size hold for the whole launch
   int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaWarps + warp) * stride : nullptr;
-  Memo memo;  // facts about immutable labels: valid whichever bucket the warp works on
+  Memo memo{s_memo[warp]};  // facts about immutable labels: valid whichever bucket the warp works on
   for (int64_t c0 = op_begin; c0 < op_end; c0 += kChunk) {
-    const int64_t clen = min((int64_t)kChunk, op_end - c0);
+    const int clen = (int)min((int64_t)kChunk, op_end - c0);
+    // 1. Per op: first-token bucket, done flag, and (for ops still to apply) the anchor.
+    for (int k = threadIdx.x; k < kAnchorSlots; k += blockDim.x) {
+      s_akey[k] = -1;
+      s_ains[k] = 0;
+      s_adel[k] = 0;
+    }
+    if (threadIdx.x < kDeltaBuckets) s_count[threadIdx.x] = 0;
+    if (threadIdx.x == 0) {
+      s_run[clen] = seg_begin[c0 + clen];
+      s_take = 0;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < clen; j += blockDim.x) {
+      const int64_t i = c0 + j;
+      const int64_t g0 = seg_begin[i], g1 = seg_begin[i + 1];
+      s_run[j] = g0;
+      int32_t b = 0;  // empty sequences: bucket 0
+      int64_t n = 0;
+      for (int64_t g = g0; g < g1; ++g) {
+        if (n == 0 && seg_len[g] > 0) b = bucket_of(pool[seg_off[g]]);
+        n += seg_len[g];
+      }
+      s_bucket[j] = (int8_t)b;
+      uint8_t fl = done[i] ? F_DONE : 0;
+      if (!fl && !s_stop[b]) {
+        int32_t anchor, next_tok;
+        find_anchor(t, root, seg_off, seg_len, pool, g0, g1, n, anchor, next_tok);
+        if (anchor >= 0) {
+          uint32_t h = ((uint32_t)anchor * 2654435761u) >> 24;
+          int slot = -1;
+          for (int it = 0; it < kAnchorSlots; ++it, h = (h + 1) & (kAnchorSlots - 1)) {
+            const int prev = atomicCAS(&s_akey[h], -1, anchor);
+            if (prev == -1 || prev == anchor) {
+              slot = (int)h;
+              break;
+            }
+          }
+          if (slot >= 0) {
+            atomicAdd(op[i] == P2P_OP_INSERT ? &s_ains[slot] : &s_adel[slot], 1);
+            s_anchor[j] = anchor;
+            s_aslot[j] = (int16_t)slot;
+            s_next[j] = next_tok;
+            fl |= F_ANCHORED;
+          }
+        }
+      }
+      s_flag[j] = fl;
+    }
+    __syncthreads();
+    // 2. Anchors that qualify: at least 3 children whatever this chunk's deletes under them do, and a table
+    //    with room for this chunk's inserts under them (grown here if needed).  One warp per anchor.
+    for (int k = warp; k < kAnchorSlots; k += kDeltaWarps) {
+      const int key = s_akey[k];
+      if (key < 0) continue;
+      int4 rec = __ldcg(t.node + key);
+      bool ok = (int64_t)rec.z - s_adel[k] >= 3;
+      if (ok && s_ains[k] > 0) ok = ensure_room(t, key, rec, s_ains[k], lane);
+      if (lane == 0) s_aok[k] = ok;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < clen; j += blockDim.x) {
+      uint8_t fl = s_flag[j];
+      if ((fl & F_ANCHORED) && !s_aok[s_aslot[j]]) s_flag[j] = fl = (uint8_t)(fl & ~F_ANCHORED);
+      if (fl & F_ANCHORED) {
+        const int a = s_aslot[j];
+        const int32_t sb = sub_bucket_of(s_anchor[j], s_next[j], s_ains[a] + s_adel[a] >= kSplitOps);
+        s_next[j] = sb;  // from here on: the op's sub-bucket
+        atomicAdd(&s_count[sb], 1);
+      }
+    }
+    __syncthreads();
+    if (warp == 0) rank_buckets(s_count, s_order, lane);
+    __syncthreads();
+    // 3. Parallel phase: the warps take sub-buckets of anchored ops, heaviest first.
+    for (;;) {
+      int idx = 0;
+      if (lane == 0) idx = atomicAdd(&s_take, 1);
+      idx = __shfl_sync(kFull, idx, 0);
+      if (idx >= kDeltaBuckets) break;
+      const int sb = s_order[idx];
+      if (s_count[sb] == 0) continue;
+      bool stopped = false;
+      for (int j0 = 0; j0 < clen; j0 += 32) {
+        const int j = j0 + lane;
+        unsigned mine = __ballot_sync(kFull, j < clen && (s_flag[j] & (F_ANCHORED | F_DONE)) == F_ANCHORED &&
+                                                  s_next[j] == sb);
+        while (mine) {
+          const int jj = j0 + (__ffs(mine) - 1);
+          mine &= mine - 1;
+          if (stopped) {  // ops held back behind a stopped op: hold back their first-token buckets too
+            if (lane == 0) s_stop[s_bucket[jj]] = 1;
+            continue;
+          }
+          const int64_t i = c0 + jj;
+          const int r = apply_op(t, root, s_anchor[jj], op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool,
+                                 buf, lane, memo);
+          if (lane == 0) {
+            if (r == OP_DONE) {
+              done[i] = 1;
+              s_flag[jj] |= F_DONE;
+            } else if (r == OP_DEFER) {
+              s_flag[jj] |= F_DEFERRED;
+            } else {
+              s_stop[s_bucket[jj]] = 1;
+              if (r == OP_CORRUPT) atomicOr(&gs->status, DELTA_CORRUPT);
+            }
+          }
+          stopped = stopped || (r != OP_DONE && r != OP_DEFER);
+          __syncwarp();
+        }
+      }
+    }
+    __syncthreads();
+    // 4. Serial phase: the warps take first-token buckets of the other ops, heaviest first.
     if (threadIdx.x < kDeltaBuckets) s_count[threadIdx.x] = 0;
     if (threadIdx.x == 0) s_take = 0;
     __syncthreads();
-    if (threadIdx.x == 0) s_run[clen] = seg_begin[c0 + clen];
-    for (int64_t j = threadIdx.x; j < clen; j += blockDim.x) {
-      const int64_t i = c0 + j;
-      int32_t b = 0;  // empty sequences: bucket 0
-      const int64_t g0 = seg_begin[i];
-      s_run[j] = g0;
-      for (int64_t g = g0; g < seg_begin[i + 1]; ++g) {
-        if (seg_len[g] > 0) {
-          b = bucket_of(pool[seg_off[g]]);
-          break;
-        }
-      }
-      s_bucket[j] = (int8_t)b;
-      atomicAdd(&s_count[b], 1);
+    for (int j = threadIdx.x; j < clen; j += blockDim.x) {
+      const uint8_t fl = s_flag[j];
+      if (!(fl & F_DONE) && (!(fl & F_ANCHORED) || (fl & F_DEFERRED))) atomicAdd(&s_count[s_bucket[j]], 1);
     }
     __syncthreads();
-    if (warp == 0) {  // rank the buckets by op count (ties: lower bucket first)
-      const int mine = s_count[lane];
-      int rank = 0;
-      for (int o = 0; o < kDeltaBuckets; ++o) {
-        const int other = s_count[o];
-        rank += other > mine || (other == mine && o < lane);
-      }
-      s_order[rank] = lane;
-    }
+    if (warp == 0) rank_buckets(s_count, s_order, lane);
     __syncthreads();
     for (;;) {
       int idx = 0;
@@ -590,58 +845,38 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 3)
       idx = __shfl_sync(kFull, idx, 0);
       if (idx >= kDeltaBuckets) break;
       const int bk = s_order[idx];
-      if (s_count[bk] == 0 || s_stopped[bk]) continue;
-      int64_t next = my_cursors[bk];
-      if (next >= c0 + clen) continue;
+      if (s_count[bk] == 0 || *(volatile int*)&s_stop[bk]) continue;
       bool stopped = false;
-      for (int64_t j0 = max((int64_t)0, next - c0); j0 < clen && !stopped; j0 += 32) {
-        const int64_t j = j0 + lane;
-        unsigned mine = __ballot_sync(kFull, j < clen && s_bucket[j] == bk);
+      for (int j0 = 0; j0 < clen && !stopped; j0 += 32) {
+        const int j = j0 + lane;
+        bool mine_op = false;
+        if (j < clen) {
+          const uint8_t fl = s_flag[j];
+          mine_op = s_bucket[j] == bk && !(fl & F_DONE) && (!(fl & F_ANCHORED) || (fl & F_DEFERRED));
+        }
+        unsigned mine = __ballot_sync(kFull, mine_op);
         while (mine && !stopped) {
-          const int64_t jj = j0 + (__ffs(mine) - 1), i = c0 + jj;
+          const int jj = j0 + (__ffs(mine) - 1);
           mine &= mine - 1;
-          // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
-          const int64_t g0 = s_run[jj], g1 = s_run[jj + 1];
-          Seq q;
-          if (g1 - g0 <= 2) {
-            q.a = pool + (g1 > g0 ? seg_off[g0] : 0);
-            q.na = g1 > g0 ? seg_len[g0] : 0;
-            q.b = g1 - g0 == 2 ? pool + seg_off[g0 + 1] : q.a;
-            q.n = q.na + (g1 - g0 == 2 ? seg_len[g0 + 1] : 0);
-          } else {
-            if (!buf) {  // the host gives gather scratch whenever an op has more than two runs
-              if (lane == 0) atomicOr(&gs->status, DELTA_CORRUPT);
-              stopped = true;
-              next = i;
-              break;
+          const int64_t i = c0 + jj;
+          const int r = apply_op(t, root, -1, op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool, buf, lane,
+                                 memo);
+          if (lane == 0) {
+            if (r == OP_DONE) {
+              done[i] = 1;
+              s_flag[jj] |= F_DONE;
+            } else {
+              s_stop[bk] = 1;
+              if (r != OP_NEED) atomicOr(&gs->status, DELTA_CORRUPT);
             }
-            int64_t len = 0;
-            for (int64_t g = g0; g < g1; ++g) {
-              copy_tokens(buf + len, pool + seg_off[g], seg_len[g], lane);
-              len += seg_len[g];
-            }
-            __syncwarp();
-            q.a = q.b = buf;
-            q.na = q.n = len;
           }
-          const int r = op[i] == P2P_OP_INSERT ? insert(t, q, root, lane, memo) : remove(t, q, root, lane, memo);
-          if (r != OP_DONE) {
-            stopped = true;
-            next = i;
-            if (r == OP_CORRUPT && lane == 0) atomicOr(&gs->status, DELTA_CORRUPT);
-          }
+          stopped = r != OP_DONE;
+          __syncwarp();
         }
       }
-      if (lane == 0) {
-        my_cursors[bk] = stopped ? next : c0 + clen;
-        if (stopped) s_stopped[bk] = 1;
-      }
-      __syncwarp();
     }
     __syncthreads();
   }
-  // Buckets that never stopped have applied all their ops.
-  if (threadIdx.x < kDeltaBuckets && !s_stopped[threadIdx.x]) my_cursors[threadIdx.x] = op_end;
 }
 
 // Validates a device-resident delta into header (int32 words: [0..1] longest sequence as u64, [2] error
@@ -695,10 +930,6 @@ __global__ void init_ranges_kernel(TreeState* states, int32_t nt, const int64_t*
   states[i].n_absent = 0;
 }
 
-__global__ void init_cursors_kernel(const TreeState* states, int64_t* cursors, int32_t nt) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i < (int64_t)nt * kDeltaBuckets) cursors[i] = states[i / kDeltaBuckets].op_begin;
-}
 
 constexpr int kCompactThreads = 512;   // two CTAs per SM: every tree of a 256-tree router at once
 constexpr int kSmallBits = 4;   // tables of at most 16 slots are copied by one thread
@@ -921,18 +1152,11 @@ cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, cudaStream_t st) 
   return cudaGetLastError();
 }
 
-cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int32_t n_trees, cudaStream_t st) {
-  if (n_trees <= 0) return cudaSuccess;
-  const int64_t total = (int64_t)n_trees * kDeltaBuckets;
-  init_cursors_kernel<<<(int)((total + 255) / 256), 256, 0, st>>>(d_states, cursors, n_trees);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
+cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st) {
   if (n_trees <= 0) return cudaSuccess;
-  delta_kernel<<<n_trees, kDeltaWarps * 32, 0, st>>>(d_states, cursors, op, seg_begin, seg_off, seg_len, pool, gather,
+  delta_kernel<<<n_trees, kDeltaWarps * 32, 0, st>>>(d_states, done, op, seg_begin, seg_off, seg_len, pool, gather,
                                                      gather_stride, shared);
   return cudaGetLastError();
 }

@@ -111,13 +111,12 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          cudaStream_t st);
 
 // Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaWarps warps
-// per tree.  cursors[n_trees * kDeltaBuckets] holds each bucket's next op (set by launch_init_cursors,
-// kept across relaunches).  gather (n_trees * kDeltaWarps * gather_stride tokens) is needed only when an
-// op's sequence has more than two pool runs; otherwise it may be NULL.
-cudaError_t launch_delta(TreeState* d_states, int64_t* cursors, int32_t n_trees, const int32_t* op,
+// per tree.  done[i] (one byte per op of the call, zero before the first launch, kept across relaunches)
+// marks the ops applied so far.  gather (n_trees * kDeltaWarps * gather_stride tokens) is needed only when
+// an op's sequence has more than two pool runs; otherwise it may be NULL.
+cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st);
-cudaError_t launch_init_cursors(const TreeState* d_states, int64_t* cursors, int32_t n_trees, cudaStream_t st);
 
 // Compaction: copies the live part of a tree (everything reachable from the root) into fresh arrays, with
 // nodes renumbered in breadth-first order, every live table rehashed at its size without tombstones, and

@@ -84,7 +84,7 @@ struct p2p_router {
   int32_t* h_err = nullptr;       // pinned
   TreeState* h_states = nullptr;  // pinned, P entries
   DevBuf req_tok, req_off, out_match, out_peer;
-  DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_cursors, d_gather;
+  DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_done, d_gather;
   DevBuf grp_keys, grp_vals, grp_req;  // shared-prefix grouping of a batch
   DevBuf cmp_jobs, cmp_queue;          // device compaction
   int64_t launches = 0;  // kernels this router has launched
@@ -647,7 +647,7 @@ void p2p_router_destroy(p2p_router* r) {
   if (r->pool) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
-                      &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_cursors, &r->d_gather,
+                      &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
                       &r->grp_keys, &r->grp_vals, &r->grp_req, &r->cmp_jobs, &r->cmp_queue})
       dfree(r, b->p);
     dfree(r, r->d_views);
@@ -807,26 +807,26 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
     d_sl = (const int32_t*)r->d_seg_len.p;
     d_pool = (const int32_t*)r->d_pool.p;
   }
-  CK(ensure(r, r->d_cursors, (size_t)nt * p2p::kDeltaBuckets * sizeof(int64_t)));
+  CK(ensure(r, r->d_done, (size_t)std::max<int64_t>(n, 1)));
   int32_t* gather = nullptr;
   const int64_t stride = std::max<int64_t>(max_len, 1);
   if (max_runs > 2) {
     CK(ensure(r, r->d_gather, (size_t)nt * p2p::kDeltaWarps * stride * sizeof(int32_t)));
     gather = (int32_t*)r->d_gather.p;
   }
-  int64_t* cursors = (int64_t*)r->d_cursors.p;
-  // Device states = host mirror, then this call's op ranges and bucket cursors (set on the device).
+  uint8_t* done = (uint8_t*)r->d_done.p;
+  // Device states = host mirror, then this call's op ranges (set on the device) and cleared done flags.
   if (int rc = push_states(r, p0, p1)) return rc;
   CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d_pb : nullptr, n, r->stream));
-  CK(p2p::launch_init_cursors(r->d_states + p0, cursors, nt, r->stream));
-  r->launches += 2;
+  if (n) CK(cudaMemsetAsync(done, 0, (size_t)n, r->stream));
+  r->launches += 1;
   int rc = P2P_OK;
   for (int round = 0;; ++round) {
     if (round == 64) {
       rc = fail(r, P2P_E_NOMEM, "delta did not fit after 64 arena growths");
       break;
     }
-    CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->d_shared,
+    CK(p2p::launch_delta(r->d_states + p0, done, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->d_shared,
                          r->stream));
     r->launches += 1;
     if (int e = pull_states(r, p0, p1)) return e;
@@ -894,22 +894,22 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
   if (bits & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
   const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
   const int32_t nt = p1 - p0;
-  // Scratch: one int64 cursor per (tree, bucket); gathered sequences only when an op has > 2 pool runs.
-  const int64_t cursor_ints = (int64_t)nt * p2p::kDeltaBuckets * 2;
+  // Scratch: one done byte per op (in whole words); gathered sequences only when an op has > 2 pool runs.
+  const int64_t done_ints = (S.n + 3) / 4;
   const int64_t stride = max_len > 0 ? (int64_t)max_len : 1;
   const int64_t gather_ints = max_runs > 2 ? (int64_t)nt * p2p::kDeltaWarps * stride : 0;
-  if (cursor_ints + gather_ints > p2p::static_scratch_tokens())
-    return fail(r, P2P_E_INVAL, "the delta needs " + std::to_string(cursor_ints + gather_ints) +
+  if (done_ints + gather_ints > p2p::static_scratch_tokens())
+    return fail(r, P2P_E_INVAL, "the delta needs " + std::to_string(done_ints + gather_ints) +
                                     " words of scratch, more than the static scratch of " +
                                     std::to_string(p2p::static_scratch_tokens()) +
                                     " (exceeds the static scratch: split the delta or its sequences' runs)");
-  int64_t* cursors = reinterpret_cast<int64_t*>(tokens);
-  int32_t* gather = gather_ints ? tokens + cursor_ints : nullptr;
+  uint8_t* done = reinterpret_cast<uint8_t*>(tokens);
+  int32_t* gather = gather_ints ? tokens + done_ints : nullptr;
   CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d->peer_begin : nullptr, S.n, r->stream));
-  CK(p2p::launch_init_cursors(r->d_states + p0, cursors, nt, r->stream));
-  CK(p2p::launch_delta(r->d_states + p0, cursors, nt, d->op, S.seg_begin, S.seg_off, S.seg_len, S.pool, gather, stride,
+  if (S.n) CK(cudaMemsetAsync(done, 0, (size_t)S.n, r->stream));
+  CK(p2p::launch_delta(r->d_states + p0, done, nt, d->op, S.seg_begin, S.seg_off, S.seg_len, S.pool, gather, stride,
                        r->d_shared, r->stream));
-  r->launches += 3;
+  r->launches += 2;
   CK(cudaMemcpyAsync(r->h_states, r->d_states + p0, (size_t)nt * sizeof(TreeState), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaStreamSynchronize(r->stream));
   std::memcpy(r->hs.data() + p0, r->h_states, (size_t)nt * sizeof(TreeState));
