@@ -933,7 +933,8 @@ __global__ void init_ranges_kernel(TreeState* states, int32_t nt, const int64_t*
 
 constexpr int kCompactThreads = 512;   // two CTAs per SM: every tree of a 256-tree router at once
 constexpr int kSmallBits = 4;   // tables of at most 16 slots are copied by one thread
-constexpr int kBigCap = 2048;   // big tables queued per level for the warps (more are copied by threads)
+constexpr int kUnitSlots = 1024;  // slots of a big table per unit of warp work
+constexpr int kUnitCap = 2048;    // units queued per level (a table whose units do not fit is copied by a thread)
 
 // One thread copies n tokens, 8 loads in flight before their stores.
 __device__ __forceinline__ void copy_run(int32_t* __restrict__ dst, const int32_t* __restrict__ src, int32_t n) {
@@ -949,8 +950,8 @@ __device__ __forceinline__ void copy_run(int32_t* __restrict__ dst, const int32_
 }
 
 struct CompactShared {
-  int node, child, label, tail, fail, nbig;
-  int big[kBigCap];
+  int node, child, label, tail, fail, nunits;
+  int2 units[kUnitCap];  // (queue index, first slot) of kUnitSlots slots of a big table; queue index -1: none
 };
 
 // Copies queued node q (old id, new id) and its table, one thread.
@@ -987,26 +988,18 @@ __device__ void compact_node_thread(CompactJob& J, CompactShared& S, int2 q, con
   J.nnode[q.y] = make_int4(noff, make_meta(bits, live), rec.z, rec.w);
 }
 
-// Copies queued node q and its (large) table, one warp: lane j takes slot base + j, and new ids, queue
-// entries and label offsets of the live slots come from one reservation per 32 slots (ranks and a prefix
-// sum of label lengths); entries go into the new table with a 64-bit compare-and-swap.
-__device__ void compact_node_warp(CompactJob& J, CompactShared& S, int2 q, const int4& rec, int lane) {
+// Copies slots [start, end) of a big table (node q, old record rec) into its new table at noff, one warp:
+// lane j takes slot base + j, and new ids, queue entries and label offsets of the live slots come from one
+// reservation per 32 slots (ranks and a prefix sum of label lengths); entries go into the new table with a
+// 64-bit compare-and-swap, since other warps fill other ranges of the same table.
+__device__ void compact_range_warp(CompactJob& J, CompactShared& S, const int4& rec, int32_t noff, int32_t start,
+                                   int32_t end, int lane) {
   const int32_t bits = tab_bits(rec.y);
-  const int32_t size = 1 << bits;
-  const uint32_t mask = (uint32_t)size - 1;
-  int32_t noff = 0, live = 0;
-  if (lane == 0) {
-    noff = atomicAdd(&S.child, size);
-    if ((int64_t)noff + size > J.cap_child) atomicOr(&S.fail, 1);
-  }
-  noff = __shfl_sync(kFull, noff, 0);
-  if (__shfl_sync(kFull, *(volatile int*)&S.fail, 0)) return;  // one decision for the whole warp
-  for (int32_t j = lane; j < size; j += 32) J.nchild[noff + j] = make_int4(0, 0, 0, 0);
-  __syncwarp();
-  for (int32_t base = 0; base < size; base += 32) {
+  const uint32_t mask = (1u << bits) - 1;
+  for (int32_t base = start; base < end; base += 32) {
     const int32_t j = base + lane;
-    const int4 e = j < size ? J.child[rec.x + j] : make_int4(0, 0, 0, 0);
-    const bool is_live = j < size && e.y >= 1;
+    const int4 e = j < end ? J.child[rec.x + j] : make_int4(0, 0, 0, 0);
+    const bool is_live = j < end && e.y >= 1;
     const unsigned m = __ballot_sync(kFull, is_live);
     if (!m) continue;
     const int32_t cnt = __popc(m), rank = __popc(m & ((1u << lane) - 1));
@@ -1066,26 +1059,27 @@ __device__ void compact_node_warp(CompactJob& J, CompactShared& S, int2 q, const
         }
       }
     }
-    live += cnt;
   }
-  __syncwarp();
-  if (lane == 0) J.nnode[q.y] = make_int4(noff, make_meta(bits, live), rec.z, rec.w);
 }
 
-// One CTA per tree: level-synchronous breadth-first copy from the root.  A thread takes each queued node;
-// nodes whose table has more than 2^kSmallBits slots are listed and then copied by whole warps.  Every node
-// is queued with a new id below cap_node (checked before the append), so the queue needs cap_node entries.
+// One CTA per tree: level-synchronous breadth-first copy from the root.  A thread takes each queued node.
+// A node whose table has more than 2^kSmallBits slots gets its new table range and record from that
+// thread, and its slots are cut into units of kUnitSlots that all warps then zero and fill; smaller tables
+// are copied by the thread.  Every node is queued with a new id below cap_node (checked before the
+// append), so the queue needs cap_node entries.  A big table's record counts its children from the old
+// record (the live-child count), so no pass has to count them.
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jobs) {
   CompactJob& J = jobs[blockIdx.x];
   __shared__ CompactShared S;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kWarps = kCompactThreads / 32;
   if (threadIdx.x == 0) {
     S.node = 1;
     S.child = 0;
     S.label = 0;
     S.tail = 1;
     S.fail = 0;
-    S.nbig = 0;
+    S.nunits = 0;
     J.queue[0] = make_int2(0, 0);
   }
   __syncthreads();
@@ -1094,23 +1088,45 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jo
     for (int i = begin + threadIdx.x; i < end; i += kCompactThreads) {
       const int2 q = J.queue[i];
       const int4 rec = J.node[q.x];
-      if (tab_bits(rec.y) > kSmallBits) {
-        const int k = atomicAdd(&S.nbig, 1);
-        if (k < kBigCap) {
-          S.big[k] = i;
+      const int32_t bits = tab_bits(rec.y);
+      if (bits > kSmallBits) {
+        const int32_t size = 1 << bits, nu = (size + kUnitSlots - 1) / kUnitSlots;
+        const int u0 = atomicAdd(&S.nunits, nu);
+        if (u0 + nu <= kUnitCap) {
+          const int32_t noff = atomicAdd(&S.child, size);
+          if ((int64_t)noff + size > J.cap_child) {
+            atomicOr(&S.fail, 1);
+            for (int k = 0; k < nu; ++k) S.units[u0 + k] = make_int2(-1, 0);
+            continue;
+          }
+          J.nnode[q.y] = make_int4(noff, make_meta(bits, rec.z), rec.z, rec.w);
+          for (int k = 0; k < nu; ++k) S.units[u0 + k] = make_int2(i, k * kUnitSlots);
           continue;
         }
+        for (int k = u0; k < kUnitCap; ++k) S.units[k] = make_int2(-1, 0);  // no room: this thread copies it
       }
       compact_node_thread(J, S, q, rec);
     }
     __syncthreads();
-    const int nbig = min(S.nbig, kBigCap);
-    for (int k = warp; k < nbig; k += kCompactThreads / 32) {
-      const int2 q = J.queue[S.big[k]];
-      compact_node_warp(J, S, q, J.node[q.x], lane);
+    const int nunits = min(S.nunits, kUnitCap);
+    for (int k = warp; k < nunits; k += kWarps) {  // zero every unit's slots first: inserts may wrap into them
+      const int2 u = S.units[k];
+      if (u.x < 0) continue;
+      const int4 nrec = J.nnode[J.queue[u.x].y];
+      const int32_t n = min(kUnitSlots, (1 << tab_bits(nrec.y)) - u.y);
+      for (int32_t j = lane; j < n; j += 32) J.nchild[nrec.x + u.y + j] = make_int4(0, 0, 0, 0);
     }
     __syncthreads();
-    if (threadIdx.x == 0) S.nbig = 0;
+    for (int k = warp; k < nunits; k += kWarps) {
+      const int2 u = S.units[k];
+      if (u.x < 0 || __shfl_sync(kFull, *(volatile int*)&S.fail, 0)) continue;
+      const int2 q = J.queue[u.x];
+      const int4 rec = J.node[q.x];
+      const int32_t noff = J.nnode[q.y].x;
+      compact_range_warp(J, S, rec, noff, u.y, min(u.y + kUnitSlots, 1 << tab_bits(rec.y)), lane);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) S.nunits = 0;
     begin = end;
     end = *(volatile int*)&S.fail ? end : *(volatile int*)&S.tail;
     __syncthreads();

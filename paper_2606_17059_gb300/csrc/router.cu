@@ -25,6 +25,11 @@ struct DevBuf {
 
 int32_t clamp_i32(int64_t v) { return (int32_t)std::min<int64_t>(v, INT32_MAX); }
 
+// Capacity of a tree's own label arena holding `own` live tokens.  Deltas leave replaced labels behind as
+// stale space, and a tree is compacted once that passes its live space; twice the live tokens plus a
+// quarter is enough to get there without growing the arena on the way.
+int32_t label_cap(int64_t own) { return clamp_i32(2 * own + std::max<int64_t>(own / 4, 65536)); }
+
 int64_t next_pow2(int64_t v) {
   int64_t p = 1;
   while (p < v) p <<= 1;
@@ -362,7 +367,7 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   // Headroom for device deltas (no regrowth for a few anti-entropy rounds of a few percent each).
   const int32_t cap_node = clamp_i32(2 * N + 1024);
   const int32_t cap_child = clamp_i32(2 * slots + 1024);
-  const int32_t cap_label = clamp_i32(n_own + std::max<int64_t>(NL / 2, 4096));
+  const int32_t cap_label = std::max(label_cap(n_own), clamp_i32(n_own + NL / 2));
   TreeState nt;
   cudaError_t e = alloc_tree_arrays(r, nt, cap_node, cap_child, cap_label);
   if (e != cudaSuccess) return fail(r, P2P_E_NOMEM, std::string("allocating the tree: ") + cudaGetErrorString(e));
@@ -515,7 +520,7 @@ int compact_trees(p2p_router* r, const std::vector<int32_t>& ps, int32_t p0, int
     const int64_t slots = std::max<int64_t>((int64_t)t.n_child - t.stale_child, 0);
     const int64_t own = std::max<int64_t>((int64_t)t.n_label - t.stale_label, 0);
     cudaError_t e = alloc_tree_arrays(r, fresh[i], clamp_i32(2 * nodes + 1024), clamp_i32(2 * slots + 1024),
-                                      clamp_i32(own + std::max<int64_t>(own, 65536)));
+                                      label_cap(own));
     if (e != cudaSuccess) {
       for (size_t j = 0; j < i; ++j) free_tree_arrays(r, fresh[j]);
       return fail(r, P2P_E_NOMEM, std::string("allocating a compacted tree: ") + cudaGetErrorString(e));
@@ -815,6 +820,11 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
     gather = (int32_t*)r->d_gather.p;
   }
   uint8_t* done = (uint8_t*)r->d_done.p;
+  std::vector<int4> before((size_t)nt);  // arena use at the start of the call
+  for (int32_t p = p0; p < p1; ++p) {
+    const TreeState& t = r->hs[(size_t)p];
+    before[(size_t)(p - p0)] = make_int4(t.n_node, t.n_child, t.n_label, 0);
+  }
   // Device states = host mirror, then this call's op ranges (set on the device) and cleared done flags.
   if (int rc = push_states(r, p0, p1)) return rc;
   CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d_pb : nullptr, n, r->stream));
@@ -842,6 +852,24 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
     }
     if (rc != P2P_OK || !again) break;
     if (int e = push_states(r, p0, p1)) return e;
+  }
+  // Room ahead of the next call: a tree (not about to be compacted) whose free room in an arena is below
+  // twice what this call used there is grown now, so the next call's kernel does not stop for room.
+  for (int32_t p = p0; p < p1 && rc == P2P_OK; ++p) {
+    TreeState& t = r->hs[(size_t)p];
+    if (needs_compaction(t)) continue;
+    const int4 b = before[(size_t)(p - p0)];
+    const int64_t dn = 2 * std::max<int64_t>((int64_t)t.n_node - b.x, 0);
+    const int64_t dc = 2 * std::max<int64_t>((int64_t)t.n_child - b.y, 0);
+    const int64_t dl = 2 * std::max<int64_t>((int64_t)t.n_label - b.z, 0);
+    const bool short_n = (int64_t)t.cap_node - t.n_node < dn, short_c = (int64_t)t.cap_child - t.n_child < dc,
+               short_l = (int64_t)t.cap_label - t.n_label < dl;
+    if (!short_n && !short_c && !short_l) continue;
+    t.need_node = short_n ? clamp_i32(dn) : 0;
+    t.need_child = short_c ? clamp_i32(dc) : 0;
+    t.need_label = short_l ? clamp_i32(dl) : 0;
+    t.need_root = 0;
+    rc = grow_tree(r, p);
   }
   // Publish the (possibly moved) arrays to the route kernel's view table; compact very stale trees.
   if (int e = push_states(r, p0, p1)) return e;
