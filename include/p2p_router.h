@@ -180,7 +180,7 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
  * array of the library (8 MiB plus a 256-byte header, held by every GPU that loads the library until the
  * process exits); trees are never grown or compacted.
  * Limits: the scratch holds one byte per op of the delta (rounded up to whole 4-byte words), plus, only
- * when some op's sequence is split into more than two pool runs, 32 bytes x (longest sequence in tokens)
+ * when some op's sequence is split into more than two pool runs, 64 bytes x (longest sequence in tokens)
  * per tree the call touches; a delta that needs more gets P2P_E_INVAL.  If a tree's arenas run out of room, the call returns P2P_E_NOMEM and that
  * tree holds only part of its ops (each op applied whole or not at all); p2p_tree_apply_delta, which may
  * allocate, grows trees.

@@ -43,7 +43,7 @@ namespace p2p {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 2048;        // ops staged in shared memory at a time
+constexpr int kChunk = 1536;        // ops staged in shared memory at a time
 constexpr int kWide = 64;           // children that make a node an anchor of parallel sub-buckets
 constexpr int kAnchorDepth = 3;     // tree levels the pre-walk descends looking for an anchor
 constexpr int kAnchorSlots = 256;   // distinct anchors per chunk (ops beyond stay in the serial phase)
@@ -672,7 +672,7 @@ __device__ void rank_buckets(const int* count, int* order, int lane) {
   order[rank] = lane;
 }
 
-__global__ void __launch_bounds__(kDeltaWarps * 32, 3)
+__global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     delta_kernel(TreeState* states, uint8_t* done, const int32_t* __restrict__ op,
                  const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
                  const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int32_t* gather,

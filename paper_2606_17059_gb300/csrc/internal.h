@@ -71,7 +71,7 @@ enum { DELTA_OK = 0, DELTA_NEED_SPACE = 1, DELTA_CORRUPT = 2 };
 // kDeltaWarps warps per tree takes the buckets heaviest first.
 constexpr int kDeltaBucketBits = 5;
 constexpr int kDeltaBuckets = 1 << kDeltaBucketBits;
-constexpr int kDeltaWarps = 8;
+constexpr int kDeltaWarps = 16;
 
 // Children tables: at least 4 slots; grown (doubled) when claimed slots would pass 3/4 of the table.
 constexpr int kMinTabBits = 2;
