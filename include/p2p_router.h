@@ -209,9 +209,12 @@ int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]);
 int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
                     const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
 
-/* As p2p_route_batch with every pointer in HOST memory (pinned memory makes the copies faster):
- * copies the requests to the device, routes, copies both outputs back and waits.  Offsets are
- * validated on the host (P2P_E_INVAL).  Requests are tokens[offsets[0] .. offsets[B]). */
+/* As p2p_route_batch with every pointer in HOST memory: copies the requests to the device, routes,
+ * copies both outputs back and waits.  Large batches go in up to 8 chunks of at least 131,072 requests:
+ * a chunk's inputs are copied in while the chunk before it is routed and the one before that is copied
+ * out (two copy streams of the router, ordered by events against the router stream).  Results equal
+ * those of one p2p_route_batch of the whole batch.  The copies overlap only from pinned host memory.
+ * Offsets are validated on the host (P2P_E_INVAL).  Requests are tokens[offsets[0] .. offsets[B]). */
 int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* offsets, int64_t B,
                          const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
 

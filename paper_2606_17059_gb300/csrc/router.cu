@@ -17,6 +17,10 @@ using p2p::TreeView;
 namespace {
 
 constexpr int kLoadRing = 8;
+// p2p_route_batch_host pipelines its copies with the routing in up to kPipe chunks of at least
+// kPipeRequests requests each.
+constexpr int kPipe = 8;
+constexpr int64_t kPipeRequests = 131072;
 
 struct DevBuf {
   void* p = nullptr;
@@ -85,6 +89,9 @@ struct p2p_router {
   int32_t* d_hdr = nullptr;  // validation result of device-resident deltas
   int32_t* h_load = nullptr;  // pinned, kLoadRing slots of P values
   cudaEvent_t load_ev[kLoadRing] = {};
+  // Copy streams of p2p_route_batch_host (inputs in, results out) and the events that order them.
+  cudaStream_t cp_in = nullptr, cp_out = nullptr;
+  cudaEvent_t ev_start = nullptr, ev_done = nullptr, ev_in[kPipe] = {}, ev_routed[kPipe] = {};
   int load_slot = 0;
   int32_t* h_err = nullptr;       // pinned
   TreeState* h_states = nullptr;  // pinned, P entries
@@ -627,6 +634,14 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_err, sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_states, (size_t)P * sizeof(TreeState));
   for (int i = 0; i < kLoadRing && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&r->load_ev[i], cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&r->cp_in, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&r->cp_out, cudaStreamNonBlocking);
+  for (cudaEvent_t* ev : {&r->ev_start, &r->ev_done})
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
+  for (int i = 0; i < kPipe && e == cudaSuccess; ++i) {
+    e = cudaEventCreateWithFlags(&r->ev_in[i], cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&r->ev_routed[i], cudaEventDisableTiming);
+  }
   if (e == cudaSuccess) e = cudaMemsetAsync(r->d_err, 0, sizeof(int32_t), r->stream);
   if (e != cudaSuccess) {
     fail(r, P2P_E_NOMEM, std::string("allocating router state: ") + cudaGetErrorString(e));
@@ -666,6 +681,17 @@ void p2p_router_destroy(p2p_router* r) {
   }
   for (cudaEvent_t ev : r->load_ev)
     if (ev) cudaEventDestroy(ev);
+  for (cudaStream_t s : {r->cp_in, r->cp_out})
+    if (s) {
+      cudaStreamSynchronize(s);
+      cudaStreamDestroy(s);
+    }
+  for (cudaEvent_t ev : {r->ev_start, r->ev_done})
+    if (ev) cudaEventDestroy(ev);
+  for (int i = 0; i < kPipe; ++i) {
+    if (r->ev_in[i]) cudaEventDestroy(r->ev_in[i]);
+    if (r->ev_routed[i]) cudaEventDestroy(r->ev_routed[i]);
+  }
   if (r->h_load) cudaFreeHost(r->h_load);
   if (r->h_err) cudaFreeHost(r->h_err);
   if (r->h_states) cudaFreeHost(r->h_states);
@@ -986,14 +1012,40 @@ int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* of
   CK(ensure(r, r->req_off, (size_t)(B + 1) * sizeof(int64_t)));
   CK(ensure(r, r->out_match, (size_t)B * r->P * sizeof(int32_t)));
   CK(ensure(r, r->out_peer, (size_t)B * sizeof(int32_t)));
-  if (n_tok) CK(cudaMemcpyAsync(r->req_tok.p, tokens + offsets[0], (size_t)n_tok * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
-  CK(cudaMemcpyAsync(r->req_off.p, offsets, (size_t)(B + 1) * sizeof(int64_t), cudaMemcpyHostToDevice, r->stream));
   if (int rc = stage_load(r, load)) return rc;
-  if (int rc = route(r, (const int32_t*)r->req_tok.p, n_tok, offsets[0], (const int64_t*)r->req_off.p, B, alpha,
-                     (int32_t*)r->out_match.p, (int32_t*)r->out_peer.p))
-    return rc;
-  CK(cudaMemcpyAsync(out_match, r->out_match.p, (size_t)B * r->P * sizeof(int32_t), cudaMemcpyDeviceToHost, r->stream));
-  CK(cudaMemcpyAsync(out_peer, r->out_peer.p, (size_t)B * sizeof(int32_t), cudaMemcpyDeviceToHost, r->stream));
+  // The batch goes in chunks: chunk k's inputs are copied in on cp_in while chunk k-1 is routed on the
+  // router stream and chunk k-2's results are copied out on cp_out.  Each chunk is grouped and routed on
+  // its own (groups never span chunks), which gives the same results as one pass.
+  const int K = (int)std::min<int64_t>(kPipe, std::max<int64_t>(1, B / kPipeRequests));
+  const int64_t Bc = (B + K - 1) / K;
+  int32_t* d_tok = static_cast<int32_t*>(r->req_tok.p);
+  int64_t* d_off = static_cast<int64_t*>(r->req_off.p);
+  int32_t* d_match = static_cast<int32_t*>(r->out_match.p);
+  int32_t* d_peer = static_cast<int32_t*>(r->out_peer.p);
+  CK(cudaEventRecord(r->ev_start, r->stream));  // the buffers are ready (allocated, no longer in use)
+  CK(cudaStreamWaitEvent(r->cp_in, r->ev_start, 0));
+  CK(cudaStreamWaitEvent(r->cp_out, r->ev_start, 0));
+  for (int k = 0; k < K; ++k) {
+    const int64_t b0 = k * Bc, b1 = std::min(B, b0 + Bc);
+    if (b0 >= b1) break;
+    const int64_t t0 = offsets[b0] - offsets[0], t1 = offsets[b1] - offsets[0];
+    if (t1 > t0)
+      CK(cudaMemcpyAsync(d_tok + t0, tokens + offsets[b0], (size_t)(t1 - t0) * sizeof(int32_t), cudaMemcpyHostToDevice,
+                         r->cp_in));
+    CK(cudaMemcpyAsync(d_off + b0, offsets + b0, (size_t)(b1 - b0 + 1) * sizeof(int64_t), cudaMemcpyHostToDevice,
+                       r->cp_in));
+    CK(cudaEventRecord(r->ev_in[k], r->cp_in));
+    CK(cudaStreamWaitEvent(r->stream, r->ev_in[k], 0));
+    if (int rc = route(r, d_tok + t0, t1 - t0, offsets[b0], d_off + b0, b1 - b0, alpha, d_match + b0 * r->P, d_peer + b0))
+      return rc;
+    CK(cudaEventRecord(r->ev_routed[k], r->stream));
+    CK(cudaStreamWaitEvent(r->cp_out, r->ev_routed[k], 0));
+    CK(cudaMemcpyAsync(out_match + b0 * r->P, d_match + b0 * r->P, (size_t)(b1 - b0) * r->P * sizeof(int32_t),
+                       cudaMemcpyDeviceToHost, r->cp_out));
+    CK(cudaMemcpyAsync(out_peer + b0, d_peer + b0, (size_t)(b1 - b0) * sizeof(int32_t), cudaMemcpyDeviceToHost, r->cp_out));
+  }
+  CK(cudaEventRecord(r->ev_done, r->cp_out));
+  CK(cudaStreamWaitEvent(r->stream, r->ev_done, 0));
   return do_sync(r);
 }
 

@@ -47,6 +47,10 @@ def test_stale_replica_workload_full_size():
     gm, gp = _route_full(r, tok, off, W.load(), W.alpha)
     om, op, _ = oracle.route(trees, tok, off, W.load(), W.alpha, n_threads=16)
     assert_same_route(gm, gp, om, op, "stale replicas, full size")
+    # The host-pointer call pipelines 262,144 requests as two chunks (copies overlapping the routing, groups
+    # formed per chunk): its results must be those of the one-pass device call.
+    hm, hp = r.route_host(tok, off, W.load(), W.alpha)
+    assert_same_route(hm, hp, gm, gp, "host-pointer call in chunks")
 
 
 def test_scale_workload_sampled_outputs():
