@@ -188,11 +188,22 @@ __device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ la
 // length clamped to 2^31 - 1 (no match can be longer than a tree path).  The first `known` tokens are known
 // to be matched (known <= match(r, T)): the walk still follows their path but does not compare them.
 template <int U>
+__device__ int32_t walk_from(const TreeView& t, int4 ce, const int32_t* s_req, int32_t n_s, const int32_t* g_req,
+                             int32_t len, int32_t known, int lane, int32_t* err);
+
+template <int U>
 __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t len,
                         int32_t known, int lane, int32_t* err) {
   if (len == 0) return 0;
   int4 ce;
   if (!find_child(t.child + t.root_off, t.root_bits, req_at(s_req, n_s, g_req, 0), lane, ce)) return 0;
+  return walk_from<U>(t, ce, s_req, n_s, g_req, len, known, lane, err);
+}
+
+// The walk below the root, from the root's child entry ce for the request's first token (len >= 1).
+template <int U>
+__device__ int32_t walk_from(const TreeView& t, int4 ce, const int32_t* s_req, int32_t n_s, const int32_t* g_req,
+                             int32_t len, int32_t known, int lane, int32_t* err) {
   int32_t pos = 0;
   for (;;) {
     if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree; keeps the loop finite if it does
@@ -238,6 +249,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
   extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
+  __shared__ int4 s_root[kWarps][32];  // per warp: the item's root-table windows
   __shared__ unsigned long long s_next;
   const int lane = threadIdx.x & 31;
   if (threadIdx.x < kSlots) {
@@ -347,9 +359,47 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const int32_t* req = st + *(volatile int*)&sl.shift;
     const int32_t len32 = (int32_t)min(len, (int64_t)INT32_MAX);
     const int32_t p1 = min(P, (c + 1) * G);
+    // The request's first token in the root tables of the item's trees at once: lanes 4i .. 4i+3 read four
+    // consecutive slots of tree c*G + i's table (G <= 8).  A tree whose window holds the token before any
+    // empty slot starts its walk below the root; one whose window has an empty slot first does not hold
+    // the token; one whose window is all other keys probes again in full.
+    unsigned hit_mask = 0, empty_mask = 0;
+    int4* s_re = s_root[threadIdx.x >> 5];  // this warp's window entries
+    if (len > 0) {
+      int4 re = make_int4(0, 0, 0, 0);
+      const int32_t tp = c * G + (lane >> 2);
+      const int32_t tok0 = req_at(req, n_s, tokens + start, 0);
+      bool hit = false, empty = false;
+      if (tp < p1) {
+        const int32_t bits = trees[tp].root_bits;
+        if (bits > 0) {
+          const uint32_t mask = (1u << bits) - 1;
+          re = __ldg(trees[tp].child + trees[tp].root_off + ((slot_hash(tok0, bits) + (lane & 3)) & mask));
+          hit = re.y >= 1 && re.x == tok0;
+          empty = re.y == 0;
+        } else {
+          empty = true;  // an empty root table holds nothing
+        }
+      }
+      s_re[lane] = re;
+      __syncwarp();
+      hit_mask = __ballot_sync(kFull, hit);
+      empty_mask = __ballot_sync(kFull, empty);
+    }
     unsigned long long best = 0;
     for (int32_t p = c * G; p < p1; ++p) {
-      const int32_t m = len > 0 ? walk<kUnroll>(trees[p], req, n_s, tokens + start, len32, 0, lane, err) : 0;
+      int32_t m = 0;
+      if (len > 0) {
+        const int sh = 4 * (p - c * G);
+        const unsigned gh = (hit_mask >> sh) & 0xFu, ge = (empty_mask >> sh) & 0xFu;
+        const int fh = gh ? __ffs(gh) : 64, fe = ge ? __ffs(ge) : 64;
+        if (fh < fe) {
+          const int4 ce = s_re[sh + fh - 1];  // written by this warp before its ballots
+          m = walk_from<kUnroll>(trees[p], ce, req, n_s, tokens + start, len32, 0, lane, err);
+        } else if (fe == 64) {
+          m = walk<kUnroll>(trees[p], req, n_s, tokens + start, len32, 0, lane, err);
+        }
+      }
       if (lane == 0) {
         out_match[b * P + p] = m;
         const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
