@@ -103,11 +103,13 @@ __device__ int64_t lcp_warp(const int32_t* __restrict__ a, const int32_t* __rest
 }
 
 // One warp per request: its leader, the exact common prefix with it, and the request appended to the leader
-// list (lists[0 ..)) or the follower list (lists[B ..)); counts[0] and counts[1] must start at zero.
+// list (lists[0 ..)) or the follower list (lists[B ..)); counts must start at zero, gid at -1 and cmin at
+// INT32_MAX.  A leader with followers gets the smallest of their common prefixes in cmin and, while rows
+// last, a checkpoint row in gid.
 __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
     const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
     int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
-    int32_t* lists, int32_t* counts) {
+    int32_t* lists, int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
   for (int64_t b = ((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5; b < B; b += warps) {
@@ -129,6 +131,11 @@ __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
         lead[b] = l;
         cpre[b] = (int32_t)c;
         lists[B + atomicAdd(&counts[1], 1)] = (int32_t)b;
+        atomicMin(&cmin[l], (int32_t)c);
+        if (atomicCAS(&gid[l], -1, -2) == -1) {  // the leader's first follower gives it a row
+          const int32_t row = atomicAdd(&counts[2], 1);
+          atomicExch(&gid[l], row < gcap ? row : -1);
+        }
       }
     }
   }
@@ -142,7 +149,9 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   const size_t slots = (size_t)1 << g.bits;
   cudaError_t e = cudaMemsetAsync(g.keys, 0, slots * sizeof(unsigned long long), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g.vals, 0x7f, slots * sizeof(int32_t), st);  // 0x7f7f7f7f > any index
-  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 2 * sizeof(int32_t), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 3 * sizeof(int32_t), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.gid, 0xff, (size_t)B * sizeof(int32_t), st);   // -1
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.cmin, 0x7f, (size_t)B * sizeof(int32_t), st);  // > any prefix
   if (e != cudaSuccess) return e;
   const int64_t want = (B + kGroupThreads / 32 - 1) / (kGroupThreads / 32);
   const int grid = (int)std::min<int64_t>(want, (int64_t)num_sms * 8);
@@ -151,7 +160,7 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   group_resolve_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
-                                                       g.lead, g.cpre, g.lists, g.counts);
+                                                       g.lead, g.cpre, g.lists, g.counts, g.gid, g.cmin, g.gcap);
   return cudaGetLastError();
 }
 

@@ -43,6 +43,8 @@ struct Slot {
   int len_s;        // tokens held in shared memory
   int shift;        // token j of the request sits at slot token shift + j (keeps bulk copies 16-byte aligned)
   int done;         // items of the request finished
+  int row;          // grouped batch: the leader's checkpoint row (-1: none)
+  int climit;       // grouped batch: checkpoints are taken at positions <= climit
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -189,21 +191,28 @@ __device__ __forceinline__ int32_t first_mismatch(const int32_t* __restrict__ la
 // to be matched (known <= match(r, T)): the walk still follows their path but does not compare them.
 template <int U>
 __device__ int32_t walk_from(const TreeView& t, int4 ce, const int32_t* s_req, int32_t n_s, const int32_t* g_req,
-                             int32_t len, int32_t known, int lane, int32_t* err);
+                             int32_t len, int32_t known, int lane, int32_t* err, int32_t climit, int4* ck);
+
+// Checkpoint of a walk at the root: {position 0, the root's table offset, its meta, "has children"}.
+__device__ __forceinline__ int4 root_checkpoint(const TreeView& t) {
+  return make_int4(0, t.root_off, make_meta(t.root_bits, 0), 1);
+}
 
 template <int U>
 __device__ int32_t walk(const TreeView& t, const int32_t* s_req, int32_t n_s, const int32_t* g_req, int32_t len,
-                        int32_t known, int lane, int32_t* err) {
+                        int32_t known, int lane, int32_t* err, int32_t climit, int4* ck) {
   if (len == 0) return 0;
   int4 ce;
   if (!find_child(t.child + t.root_off, t.root_bits, req_at(s_req, n_s, g_req, 0), lane, ce)) return 0;
-  return walk_from<U>(t, ce, s_req, n_s, g_req, len, known, lane, err);
+  return walk_from<U>(t, ce, s_req, n_s, g_req, len, known, lane, err, climit, ck);
 }
 
-// The walk below the root, from the root's child entry ce for the request's first token (len >= 1).
+// The walk below the root, from the root's child entry ce for the request's first token (len >= 1).  If ck
+// is not NULL, lane 0 stores there each node boundary the walk reaches at a position <= climit (so the
+// deepest one stays): {position, the node's table offset, its meta, its child count}.
 template <int U>
 __device__ int32_t walk_from(const TreeView& t, int4 ce, const int32_t* s_req, int32_t n_s, const int32_t* g_req,
-                             int32_t len, int32_t known, int lane, int32_t* err) {
+                             int32_t len, int32_t known, int lane, int32_t* err, int32_t climit, int4* ck) {
   int32_t pos = 0;
   for (;;) {
     if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree; keeps the loop finite if it does
@@ -215,6 +224,7 @@ __device__ int32_t walk_from(const TreeView& t, int4 ce, const int32_t* s_req, i
     const int32_t k = first_mismatch<U>(label_ptr(t.label, t.shared, ce.z), s_req, n_s, g_req, pos, lim,
                                         max(1, known - pos), lane);
     pos += k;
+    if (ck && k == ce.w && pos <= climit && lane == 0) *ck = make_int4(pos, nn.x, nn.y, nn.z);
     if (k < ce.w || pos >= len || nn.z <= 0) break;
     if (!find_child(t.child + nn.x, tab_bits(nn.y), req_at(s_req, n_s, g_req, pos), lane, ce)) break;
   }
@@ -245,8 +255,9 @@ __device__ __forceinline__ unsigned long long route_key(int32_t m, int32_t ld, i
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ list,
-    const int32_t* __restrict__ count, const int32_t* __restrict__ load, int32_t alpha,
-    int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
+    const int32_t* __restrict__ count, const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin,
+    int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match,
+    int32_t* __restrict__ out_peer, int32_t* err) {
   extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
   __shared__ int4 s_root[kWarps][32];  // per warp: the item's root-table windows
@@ -335,6 +346,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
         sl.shift = shift;
         sl.best = 0;
         sl.done = 0;
+        sl.row = gid ? __ldg(gid + b) : -1;
+        sl.climit = gid ? __ldg(cmin + b) : -1;
         __threadfence_block();
         *(volatile int*)&sl.ready = (int)k;
       }
@@ -359,6 +372,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const int32_t* req = st + *(volatile int*)&sl.shift;
     const int32_t len32 = (int32_t)min(len, (int64_t)INT32_MAX);
     const int32_t p1 = min(P, (c + 1) * G);
+    const int32_t row = *(volatile int*)&sl.row, climit = row >= 0 ? *(volatile int*)&sl.climit : -1;
     // The request's first token in the root tables of the item's trees at once: lanes 4i .. 4i+3 read four
     // consecutive slots of tree c*G + i's table (G <= 8).  A tree whose window holds the token before any
     // empty slot starts its walk below the root; one whose window has an empty slot first does not hold
@@ -393,11 +407,16 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
         const int sh = 4 * (p - c * G);
         const unsigned gh = (hit_mask >> sh) & 0xFu, ge = (empty_mask >> sh) & 0xFu;
         const int fh = gh ? __ffs(gh) : 64, fe = ge ? __ffs(ge) : 64;
+        int4* ck = nullptr;
+        if (row >= 0) {  // the walk overwrites the root checkpoint with deeper boundaries
+          ck = ckpt + (int64_t)row * P + p;
+          if (lane == 0) *ck = root_checkpoint(trees[p]);
+        }
         if (fh < fe) {
           const int4 ce = s_re[sh + fh - 1];  // written by this warp before its ballots
-          m = walk_from<kUnroll>(trees[p], ce, req, n_s, tokens + start, len32, 0, lane, err);
+          m = walk_from<kUnroll>(trees[p], ce, req, n_s, tokens + start, len32, 0, lane, err, climit, ck);
         } else if (fe == 64) {
-          m = walk<kUnroll>(trees[p], req, n_s, tokens + start, len32, 0, lane, err);
+          m = walk<kUnroll>(trees[p], req, n_s, tokens + start, len32, 0, lane, err, climit, ck);
         }
       }
       if (lane == 0) {
@@ -478,14 +497,11 @@ __device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab,
   return lim;
 }
 
-// One thread: match(r, T) with the first `known` tokens known to match (1 <= known < len).  state = 1 when
-// a compare longer than kThreadSpan remains (the result is then left to the warp), 2 on a corrupt entry.
-__device__ int32_t walk_1(const TreeView& t, const int32_t* __restrict__ req, int32_t len, int32_t known,
-                          int& state) {
-  state = 0;
-  int4 ce;
-  if (!find_child_1(t.child + t.root_off, t.root_bits, __ldg(req), ce)) return 0;
-  int32_t pos = 0;
+// One thread: the walk from child entry ce at position pos, with the first `known` tokens known to match
+// (known < len).  state = 1 when a compare longer than kThreadSpan remains (the result is then left to the
+// warp), 2 on a corrupt entry.
+__device__ int32_t walk_1_loop(const TreeView& t, int4 ce, int32_t pos, const int32_t* __restrict__ req, int32_t len,
+                               int32_t known, int& state) {
   for (;;) {  // pos grows by >= 1 per step (the child's first token matched), so at most len steps
     if (ce.w <= 0 || ce.y <= 0) {
       state = 2;
@@ -508,13 +524,26 @@ __device__ int32_t walk_1(const TreeView& t, const int32_t* __restrict__ req, in
   }
 }
 
+// One thread: match(r, T) resumed at a checkpoint of the leader's walk (a node boundary at position
+// ck.x <= known, see walk_from); the root checkpoint makes it a whole walk.
+__device__ int32_t walk_1(const TreeView& t, const int4& ck, const int32_t* __restrict__ req, int32_t len,
+                          int32_t known, int& state) {
+  state = 0;
+  const int32_t pos = ck.x;
+  if (pos >= len) return len;
+  if (ck.w <= 0) return pos;
+  int4 ce;
+  if (!find_child_1(t.child + ck.y, tab_bits(ck.z), __ldg(req + pos), ce)) return pos;
+  return walk_1_loop(t, ce, pos, req, len, known, state);
+}
+
 // One warp per follower list[i], i < *count; lane j takes trees j, j + 32, ...
 __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, const int32_t* __restrict__ list,
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
-    const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int32_t* err) {
+    const int32_t* __restrict__ gid, const int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha,
+    int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
@@ -531,7 +560,8 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kerne
     const int32_t* req = tokens + start;
     const int32_t len = (int32_t)min(end - start, (int64_t)INT32_MAX);
     const int32_t c = __ldg(cpre + f);
-    const int64_t lrow = (int64_t)__ldg(lead + f) * P, frow = f * P;
+    const int32_t l = __ldg(lead + f), row = __ldg(gid + l);
+    const int64_t lrow = (int64_t)l * P, frow = f * P;
     unsigned long long best = 0;
     for (int32_t p0 = 0; p0 < P; p0 += 32) {
       const int32_t p = p0 + lane;
@@ -539,12 +569,19 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kerne
       int state = 0;
       if (p < P) {
         const int32_t ml = out_match[lrow + p];  // the leaders' pass has finished
-        m = ml < c ? ml : c >= len ? len : walk_1(trees[p], req, len, c, state);
+        if (ml < c) {
+          m = ml;
+        } else if (c >= len) {
+          m = len;
+        } else {
+          const int4 ck = row >= 0 ? __ldg(ckpt + (int64_t)row * P + p) : root_checkpoint(trees[p]);
+          m = walk_1(trees[p], ck, req, len, c, state);
+        }
       }
       if (state == 2) atomicOr(err, ERR_CORRUPT_TREE);
       for (unsigned need = __ballot_sync(kFull, state == 1); need; need &= need - 1) {
         const int j = __ffs(need) - 1;
-        const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err);
+        const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err, -1, nullptr);
         if (lane == j) m = mm;
       }
       if (p < P) {
@@ -574,15 +611,16 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
   const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
   const int grid = (int)(B < max_ctas ? B : max_ctas);
   route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B,
-                                             g ? g->lists : nullptr, g ? g->counts : nullptr, d_load, alpha, out_match,
+                                             g ? g->lists : nullptr, g ? g->counts : nullptr, g ? g->gid : nullptr,
+                                             g ? g->cmin : nullptr, g ? g->ckpt : nullptr, d_load, alpha, out_match,
                                              out_peer, d_err);
   e = cudaGetLastError();
   if (e != cudaSuccess || !g) return e;
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
   follow_kernel<<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
-                                                  g->counts + 1, g->lead, g->cpre, d_load, alpha, out_match, out_peer,
-                                                  d_err);
+                                                  g->counts + 1, g->lead, g->cpre, g->gid, g->ckpt, d_load, alpha,
+                                                  out_match, out_peer, d_err);
   return cudaGetLastError();
 }
 
