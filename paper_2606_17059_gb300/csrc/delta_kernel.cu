@@ -887,6 +887,10 @@ __global__ void validate_kernel(int32_t* header, const int32_t* __restrict__ op,
   unsigned long long* max_len = reinterpret_cast<unsigned long long*>(header);
   int32_t* err = header + 2;
   int32_t* max_runs = header + 3;
+  // Each thread keeps its own maxima and error bits; the warp reduces them and one lane updates the header,
+  // so a delta of millions of ops makes a few thousand atomics, not millions on two words.
+  unsigned long long my_len = 0;
+  int32_t my_runs = 0, my_bits = 0;
   const int64_t stride = (int64_t)gridDim.x * blockDim.x;
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
     int bits = 0;
@@ -905,10 +909,20 @@ __global__ void validate_kernel(int32_t* header, const int32_t* __restrict__ op,
         len += l;
       }
       if (len > INT32_MAX) bits |= STATIC_TOO_LONG;
-      atomicMax(max_len, (unsigned long long)len);
-      atomicMax(max_runs, (int32_t)min(b - a, (int64_t)INT32_MAX));
+      my_len = max(my_len, (unsigned long long)len);
+      my_runs = max(my_runs, (int32_t)min(b - a, (int64_t)INT32_MAX));
     }
-    if (bits) atomicOr(err, bits);
+    my_bits |= bits;
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    my_len = max(my_len, __shfl_xor_sync(kFull, my_len, o));
+    my_runs = max(my_runs, __shfl_xor_sync(kFull, my_runs, o));
+    my_bits |= __shfl_xor_sync(kFull, my_bits, o);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    if (my_len) atomicMax(max_len, my_len);
+    if (my_runs) atomicMax(max_runs, my_runs);
+    if (my_bits) atomicOr(err, my_bits);
   }
   if (peer_begin && blockIdx.x == 0) {
     for (int32_t p = threadIdx.x; p <= P; p += blockDim.x) {

@@ -37,8 +37,10 @@ __device__ __forceinline__ bool request_range(const int64_t* offsets, int64_t b,
   return start >= 0 && start <= end && end <= n_tokens;
 }
 
-// One warp per request: hash of the first kGroupHead tokens (one token per lane and position, each mixed
-// with its position, summed), then lane 0 finds or claims the key's slot and lowers its leader index.
+// One warp per 32 consecutive requests (lane i owns request base + i).  The warp hashes each request's
+// first kGroupHead tokens in turn (one token per lane and position, each mixed with its position, summed);
+// then every distinct key of the 32 is looked up or claimed once, by its lowest lane, which also lowers
+// the key's leader index to that lane's request (the smallest of the warp's requests with the key).
 __global__ void __launch_bounds__(kGroupThreads) group_hash_kernel(
     const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
     int64_t B, unsigned long long* keys, int32_t* vals, int32_t bits, int32_t* slot_of) {
@@ -46,32 +48,36 @@ __global__ void __launch_bounds__(kGroupThreads) group_hash_kernel(
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
   const uint32_t mask = (1u << bits) - 1;
-  for (int64_t b = ((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5; b < B; b += warps) {
-    int64_t start, len;
-    if (!request_range(offsets, b, tok_base, n_tokens, start, len) || len < kGroupHead) {
-      if (lane == 0) slot_of[b] = -1;
-      continue;
-    }
-    const int32_t* g = tokens + start;
-    unsigned long long h = mix64((unsigned long long)(uint32_t)__ldg(g + lane) | ((unsigned long long)lane << 32)) +
-                           mix64((unsigned long long)(uint32_t)__ldg(g + lane + 32) |
-                                 ((unsigned long long)(lane + 32) << 32));
+  for (int64_t base = (((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5) * 32; base < B; base += warps * 32) {
+    unsigned long long my_h = 0;  // 0: the lane's request is not grouped
+    for (int r = 0; r < 32 && base + r < B; ++r) {
+      int64_t start, len;
+      if (!request_range(offsets, base + r, tok_base, n_tokens, start, len) || len < kGroupHead) continue;
+      const int32_t* g = tokens + start;
+      unsigned long long h = mix64((unsigned long long)(uint32_t)__ldg(g + lane) | ((unsigned long long)lane << 32)) +
+                             mix64((unsigned long long)(uint32_t)__ldg(g + lane + 32) |
+                                   ((unsigned long long)(lane + 32) << 32));
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) h += __shfl_xor_sync(kFull, h, o);
-    h |= 1ull;  // 0 marks an empty slot
-    if (lane == 0) {
-      int32_t slot = -1;
-      uint32_t s = (uint32_t)h & mask;
-      for (uint32_t it = 0; it <= mask; ++it, s = (s + 1) & mask) {
-        const unsigned long long prev = atomicCAS(&keys[s], 0ull, h);
-        if (prev == 0ull || prev == h) {
-          slot = (int32_t)s;
+      for (int o = 16; o > 0; o >>= 1) h += __shfl_xor_sync(kFull, h, o);
+      h |= 1ull;  // 0 marks an empty slot
+      if (lane == r) my_h = h;
+    }
+    const unsigned same = __match_any_sync(kFull, my_h);
+    const int first = __ffs(same) - 1;
+    int32_t slot = -1;
+    if (my_h && lane == first) {
+      uint32_t sl = (uint32_t)my_h & mask;
+      for (uint32_t it = 0; it <= mask; ++it, sl = (sl + 1) & mask) {
+        const unsigned long long prev = atomicCAS(&keys[sl], 0ull, my_h);
+        if (prev == 0ull || prev == my_h) {
+          slot = (int32_t)sl;
           break;
         }
       }
-      if (slot >= 0) atomicMin(&vals[slot], (int32_t)b);
-      slot_of[b] = slot;
+      if (slot >= 0) atomicMin(&vals[slot], (int32_t)(base + lane));
     }
+    slot = __shfl_sync(kFull, slot, first);
+    if (base + lane < B) slot_of[base + lane] = my_h ? slot : -1;
   }
 }
 
@@ -102,36 +108,56 @@ __device__ int64_t lcp_warp(const int32_t* __restrict__ a, const int32_t* __rest
   return n;
 }
 
-// One warp per request: its leader, the exact common prefix with it, and the request appended to the leader
-// list (lists[0 ..)) or the follower list (lists[B ..)); counts must start at zero, gid at -1 and cmin at
-// INT32_MAX.  A leader with followers gets the smallest of their common prefixes in cmin and, while rows
-// last, a checkpoint row in gid.
+// One warp per 32 consecutive requests (lane i owns request base + i): each request's leader; for each
+// follower in turn, the exact common prefix with its leader (the whole warp compares); then the warp's
+// leaders and followers are appended to lists[0 ..) and lists[B ..) with one counter update each.  counts
+// must start at zero, gid at -1 and cmin at INT32_MAX.  A leader with followers gets the smallest of their
+// common prefixes in cmin and, while rows last, a checkpoint row in gid (one update per distinct leader of
+// the warp's followers).
 __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
     const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
     int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
     int32_t* lists, int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
-  for (int64_t b = ((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5; b < B; b += warps) {
-    const int32_t s = slot_of[b];
+  for (int64_t base = (((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5) * 32; base < B; base += warps * 32) {
+    const int64_t b = base + lane;
+    const bool valid = b < B;
+    const int32_t s = valid ? slot_of[b] : -1;
     const int32_t l = s >= 0 ? vals[s] : (int32_t)b;
-    int64_t c = -1;
-    if (l != (int32_t)b) {  // both requests are valid and hold at least kGroupHead tokens
-      int64_t sb, nb, sl, nl;
-      request_range(offsets, b, tok_base, n_tokens, sb, nb);
-      request_range(offsets, l, tok_base, n_tokens, sl, nl);
-      c = lcp_warp(tokens + sb, tokens + sl, min(nb, nl), lane);
+    int32_t my_c = -1;
+    for (unsigned fm = __ballot_sync(kFull, valid && l != (int32_t)b); fm; fm &= fm - 1) {
+      const int r = __ffs(fm) - 1;
+      const int32_t lr = __shfl_sync(kFull, l, r);
+      int64_t sb, nb, sl, nl;  // both requests are valid and hold at least kGroupHead tokens
+      request_range(offsets, base + r, tok_base, n_tokens, sb, nb);
+      request_range(offsets, lr, tok_base, n_tokens, sl, nl);
+      int64_t c = lcp_warp(tokens + sb, tokens + sl, min(nb, nl), lane);
       if (c < kGroupHead || c > INT32_MAX) c = -1;
+      if (lane == r) my_c = (int32_t)c;
     }
+    const bool is_f = my_c >= 0;
+    const unsigned lm = __ballot_sync(kFull, valid && !is_f), fm = __ballot_sync(kFull, is_f);
+    int32_t lbase = 0, fbase = 0;
     if (lane == 0) {
-      if (c < 0) {
-        lead[b] = (int32_t)b;
-        lists[atomicAdd(&counts[0], 1)] = (int32_t)b;
-      } else {
-        lead[b] = l;
-        cpre[b] = (int32_t)c;
-        lists[B + atomicAdd(&counts[1], 1)] = (int32_t)b;
-        atomicMin(&cmin[l], (int32_t)c);
+      if (lm) lbase = atomicAdd(&counts[0], __popc(lm));
+      if (fm) fbase = atomicAdd(&counts[1], __popc(fm));
+    }
+    lbase = __shfl_sync(kFull, lbase, 0);
+    fbase = __shfl_sync(kFull, fbase, 0);
+    const unsigned below = (1u << lane) - 1;
+    if (valid && !is_f) {
+      lead[b] = (int32_t)b;
+      lists[lbase + __popc(lm & below)] = (int32_t)b;
+    }
+    const unsigned same = __match_any_sync(kFull, is_f ? l : -1);
+    if (is_f) {
+      lead[b] = l;
+      cpre[b] = my_c;
+      lists[B + fbase + __popc(fm & below)] = (int32_t)b;
+      const int32_t c_min = (int32_t)__reduce_min_sync(same, (unsigned)my_c);
+      if (lane == __ffs(same) - 1) {
+        atomicMin(&cmin[l], c_min);
         if (atomicCAS(&gid[l], -1, -2) == -1) {  // the leader's first follower gives it a row
           const int32_t row = atomicAdd(&counts[2], 1);
           atomicExch(&gid[l], row < gcap ? row : -1);
@@ -153,7 +179,7 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   if (e == cudaSuccess) e = cudaMemsetAsync(g.gid, 0xff, (size_t)B * sizeof(int32_t), st);   // -1
   if (e == cudaSuccess) e = cudaMemsetAsync(g.cmin, 0x7f, (size_t)B * sizeof(int32_t), st);  // > any prefix
   if (e != cudaSuccess) return e;
-  const int64_t want = (B + kGroupThreads / 32 - 1) / (kGroupThreads / 32);
+  const int64_t want = ((B + 31) / 32 + kGroupThreads / 32 - 1) / (kGroupThreads / 32);  // a warp per 32 requests
   const int grid = (int)std::min<int64_t>(want, (int64_t)num_sms * 8);
   group_hash_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.keys, g.vals, g.bits,
                                                     g.slot_of);
