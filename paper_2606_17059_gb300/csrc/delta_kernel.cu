@@ -364,10 +364,21 @@ __device__ bool ensure_room(Tree& t, int32_t cur, int4& nd, int32_t extra, int l
   return true;
 }
 
+// A warp's shortcut to the anchor it last reached in a chunk's parallel phase.  Nothing above an anchor
+// changes in that phase, so an op whose first pool run is the same run (same address, same tokens) and
+// covers the anchor's position reaches the anchor by the same path: it may start there.
+struct AnchorStart {
+  int32_t node;         // the anchor (-1: none)
+  int32_t pos;          // tokens consumed on reaching it
+  const int32_t* seq;   // the first pool run of the op that reached it
+  int4 rec;             // its record then (its table offset and size hold for the phase)
+};
+
 // root: the root's node record as of the launch (its table moves only between launches).  anchor: in the
 // parallel phase, the op's anchor node (else -1): the op changes nothing until its walk has passed through
 // the anchor (OP_DEFER otherwise), and claims in the anchor's table are counted atomically.
-__device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo) {
+__device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo,
+                      AnchorStart* as) {
   const int64_t n = q.n;
   if (n == 0) {
     if (lane == 0) atomicAdd(&t.node[0].w, 1);
@@ -379,6 +390,12 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   int32_t n0, c0, l0;
   int4 nd = root;  // record of node cur: below the root (and the anchor) only this warp writes it
   bool passed = anchor < 0;
+  if (anchor >= 0 && as->node == anchor && as->seq == q.a && q.na >= as->pos && n > as->pos) {
+    cur = anchor;
+    pos = as->pos;
+    nd = as->rec;
+    passed = true;
+  }
   for (int64_t guard = 0; guard <= n + 1; ++guard) {
     if (pos == n) {  // the sequence ends exactly at node cur (never the root here: n > 0)
       if (!passed || cur == anchor) return OP_DEFER;
@@ -448,7 +465,11 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
       cur = ce.y;
       pos += k;
       nd = nn;
-      passed = passed || cur == anchor;
+      if (!passed && cur == anchor) {
+        passed = true;
+        if (pos <= q.na && lane == 0) *as = AnchorStart{anchor, (int32_t)pos, q.a, nd};
+        __syncwarp();
+      }
       continue;
     }
     // The sequence leaves (or ends inside) the edge after k tokens: split it there.  The new node mid
@@ -486,7 +507,8 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
 
 // anchor as for insert: nothing changes (OP_DEFER) unless the walk passed through it, and the anchor is
 // never folded here.
-__device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo) {
+__device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo,
+                      AnchorStart* as) {
   const int64_t n = q.n;
   if (n == 0) {
     int ok = 0;
@@ -504,6 +526,12 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   int64_t pos = 0;
   int4 nd = root, pn = root;  // records of cur and par (below the root and the anchor only this warp writes them)
   bool passed = anchor < 0;
+  if (anchor >= 0 && as->node == anchor && as->seq == q.a && q.na >= as->pos && n > as->pos) {
+    cur = anchor;  // par and e_cur stay unknown: the anchor is never folded here
+    pos = as->pos;
+    nd = as->rec;
+    passed = true;
+  }
   for (int64_t guard = 0; pos < n; ++guard) {
     if (guard > n) return OP_CORRUPT;
     int32_t slot;
@@ -528,7 +556,11 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     cur = ce.y;
     pos += ce.w;
     nd = nn;
-    passed = passed || cur == anchor;
+    if (!passed && cur == anchor) {
+      passed = true;
+      if (pos <= q.na && lane == 0) *as = AnchorStart{anchor, (int32_t)pos, q.a, nd};
+      __syncwarp();
+    }
   }
   if (!passed || cur == anchor) return OP_DEFER;
   if (nd.w == 0) {
@@ -639,7 +671,7 @@ __device__ void find_anchor(const Tree& t, const int4& root, const int64_t* __re
 // Applies op i (one warp); anchor as for insert/remove.
 __device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcode, int64_t g0, int64_t g1,
                         const int64_t* __restrict__ seg_off, const int32_t* __restrict__ seg_len,
-                        const int32_t* __restrict__ pool, int32_t* buf, int lane, Memo& memo) {
+                        const int32_t* __restrict__ pool, int32_t* buf, int lane, Memo& memo, AnchorStart* as) {
   // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
   Seq q;
   if (g1 - g0 <= 2) {
@@ -658,7 +690,8 @@ __device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcod
     q.a = q.b = buf;
     q.na = q.n = len;
   }
-  return opcode == P2P_OP_INSERT ? insert(t, q, root, anchor, lane, memo) : remove(t, q, root, anchor, lane, memo);
+  return opcode == P2P_OP_INSERT ? insert(t, q, root, anchor, lane, memo, as)
+                                 : remove(t, q, root, anchor, lane, memo, as);
 }
 
 // Ranks kDeltaBuckets buckets by count (heaviest first, ties to the lower bucket) into order; one warp.
@@ -690,6 +723,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   __shared__ int s_take;
   __shared__ int s_any;
   __shared__ MemoEntry s_memo[kDeltaWarps][kMemoSlots];
+  __shared__ AnchorStart s_astart[kDeltaWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   TreeState* gs = states + blockIdx.x;
   if (lane < kMemoSlots) s_memo[warp][lane] = MemoEntry{nullptr, nullptr, 0};
@@ -788,7 +822,10 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     __syncthreads();
     if (warp == 0) rank_buckets(s_count, s_order, lane);
     __syncthreads();
-    // 3. Parallel phase: the warps take sub-buckets of anchored ops, heaviest first.
+    // 3. Parallel phase: the warps take sub-buckets of anchored ops, heaviest first.  (Each warp's anchor
+    //    shortcut is cleared first: an anchor's table may have grown in step 2.)
+    if (lane == 0) s_astart[warp].node = -1;
+    __syncwarp();
     for (;;) {
       int idx = 0;
       if (lane == 0) idx = atomicAdd(&s_take, 1);
@@ -810,7 +847,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
           }
           const int64_t i = c0 + jj;
           const int r = apply_op(t, root, s_anchor[jj], op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool,
-                                 buf, lane, memo);
+                                 buf, lane, memo, &s_astart[warp]);
           if (lane == 0) {
             if (r == OP_DONE) {
               done[i] = 1;
@@ -860,7 +897,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
           mine &= mine - 1;
           const int64_t i = c0 + jj;
           const int r = apply_op(t, root, -1, op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool, buf, lane,
-                                 memo);
+                                 memo, &s_astart[warp]);
           if (lane == 0) {
             if (r == OP_DONE) {
               done[i] = 1;
