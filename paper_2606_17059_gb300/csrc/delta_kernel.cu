@@ -265,8 +265,38 @@ struct Memo {
   MemoEntry* e;
 };
 
+// First j in [from, lim) with a[j] != b[j], or lim (one warp; both arrays contiguous in global memory).
+// kDiffUnroll loads of 32 tokens in flight per lane and side; a block is folded into one OR of XORs per
+// lane and one vote, and only a block that holds a mismatch is searched again.
+constexpr int kDiffUnroll = 8;
+__device__ int64_t first_diff_arrays(const int32_t* a, const int32_t* b, int64_t from, int64_t lim, int lane) {
+  int64_t j0 = from;
+  for (; j0 + 32 * kDiffUnroll <= lim; j0 += 32 * kDiffUnroll) {
+    int32_t x[kDiffUnroll];
+#pragma unroll
+    for (int u = 0; u < kDiffUnroll; ++u) x[u] = a[j0 + u * 32 + lane];
+    int32_t diff = 0;
+#pragma unroll
+    for (int u = 0; u < kDiffUnroll; ++u) diff |= x[u] ^ b[j0 + u * 32 + lane];
+    if (__any_sync(kFull, diff != 0)) {
+#pragma unroll
+      for (int u = 0; u < kDiffUnroll; ++u) {
+        const unsigned m = __ballot_sync(kFull, x[u] != b[j0 + u * 32 + lane]);
+        if (m) return j0 + u * 32 + (__ffs(m) - 1);
+      }
+    }
+  }
+  for (; j0 < lim; j0 += 32) {
+    const int64_t j = j0 + lane;
+    const unsigned m = __ballot_sync(kFull, j < lim && a[j] != b[j]);
+    if (m) return j0 + (__ffs(m) - 1);
+  }
+  return lim;
+}
+
 // First j in [from, lim) with lab[j] != q[pos + j], or lim.  Lane k looks at memo entry k, so a lookup is
-// one step.
+// one step.  The sequence side is compared run by run (its first pool run, then the second), so both
+// sides of every compare are contiguous.
 __device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int64_t from, int64_t lim, int lane,
                               Memo& memo) {
   const bool in_a = pos < q.na;  // q[pos ..] starts in the first pool run, which the memo can describe
@@ -280,24 +310,10 @@ __device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int
     from = max(from, (int64_t)__reduce_max_sync(kFull, (unsigned)skip));
   }
   int64_t k = lim;
-  for (int64_t j0 = from; j0 < lim; j0 += 128) {
-    int32_t x[4], y[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const int64_t j = j0 + u * 32 + lane;
-      x[u] = j < lim ? lab[j] : 0;
-      y[u] = j < lim ? q.at(pos + j) : 0;
-    }
-    bool hit = false;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const unsigned m = __ballot_sync(kFull, x[u] != y[u]);
-      if (m && !hit) {
-        k = j0 + u * 32 + (__ffs(m) - 1);
-        hit = true;
-      }
-    }
-    if (hit) break;
+  if (from < lim) {
+    const int64_t split = max(from, min(lim, q.na - pos));  // positions below split lie in the first run
+    k = from < split ? first_diff_arrays(lab, q.a + pos, from, split, lane) : split;
+    if (k == split && split < lim) k = first_diff_arrays(lab, q.b + (pos - q.na), split, lim, lane);
   }
   if (in_a && k >= 64) {  // remember a long verified run (within the first pool run), slot by label address
     if (lane == 0) {
