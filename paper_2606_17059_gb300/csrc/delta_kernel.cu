@@ -43,7 +43,7 @@ namespace p2p {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 1536;        // ops staged in shared memory at a time
+constexpr int kChunk = 1024;        // ops staged in shared memory at a time
 constexpr int kWide = 64;           // children that make a node an anchor of parallel sub-buckets
 constexpr int kAnchorDepth = 3;     // tree levels the pre-walk descends looking for an anchor
 constexpr int kAnchorSlots = 256;   // distinct anchors per chunk (ops beyond stay in the serial phase)
@@ -380,21 +380,51 @@ __device__ bool ensure_room(Tree& t, int32_t cur, int4& nd, int32_t extra, int l
   return true;
 }
 
-// A warp's shortcut to the anchor it last reached in a chunk's parallel phase.  Nothing above an anchor
-// changes in that phase, so an op whose first pool run is the same run (same address, same tokens) and
-// covers the anchor's position reaches the anchor by the same path: it may start there.
-struct AnchorStart {
-  int32_t node;         // the anchor (-1: none)
-  int32_t pos;          // tokens consumed on reaching it
-  const int32_t* seq;   // the first pool run of the op that reached it
-  int4 rec;             // its record then (its table offset and size hold for the phase)
+// A shortcut to an anchor, shared by the CTA's warps for one chunk's parallel phase.  Nothing above an
+// anchor changes in that phase, so an op whose first pool run is the run (same address, same tokens) of
+// the op that first reached the anchor, and covers the anchor's position, reaches it by the same path: it
+// may start there.  The first op to reach the anchor claims the entry, writes pos and rec, and publishes
+// seq last; the entry is not written again in the phase.
+struct AnchorEntry {
+  const int32_t* seq;  // the first pool run of the op that reached the anchor (NULL: not published)
+  int32_t pos;         // tokens consumed on reaching it
+  int32_t claim;
+  int4 rec;            // its record then (its table offset and size hold for the phase)
 };
+
+// The shortcut test, taken by lane 0 for the whole warp: true (with pos and rec) if op q may start at the
+// anchor of entry ae.
+__device__ __forceinline__ bool anchor_start(const AnchorEntry* ae, const Seq& q, int lane, int64_t& pos, int4& rec) {
+  int ok = 0;
+  if (lane == 0 && ae) {
+    const int32_t* sp = *(const int32_t* const volatile*)&ae->seq;
+    ok = sp == q.a && sp != nullptr;
+  }
+  if (!__shfl_sync(kFull, ok, 0)) return false;
+  __threadfence_block();
+  pos = *(const volatile int32_t*)&ae->pos;
+  rec = make_int4(*(const volatile int*)&ae->rec.x, *(const volatile int*)&ae->rec.y,
+                  *(const volatile int*)&ae->rec.z, *(const volatile int*)&ae->rec.w);
+  return q.na >= pos && q.n > pos;
+}
+
+// Publishes the shortcut for the op that first reached its anchor (at pos, record rec), if the entry is free
+// and the op's first pool run covers the anchor's position.
+__device__ __forceinline__ void anchor_publish(AnchorEntry* ae, const Seq& q, int64_t pos, const int4& rec, int lane) {
+  if (lane == 0 && ae && pos <= q.na && atomicCAS(&ae->claim, 0, 1) == 0) {
+    ae->pos = (int32_t)pos;
+    ae->rec = rec;
+    __threadfence_block();
+    *(const int32_t* volatile*)&ae->seq = q.a;
+  }
+  __syncwarp();
+}
 
 // root: the root's node record as of the launch (its table moves only between launches).  anchor: in the
 // parallel phase, the op's anchor node (else -1): the op changes nothing until its walk has passed through
 // the anchor (OP_DEFER otherwise), and claims in the anchor's table are counted atomically.
 __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo,
-                      AnchorStart* as) {
+                      AnchorEntry* ae) {
   const int64_t n = q.n;
   if (n == 0) {
     if (lane == 0) atomicAdd(&t.node[0].w, 1);
@@ -406,11 +436,12 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   int32_t n0, c0, l0;
   int4 nd = root;  // record of node cur: below the root (and the anchor) only this warp writes it
   bool passed = anchor < 0;
-  if (anchor >= 0 && as->node == anchor && as->seq == q.a && q.na >= as->pos && n > as->pos) {
+  if (anchor >= 0 && anchor_start(ae, q, lane, pos, nd)) {
     cur = anchor;
-    pos = as->pos;
-    nd = as->rec;
     passed = true;
+  } else {
+    pos = 0;
+    nd = root;
   }
   for (int64_t guard = 0; guard <= n + 1; ++guard) {
     if (pos == n) {  // the sequence ends exactly at node cur (never the root here: n > 0)
@@ -483,8 +514,7 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
       nd = nn;
       if (!passed && cur == anchor) {
         passed = true;
-        if (pos <= q.na && lane == 0) *as = AnchorStart{anchor, (int32_t)pos, q.a, nd};
-        __syncwarp();
+        anchor_publish(ae, q, pos, nd, lane);
       }
       continue;
     }
@@ -524,7 +554,7 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
 // anchor as for insert: nothing changes (OP_DEFER) unless the walk passed through it, and the anchor is
 // never folded here.
 __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, int lane, Memo& memo,
-                      AnchorStart* as) {
+                      AnchorEntry* ae) {
   const int64_t n = q.n;
   if (n == 0) {
     int ok = 0;
@@ -542,11 +572,12 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   int64_t pos = 0;
   int4 nd = root, pn = root;  // records of cur and par (below the root and the anchor only this warp writes them)
   bool passed = anchor < 0;
-  if (anchor >= 0 && as->node == anchor && as->seq == q.a && q.na >= as->pos && n > as->pos) {
+  if (anchor >= 0 && anchor_start(ae, q, lane, pos, nd)) {
     cur = anchor;  // par and e_cur stay unknown: the anchor is never folded here
-    pos = as->pos;
-    nd = as->rec;
     passed = true;
+  } else {
+    pos = 0;
+    nd = root;
   }
   for (int64_t guard = 0; pos < n; ++guard) {
     if (guard > n) return OP_CORRUPT;
@@ -574,8 +605,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     nd = nn;
     if (!passed && cur == anchor) {
       passed = true;
-      if (pos <= q.na && lane == 0) *as = AnchorStart{anchor, (int32_t)pos, q.a, nd};
-      __syncwarp();
+      anchor_publish(ae, q, pos, nd, lane);
     }
   }
   if (!passed || cur == anchor) return OP_DEFER;
@@ -687,7 +717,7 @@ __device__ void find_anchor(const Tree& t, const int4& root, const int64_t* __re
 // Applies op i (one warp); anchor as for insert/remove.
 __device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcode, int64_t g0, int64_t g1,
                         const int64_t* __restrict__ seg_off, const int32_t* __restrict__ seg_len,
-                        const int32_t* __restrict__ pool, int32_t* buf, int lane, Memo& memo, AnchorStart* as) {
+                        const int32_t* __restrict__ pool, int32_t* buf, int lane, Memo& memo, AnchorEntry* ae) {
   // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
   Seq q;
   if (g1 - g0 <= 2) {
@@ -706,8 +736,8 @@ __device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcod
     q.a = q.b = buf;
     q.na = q.n = len;
   }
-  return opcode == P2P_OP_INSERT ? insert(t, q, root, anchor, lane, memo, as)
-                                 : remove(t, q, root, anchor, lane, memo, as);
+  return opcode == P2P_OP_INSERT ? insert(t, q, root, anchor, lane, memo, ae)
+                                 : remove(t, q, root, anchor, lane, memo, ae);
 }
 
 // Ranks kDeltaBuckets buckets by count (heaviest first, ties to the lower bucket) into order; one warp.
@@ -739,7 +769,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   __shared__ int s_take;
   __shared__ int s_any;
   __shared__ MemoEntry s_memo[kDeltaWarps][kMemoSlots];
-  __shared__ AnchorStart s_astart[kDeltaWarps];
+  __shared__ AnchorEntry s_aentry[kAnchorSlots];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   TreeState* gs = states + blockIdx.x;
   if (lane < kMemoSlots) s_memo[warp][lane] = MemoEntry{nullptr, nullptr, 0};
@@ -770,6 +800,8 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
       s_akey[k] = -1;
       s_ains[k] = 0;
       s_adel[k] = 0;
+      s_aentry[k].seq = nullptr;  // shortcuts hold for one chunk's parallel phase
+      s_aentry[k].claim = 0;
     }
     if (threadIdx.x < kDeltaBuckets) s_count[threadIdx.x] = 0;
     if (threadIdx.x == 0) {
@@ -840,8 +872,6 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     __syncthreads();
     // 3. Parallel phase: the warps take sub-buckets of anchored ops, heaviest first.  (Each warp's anchor
     //    shortcut is cleared first: an anchor's table may have grown in step 2.)
-    if (lane == 0) s_astart[warp].node = -1;
-    __syncwarp();
     for (;;) {
       int idx = 0;
       if (lane == 0) idx = atomicAdd(&s_take, 1);
@@ -863,7 +893,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
           }
           const int64_t i = c0 + jj;
           const int r = apply_op(t, root, s_anchor[jj], op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool,
-                                 buf, lane, memo, &s_astart[warp]);
+                                 buf, lane, memo, &s_aentry[s_aslot[jj]]);
           if (lane == 0) {
             if (r == OP_DONE) {
               done[i] = 1;
@@ -913,7 +943,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
           mine &= mine - 1;
           const int64_t i = c0 + jj;
           const int r = apply_op(t, root, -1, op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool, buf, lane,
-                                 memo, &s_astart[warp]);
+                                 memo, nullptr);
           if (lane == 0) {
             if (r == OP_DONE) {
               done[i] = 1;
