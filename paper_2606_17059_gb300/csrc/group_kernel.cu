@@ -114,7 +114,7 @@ __device__ int64_t lcp_warp(const int32_t* __restrict__ a, const int32_t* __rest
 // must start at zero, gid at -1 and cmin at INT32_MAX.  A leader with followers gets the smallest of their
 // common prefixes in cmin and, while rows last, a checkpoint row in gid (one update per distinct leader of
 // the warp's followers).
-__global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
+__global__ void __launch_bounds__(kGroupThreads) group_resolve32_kernel(
     const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
     int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
     int32_t* lists, int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap) {
@@ -167,6 +167,63 @@ __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
   }
 }
 
+// One warp per request: its leader and the exact common prefix with it; the CTA's 8 requests of a round are
+// then appended to lists[0 ..) (leaders) or lists[B ..) (followers) with one counter update per list and
+// round.  counts must start at zero, gid at -1 and cmin at INT32_MAX.  A leader with followers gets the
+// smallest of their common prefixes in cmin (updated only when a follower lowers it, so popular groups
+// make few atomics) and, while rows last, a checkpoint row in gid.
+__global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
+    const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
+    int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
+    int32_t* lists, int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap) {
+  constexpr int kWarps = kGroupThreads / 32;
+  __shared__ int s_kind[kWarps];  // 0: none, 1: leader, 2: follower
+  __shared__ int s_pos[kWarps];   // the request's index in its list
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int64_t r0 = (int64_t)blockIdx.x * kWarps; r0 < B; r0 += (int64_t)gridDim.x * kWarps) {
+    const int64_t b = r0 + warp;
+    int kind = 0;
+    int32_t l = -1, c32 = -1;
+    if (b < B) {
+      const int32_t s = slot_of[b];
+      l = s >= 0 ? vals[s] : (int32_t)b;
+      int64_t c = -1;
+      if (l != (int32_t)b) {  // both requests are valid and hold at least kGroupHead tokens
+        int64_t sb, nb, sl, nl;
+        request_range(offsets, b, tok_base, n_tokens, sb, nb);
+        request_range(offsets, l, tok_base, n_tokens, sl, nl);
+        c = lcp_warp(tokens + sb, tokens + sl, min(nb, nl), lane);
+        if (c < kGroupHead || c > INT32_MAX) c = -1;
+      }
+      kind = c < 0 ? 1 : 2;
+      c32 = (int32_t)c;
+    }
+    if (lane == 0) s_kind[warp] = kind;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int nl = 0, nf = 0;
+      for (int w = 0; w < kWarps; ++w) nl += s_kind[w] == 1, nf += s_kind[w] == 2;
+      const int bl = nl ? atomicAdd(&counts[0], nl) : 0, bf = nf ? atomicAdd(&counts[1], nf) : 0;
+      for (int w = 0, il = 0, jf = 0; w < kWarps; ++w) s_pos[w] = s_kind[w] == 1 ? bl + il++ : s_kind[w] == 2 ? bf + jf++ : 0;
+    }
+    __syncthreads();
+    if (lane == 0 && kind == 1) {
+      lead[b] = (int32_t)b;
+      lists[s_pos[warp]] = (int32_t)b;
+    } else if (lane == 0 && kind == 2) {
+      lead[b] = l;
+      cpre[b] = c32;
+      lists[B + s_pos[warp]] = (int32_t)b;
+      if (c32 < *(volatile int32_t*)&cmin[l]) atomicMin(&cmin[l], c32);
+      if (*(volatile int32_t*)&gid[l] == -1 && atomicCAS(&gid[l], -1, -2) == -1) {
+        const int32_t row = atomicAdd(&counts[2], 1);  // the leader's first follower gives it a row
+        atomicExch(&gid[l], row < gcap ? row : -1);
+      }
+    }
+    __syncthreads();  // s_kind and s_pos are reused next round
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
@@ -179,14 +236,24 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   if (e == cudaSuccess) e = cudaMemsetAsync(g.gid, 0xff, (size_t)B * sizeof(int32_t), st);   // -1
   if (e == cudaSuccess) e = cudaMemsetAsync(g.cmin, 0x7f, (size_t)B * sizeof(int32_t), st);  // > any prefix
   if (e != cudaSuccess) return e;
-  const int64_t want = ((B + 31) / 32 + kGroupThreads / 32 - 1) / (kGroupThreads / 32);  // a warp per 32 requests
-  const int grid = (int)std::min<int64_t>(want, (int64_t)num_sms * 8);
+  const int64_t hash_ctas = ((B + 31) / 32 + kGroupThreads / 32 - 1) / (kGroupThreads / 32);  // a warp per 32 requests
+  const int64_t resolve_ctas = (B + kGroupThreads / 32 - 1) / (kGroupThreads / 32);            // a warp per request
+  const int grid = (int)std::min<int64_t>(hash_ctas, (int64_t)num_sms * 8);
+  const int grid2 = (int)std::min<int64_t>(resolve_ctas, (int64_t)num_sms * 8);
   group_hash_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.keys, g.vals, g.bits,
                                                     g.slot_of);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  group_resolve_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
-                                                       g.lead, g.cpre, g.lists, g.counts, g.gid, g.cmin, g.gcap);
+  // Large batches: a warp per 32 requests (at least 32 warps per SM still busy; fewest atomics).  Smaller
+  // ones: a warp per request, so that the common-prefix compares spread over as many warps as there are
+  // requests.
+  if (B >= (int64_t)num_sms * 32 * 32) {
+    group_resolve32_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
+                                                           g.lead, g.cpre, g.lists, g.counts, g.gid, g.cmin, g.gcap);
+  } else {
+    group_resolve_kernel<<<grid2, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
+                                                          g.lead, g.cpre, g.lists, g.counts, g.gid, g.cmin, g.gcap);
+  }
   return cudaGetLastError();
 }
 
