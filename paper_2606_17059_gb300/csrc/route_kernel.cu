@@ -498,10 +498,11 @@ __device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab,
 }
 
 // One thread: the walk from child entry ce at position pos, with the first `known` tokens known to match
-// (known < len).  state = 1 when a compare longer than kThreadSpan remains (the result is then left to the
-// warp), 2 on a corrupt entry.
+// (known < len).  state = 1 when a label compare matches its first 8 tokens and more than kThreadSpan remain
+// (the result is then left to the warp), 2 on a corrupt entry.  If ck is not NULL, each node
+// boundary reached at a position <= climit is stored there (see walk_from).
 __device__ int32_t walk_1_loop(const TreeView& t, int4 ce, int32_t pos, const int32_t* __restrict__ req, int32_t len,
-                               int32_t known, int& state) {
+                               int32_t known, int& state, int32_t climit, int4* ck) {
   for (;;) {  // pos grows by >= 1 per step (the child's first token matched), so at most len steps
     if (ce.w <= 0 || ce.y <= 0) {
       state = 2;
@@ -512,45 +513,63 @@ __device__ int32_t walk_1_loop(const TreeView& t, int4 ce, int32_t pos, const in
     const int32_t from = max(1, known - pos);
     int32_t k = lim;
     if (from < lim) {
-      if (lim - from > kThreadSpan) {
-        state = 1;
-        return 0;
+      // One step of 8 tokens first (a request that leaves the edge early, the common case, stops there);
+      // then a remainder of up to kThreadSpan tokens here, a longer one by the warp.
+      const int32_t* lab = label_ptr(t.label, t.shared, ce.z);
+      const int32_t first = min(lim, from + 8);
+      k = first_diff_1(lab, req + pos, from, first);
+      if (k == first && first < lim) {
+        if (lim - first > kThreadSpan) {
+          state = 1;
+          return 0;
+        }
+        k = first_diff_1(lab, req + pos, first, lim);
       }
-      k = first_diff_1(label_ptr(t.label, t.shared, ce.z), req + pos, from, lim);
     }
     pos += k;
+    if (ck && k == ce.w && pos <= climit) *ck = make_int4(pos, nn.x, nn.y, nn.z);
     if (k < ce.w || pos >= len || nn.z <= 0) return pos;
     if (!find_child_1(t.child + nn.x, tab_bits(nn.y), __ldg(req + pos), ce)) return pos;
   }
 }
 
 // One thread: match(r, T) resumed at a checkpoint of the leader's walk (a node boundary at position
-// ck.x <= known, see walk_from); the root checkpoint makes it a whole walk.
+// ck.x <= known, see walk_from); the root checkpoint makes it a whole walk.  climit/ck_out as for
+// walk_1_loop.
 __device__ int32_t walk_1(const TreeView& t, const int4& ck, const int32_t* __restrict__ req, int32_t len,
-                          int32_t known, int& state) {
+                          int32_t known, int& state, int32_t climit, int4* ck_out) {
   state = 0;
   const int32_t pos = ck.x;
   if (pos >= len) return len;
   if (ck.w <= 0) return pos;
   int4 ce;
   if (!find_child_1(t.child + ck.y, tab_bits(ck.z), __ldg(req + pos), ce)) return pos;
-  return walk_1_loop(t, ce, pos, req, len, known, state);
+  return walk_1_loop(t, ce, pos, req, len, known, state, climit, ck_out);
 }
 
-// One warp per follower list[i], i < *count; lane j takes trees j, j + 32, ...
-__global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kernel(
+// One warp per request list[i], i < *count; lane j walks trees j, j + 32, ...
+//   kLeader: the request is a group leader (or ungrouped): whole walks, and for a leader with a checkpoint
+//   row, the checkpoints its followers resume from.
+//   !kLeader: the request follows leader lead[f] with common prefix c = cpre[f]: match(f, T) = match(lead,
+//   T) if that is < c, else a walk resumed at the leader's checkpoint that does not compare f's first c
+//   tokens.
+template <bool kLeader>
+__global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, const int32_t* __restrict__ list,
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
-    const int32_t* __restrict__ gid, const int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha,
-    int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer, int32_t* err) {
+    const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
+    const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
+    int32_t* err) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
   for (int64_t i = ((int64_t)blockIdx.x * kFollowThreads + threadIdx.x) >> 5; i < n; i += warps) {
     const int64_t f = __ldg(list + i);
     const int64_t start = __ldg(offsets + f) - tok_base, end = __ldg(offsets + f + 1) - tok_base;
-    if (!(start >= 0 && start <= end && end <= n_tokens)) {  // cannot happen: only valid requests are grouped
+    const int64_t frow = f * P;
+    if (!(start >= 0 && start <= end && end <= n_tokens)) {  // (followers are always valid)
+      for (int32_t p = lane; p < P; p += 32) out_match[frow + p] = 0;
       if (lane == 0) {
         out_peer[f] = -1;
         atomicOr(err, ERR_BAD_OFFSETS);
@@ -559,29 +578,45 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) follow_kerne
     }
     const int32_t* req = tokens + start;
     const int32_t len = (int32_t)min(end - start, (int64_t)INT32_MAX);
-    const int32_t c = __ldg(cpre + f);
-    const int32_t l = __ldg(lead + f), row = __ldg(gid + l);
-    const int64_t lrow = (int64_t)l * P, frow = f * P;
+    int32_t c = 0, climit = -1;
+    int64_t lrow = 0;
+    int32_t row;
+    if (kLeader) {
+      row = __ldg(gid + f);
+      climit = row >= 0 ? __ldg(cmin + f) : -1;
+    } else {
+      c = __ldg(cpre + f);
+      const int32_t l = __ldg(lead + f);
+      row = __ldg(gid + l);
+      lrow = (int64_t)l * P;
+    }
     unsigned long long best = 0;
     for (int32_t p0 = 0; p0 < P; p0 += 32) {
       const int32_t p = p0 + lane;
       int32_t m = 0;
       int state = 0;
       if (p < P) {
-        const int32_t ml = out_match[lrow + p];  // the leaders' pass has finished
-        if (ml < c) {
-          m = ml;
-        } else if (c >= len) {
-          m = len;
+        if (kLeader) {
+          int4* ck = row >= 0 ? ckpt + (int64_t)row * P + p : nullptr;
+          if (ck) *ck = root_checkpoint(trees[p]);
+          m = len > 0 ? walk_1(trees[p], root_checkpoint(trees[p]), req, len, 0, state, climit, ck) : 0;
         } else {
-          const int4 ck = row >= 0 ? __ldg(ckpt + (int64_t)row * P + p) : root_checkpoint(trees[p]);
-          m = walk_1(trees[p], ck, req, len, c, state);
+          const int32_t ml = out_match[lrow + p];  // the leaders' pass has finished
+          if (ml < c) {
+            m = ml;
+          } else if (c >= len) {
+            m = len;
+          } else {
+            const int4 ck = row >= 0 ? ckpt[(int64_t)row * P + p] : root_checkpoint(trees[p]);
+            m = walk_1(trees[p], ck, req, len, c, state, -1, nullptr);
+          }
         }
       }
       if (state == 2) atomicOr(err, ERR_CORRUPT_TREE);
       for (unsigned need = __ballot_sync(kFull, state == 1); need; need &= need - 1) {
         const int j = __ffs(need) - 1;
-        const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err, -1, nullptr);
+        int4* ck = kLeader && row >= 0 ? ckpt + (int64_t)row * P + p0 + j : nullptr;
+        const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err, climit, ck);
         if (lane == j) m = mm;
       }
       if (p < P) {
@@ -605,22 +640,40 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
                          int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
-  const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
-  cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
-  const int grid = (int)(B < max_ctas ? B : max_ctas);
-  route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B,
-                                             g ? g->lists : nullptr, g ? g->counts : nullptr, g ? g->gid : nullptr,
-                                             g ? g->cmin : nullptr, g ? g->ckpt : nullptr, d_load, alpha, out_match,
-                                             out_peer, d_err);
-  e = cudaGetLastError();
-  if (e != cudaSuccess || !g) return e;
+  if (!g) {  // ungrouped: the staged kernel over every request
+    const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
+    cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
+    const int grid = (int)(B < max_ctas ? B : max_ctas);
+    route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, nullptr, nullptr,
+                                               nullptr, nullptr, nullptr, d_load, alpha, out_match, out_peer, d_err);
+    return cudaGetLastError();
+  }
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
-  follow_kernel<<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
-                                                  g->counts + 1, g->lead, g->cpre, g->gid, g->ckpt, d_load, alpha,
-                                                  out_match, out_peer, d_err);
+  cudaError_t e;
+  if (n_tokens >= B * (int64_t)kSlotTokens) {
+    // Requests of a staging window or longer on average: the leaders' walks are long compares, which the
+    // staged kernel's warps do from shared memory.
+    const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
+    e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
+    const int grid = (int)(B < max_ctas ? B : max_ctas);
+    route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists, g->counts,
+                                               g->gid, g->cmin, g->ckpt, d_load, alpha, out_match, out_peer, d_err);
+  } else {
+    // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
+    lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists,
+                                                        g->counts, nullptr, nullptr, g->gid, g->cmin, g->ckpt, d_load,
+                                                        alpha, out_match, out_peer, d_err);
+  }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
+                                                       g->counts + 1, g->lead, g->cpre, g->gid, nullptr, g->ckpt, d_load,
+                                                       alpha, out_match, out_peer, d_err);
   return cudaGetLastError();
 }
 
