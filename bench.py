@@ -359,7 +359,8 @@ def run_ours(args):
             bytes_per_launch = orc.touched_bytes(ctr) / n_acc * B
             achieved = bytes_per_launch / (route_avg_ms / 1e3) / 1e9
             roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                    "traffic": None, "kernel": "route_kernel", "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
+                    "traffic": None,
+                    "kernel": "route step: group_hash + group_resolve + lane_kernel (leaders, followers)", "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
                     "bytes_per_launch": bytes_per_launch, "route_ms": route_avg_ms,
                     "bytes_basis": f"oracle touched-byte counters over {n_acc} requests x {P} trees, "
                                    f"scaled to {B} requests per launch"}
