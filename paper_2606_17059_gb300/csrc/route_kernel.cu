@@ -560,7 +560,8 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
     const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
     const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int32_t* err) {
+    int4* __restrict__ walks, int32_t* wcount, int32_t wcap, unsigned long long* __restrict__ rkey,
+    int32_t* __restrict__ rpend, int32_t* err) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
@@ -591,6 +592,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
       lrow = (int64_t)l * P;
     }
     unsigned long long best = 0;
+    int pend = 0;  // walks of this request handed to the queue
     for (int32_t p0 = 0; p0 < P; p0 += 32) {
       const int32_t p = p0 + lane;
       int32_t m = 0;
@@ -613,13 +615,28 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
         }
       }
       if (state == 2) atomicOr(err, ERR_CORRUPT_TREE);
-      for (unsigned need = __ballot_sync(kFull, state == 1); need; need &= need - 1) {
+      // Long matches go to the queue, which every warp drains afterwards (so that a request with many of
+      // them does not keep one warp busy while the others idle); if it is full, this warp walks them.
+      unsigned need = __ballot_sync(kFull, state == 1);
+      bool queued = false;
+      if (need) {
+        int base = 0;
+        if (lane == 0) base = atomicAdd(wcount, __popc(need));
+        base = __shfl_sync(kFull, base, 0);
+        if ((int64_t)base + __popc(need) <= wcap) {
+          if (state == 1) walks[base + __popc(need & ((1u << lane) - 1))] = make_int4((int32_t)f, p, c, 0);
+          pend += __popc(need);
+          queued = state == 1;
+          need = 0;
+        }
+      }
+      for (; need; need &= need - 1) {
         const int j = __ffs(need) - 1;
         int4* ck = kLeader && row >= 0 ? ckpt + (int64_t)row * P + p0 + j : nullptr;
         const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err, climit, ck);
         if (lane == j) m = mm;
       }
-      if (p < P) {
+      if (p < P && !queued) {
         out_match[frow + p] = m;
         const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
         best = key > best ? key : best;
@@ -630,7 +647,56 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
       const unsigned long long other = __shfl_xor_sync(kFull, best, o);
       best = other > best ? other : best;
     }
-    if (lane == 0) out_peer[f] = 0xFFFF - (int32_t)(best & 0xFFFFull);
+    if (lane == 0) {
+      if (pend == 0) {
+        out_peer[f] = 0xFFFF - (int32_t)(best & 0xFFFFull);
+      } else {  // the queue's walks finish the route (drain_kernel)
+        rkey[f] = best;
+        rpend[f] = pend;
+      }
+    }
+  }
+}
+
+// One warp per queued walk {request f, tree p, known prefix c}: the walk, its match, its key merged into the
+// request's; the request's last queued walk writes the route.  kLeader: also the leader's checkpoints.
+template <bool kLeader>
+__global__ void __launch_bounds__(kFollowThreads) drain_kernel(
+    const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
+    int64_t tok_base, const int64_t* __restrict__ offsets, const int4* __restrict__ walks,
+    const int32_t* __restrict__ wcount, int32_t wcap, const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin,
+    int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match,
+    int32_t* __restrict__ out_peer, unsigned long long* rkey, int32_t* rpend, int32_t* err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
+  const int64_t n = min((int64_t)*wcount, (int64_t)wcap);
+  for (int64_t i = ((int64_t)blockIdx.x * kFollowThreads + threadIdx.x) >> 5; i < n; i += warps) {
+    const int4 w = walks[i];
+    const int64_t f = w.x;
+    const int32_t p = w.y, c = w.z;
+    const int64_t start = __ldg(offsets + f) - tok_base;
+    const int32_t len = (int32_t)min(__ldg(offsets + f + 1) - tok_base - start, (int64_t)INT32_MAX);
+    const int32_t* req = tokens + start;
+    int32_t climit = -1;
+    int4* ck = nullptr;
+    if (kLeader) {
+      const int32_t row = __ldg(gid + f);
+      if (row >= 0) {
+        climit = __ldg(cmin + f);
+        ck = ckpt + (int64_t)row * P + p;
+      }
+    }
+    const int32_t m = walk<8>(trees[p], req, 0, req, len, c, lane, err, climit, ck);
+    if (lane == 0) {
+      out_match[f * P + p] = m;
+      atomicMax(&rkey[f], route_key(m, __ldg(load + p), p, alpha));
+      __threadfence();
+      if (atomicSub(&rpend[f], 1) == 1) {  // the request's last walk: every other key is merged
+        __threadfence();
+        const unsigned long long bk = atomicMax(&rkey[f], 0ull);
+        out_peer[f] = 0xFFFF - (int32_t)(bk & 0xFFFFull);
+      }
+    }
   }
 }
 
@@ -638,7 +704,9 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
 
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
                          const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
-                         int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st) {
+                         int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st,
+                         int* launched) {
+  *launched = 0;
   if (B <= 0) return cudaSuccess;
   if (!g) {  // ungrouped: the staged kernel over every request
     const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
@@ -648,10 +716,12 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
     const int grid = (int)(B < max_ctas ? B : max_ctas);
     route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, nullptr, nullptr,
                                                nullptr, nullptr, nullptr, d_load, alpha, out_match, out_peer, d_err);
+    *launched = 1;
     return cudaGetLastError();
   }
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
+  const int drain_grid = num_sms * kFollowCtasPerSm;  // drains read their walk count on the device
   cudaError_t e;
   if (n_tokens >= B * (int64_t)kSlotTokens) {
     // Requests of a staging window or longer on average: the leaders' walks are long compares, which the
@@ -663,17 +733,33 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
     const int grid = (int)(B < max_ctas ? B : max_ctas);
     route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists, g->counts,
                                                g->gid, g->cmin, g->ckpt, d_load, alpha, out_match, out_peer, d_err);
+    *launched = 1;
   } else {
     // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
     lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists,
                                                         g->counts, nullptr, nullptr, g->gid, g->cmin, g->ckpt, d_load,
-                                                        alpha, out_match, out_peer, d_err);
+                                                        alpha, out_match, out_peer, g->walks, g->counts + 3, g->wcap,
+                                                        g->rkey, g->rpend, d_err);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    drain_kernel<true><<<drain_grid, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
+                                                              g->walks, g->counts + 3, g->wcap, g->gid, g->cmin,
+                                                              g->ckpt, d_load, alpha, out_match, out_peer, g->rkey,
+                                                              g->rpend, d_err);
+    *launched = 2;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
                                                        g->counts + 1, g->lead, g->cpre, g->gid, nullptr, g->ckpt, d_load,
-                                                       alpha, out_match, out_peer, d_err);
+                                                       alpha, out_match, out_peer, g->walks, g->counts + 4, g->wcap,
+                                                       g->rkey, g->rpend, d_err);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  drain_kernel<false><<<drain_grid, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->walks,
+                                                             g->counts + 4, g->wcap, nullptr, nullptr, nullptr, d_load,
+                                                             alpha, out_match, out_peer, g->rkey, g->rpend, d_err);
+  *launched += 2;
   return cudaGetLastError();
 }
 
