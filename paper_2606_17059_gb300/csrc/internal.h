@@ -98,23 +98,18 @@ struct GroupScratch {
   int32_t* lead;     // [B]
   int32_t* cpre;     // [B]
   int32_t* lists;    // [2B]
-  int32_t* counts;   // [5]: leaders, followers, groups with a checkpoint row, handed-off walks (leader
-                     // pass, follower pass)
+  int32_t* counts;   // [3]: leaders, followers, groups with a checkpoint row
   int32_t* gid;      // [B]: a leader's checkpoint row (-1: none)
   int32_t* cmin;     // [B]: a leader's smallest common prefix with its followers
   int4* ckpt;        // [gcap * P]: per (row, tree) the leader's walk state to resume from (see route_kernel.cu)
   int32_t gcap;      // checkpoint rows
-  int4* walks;       // [wcap]: long walks handed off by the lane kernels {request, tree, known prefix, 0}
-  int32_t wcap;
-  unsigned long long* rkey;  // [B]: a request's route key over its walks not handed off
-  int32_t* rpend;            // [B]: its handed-off walks still to finish
 };
 cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
                          const GroupScratch& g, int num_sms, cudaStream_t st);
 
 // Route kernels (lookup + route decision), see route_kernel.cu.  Without groups (g == nullptr) one launch
-// routes every request; with groups, a leader pass and a follower pass, each with a drain of the long walks
-// it handed off.  *launched is set to the number of kernels launched.
+// routes every request; with groups, a leader pass and a follower pass.  *launched is set to the number of
+// kernels launched.
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens,
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
                          int32_t* out_match, int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms,

@@ -4,20 +4,23 @@
 // number of leading request tokens found along one path of T_p, a partial edge included), and the
 // chosen peer argmax_p (match - alpha*load_p, -load_p, -p) (Algorithm 1's argmax with a load term).
 //
-// Schedule.  A CTA takes requests b = blockIdx.x, blockIdx.x + gridDim.x, ...; its work items are
-// (request, group of G consecutive trees) in that order, handed to warps from a shared counter, so a warp
-// that finishes short walks immediately takes the next item instead of waiting for the slowest walk of the
-// request.  Requests are staged in shared memory in kSlots slots: the warp that takes a request's first item
-// copies its tokens in with one bulk (TMA) copy (up to kSlotTokens; longer requests read the rest through
-// the read-only path); warps with later items of that request wait until it is staged; the last warp to
-// finish one of its items writes the route and frees the slot for the request kSlots later.  Every wait is
-// bounded.
+// Passes.  A grouped batch (group_kernel.cu) is routed by a leader pass and a follower pass.  Leaders of
+// short requests, and all followers, are walked by lane_kernel (a lane per tree; below).  Leaders whose
+// requests are longer than a staging window on average, and batches too large to group, go to route_kernel:
 //
-// A walk is warp-cooperative: a child lookup probes 32 slots of the node's children hash table at once
-// (one coalesced load, whatever the fan-out), and an edge label is compared 32 consecutive tokens per warp
-// load, up to kUnroll loads in flight per lane, folded into one vote per block; the first mismatch is
-// searched only inside the block that holds it.  The route decision keeps the max of a packed 64-bit key
-// per request.  Integer work only: no tensor cores.
+// route_kernel schedule.  A CTA takes requests b = list[blockIdx.x], list[blockIdx.x + gridDim.x], ...; its
+// work items are (request, group of G consecutive trees) in that order, handed to warps from a shared
+// counter, so a warp that finishes short walks immediately takes the next item.  Requests are staged in
+// shared memory in kSlots slots: the warp that takes a request's first item copies its tokens in with one
+// bulk (TMA) copy (up to kSlotTokens; longer requests read the rest through the read-only path); warps with
+// later items of that request wait until it is staged; the last warp to finish one of its items writes the
+// route and frees the slot for the request kSlots later.  Every wait is bounded.
+//
+// A warp-cooperative walk: a child lookup probes 32 slots of the node's children hash table at once (one
+// coalesced load, whatever the fan-out), and an edge label is compared 32 consecutive tokens per warp load,
+// up to kUnroll loads in flight per lane, folded into one vote per block; the first mismatch is searched
+// only inside the block that holds it.  The route decision keeps the max of a packed 64-bit key per
+// request.  Integer work only: no tensor cores.
 #include "internal.h"
 
 namespace p2p {
@@ -445,13 +448,15 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
   }
 }
 
-// ---- Follower pass of a grouped batch -------------------------------------------------------------------
+// ---- Lane walks (leaders of short requests, and followers) ----------------------------------------------
 //
-// A follower f with leader l and exact common prefix c: in tree p, match(f) = match(l) if match(l) < c, else
-// a walk that does not compare f's first c tokens.  Such a walk is short (a child lookup at each node on
-// the known part, then the compare past c), so each lane walks its own (follower, tree) pair: a warp keeps
-// 32 independent chains of dependent loads in flight.  A lane whose remaining compare is longer than
-// kThreadSpan tokens hands that pair to the whole warp (the cooperative walk above).
+// A warp takes one request and each lane one tree (lanes j, j + 32, ...), so a warp keeps 32 independent
+// chains of dependent loads in flight.  Edges are walked by their lane; a label compare that goes on past
+// its first 8 tokens with more than kThreadSpan tokens left is done by the whole warp, once for every lane
+// waiting at the same label address and request position.
+//   Leaders: whole walks, and the checkpoints their followers resume from.
+//   A follower f with leader l and exact common prefix c: in tree p, match(f) = match(l) if match(l) < c,
+//   else a walk resumed at the leader's checkpoint that does not compare f's first c tokens.
 
 constexpr int kFollowThreads = 256;
 constexpr int kFollowCtasPerSm = 4;
@@ -497,56 +502,6 @@ __device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab,
   return lim;
 }
 
-// One thread: the walk from child entry ce at position pos, with the first `known` tokens known to match
-// (known < len).  state = 1 when a label compare matches its first 8 tokens and more than kThreadSpan remain
-// (the result is then left to the warp), 2 on a corrupt entry.  If ck is not NULL, each node
-// boundary reached at a position <= climit is stored there (see walk_from).
-__device__ int32_t walk_1_loop(const TreeView& t, int4 ce, int32_t pos, const int32_t* __restrict__ req, int32_t len,
-                               int32_t known, int& state, int32_t climit, int4* ck) {
-  for (;;) {  // pos grows by >= 1 per step (the child's first token matched), so at most len steps
-    if (ce.w <= 0 || ce.y <= 0) {
-      state = 2;
-      return pos;
-    }
-    const int4 nn = __ldg(t.node + ce.y);  // the child's record, fetched while the label is compared
-    const int32_t lim = min(ce.w, len - pos);
-    const int32_t from = max(1, known - pos);
-    int32_t k = lim;
-    if (from < lim) {
-      // One step of 8 tokens first (a request that leaves the edge early, the common case, stops there);
-      // then a remainder of up to kThreadSpan tokens here, a longer one by the warp.
-      const int32_t* lab = label_ptr(t.label, t.shared, ce.z);
-      const int32_t first = min(lim, from + 8);
-      k = first_diff_1(lab, req + pos, from, first);
-      if (k == first && first < lim) {
-        if (lim - first > kThreadSpan) {
-          state = 1;
-          return 0;
-        }
-        k = first_diff_1(lab, req + pos, first, lim);
-      }
-    }
-    pos += k;
-    if (ck && k == ce.w && pos <= climit) *ck = make_int4(pos, nn.x, nn.y, nn.z);
-    if (k < ce.w || pos >= len || nn.z <= 0) return pos;
-    if (!find_child_1(t.child + nn.x, tab_bits(nn.y), __ldg(req + pos), ce)) return pos;
-  }
-}
-
-// One thread: match(r, T) resumed at a checkpoint of the leader's walk (a node boundary at position
-// ck.x <= known, see walk_from); the root checkpoint makes it a whole walk.  climit/ck_out as for
-// walk_1_loop.
-__device__ int32_t walk_1(const TreeView& t, const int4& ck, const int32_t* __restrict__ req, int32_t len,
-                          int32_t known, int& state, int32_t climit, int4* ck_out) {
-  state = 0;
-  const int32_t pos = ck.x;
-  if (pos >= len) return len;
-  if (ck.w <= 0) return pos;
-  int4 ce;
-  if (!find_child_1(t.child + ck.y, tab_bits(ck.z), __ldg(req + pos), ce)) return pos;
-  return walk_1_loop(t, ce, pos, req, len, known, state, climit, ck_out);
-}
-
 // One warp per request list[i], i < *count; lane j walks trees j, j + 32, ...
 //   kLeader: the request is a group leader (or ungrouped): whole walks, and for a leader with a checkpoint
 //   row, the checkpoints its followers resume from.
@@ -560,8 +515,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
     const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
     const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int4* __restrict__ walks, int32_t* wcount, int32_t wcap, unsigned long long* __restrict__ rkey,
-    int32_t* __restrict__ rpend, int32_t* err) {
+    int32_t* err) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
@@ -592,51 +546,94 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
       lrow = (int64_t)l * P;
     }
     unsigned long long best = 0;
-    int pend = 0;  // walks of this request handed to the queue
     for (int32_t p0 = 0; p0 < P; p0 += 32) {
       const int32_t p = p0 + lane;
-      int32_t m = 0;
-      int state = 0;
-      if (p < P) {
+      int32_t m = 0, pos = 0, known = c;
+      bool act = false;  // the lane has an edge to walk (ce, at position pos)
+      int4 ce = make_int4(0, 0, 0, 0);
+      int4* ck = nullptr;
+      if (p < P && len > 0) {
+        int4 start = root_checkpoint(trees[p]);
+        bool walk_it = true;
         if (kLeader) {
-          int4* ck = row >= 0 ? ckpt + (int64_t)row * P + p : nullptr;
-          if (ck) *ck = root_checkpoint(trees[p]);
-          m = len > 0 ? walk_1(trees[p], root_checkpoint(trees[p]), req, len, 0, state, climit, ck) : 0;
+          if (row >= 0) {
+            ck = ckpt + (int64_t)row * P + p;
+            *ck = start;
+          }
         } else {
           const int32_t ml = out_match[lrow + p];  // the leaders' pass has finished
-          if (ml < c) {
-            m = ml;
-          } else if (c >= len) {
-            m = len;
-          } else {
-            const int4 ck = row >= 0 ? ckpt[(int64_t)row * P + p] : root_checkpoint(trees[p]);
-            m = walk_1(trees[p], ck, req, len, c, state, -1, nullptr);
+          if (ml < c || c >= len) {
+            m = ml < c ? ml : len;
+            walk_it = false;
+          } else if (row >= 0) {
+            start = ckpt[(int64_t)row * P + p];
           }
         }
-      }
-      if (state == 2) atomicOr(err, ERR_CORRUPT_TREE);
-      // Long matches go to the queue, which every warp drains afterwards (so that a request with many of
-      // them does not keep one warp busy while the others idle); if it is full, this warp walks them.
-      unsigned need = __ballot_sync(kFull, state == 1);
-      bool queued = false;
-      if (need) {
-        int base = 0;
-        if (lane == 0) base = atomicAdd(wcount, __popc(need));
-        base = __shfl_sync(kFull, base, 0);
-        if ((int64_t)base + __popc(need) <= wcap) {
-          if (state == 1) walks[base + __popc(need & ((1u << lane) - 1))] = make_int4((int32_t)f, p, c, 0);
-          pend += __popc(need);
-          queued = state == 1;
-          need = 0;
+        if (walk_it) {
+          pos = min(start.x, len);
+          m = pos;
+          act = pos < len && start.w > 0 &&
+                find_child_1(trees[p].child + start.y, tab_bits(start.z), __ldg(req + pos), ce);
         }
       }
-      for (; need; need &= need - 1) {
-        const int j = __ffs(need) - 1;
-        int4* ck = kLeader && row >= 0 ? ckpt + (int64_t)row * P + p0 + j : nullptr;
-        const int32_t mm = walk<8>(trees[p0 + j], req, 0, req, len, c, lane, err, climit, ck);
-        if (lane == j) m = mm;
+      // The walks advance edge by edge.  A lane compares an edge's label itself when it leaves within the
+      // first 8 tokens or the edge has at most kThreadSpan tokens left; longer compares are done by the
+      // whole warp, once per distinct (label address, request position): the long prompt prefixes are
+      // interned labels shared by many trees, so one compare serves every lane at that label.
+      while (__ballot_sync(kFull, act)) {
+        int4 nn = make_int4(0, 0, 0, 0);
+        int32_t k = 0, lim = 0, from2 = 0;
+        const int32_t* lab = nullptr;
+        bool need = false;
+        if (act) {
+          if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree
+            atomicOr(err, ERR_CORRUPT_TREE);
+            act = false;
+          } else {
+            nn = __ldg(trees[p].node + ce.y);
+            lab = label_ptr(trees[p].label, trees[p].shared, ce.z);
+            lim = min(ce.w, len - pos);
+            const int32_t from = max(1, known - pos);
+            k = lim;
+            if (from < lim) {
+              const int32_t first = min(lim, from + 8);
+              k = first_diff_1(lab, req + pos, from, first);
+              if (k == first && first < lim) {
+                if (lim - first <= kThreadSpan) {
+                  k = first_diff_1(lab, req + pos, first, lim);
+                } else {
+                  need = true;
+                  from2 = first;
+                }
+              }
+            }
+          }
+        }
+        for (unsigned needm = __ballot_sync(kFull, need); needm;) {
+          const int j = __ffs(needm) - 1;
+          const unsigned long long la = __shfl_sync(kFull, (unsigned long long)(uintptr_t)(lab + from2), j);
+          const int32_t rp = __shfl_sync(kFull, pos + from2, j);
+          const bool mine = need && (unsigned long long)(uintptr_t)(lab + from2) == la && pos + from2 == rp;
+          const unsigned grp = __ballot_sync(kFull, mine);
+          int32_t cmax = mine ? lim - from2 : 0;
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) cmax = max(cmax, __shfl_xor_sync(kFull, cmax, o));
+          const int32_t kk = compare_range<8, true>(reinterpret_cast<const int32_t*>(la), req + rp, 0, cmax, lane);
+          if (mine) {
+            k = from2 + min(kk < 0 ? cmax : kk, lim - from2);
+            need = false;
+          }
+          needm &= ~grp;
+        }
+        if (act) {
+          pos += k;
+          m = pos;
+          if (kLeader && ck && k == ce.w && pos <= climit) *ck = make_int4(pos, nn.x, nn.y, nn.z);
+          act = k == ce.w && pos < len && nn.z > 0 &&
+                find_child_1(trees[p].child + nn.x, tab_bits(nn.y), __ldg(req + pos), ce);
+        }
       }
-      if (p < P && !queued) {
+      if (p < P) {
         out_match[frow + p] = m;
         const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
         best = key > best ? key : best;
@@ -647,56 +644,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
       const unsigned long long other = __shfl_xor_sync(kFull, best, o);
       best = other > best ? other : best;
     }
-    if (lane == 0) {
-      if (pend == 0) {
-        out_peer[f] = 0xFFFF - (int32_t)(best & 0xFFFFull);
-      } else {  // the queue's walks finish the route (drain_kernel)
-        rkey[f] = best;
-        rpend[f] = pend;
-      }
-    }
-  }
-}
-
-// One warp per queued walk {request f, tree p, known prefix c}: the walk, its match, its key merged into the
-// request's; the request's last queued walk writes the route.  kLeader: also the leader's checkpoints.
-template <bool kLeader>
-__global__ void __launch_bounds__(kFollowThreads) drain_kernel(
-    const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
-    int64_t tok_base, const int64_t* __restrict__ offsets, const int4* __restrict__ walks,
-    const int32_t* __restrict__ wcount, int32_t wcap, const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin,
-    int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match,
-    int32_t* __restrict__ out_peer, unsigned long long* rkey, int32_t* rpend, int32_t* err) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
-  const int64_t n = min((int64_t)*wcount, (int64_t)wcap);
-  for (int64_t i = ((int64_t)blockIdx.x * kFollowThreads + threadIdx.x) >> 5; i < n; i += warps) {
-    const int4 w = walks[i];
-    const int64_t f = w.x;
-    const int32_t p = w.y, c = w.z;
-    const int64_t start = __ldg(offsets + f) - tok_base;
-    const int32_t len = (int32_t)min(__ldg(offsets + f + 1) - tok_base - start, (int64_t)INT32_MAX);
-    const int32_t* req = tokens + start;
-    int32_t climit = -1;
-    int4* ck = nullptr;
-    if (kLeader) {
-      const int32_t row = __ldg(gid + f);
-      if (row >= 0) {
-        climit = __ldg(cmin + f);
-        ck = ckpt + (int64_t)row * P + p;
-      }
-    }
-    const int32_t m = walk<8>(trees[p], req, 0, req, len, c, lane, err, climit, ck);
-    if (lane == 0) {
-      out_match[f * P + p] = m;
-      atomicMax(&rkey[f], route_key(m, __ldg(load + p), p, alpha));
-      __threadfence();
-      if (atomicSub(&rpend[f], 1) == 1) {  // the request's last walk: every other key is merged
-        __threadfence();
-        const unsigned long long bk = atomicMax(&rkey[f], 0ull);
-        out_peer[f] = 0xFFFF - (int32_t)(bk & 0xFFFFull);
-      }
-    }
+    if (lane == 0) out_peer[f] = 0xFFFF - (int32_t)(best & 0xFFFFull);
   }
 }
 
@@ -721,7 +669,6 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
   }
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
-  const int drain_grid = num_sms * kFollowCtasPerSm;  // drains read their walk count on the device
   cudaError_t e;
   if (n_tokens >= B * (int64_t)kSlotTokens) {
     // Requests of a staging window or longer on average: the leaders' walks are long compares, which the
@@ -738,28 +685,15 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
     // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
     lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists,
                                                         g->counts, nullptr, nullptr, g->gid, g->cmin, g->ckpt, d_load,
-                                                        alpha, out_match, out_peer, g->walks, g->counts + 3, g->wcap,
-                                                        g->rkey, g->rpend, d_err);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    drain_kernel<true><<<drain_grid, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
-                                                              g->walks, g->counts + 3, g->wcap, g->gid, g->cmin,
-                                                              g->ckpt, d_load, alpha, out_match, out_peer, g->rkey,
-                                                              g->rpend, d_err);
-    *launched = 2;
+                                                        alpha, out_match, out_peer, d_err);
+    *launched = 1;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
                                                        g->counts + 1, g->lead, g->cpre, g->gid, nullptr, g->ckpt, d_load,
-                                                       alpha, out_match, out_peer, g->walks, g->counts + 4, g->wcap,
-                                                       g->rkey, g->rpend, d_err);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  drain_kernel<false><<<drain_grid, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->walks,
-                                                             g->counts + 4, g->wcap, nullptr, nullptr, nullptr, d_load,
-                                                             alpha, out_match, out_peer, g->rkey, g->rpend, d_err);
-  *launched += 2;
+                                                       alpha, out_match, out_peer, d_err);
+  *launched += 1;
   return cudaGetLastError();
 }
 

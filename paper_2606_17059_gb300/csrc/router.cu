@@ -97,7 +97,7 @@ struct p2p_router {
   TreeState* h_states = nullptr;  // pinned, P entries
   DevBuf req_tok, req_off, out_match, out_peer;
   DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_done, d_gather;
-  DevBuf grp_keys, grp_vals, grp_req, grp_ckpt, grp_walk;  // shared-prefix grouping of a batch
+  DevBuf grp_keys, grp_vals, grp_req, grp_ckpt;  // shared-prefix grouping of a batch
   DevBuf cmp_jobs, cmp_queue;          // device compaction
   int64_t launches = 0;  // kernels this router has launched
   // Shared label pool: long labels interned across trees (device array, host mirror, content index).
@@ -167,10 +167,8 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
   const int64_t gcap = std::max<int64_t>(1, std::min<int64_t>(B / 2 + 1, ((int64_t)256 << 20) / ((int64_t)r->P * 16)));
   cudaError_t e = ensure(r, r->grp_keys, (size_t)slots * sizeof(unsigned long long));
   if (e == cudaSuccess) e = ensure(r, r->grp_vals, (size_t)slots * sizeof(int32_t));
-  const int64_t wcap = (int64_t)1 << 22;  // handed-off walks queued per pass (more are walked by their warp)
-  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(7 * B + 5) * sizeof(int32_t));
+  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(7 * B + 3) * sizeof(int32_t));
   if (e == cudaSuccess) e = ensure(r, r->grp_ckpt, (size_t)gcap * r->P * sizeof(int4));
-  if (e == cudaSuccess) e = ensure(r, r->grp_walk, (size_t)wcap * sizeof(int4) + (size_t)B * (sizeof(unsigned long long) + sizeof(int32_t)));
   if (e != cudaSuccess) return e;
   int32_t* q = static_cast<int32_t*>(r->grp_req.p);
   g.keys = static_cast<unsigned long long*>(r->grp_keys.p);
@@ -185,10 +183,6 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
   g.counts = q + 7 * B;
   g.ckpt = static_cast<int4*>(r->grp_ckpt.p);
   g.gcap = (int32_t)gcap;
-  g.walks = static_cast<int4*>(r->grp_walk.p);
-  g.wcap = (int32_t)wcap;
-  g.rkey = reinterpret_cast<unsigned long long*>(g.walks + wcap);
-  g.rpend = reinterpret_cast<int32_t*>(g.rkey + B);
   return cudaSuccess;
 }
 
@@ -683,7 +677,7 @@ void p2p_router_destroy(p2p_router* r) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
-                      &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->grp_walk, &r->cmp_jobs, &r->cmp_queue})
+                      &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
