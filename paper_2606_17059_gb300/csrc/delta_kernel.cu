@@ -44,8 +44,8 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kChunk = 1024;        // ops staged in shared memory at a time
-constexpr int kWide = 64;           // children that make a node an anchor of parallel sub-buckets
-constexpr int kAnchorDepth = 3;     // tree levels the pre-walk descends looking for an anchor
+constexpr int kWide = 8;            // children that make a node an anchor of parallel sub-buckets
+constexpr int kAnchorDepth = 4;     // tree levels the pre-walk descends looking for an anchor
 constexpr int kAnchorSlots = 256;   // distinct anchors per chunk (ops beyond stay in the serial phase)
 constexpr int kSplitOps = 32;       // an anchor with this many ops in a chunk is split by next token
 enum { OP_DONE = 0, OP_NEED = 1, OP_CORRUPT = 2, OP_DEFER = 3 };
