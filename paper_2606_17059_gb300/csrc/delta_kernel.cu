@@ -1030,29 +1030,23 @@ __global__ void init_ranges_kernel(TreeState* states, int32_t nt, const int64_t*
 
 constexpr int kCompactThreads = 512;   // two CTAs per SM: every tree of a 256-tree router at once
 constexpr int kSmallBits = 4;   // tables of at most 16 slots are copied by one thread
+constexpr int kSlotBatch = 4;   // slots of a small table a thread loads before it handles them
 constexpr int kUnitSlots = 1024;  // slots of a big table per unit of warp work
 constexpr int kUnitCap = 2048;    // units queued per level (a table whose units do not fit is copied by a thread)
-
-// One thread copies n tokens, 8 loads in flight before their stores.
-__device__ __forceinline__ void copy_run(int32_t* __restrict__ dst, const int32_t* __restrict__ src, int32_t n) {
-  int32_t t = 0;
-  for (; t + 8 <= n; t += 8) {
-    int32_t x[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) x[u] = src[t + u];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) dst[t + u] = x[u];
-  }
-  for (; t < n; ++t) dst[t] = src[t];
-}
+constexpr int kLabelThreads = 256;  // compact_labels_kernel: CTAs of 8 warps, a warp per 32 new nodes
+constexpr int kLabelCtasPerSm = 8;
 
 struct CompactShared {
-  int node, child, label, tail, fail, nunits;
-  int2 units[kUnitCap];  // (queue index, first slot) of kUnitSlots slots of a big table; queue index -1: none
+  int node, child, label, fail, nunits;
+  int2 units[kUnitCap];  // (new node id, first slot) of kUnitSlots slots of a big table; id -1: none
 };
 
-// Copies queued node q (old id, new id) and its table, one thread.
-__device__ void compact_node_thread(CompactJob& J, CompactShared& S, int2 q, const int4& rec) {
+// Copies the table of node cid (old record rec) into a fresh table of the same size, one thread.  The
+// slots are loaded kSlotBatch at a time; each batch takes its new ids and label space with one reservation,
+// and the thread places its entries by linear probing on a bit mask of the slots it has filled, so the new
+// table is written once, with no read-back.  Labels are not copied here: each child's scratch entry
+// records where its label moves, and compact_labels_kernel moves them all afterwards.
+__device__ void compact_node_thread(CompactJob& J, CompactShared& S, int32_t cid, const int4& rec) {
   const int32_t bits = tab_bits(rec.y);
   int32_t noff = 0, live = 0;
   if (bits) {
@@ -1063,39 +1057,59 @@ __device__ void compact_node_thread(CompactJob& J, CompactShared& S, int2 q, con
       atomicOr(&S.fail, 1);
       return;
     }
-    for (int32_t j = 0; j < size; ++j) J.nchild[noff + j] = make_int4(0, 0, 0, 0);
-    for (int32_t j = 0; j < size; ++j) {
-      const int4 e = J.child[rec.x + j];
-      if (e.y < 1) continue;
-      const int32_t cid = atomicAdd(&S.node, 1);
-      int32_t nz = e.z;
-      if (e.z >= 0) nz = atomicAdd(&S.label, e.w);
-      if (cid >= J.cap_node || (e.z >= 0 && (int64_t)nz + e.w > J.cap_label)) {
+    uint32_t used = 0;
+    for (int32_t j0 = 0; j0 < size; j0 += kSlotBatch) {
+      int4 e[kSlotBatch];
+#pragma unroll
+      for (int u = 0; u < kSlotBatch; ++u)
+        e[u] = j0 + u < size ? __ldg(J.child + rec.x + j0 + u) : make_int4(0, 0, 0, 0);
+      int32_t cnt = 0, tot = 0;
+#pragma unroll
+      for (int u = 0; u < kSlotBatch; ++u)
+        if (e[u].y >= 1) {
+          ++cnt;
+          tot += e[u].z >= 0 ? e[u].w : 0;
+        }
+      if (!cnt) continue;
+      int32_t c = atomicAdd(&S.node, cnt);
+      int32_t nz = tot ? atomicAdd(&S.label, tot) : 0;
+      if ((int64_t)c + cnt > J.cap_node || (int64_t)nz + tot > J.cap_label) {
         atomicOr(&S.fail, 1);
         return;
       }
-      if (e.z >= 0) copy_run(J.nlabel + nz, J.label + e.z, e.w);
-      J.queue[atomicAdd(&S.tail, 1)] = make_int2(e.y, cid);
-      uint32_t sl = slot_hash(e.x, bits);
-      for (uint32_t it = 0; it < mask && J.nchild[noff + sl].y != 0; ++it) sl = (sl + 1) & mask;
-      J.nchild[noff + sl] = make_int4(e.x, cid, nz, e.w);
-      ++live;
+#pragma unroll
+      for (int u = 0; u < kSlotBatch; ++u) {
+        if (e[u].y < 1) continue;
+        const bool own = e[u].z >= 0;
+        const int32_t z = own ? nz : e[u].z;
+        J.queue[c] = make_int4(e[u].y, e[u].z, z, own ? e[u].w : 0);
+        uint32_t sl = slot_hash(e[u].x, bits);
+        while ((used >> sl) & 1u) sl = (sl + 1) & mask;
+        used |= 1u << sl;
+        J.nchild[noff + sl] = make_int4(e[u].x, c, z, e[u].w);
+        ++c;
+        nz += own ? e[u].w : 0;
+        ++live;
+      }
     }
+    for (int32_t j = 0; j < size; ++j)
+      if (!((used >> j) & 1u)) J.nchild[noff + j] = make_int4(0, 0, 0, 0);
   }
-  J.nnode[q.y] = make_int4(noff, make_meta(bits, live), rec.z, rec.w);
+  J.nnode[cid] = make_int4(noff, make_meta(bits, live), rec.z, rec.w);
 }
 
-// Copies slots [start, end) of a big table (node q, old record rec) into its new table at noff, one warp:
-// lane j takes slot base + j, and new ids, queue entries and label offsets of the live slots come from one
-// reservation per 32 slots (ranks and a prefix sum of label lengths); entries go into the new table with a
-// 64-bit compare-and-swap, since other warps fill other ranges of the same table.
+// Copies slots [start, end) of a big table (old record rec) into its new table at noff, one warp: lane j
+// takes slot base + j, and new ids and label space for the live slots come from one reservation per 32
+// slots (ranks and a prefix sum of label lengths); entries go into the new table with a 64-bit
+// compare-and-swap, since other warps fill other ranges of the same table.  As for small tables, the
+// labels themselves move later.
 __device__ void compact_range_warp(CompactJob& J, CompactShared& S, const int4& rec, int32_t noff, int32_t start,
                                    int32_t end, int lane) {
   const int32_t bits = tab_bits(rec.y);
   const uint32_t mask = (1u << bits) - 1;
   for (int32_t base = start; base < end; base += 32) {
     const int32_t j = base + lane;
-    const int4 e = j < end ? J.child[rec.x + j] : make_int4(0, 0, 0, 0);
+    const int4 e = j < end ? __ldg(J.child + rec.x + j) : make_int4(0, 0, 0, 0);
     const bool is_live = j < end && e.y >= 1;
     const unsigned m = __ballot_sync(kFull, is_live);
     if (!m) continue;
@@ -1108,44 +1122,20 @@ __device__ void compact_range_warp(CompactJob& J, CompactShared& S, const int4& 
       if (lane >= o) incl += y;
     }
     const int32_t total = __shfl_sync(kFull, incl, 31);
-    int32_t lbase = 0, nbase = 0, qbase = 0, bad = 0;
+    int32_t lbase = 0, nbase = 0, bad = 0;
     if (lane == 0) {
       lbase = atomicAdd(&S.label, total);
       nbase = atomicAdd(&S.node, cnt);
-      qbase = atomicAdd(&S.tail, cnt);
       bad = (int64_t)lbase + total > J.cap_label || (int64_t)nbase + cnt > J.cap_node;
       if (bad) atomicOr(&S.fail, 1);
     }
     if (__shfl_sync(kFull, bad, 0)) return;
     lbase = __shfl_sync(kFull, lbase, 0);
     nbase = __shfl_sync(kFull, nbase, 0);
-    qbase = __shfl_sync(kFull, qbase, 0);
-    // The 32 slots' own-arena labels as one run of `total` tokens: token i of the run belongs to the first
-    // lane whose inclusive prefix sum exceeds i (a binary search over the lanes, every lane taking part in
-    // the shuffles); lanes move 8 tokens each per step, loads before stores.
-    for (int32_t i0 = 0; i0 < total; i0 += 256) {
-      int32_t x[8], dst[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int32_t i = i0 + u * 32 + lane;
-        int lo = 0;
-#pragma unroll
-        for (int step = 16; step > 0; step >>= 1)
-          if (__shfl_sync(kFull, incl, lo + step - 1) <= i) lo += step;
-        const int32_t k_end = __shfl_sync(kFull, incl, lo & 31), k_w = __shfl_sync(kFull, w, lo & 31);
-        const int32_t k_src = __shfl_sync(kFull, e.z, lo & 31);
-        const bool ok = i < total;
-        x[u] = ok ? J.label[k_src + (i - (k_end - k_w))] : 0;
-        dst[u] = ok ? lbase + i : -1;
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (dst[u] >= 0) J.nlabel[dst[u]] = x[u];
-    }
     if (is_live) {
       const int32_t cid = nbase + rank;
       const int32_t nz = e.z >= 0 ? lbase + incl - w : e.z;
-      J.queue[qbase + rank] = make_int2(e.y, cid);
+      J.queue[cid] = make_int4(e.y, e.z, nz, w);
       const unsigned long long kv = (unsigned long long)(uint32_t)e.x | ((unsigned long long)(uint32_t)cid << 32);
       uint32_t sl = slot_hash(e.x, bits);
       for (uint32_t it = 0; it <= mask; ++it, sl = (sl + 1) & mask) {
@@ -1159,12 +1149,13 @@ __device__ void compact_range_warp(CompactJob& J, CompactShared& S, const int4& 
   }
 }
 
-// One CTA per tree: level-synchronous breadth-first copy from the root.  A thread takes each queued node.
-// A node whose table has more than 2^kSmallBits slots gets its new table range and record from that
-// thread, and its slots are cut into units of kUnitSlots that all warps then zero and fill; smaller tables
-// are copied by the thread.  Every node is queued with a new id below cap_node (checked before the
-// append), so the queue needs cap_node entries.  A big table's record counts its children from the old
-// record (the live-child count), so no pass has to count them.
+// One CTA per tree: level-synchronous breadth-first copy of the structure from the root.  New ids are
+// handed out level by level, so the nodes of the next level are the ids [end, S.node) and the scratch
+// entry of id c (old id, old and new label offsets, own-arena label length) is written by the parent's
+// copy.  A thread takes each node of the level.  A node whose table has more than 2^kSmallBits slots gets
+// its new table range and record from that thread, and its slots are cut into units of kUnitSlots that all
+// warps then zero and fill; smaller tables are copied by the thread.  A big table's record counts its
+// children from the old record (the live-child count), so no pass has to count them.
 __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jobs) {
   CompactJob& J = jobs[blockIdx.x];
   __shared__ CompactShared S;
@@ -1174,17 +1165,15 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jo
     S.node = 1;
     S.child = 0;
     S.label = 0;
-    S.tail = 1;
     S.fail = 0;
     S.nunits = 0;
-    J.queue[0] = make_int2(0, 0);
+    J.queue[0] = make_int4(0, 0, 0, 0);
   }
   __syncthreads();
   int begin = 0, end = 1;
   while (begin < end) {
-    for (int i = begin + threadIdx.x; i < end; i += kCompactThreads) {
-      const int2 q = J.queue[i];
-      const int4 rec = J.node[q.x];
+    for (int cid = begin + threadIdx.x; cid < end; cid += kCompactThreads) {
+      const int4 rec = __ldg(J.node + J.queue[cid].x);
       const int32_t bits = tab_bits(rec.y);
       if (bits > kSmallBits) {
         const int32_t size = 1 << bits, nu = (size + kUnitSlots - 1) / kUnitSlots;
@@ -1196,20 +1185,20 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jo
             for (int k = 0; k < nu; ++k) S.units[u0 + k] = make_int2(-1, 0);
             continue;
           }
-          J.nnode[q.y] = make_int4(noff, make_meta(bits, rec.z), rec.z, rec.w);
-          for (int k = 0; k < nu; ++k) S.units[u0 + k] = make_int2(i, k * kUnitSlots);
+          J.nnode[cid] = make_int4(noff, make_meta(bits, rec.z), rec.z, rec.w);
+          for (int k = 0; k < nu; ++k) S.units[u0 + k] = make_int2(cid, k * kUnitSlots);
           continue;
         }
         for (int k = u0; k < kUnitCap; ++k) S.units[k] = make_int2(-1, 0);  // no room: this thread copies it
       }
-      compact_node_thread(J, S, q, rec);
+      compact_node_thread(J, S, cid, rec);
     }
     __syncthreads();
     const int nunits = min(S.nunits, kUnitCap);
     for (int k = warp; k < nunits; k += kWarps) {  // zero every unit's slots first: inserts may wrap into them
       const int2 u = S.units[k];
       if (u.x < 0) continue;
-      const int4 nrec = J.nnode[J.queue[u.x].y];
+      const int4 nrec = J.nnode[u.x];
       const int32_t n = min(kUnitSlots, (1 << tab_bits(nrec.y)) - u.y);
       for (int32_t j = lane; j < n; j += 32) J.nchild[nrec.x + u.y + j] = make_int4(0, 0, 0, 0);
     }
@@ -1217,15 +1206,14 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jo
     for (int k = warp; k < nunits; k += kWarps) {
       const int2 u = S.units[k];
       if (u.x < 0 || __shfl_sync(kFull, *(volatile int*)&S.fail, 0)) continue;
-      const int2 q = J.queue[u.x];
-      const int4 rec = J.node[q.x];
-      const int32_t noff = J.nnode[q.y].x;
+      const int4 rec = __ldg(J.node + J.queue[u.x].x);
+      const int32_t noff = J.nnode[u.x].x;
       compact_range_warp(J, S, rec, noff, u.y, min(u.y + kUnitSlots, 1 << tab_bits(rec.y)), lane);
     }
     __syncthreads();
     if (threadIdx.x == 0) S.nunits = 0;
     begin = end;
-    end = *(volatile int*)&S.fail ? end : *(volatile int*)&S.tail;
+    end = *(volatile int*)&S.fail ? end : *(volatile int*)&S.node;
     __syncthreads();
   }
   if (threadIdx.x == 0) {
@@ -1233,6 +1221,54 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jo
     J.n_child = S.child;
     J.n_label = S.label;
     J.status = S.fail;
+  }
+}
+
+// Moves the own-arena labels of every compacted tree, after compact_kernel: a warp takes 32 consecutive
+// new ids of one job, whose scratch entries give each label's old and new offsets and length, and copies
+// their labels as one run of `total` tokens.  Token i of the run belongs to the first lane whose inclusive
+// prefix sum of lengths exceeds i (a binary search over the lanes, every lane taking part in the shuffles);
+// lanes move 8 tokens each per step, loads before stores.  Items are (job, group of 32 ids), grid-strided,
+// so one big tree's labels spread over the whole GPU.
+__global__ void __launch_bounds__(kLabelThreads) compact_labels_kernel(const CompactJob* __restrict__ jobs,
+                                                                       int64_t n_items, int32_t groups_per_job) {
+  const int lane = threadIdx.x & 31;
+  const int64_t n_warps = (int64_t)gridDim.x * (kLabelThreads / 32);
+  for (int64_t it = ((int64_t)blockIdx.x * kLabelThreads + threadIdx.x) >> 5; it < n_items; it += n_warps) {
+    const CompactJob& J = jobs[it / groups_per_job];
+    const int32_t c0 = (int32_t)(it % groups_per_job) * 32;
+    if (J.status != 0 || c0 >= J.n_node) continue;
+    const int32_t c = c0 + lane;
+    const int4 s = c < J.n_node ? J.queue[c] : make_int4(0, 0, 0, 0);
+    int32_t incl = s.w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const int32_t total = __shfl_sync(kFull, incl, 31);
+    // Token i of the run, owned by lane k, is old token sbase[k] + i and new token dbase[k] + i.
+    const int32_t sbase = s.y - (incl - s.w), dbase = s.z - (incl - s.w);
+    const int32_t* __restrict__ src = J.label;
+    int32_t* __restrict__ dst = J.nlabel;
+    for (int32_t i0 = 0; i0 < total; i0 += 256) {
+      int32_t x[8], to[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int32_t i = i0 + u * 32 + lane;
+        int lo = 0;
+#pragma unroll
+        for (int step = 16; step > 0; step >>= 1)
+          if (__shfl_sync(kFull, incl, lo + step - 1) <= i) lo += step;
+        const int32_t k_src = __shfl_sync(kFull, sbase, lo & 31), k_dst = __shfl_sync(kFull, dbase, lo & 31);
+        const bool ok = i < total;
+        x[u] = ok ? __ldg(src + k_src + i) : 0;
+        to[u] = ok ? k_dst + i : -1;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (to[u] >= 0) dst[to[u]] = x[u];
+    }
   }
 }
 
@@ -1259,9 +1295,12 @@ cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, i
   return cudaGetLastError();
 }
 
-cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, cudaStream_t st) {
+cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, int32_t max_cap_node, int num_sms, cudaStream_t st) {
   if (n_jobs <= 0) return cudaSuccess;
   compact_kernel<<<n_jobs, kCompactThreads, 0, st>>>(d_jobs);
+  const int32_t groups = (max_cap_node + 31) / 32;
+  compact_labels_kernel<<<std::max(num_sms, 1) * kLabelCtasPerSm, kLabelThreads, 0, st>>>(
+      d_jobs, (int64_t)n_jobs * groups, groups);
   return cudaGetLastError();
 }
 

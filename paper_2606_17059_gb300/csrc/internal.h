@@ -133,13 +133,16 @@ struct CompactJob {
   int4* nnode;  // new arrays and their capacities
   int4* nchild;
   int32_t* nlabel;
-  int2* queue;  // cap_node entries of scratch (a node is queued only with a new id below cap_node)
+  int4* queue;  // cap_node entries of scratch, by new id: (old id, old label offset, new label offset,
+                //   own-arena label length or 0)
   int32_t cap_node, cap_child, cap_label;
   int32_t n_node, n_child, n_label;  // out: the new counts
   int32_t status;                    // out: 0, or 1 if a new array was too small (the job is then void)
   int32_t pad_;
 };
-cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, cudaStream_t st);
+// Two launches: compact_kernel (one CTA per job) copies the structure, then compact_labels_kernel moves the
+// labels of every job over the whole GPU.  max_cap_node bounds every job's cap_node.
+cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, int32_t max_cap_node, int num_sms, cudaStream_t st);
 
 // Home slot of a first token in a children table of 2^bits slots (host table builder and kernels).
 inline __host__ __device__ uint32_t slot_hash(int32_t tok, int32_t bits) {

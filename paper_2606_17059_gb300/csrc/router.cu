@@ -82,6 +82,9 @@ struct p2p_router {
   cudaStream_t stream = nullptr;
   cudaMemPool_t pool = nullptr;
   std::vector<TreeState> hs;  // host mirror of every tree's state
+  // Per tree, a second set of arrays (pointers and capacities) that a device compaction copies the tree
+  // into; the old set then becomes the spare.  Empty when it could not be allocated.
+  std::vector<TreeState> spare;
   TreeView* d_views = nullptr;
   TreeState* d_states = nullptr;
   int32_t* d_load = nullptr;
@@ -387,6 +390,20 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   TreeState nt;
   cudaError_t e = alloc_tree_arrays(r, nt, cap_node, cap_child, cap_label);
   if (e != cudaSuccess) return fail(r, P2P_E_NOMEM, std::string("allocating the tree: ") + cudaGetErrorString(e));
+  // The tree's spare set of arrays, a quarter larger than the live one (deltas grow the tree before it is
+  // compacted): a later device compaction copies the tree into it, so the delta call that compacts maps no
+  // new memory.  Without room for it there is none.
+  TreeState& sp = r->spare[(size_t)peer];
+  const int32_t sp_node = clamp_i32(cap_node + (int64_t)cap_node / 4),
+                sp_child = clamp_i32(cap_child + (int64_t)cap_child / 4),
+                sp_label = clamp_i32(cap_label + (int64_t)cap_label / 4);
+  if (sp.cap_node < sp_node || sp.cap_child < sp_child || sp.cap_label < sp_label) {
+    free_tree_arrays(r, sp);
+    if (alloc_tree_arrays(r, sp, sp_node, sp_child, sp_label) != cudaSuccess) {
+      sp = TreeState{};
+      (void)cudaGetLastError();
+    }
+  }
   CK(cudaMemcpyAsync(nt.node, node.data(), (size_t)N * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   if (slots) CK(cudaMemcpyAsync(nt.child, child.data(), (size_t)slots * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   if (n_own) CK(cudaMemcpyAsync(nt.label, own.data(), (size_t)n_own * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
@@ -520,49 +537,80 @@ int compact_tree(p2p_router* r, int32_t p) {
   return upload_flat(r, p, &v);
 }
 
-// Compacts trees ps on the device (compact_kernel): fresh arrays sized from the live counts with the same
-// headroom as an upload, one CTA per tree, then the states and views of [p0, p1) are republished.  A tree
+// Compacts trees ps on the device: fresh arrays sized from the live counts with the same headroom as an
+// upload; compact_kernel copies each tree's structure (one CTA per tree) and compact_labels_kernel moves all
+// their labels over the whole GPU; then the states and views of [p0, p1) are republished.  A tree
 // whose fresh arrays turn out too small keeps its old arrays and is compacted through the host instead.
 int compact_trees(p2p_router* r, const std::vector<int32_t>& ps, int32_t p0, int32_t p1) {
   if (ps.empty()) return P2P_OK;
   const size_t n = ps.size();
   std::vector<p2p::CompactJob> jobs(n);
   std::vector<TreeState> fresh(n);
+  std::vector<char> from_spare(n, 0);
+  // Fresh arrays that are not used after all: a spare goes back to its tree, the rest to the pool.
+  auto release = [&](size_t j) {
+    if (from_spare[j])
+      r->spare[(size_t)ps[j]] = fresh[j];
+    else
+      free_tree_arrays(r, fresh[j]);
+  };
   std::vector<int64_t> qoff(n);
   int64_t qtotal = 0;
+  int32_t max_cap_node = 0;
   for (size_t i = 0; i < n; ++i) {
     const TreeState& t = r->hs[(size_t)ps[i]];
     const int64_t nodes = std::max<int64_t>((int64_t)t.n_node - t.dead_nodes, 1);
     const int64_t slots = std::max<int64_t>((int64_t)t.n_child - t.stale_child, 0);
     const int64_t own = std::max<int64_t>((int64_t)t.n_label - t.stale_label, 0);
-    cudaError_t e = alloc_tree_arrays(r, fresh[i], clamp_i32(2 * nodes + 1024), clamp_i32(2 * slots + 1024),
-                                      label_cap(own));
-    if (e != cudaSuccess) {
-      for (size_t j = 0; j < i; ++j) free_tree_arrays(r, fresh[j]);
-      return fail(r, P2P_E_NOMEM, std::string("allocating a compacted tree: ") + cudaGetErrorString(e));
+    const int32_t cn = clamp_i32(2 * nodes + 1024), cc = clamp_i32(2 * slots + 1024), cl = label_cap(own);
+    // The spare serves when it holds the live tree with a quarter to spare; growth ahead of later calls
+    // (apply_delta) adds room from there.
+    TreeState& sp = r->spare[(size_t)ps[i]];
+    if (sp.node && sp.cap_node >= nodes + nodes / 4 + 1024 && sp.cap_child >= slots + slots / 4 + 1024 &&
+        sp.cap_label >= own + own / 4 + 65536) {
+      fresh[i] = sp;
+      from_spare[i] = 1;
+      sp = TreeState{};
+    } else {
+      cudaError_t e = alloc_tree_arrays(r, fresh[i], cn, cc, cl);
+      if (e != cudaSuccess) {
+        for (size_t j = 0; j < i; ++j) release(j);
+        return fail(r, P2P_E_NOMEM, std::string("allocating a compacted tree: ") + cudaGetErrorString(e));
+      }
     }
     const TreeState& f = fresh[i];
     jobs[i] = p2p::CompactJob{t.node, t.child, t.label, f.node, f.child, f.label, nullptr,
                               f.cap_node, f.cap_child, f.cap_label, 0, 0, 0, 0, 0};
     qoff[i] = qtotal;
     qtotal += f.cap_node;
+    max_cap_node = std::max(max_cap_node, f.cap_node);
   }
-  CK(ensure(r, r->cmp_queue, (size_t)qtotal * sizeof(int2)));
+  CK(ensure(r, r->cmp_queue, (size_t)qtotal * sizeof(int4)));
   CK(ensure(r, r->cmp_jobs, n * sizeof(p2p::CompactJob)));
-  for (size_t i = 0; i < n; ++i) jobs[i].queue = static_cast<int2*>(r->cmp_queue.p) + qoff[i];
+  for (size_t i = 0; i < n; ++i) jobs[i].queue = static_cast<int4*>(r->cmp_queue.p) + qoff[i];
   CK(cudaMemcpyAsync(r->cmp_jobs.p, jobs.data(), n * sizeof(p2p::CompactJob), cudaMemcpyHostToDevice, r->stream));
-  CK(p2p::launch_compact(static_cast<p2p::CompactJob*>(r->cmp_jobs.p), (int32_t)n, r->stream));
-  r->launches += 1;
+  CK(p2p::launch_compact(static_cast<p2p::CompactJob*>(r->cmp_jobs.p), (int32_t)n, max_cap_node, r->num_sms,
+                         r->stream));
+  r->launches += 2;
   CK(d2h(r, jobs.data(), r->cmp_jobs.p, n * sizeof(p2p::CompactJob)));
   std::vector<int32_t> retry;
   for (size_t i = 0; i < n; ++i) {
     TreeState& t = r->hs[(size_t)ps[i]];
     if (jobs[i].status != 0) {
-      free_tree_arrays(r, fresh[i]);
+      release(i);
       retry.push_back(ps[i]);
       continue;
     }
-    free_tree_arrays(r, t);
+    // The old arrays become the tree's spare (a smaller spare goes back to the pool).
+    TreeState& sp = r->spare[(size_t)ps[i]];
+    free_tree_arrays(r, sp);
+    sp = TreeState{};
+    sp.node = t.node;
+    sp.child = t.child;
+    sp.label = t.label;
+    sp.cap_node = t.cap_node;
+    sp.cap_child = t.cap_child;
+    sp.cap_label = t.cap_label;
     t = fresh[i];
     t.n_node = jobs[i].n_node;
     t.n_child = jobs[i].n_child;
@@ -580,6 +628,15 @@ bool needs_compaction(const TreeState& t) {
   return (t.stale_label > 65536 && 2 * t.stale_label > t.n_label) ||
          (t.stale_child > 65536 && 2 * t.stale_child > t.n_child) ||
          (t.dead_nodes > 16384 && 2 * t.dead_nodes > t.n_node);
+}
+
+// A tree at least 70% of the way to needs_compaction.  When some tree of a call is compacted, these go
+// along in the same launch: replicas that receive deltas at the same rate reach the threshold within a few
+// calls of one another, and one compaction wave costs about as much as one of a handful of trees.
+bool nears_compaction(const TreeState& t) {
+  return (t.stale_label > 45875 && 20 * t.stale_label > 7 * (int64_t)t.n_label) ||
+         (t.stale_child > 45875 && 20 * t.stale_child > 7 * (int64_t)t.n_child) ||
+         (t.dead_nodes > 11468 && 20 * t.dead_nodes > 7 * (int64_t)t.n_node);
 }
 
 // Resets the per-call fields of trees [p0, p1) and copies their states to the device.
@@ -634,6 +691,7 @@ int p2p_router_create(int32_t P, p2p_router** out) {
     return bail(P2P_E_CUDA);
   }
   r->hs.assign((size_t)P, TreeState{});
+  r->spare.assign((size_t)P, TreeState{});
   e = dalloc(r, (void**)&r->d_views, (size_t)P * sizeof(TreeView));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_states, (size_t)P * sizeof(TreeState));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_load, (size_t)P * sizeof(int32_t));
@@ -675,6 +733,7 @@ void p2p_router_destroy(p2p_router* r) {
   cudaStreamSynchronize(r->stream);
   if (r->pool) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
+    for (TreeState& t : r->spare) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
                       &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue})
@@ -916,6 +975,11 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
     const TreeState& t = r->hs[(size_t)p];
     absent += t.n_absent;
     if (needs_compaction(t)) stale.push_back(p);
+  }
+  if (!stale.empty()) {
+    stale.clear();
+    for (int32_t p = p0; p < p1; ++p)
+      if (nears_compaction(r->hs[(size_t)p])) stale.push_back(p);
   }
   if (rc == P2P_OK) rc = compact_trees(r, stale, p0, p1);
   if (n_absent) *n_absent = absent;
