@@ -151,6 +151,9 @@ int p2p_flat_tree_validate(const p2p_flat_tree* t);
 /* Replaces tree `peer` with the full snapshot t (host pointers, copied before return).  This is the
  * receive side of the anti-entropy broadcast: delivering the same snapshot twice gives the same tree
  * (Section 3, "Trie-broadcast loss").  Enqueued on the router stream after earlier routes.
+ * Device memory: the tree's arrays with headroom for deltas, plus a spare set a quarter larger that a
+ * later device compaction copies the tree into (the old set then becomes the spare); the spare is skipped
+ * when there is no room for it.
  * Errors: P2P_E_INVAL (peer), P2P_E_FORMAT (invalid tree; nothing changes), P2P_E_NOMEM, P2P_E_CUDA. */
 int p2p_tree_upload(p2p_router* r, int32_t peer, const p2p_flat_tree* t);
 
@@ -165,7 +168,9 @@ int p2p_tree_download(p2p_router* r, int32_t peer, p2p_snapshot** out);
  * ops peer_begin[p] .. peer_begin[p+1]-1.  INSERT adds one occurrence of the sequence (Section 2,
  * updateTrie / updateTrieEstimate); DELETE removes one occurrence, and is a counted no-op when the
  * sequence is not stored.  Trees stay edge-compressed and canonical.  Runs on the device; the call
- * returns when the delta is applied (device arrays are only read, host arrays are copied).
+ * returns when the delta is applied (device arrays are only read, host arrays are copied).  A tree whose
+ * stale arena space has passed its live space is then compacted on the device, and with it every tree of
+ * the call at least 70% of the way there.
  * *n_absent (nullable) receives the number of no-op DELETEs.
  * Errors: P2P_E_INVAL (bad op code, peer, ranges or segments; nothing changes), P2P_E_NOMEM,
  * P2P_E_CUDA, P2P_E_DEVICE. */

@@ -232,7 +232,7 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   const size_t slots = (size_t)1 << g.bits;
   cudaError_t e = cudaMemsetAsync(g.keys, 0, slots * sizeof(unsigned long long), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g.vals, 0x7f, slots * sizeof(int32_t), st);  // 0x7f7f7f7f > any index
-  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 3 * sizeof(int32_t), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 4 * sizeof(int32_t), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g.gid, 0xff, (size_t)B * sizeof(int32_t), st);   // -1
   if (e == cudaSuccess) e = cudaMemsetAsync(g.cmin, 0x7f, (size_t)B * sizeof(int32_t), st);  // > any prefix
   if (e != cudaSuccess) return e;

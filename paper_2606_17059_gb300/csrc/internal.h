@@ -98,7 +98,7 @@ struct GroupScratch {
   int32_t* lead;     // [B]
   int32_t* cpre;     // [B]
   int32_t* lists;    // [2B]
-  int32_t* counts;   // [3]: leaders, followers, groups with a checkpoint row
+  int32_t* counts;   // [4]: leaders, followers, groups with a checkpoint row, the leader pass's work cursor
   int32_t* gid;      // [B]: a leader's checkpoint row (-1: none)
   int32_t* cmin;     // [B]: a leader's smallest common prefix with its followers
   int4* ckpt;        // [gcap * P]: per (row, tree) the leader's walk state to resume from (see route_kernel.cu)

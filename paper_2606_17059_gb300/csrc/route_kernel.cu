@@ -515,11 +515,21 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
     const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
     const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int32_t* err) {
+    int32_t* err, int32_t* cursor) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
-  for (int64_t i = ((int64_t)blockIdx.x * kFollowThreads + threadIdx.x) >> 5; i < n; i += warps) {
+  // Requests go to warps in a fixed stride, or, with a cursor (zero at launch), one at a time as warps
+  // become free: leaders' walks differ widely in length.  The next index is fetched while the warp
+  // routes the current request.
+  int32_t nxt = 0;
+  int64_t i0 = ((int64_t)blockIdx.x * kFollowThreads + threadIdx.x) >> 5;
+  if (cursor) {
+    if (lane == 0) nxt = atomicAdd(cursor, 1);
+    i0 = __shfl_sync(kFull, nxt, 0);
+  }
+  for (int64_t i = i0; i < n; i = cursor ? (int64_t)__shfl_sync(kFull, nxt, 0) : i + warps) {
+    if (cursor && lane == 0) nxt = atomicAdd(cursor, 1);
     const int64_t f = __ldg(list + i);
     const int64_t start = __ldg(offsets + f) - tok_base, end = __ldg(offsets + f + 1) - tok_base;
     const int64_t frow = f * P;
@@ -685,14 +695,14 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
     // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
     lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists,
                                                         g->counts, nullptr, nullptr, g->gid, g->cmin, g->ckpt, d_load,
-                                                        alpha, out_match, out_peer, d_err);
+                                                        alpha, out_match, out_peer, d_err, g->counts + 3);
     *launched = 1;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
                                                        g->counts + 1, g->lead, g->cpre, g->gid, nullptr, g->ckpt, d_load,
-                                                       alpha, out_match, out_peer, d_err);
+                                                       alpha, out_match, out_peer, d_err, nullptr);
   *launched += 1;
   return cudaGetLastError();
 }

@@ -163,14 +163,14 @@ cudaError_t ensure(p2p_router* r, DevBuf& b, size_t bytes) {
 }
 
 // Scratch of the shared-prefix grouping for a batch of B requests (B <= 2^30): a key table of at least 2B
-// slots; slot_of, lead, cpre (B each), the two request lists (2B), gid and cmin (B each) and three counts;
+// slots; slot_of, lead, cpre (B each), the two request lists (2B), gid and cmin (B each) and four counts;
 // and checkpoint rows, as many as fit in 256 MB (and at most B/2 + 1, one per leader with followers).
 cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
   const int64_t slots = std::max<int64_t>(next_pow2(2 * B), 1024);
   const int64_t gcap = std::max<int64_t>(1, std::min<int64_t>(B / 2 + 1, ((int64_t)256 << 20) / ((int64_t)r->P * 16)));
   cudaError_t e = ensure(r, r->grp_keys, (size_t)slots * sizeof(unsigned long long));
   if (e == cudaSuccess) e = ensure(r, r->grp_vals, (size_t)slots * sizeof(int32_t));
-  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(7 * B + 3) * sizeof(int32_t));
+  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(7 * B + 4) * sizeof(int32_t));
   if (e == cudaSuccess) e = ensure(r, r->grp_ckpt, (size_t)gcap * r->P * sizeof(int4));
   if (e != cudaSuccess) return e;
   int32_t* q = static_cast<int32_t*>(r->grp_req.p);
