@@ -67,52 +67,81 @@ struct Tree {
   int32_t* label;
   const int32_t* shared;  // router-wide pool of interned labels (read-only here)
   TreeState* g;
+  int2* slab;  // this warp's slabs (shared memory): per counter, the next free unit and the units left
   __device__ const int32_t* lab(int32_t off) const { return label_ptr(label, shared, off); }
 };
 
-// Reserves the room an op may need: lanes 0, 1 and 2 bump the node, child-entry and label counters at the
-// same time.  On failure the op does nothing; the units it did get are counted as stale (a later compaction
-// reclaims them), and the request is recorded for the host to grow the arenas.
-__device__ bool reserve(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, int32_t& n0, int32_t& c0, int32_t& l0,
-                        int lane) {
+// Units a warp reserves at a time for its slab of counter c: nodes, child entries, label tokens.
+__device__ __forceinline__ int32_t slab_units(int c) { return c == 0 ? 64 : c == 1 ? 256 : 4096; }
+
+// Reserves k units of counter c (0 nodes, 1 child entries, 2 label tokens) from the tree's counters by
+// compare-and-swap; -1 if they do not fit.  One lane.
+__device__ int32_t reserve_units(const Tree& t, int c, int64_t k) {
+  int32_t* ctr = c == 0 ? &t.g->n_node : c == 1 ? &t.g->n_child : &t.g->n_label;
+  const int32_t cap = c == 0 ? t.g->cap_node : c == 1 ? t.g->cap_child : t.g->cap_label;
+  int32_t old = *(volatile int32_t*)ctr;
+  for (int it = 0; it < (1 << 20); ++it) {
+    if ((int64_t)old + k > cap) return -1;
+    const int32_t prev = atomicCAS(ctr, old, (int32_t)(old + k));
+    if (prev == old) return old;
+    old = prev;
+  }
+  return -1;
+}
+
+// Counts k units of counter c as stale (dead nodes, stale child entries, stale label tokens).  One lane.
+__device__ void add_stale(const Tree& t, int c, int64_t k) {
+  if (k <= 0) return;
+  int64_t* p = c == 0 ? &t.g->dead_nodes : c == 1 ? &t.g->stale_child : &t.g->stale_label;
+  atomicAdd((unsigned long long*)p, (unsigned long long)k);
+}
+
+// Reserves the room an op may need.  Each warp keeps a slab per counter, refilled slab_units(c) units at a
+// time from the tree's counters (lanes 0, 1 and 2 at once), so most ops take their room without a global
+// atomic; a slab's rest is counted as stale when it is replaced and when the warp finishes.  A request of a
+// slab or more, or one whose refill does not fit, is reserved exactly.  On failure the op does nothing:
+// room from a slab stays in it, room reserved exactly is counted as stale (a later compaction reclaims
+// it), and the request is recorded for the host to grow the arenas.
+__device__ bool take(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, int32_t& n0, int32_t& c0, int32_t& l0,
+                     int lane) {
   int32_t r = 0;
+  int2 sl = make_int2(0, 0), ns = make_int2(0, 0);
+  int64_t exact = 0;
+  bool refilled = false;
   if (lane < 3) {
     const int64_t k = lane == 0 ? nodes : lane == 1 ? entries : tokens;
-    if (k) {
-      int32_t* ctr = lane == 0 ? &t.g->n_node : lane == 1 ? &t.g->n_child : &t.g->n_label;
-      const int32_t cap = lane == 0 ? t.g->cap_node : lane == 1 ? t.g->cap_child : t.g->cap_label;
-      r = -1;
-      int32_t old = *(volatile int32_t*)ctr;
-      for (int it = 0; it < (1 << 20); ++it) {
-        if ((int64_t)old + k > cap) break;
-        const int32_t prev = atomicCAS(ctr, old, (int32_t)(old + k));
-        if (prev == old) {
-          r = old;
-          break;
-        }
-        old = prev;
+    sl = t.slab[lane];
+    ns = sl;
+    if (k > 0) {
+      const int32_t S = slab_units(lane);
+      if (k <= sl.y) {
+        r = sl.x;
+        ns = make_int2(sl.x + (int32_t)k, sl.y - (int32_t)k);
+      } else if (k < S && (r = reserve_units(t, lane, S)) >= 0) {
+        add_stale(t, lane, sl.y);
+        refilled = true;
+        ns = make_int2(r + (int32_t)k, S - (int32_t)k);
+      } else {
+        r = reserve_units(t, lane, k);
+        exact = r >= 0 ? k : 0;
       }
     }
   }
   n0 = __shfl_sync(kFull, r, 0);
   c0 = __shfl_sync(kFull, r, 1);
   l0 = __shfl_sync(kFull, r, 2);
-  if (n0 >= 0 && c0 >= 0 && l0 >= 0) return true;
-  if (lane == 0) {
-    if (nodes && n0 >= 0) atomicAdd((unsigned long long*)&t.g->dead_nodes, (unsigned long long)nodes);
-    if (entries && c0 >= 0) atomicAdd((unsigned long long*)&t.g->stale_child, (unsigned long long)entries);
-    if (tokens && l0 >= 0) atomicAdd((unsigned long long*)&t.g->stale_label, (unsigned long long)tokens);
-    atomicOr(&t.g->status, DELTA_NEED_SPACE);
+  const bool ok = n0 >= 0 && c0 >= 0 && l0 >= 0;
+  if (lane < 3) {
+    if (!ok) {
+      if (exact) add_stale(t, lane, exact);
+      ns = refilled ? make_int2(r, slab_units(lane)) : sl;
+    }
+    t.slab[lane] = ns;
   }
-  return false;
-}
-
-// Reserves the room of one op; if it does not fit, records the request so that the host grows the arenas
-// by at least that much before the relaunch.
-__device__ bool take(Tree& t, int64_t nodes, int64_t entries, int64_t tokens, int32_t& n0, int32_t& c0, int32_t& l0,
-                     int lane) {
-  if (reserve(t, nodes, entries, tokens, n0, c0, l0, lane)) return true;
+  __syncwarp();
+  if (ok) return true;
   if (lane == 0) {
+    atomicOr(&t.g->status, DELTA_NEED_SPACE);
     atomicMax(&t.g->need_node, (int32_t)nodes);
     atomicMax(&t.g->need_child, (int32_t)entries);
     atomicMax(&t.g->need_label, (int32_t)(tokens > INT32_MAX ? INT32_MAX : tokens));
@@ -216,17 +245,17 @@ __device__ int32_t only_child(const Tree& t, int32_t off, int32_t bits, int32_t 
   return -1;
 }
 
-// Warp copies: 4 loads per lane in flight before their stores (128 tokens per step).
+// Warp copies: 8 loads per lane in flight before their stores (256 tokens per step).
 __device__ void copy_seq(int32_t* dst, const Seq& q, int64_t from, int64_t n, int lane) {
-  for (int64_t j0 = 0; j0 < n; j0 += 128) {
-    int32_t x[4];
+  for (int64_t j0 = 0; j0 < n; j0 += 256) {
+    int32_t x[8];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       const int64_t j = j0 + u * 32 + lane;
       x[u] = j < n ? q.at(from + j) : 0;
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < 8; ++u) {
       const int64_t j = j0 + u * 32 + lane;
       if (j < n) dst[j] = x[u];
     }
@@ -770,7 +799,9 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   __shared__ int s_any;
   __shared__ MemoEntry s_memo[kDeltaWarps][kMemoSlots];
   __shared__ AnchorEntry s_aentry[kAnchorSlots];
+  __shared__ int2 s_slab[kDeltaWarps][3];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane < 3) s_slab[warp][lane] = make_int2(0, 0);
   TreeState* gs = states + blockIdx.x;
   if (lane < kMemoSlots) s_memo[warp][lane] = MemoEntry{nullptr, nullptr, 0};
   const int64_t op_begin = gs->op_begin, op_end = gs->op_end;
@@ -790,6 +821,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   t.label = gs->label;
   t.shared = shared;
   t.g = gs;
+  t.slab = s_slab[warp];
   const int4 root = t.node[0];  // its table offset and size hold for the whole launch
   int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaWarps + warp) * stride : nullptr;
   Memo memo{s_memo[warp]};  // facts about immutable labels: valid whichever bucket the warp works on
@@ -960,6 +992,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     }
     __syncthreads();
   }
+  if (lane < 3) add_stale(t, lane, t.slab[lane].y);  // the rest of this warp's slabs
 }
 
 // Validates a device-resident delta into header (int32 words: [0..1] longest sequence as u64, [2] error
