@@ -28,7 +28,7 @@
 // them in op order.  Inside an op the warp cooperates: a child lookup probes 32 table slots at once, labels
 // are compared 128 tokens per step and copied 128 per step; lane 0 performs scalar stores and __syncwarp()
 // orders them before later reads.  Adding or removing a child touches one slot (a table is doubled and
-// rehashed when it passes 3/4 occupancy), so the cost of an op does not grow with the fan-out of the nodes
+// rehashed when it passes 1/2 occupancy), so the cost of an op does not grow with the fan-out of the nodes
 // it passes.
 //
 // Space.  Node, child-entry and label arenas are bump-allocated with compare-and-swap on the tree's
@@ -391,12 +391,13 @@ __device__ void fold_child(Tree& t, int32_t x, int4* ex, int32_t yslot, int32_t 
 }
 
 // Room for `extra` more children in node cur's table (cur != 0): grows the table (doubling, rehash into
-// fresh slots) when claimed slots would pass 3/4.  Returns false if the child arena is full.
+// fresh slots) when claimed slots would pass 1/2, to at most 1/4 live load.  Returns false if the child
+// arena is full.
 __device__ bool ensure_room(Tree& t, int32_t cur, int4& nd, int32_t extra, int lane) {
   const int32_t bits = tab_bits(nd.y), used = tab_used(nd.y);
   if (!tab_full(bits, (int64_t)used + extra)) return true;
   int32_t nb = bits ? bits + 1 : kMinTabBits;
-  while (nb < kMaxTabBits && ((int64_t)nd.z + extra) * 2 > ((int64_t)1 << nb)) ++nb;
+  while (nb < kMaxTabBits && ((int64_t)nd.z + extra) * 4 > ((int64_t)1 << nb)) ++nb;
   int32_t n0, c0, l0;
   if (!take(t, 0, (int64_t)1 << nb, 0, n0, c0, l0, lane)) return false;
   zero_slots(t, c0, 1 << nb, lane);
@@ -490,7 +491,7 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
       if (st == 0) {
         if (cur == anchor) {
           // The anchor's table is shared by the parallel phase's warps and was sized for the chunk's
-          // inserts under it: count the claim atomically; a table that would pass 3/4 defers the op.
+          // inserts under it: count the claim atomically; a table that would pass 1/2 defers the op.
           int32_t meta = 0;
           if (lane == 0) meta = atomicAdd(&t.node[cur].y, 1 << 5);
           meta = __shfl_sync(kFull, meta, 0);
@@ -500,7 +501,7 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
           }
         } else if (cur == 0) {
           // The root table is shared by all warps of the tree: count the claim atomically; if the table
-          // would pass 3/4 the host grows it between launches.
+          // would pass 1/2 the host grows it between launches.
           int32_t meta = 0;
           if (lane == 0) meta = atomicAdd(&t.node[0].y, 1 << 5);
           meta = __shfl_sync(kFull, meta, 0);

@@ -73,13 +73,15 @@ constexpr int kDeltaBucketBits = 5;
 constexpr int kDeltaBuckets = 1 << kDeltaBucketBits;
 constexpr int kDeltaWarps = 16;
 
-// Children tables: at least 4 slots; grown (doubled) when claimed slots would pass 3/4 of the table.
+// Children tables: at least 4 slots; grown when claimed slots (live and tombstoned) would pass 1/2 of the
+// table, to at most 1/4 live load.  A lookup of a missing child, the common case for a request that leaves
+// the cached prefixes, then scans about two slots of the linear probe.
 constexpr int kMinTabBits = 2;
 inline __host__ __device__ int32_t tab_bits(int32_t meta) { return meta & 31; }
 inline __host__ __device__ int32_t tab_used(int32_t meta) { return (int32_t)((uint32_t)meta >> 5); }
 inline __host__ __device__ int32_t make_meta(int32_t bits, int32_t used) { return bits | (int32_t)((uint32_t)used << 5); }
 inline __host__ __device__ bool tab_full(int32_t bits, int64_t used_after) {
-  return bits == 0 || used_after * 4 > ((int64_t)3 << bits);
+  return bits == 0 || used_after * 2 > ((int64_t)1 << bits);
 }
 constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits of meta
 

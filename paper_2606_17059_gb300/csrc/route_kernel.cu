@@ -72,7 +72,7 @@ __device__ __forceinline__ int32_t req_at(const int32_t* s_req, int32_t n_s, con
 }
 
 // Child with first token `tok` in the children table of 2^bits slots at tab: one coalesced probe of 32
-// consecutive slots (a table is at most 3/4 full, so the probe run almost always fits).  Returns false if
+// consecutive slots (a table is at most 1/2 full, so the probe run almost always fits).  Returns false if
 // there is no such child.
 __device__ __forceinline__ bool find_child(const int4* __restrict__ tab, int32_t bits, int32_t tok, int lane,
                                            int4& out) {

@@ -58,11 +58,11 @@ uint64_t run_hash(const int32_t* p, int64_t n) {
   return h ^ (h >> 33);
 }
 
-// Children-table sizes (log2 slots): load factor <= 1/2 at upload; the root's table gets extra room (at
-// least 64 slots) because only the host can grow it.
+// Children-table sizes (log2 slots): load factor <= 1/4 at upload (tables grow past 1/2); the root's table
+// gets extra room (at least 64 slots) because only the host can grow it.
 int32_t table_bits_for(int64_t live, bool root) {
-  if (root) return log2_exact(next_pow2(std::max<int64_t>(64, 2 * live + 32)));
-  return live == 0 ? 0 : std::max<int32_t>(p2p::kMinTabBits, log2_exact(next_pow2(2 * live)));
+  if (root) return log2_exact(next_pow2(std::max<int64_t>(64, 4 * live + 64)));
+  return live == 0 ? 0 : std::max<int32_t>(p2p::kMinTabBits, log2_exact(next_pow2(4 * live)));
 }
 
 // Inserts entry e into the table of 2^bits slots at tab (linear probing from its home slot).
