@@ -43,10 +43,11 @@ namespace p2p {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 1024;        // ops staged in shared memory at a time
+constexpr int kChunk = 2048;        // ops staged in shared memory at a time
 constexpr int kWide = 8;            // children that make a node an anchor of parallel sub-buckets
 constexpr int kAnchorDepth = 4;     // tree levels the pre-walk descends looking for an anchor
-constexpr int kAnchorSlots = 256;   // distinct anchors per chunk (ops beyond stay in the serial phase)
+constexpr int kAnchorBits = 9;
+constexpr int kAnchorSlots = 1 << kAnchorBits;  // distinct anchors per chunk (ops beyond stay in the serial phase)
 constexpr int kSplitOps = 32;       // an anchor with this many ops in a chunk is split by next token
 enum { OP_DONE = 0, OP_NEED = 1, OP_CORRUPT = 2, OP_DEFER = 3 };
 enum { F_DONE = 1, F_ANCHORED = 2, F_DEFERRED = 4 };
@@ -781,25 +782,36 @@ __device__ void rank_buckets(const int* count, int* order, int lane) {
   order[rank] = lane;
 }
 
+// Bytes of the delta kernel's dynamic shared memory (the chunk's per-op and per-anchor arrays).
+constexpr int delta_smem_bytes() {
+  return kAnchorSlots * (int)sizeof(AnchorEntry) + (kChunk + 1) * 8 + kChunk * 4 * 2 + kAnchorSlots * 4 * 4 +
+         kChunk * 2 + kChunk * 1 * 2;
+}
+
 __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     delta_kernel(TreeState* states, uint8_t* done, const int32_t* __restrict__ op,
                  const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
                  const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int32_t* gather,
                  int64_t stride, const int32_t* shared) {
-  __shared__ int64_t s_run[kChunk + 1];  // seg_begin of the chunk's ops (and of the op after them)
-  __shared__ int32_t s_anchor[kChunk];   // anchor of an anchored op
-  __shared__ int16_t s_aslot[kChunk];    // its entry in the anchor table
-  __shared__ int8_t s_bucket[kChunk];    // first-token bucket
-  __shared__ int32_t s_next[kChunk];     // an anchored op's token just past its anchor
-  __shared__ uint8_t s_flag[kChunk];     // F_* bits
-  __shared__ int s_akey[kAnchorSlots], s_ains[kAnchorSlots], s_adel[kAnchorSlots], s_aok[kAnchorSlots];
+  // The chunk's per-op and per-anchor arrays, in dynamic shared memory (delta_smem_bytes()).
+  extern __shared__ __align__(16) unsigned char s_dyn[];
+  AnchorEntry* s_aentry = reinterpret_cast<AnchorEntry*>(s_dyn);        // per anchor: its shortcut
+  int64_t* s_run = reinterpret_cast<int64_t*>(s_aentry + kAnchorSlots);  // seg_begin of the chunk's ops (+1)
+  int32_t* s_anchor = reinterpret_cast<int32_t*>(s_run + kChunk + 1);    // anchor of an anchored op
+  int32_t* s_next = s_anchor + kChunk;   // an anchored op's token just past its anchor, then its sub-bucket
+  int* s_akey = s_next + kChunk;         // per anchor slot: the anchor, its inserts, deletes, qualification
+  int* s_ains = s_akey + kAnchorSlots;
+  int* s_adel = s_ains + kAnchorSlots;
+  int* s_aok = s_adel + kAnchorSlots;
+  int16_t* s_aslot = reinterpret_cast<int16_t*>(s_aok + kAnchorSlots);  // an op's entry in the anchor table
+  int8_t* s_bucket = reinterpret_cast<int8_t*>(s_aslot + kChunk);       // first-token bucket
+  uint8_t* s_flag = reinterpret_cast<uint8_t*>(s_bucket + kChunk);      // F_* bits
   __shared__ int s_count[kDeltaBuckets];
   __shared__ int s_order[kDeltaBuckets];
   __shared__ int s_stop[kDeltaBuckets];  // first-token buckets held back for the rest of the launch
   __shared__ int s_take;
   __shared__ int s_any;
   __shared__ MemoEntry s_memo[kDeltaWarps][kMemoSlots];
-  __shared__ AnchorEntry s_aentry[kAnchorSlots];
   __shared__ int2 s_slab[kDeltaWarps][3];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (lane < 3) s_slab[warp][lane] = make_int2(0, 0);
@@ -858,7 +870,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
         int32_t anchor, next_tok;
         find_anchor(t, root, seg_off, seg_len, pool, g0, g1, n, anchor, next_tok);
         if (anchor >= 0) {
-          uint32_t h = ((uint32_t)anchor * 2654435761u) >> 24;
+          uint32_t h = ((uint32_t)anchor * 2654435761u) >> (32 - kAnchorBits);
           int slot = -1;
           for (int it = 0; it < kAnchorSlots; ++it, h = (h + 1) & (kAnchorSlots - 1)) {
             const int prev = atomicCAS(&s_akey[h], -1, anchor);
@@ -1342,8 +1354,11 @@ cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, co
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st) {
   if (n_trees <= 0) return cudaSuccess;
-  delta_kernel<<<n_trees, kDeltaWarps * 32, 0, st>>>(d_states, done, op, seg_begin, seg_off, seg_len, pool, gather,
-                                                     gather_stride, shared);
+  const int dyn = delta_smem_bytes();
+  cudaError_t e = cudaFuncSetAttribute(delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+  if (e != cudaSuccess) return e;
+  delta_kernel<<<n_trees, kDeltaWarps * 32, dyn, st>>>(d_states, done, op, seg_begin, seg_off, seg_len, pool, gather,
+                                                       gather_stride, shared);
   return cudaGetLastError();
 }
 
