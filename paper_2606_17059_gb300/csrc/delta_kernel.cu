@@ -43,11 +43,10 @@ namespace p2p {
 namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
-constexpr int kChunk = 2048;        // ops staged in shared memory at a time
+constexpr int kChunk = 3072;        // ops staged in shared memory at a time
 constexpr int kWide = 8;            // children that make a node an anchor of parallel sub-buckets
 constexpr int kAnchorDepth = 4;     // tree levels the pre-walk descends looking for an anchor
-constexpr int kAnchorBits = 9;
-constexpr int kAnchorSlots = 1 << kAnchorBits;  // distinct anchors per chunk (ops beyond stay in the serial phase)
+constexpr int kAnchorSlots = 768;  // distinct anchors per chunk (ops beyond stay in the serial phase)
 constexpr int kSplitOps = 32;       // an anchor with this many ops in a chunk is split by next token
 enum { OP_DONE = 0, OP_NEED = 1, OP_CORRUPT = 2, OP_DEFER = 3 };
 enum { F_DONE = 1, F_ANCHORED = 2, F_DEFERRED = 4 };
@@ -870,9 +869,9 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
         int32_t anchor, next_tok;
         find_anchor(t, root, seg_off, seg_len, pool, g0, g1, n, anchor, next_tok);
         if (anchor >= 0) {
-          uint32_t h = ((uint32_t)anchor * 2654435761u) >> (32 - kAnchorBits);
+          uint32_t h = (uint32_t)(((uint64_t)((uint32_t)anchor * 2654435761u) * kAnchorSlots) >> 32);
           int slot = -1;
-          for (int it = 0; it < kAnchorSlots; ++it, h = (h + 1) & (kAnchorSlots - 1)) {
+          for (int it = 0; it < kAnchorSlots; ++it, h = h + 1 == kAnchorSlots ? 0 : h + 1) {
             const int prev = atomicCAS(&s_akey[h], -1, anchor);
             if (prev == -1 || prev == anchor) {
               slot = (int)h;
