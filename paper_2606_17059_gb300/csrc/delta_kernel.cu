@@ -44,7 +44,7 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr int kChunk = 3072;        // ops staged in shared memory at a time
-constexpr int kWide = 8;            // children that make a node an anchor of parallel sub-buckets
+constexpr int kWide = 4;            // children that make a node an anchor of parallel sub-buckets
 constexpr int kAnchorDepth = 4;     // tree levels the pre-walk descends looking for an anchor
 constexpr int kAnchorSlots = 768;  // distinct anchors per chunk (ops beyond stay in the serial phase)
 constexpr int kSplitOps = 32;       // an anchor with this many ops in a chunk is split by next token
