@@ -502,12 +502,94 @@ __device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab,
   return lim;
 }
 
-// One warp per request list[i], i < *count; lane j walks trees j, j + 32, ...
-//   kLeader: the request is a group leader (or ungrouped): whole walks, and for a leader with a checkpoint
-//   row, the checkpoints its followers resume from.
+// Advances the walks of a warp's lanes edge by edge until none is left (collective: every lane of the warp
+// calls it).  Lane state: tree p, the edge ce to walk at position pos (act), m = tokens matched so far,
+// known = tokens known to match without comparing, and for leaders the checkpoint slot ck (NULL: none)
+// with the deepest position climit it records.  A lane compares an edge's label itself when it leaves
+// within the first 8 tokens or the edge has at most kThreadSpan tokens left; longer compares are done by
+// the whole warp, once per distinct (label address, request position): the long prompt prefixes are
+// interned labels shared by many trees, so one compare serves every lane at that label.
+template <bool kLeader>
+__device__ __forceinline__ void lane_walks(const TreeView* __restrict__ trees, int32_t p, const int32_t* req,
+                                           int32_t len, int32_t known, bool act, int4 ce, int32_t& pos, int32_t& m,
+                                           int4* ck, int32_t climit, int lane, int32_t* err) {
+  while (__ballot_sync(kFull, act)) {
+    int4 nn = make_int4(0, 0, 0, 0);
+    int32_t k = 0, lim = 0, from2 = 0;
+    const int32_t* lab = nullptr;
+    bool need = false;
+    if (act) {
+      if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree
+        atomicOr(err, ERR_CORRUPT_TREE);
+        act = false;
+      } else {
+        nn = __ldg(trees[p].node + ce.y);
+        lab = label_ptr(trees[p].label, trees[p].shared, ce.z);
+        lim = min(ce.w, len - pos);
+        const int32_t from = max(1, known - pos);
+        k = lim;
+        if (from < lim) {
+          const int32_t first = min(lim, from + 8);
+          k = first_diff_1(lab, req + pos, from, first);
+          if (k == first && first < lim) {
+            if (lim - first <= kThreadSpan) {
+              k = first_diff_1(lab, req + pos, first, lim);
+            } else {
+              need = true;
+              from2 = first;
+            }
+          }
+        }
+      }
+    }
+    for (unsigned needm = __ballot_sync(kFull, need); needm;) {
+      const int j = __ffs(needm) - 1;
+      const unsigned long long la = __shfl_sync(kFull, (unsigned long long)(uintptr_t)(lab + from2), j);
+      const int32_t rp = __shfl_sync(kFull, pos + from2, j);
+      const bool mine = need && (unsigned long long)(uintptr_t)(lab + from2) == la && pos + from2 == rp;
+      const unsigned grp = __ballot_sync(kFull, mine);
+      int32_t cmax = mine ? lim - from2 : 0;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) cmax = max(cmax, __shfl_xor_sync(kFull, cmax, o));
+      const int32_t kk = compare_range<8, true>(reinterpret_cast<const int32_t*>(la), req + rp, 0, cmax, lane);
+      if (mine) {
+        k = from2 + min(kk < 0 ? cmax : kk, lim - from2);
+        need = false;
+      }
+      needm &= ~grp;
+    }
+    if (act) {
+      pos += k;
+      m = pos;
+      if (kLeader && ck && k == ce.w && pos <= climit) *ck = make_int4(pos, nn.x, nn.y, nn.z);
+      act = k == ce.w && pos < len && nn.z > 0 &&
+            find_child_1(trees[p].child + nn.x, tab_bits(nn.y), __ldg(req + pos), ce);
+    }
+  }
+}
+
+// The first two slots of the linear probe for tok in a table of 2^bits slots at tab (bits >= 2): 1 with
+// e = the child, 0 if the child is absent, -1 if both slots hold other keys (the probe continues).
+__device__ __forceinline__ int probe_first2(const int4& a, const int4& b, int32_t tok, int4& e) {
+  if (a.y >= 1 && a.x == tok) {
+    e = a;
+    return 1;
+  }
+  if (a.y == 0) return 0;
+  if (b.y >= 1 && b.x == tok) {
+    e = b;
+    return 1;
+  }
+  return b.y == 0 ? 0 : -1;
+}
+
+// One warp per request list[i], i < *count.
+//   kLeader: the request is a group leader (or ungrouped): lane j walks trees j, j + 32, ..., and for a
+//   leader with a checkpoint row records the checkpoints its followers resume from.
 //   !kLeader: the request follows leader lead[f] with common prefix c = cpre[f]: match(f, T) = match(lead,
 //   T) if that is < c, else a walk resumed at the leader's checkpoint that does not compare f's first c
-//   tokens.
+//   tokens.  A lane takes two trees at a time (p and p + 32): the leader's matches, the checkpoints and the
+//   first probe step of both are loaded before either is looked at.
 template <bool kLeader>
 __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
@@ -543,110 +625,90 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     }
     const int32_t* req = tokens + start;
     const int32_t len = (int32_t)min(end - start, (int64_t)INT32_MAX);
-    int32_t c = 0, climit = -1;
-    int64_t lrow = 0;
-    int32_t row;
-    if (kLeader) {
-      row = __ldg(gid + f);
-      climit = row >= 0 ? __ldg(cmin + f) : -1;
-    } else {
-      c = __ldg(cpre + f);
-      const int32_t l = __ldg(lead + f);
-      row = __ldg(gid + l);
-      lrow = (int64_t)l * P;
-    }
     unsigned long long best = 0;
-    for (int32_t p0 = 0; p0 < P; p0 += 32) {
-      const int32_t p = p0 + lane;
-      int32_t m = 0, pos = 0, known = c;
-      bool act = false;  // the lane has an edge to walk (ce, at position pos)
-      int4 ce = make_int4(0, 0, 0, 0);
-      int4* ck = nullptr;
-      if (p < P && len > 0) {
-        int4 start = root_checkpoint(trees[p]);
-        bool walk_it = true;
-        if (kLeader) {
+    if constexpr (kLeader) {
+      const int32_t row = __ldg(gid + f);
+      const int32_t climit = row >= 0 ? __ldg(cmin + f) : -1;
+      for (int32_t p0 = 0; p0 < P; p0 += 32) {
+        const int32_t p = p0 + lane;
+        int32_t m = 0, pos = 0;
+        bool act = false;  // the lane has an edge to walk (ce, at position pos)
+        int4 ce = make_int4(0, 0, 0, 0);
+        int4* ck = nullptr;
+        if (p < P && len > 0) {
+          const int4 st = root_checkpoint(trees[p]);
           if (row >= 0) {
             ck = ckpt + (int64_t)row * P + p;
-            *ck = start;
+            *ck = st;
           }
-        } else {
-          const int32_t ml = out_match[lrow + p];  // the leaders' pass has finished
-          if (ml < c || c >= len) {
-            m = ml < c ? ml : len;
-            walk_it = false;
-          } else if (row >= 0) {
-            start = ckpt[(int64_t)row * P + p];
-          }
+          act = st.w > 0 && find_child_1(trees[p].child + st.y, tab_bits(st.z), __ldg(req), ce);
         }
-        if (walk_it) {
-          pos = min(start.x, len);
-          m = pos;
-          act = pos < len && start.w > 0 &&
-                find_child_1(trees[p].child + start.y, tab_bits(start.z), __ldg(req + pos), ce);
+        lane_walks<true>(trees, p, req, len, 0, act, ce, pos, m, ck, climit, lane, err);
+        if (p < P) {
+          out_match[frow + p] = m;
+          const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
+          best = key > best ? key : best;
         }
       }
-      // The walks advance edge by edge.  A lane compares an edge's label itself when it leaves within the
-      // first 8 tokens or the edge has at most kThreadSpan tokens left; longer compares are done by the
-      // whole warp, once per distinct (label address, request position): the long prompt prefixes are
-      // interned labels shared by many trees, so one compare serves every lane at that label.
-      while (__ballot_sync(kFull, act)) {
-        int4 nn = make_int4(0, 0, 0, 0);
-        int32_t k = 0, lim = 0, from2 = 0;
-        const int32_t* lab = nullptr;
-        bool need = false;
-        if (act) {
-          if (ce.w <= 0 || ce.y <= 0) {  // cannot happen in a valid tree
-            atomicOr(err, ERR_CORRUPT_TREE);
-            act = false;
-          } else {
-            nn = __ldg(trees[p].node + ce.y);
-            lab = label_ptr(trees[p].label, trees[p].shared, ce.z);
-            lim = min(ce.w, len - pos);
-            const int32_t from = max(1, known - pos);
-            k = lim;
-            if (from < lim) {
-              const int32_t first = min(lim, from + 8);
-              k = first_diff_1(lab, req + pos, from, first);
-              if (k == first && first < lim) {
-                if (lim - first <= kThreadSpan) {
-                  k = first_diff_1(lab, req + pos, first, lim);
-                } else {
-                  need = true;
-                  from2 = first;
-                }
-              }
-            }
-          }
+    } else {
+      const int32_t c = __ldg(cpre + f);
+      const int32_t l = __ldg(lead + f);
+      const int32_t row = __ldg(gid + l);
+      const int64_t lrow = (int64_t)l * P;  // the leaders' pass has finished: the leader's row is final
+      const int4* ckrow = ckpt + (int64_t)(row >= 0 ? row : 0) * P;
+      for (int32_t p0 = 0; p0 < P; p0 += 64) {
+        const int32_t pa = p0 + lane, pb = p0 + 32 + lane;
+        const int32_t mla = pa < P ? out_match[lrow + pa] : 0;
+        const int32_t mlb = pb < P ? out_match[lrow + pb] : 0;
+        const bool wa = pa < P && len > 0 && mla >= c && c < len;
+        const bool wb = pb < P && len > 0 && mlb >= c && c < len;
+        int4 sa = make_int4(0, 0, 0, 0), sb = make_int4(0, 0, 0, 0);
+        if (wa) sa = row >= 0 ? ckrow[pa] : root_checkpoint(trees[pa]);
+        if (wb) sb = row >= 0 ? ckrow[pb] : root_checkpoint(trees[pb]);
+        int32_t posa = min(sa.x, len), posb = min(sb.x, len);
+        int32_t ma = wa ? posa : len == 0 ? 0 : mla < c ? mla : len;
+        int32_t mb = wb ? posb : len == 0 ? 0 : mlb < c ? mlb : len;
+        bool acta = wa && posa < len && sa.w > 0 && tab_bits(sa.z) > 0;
+        bool actb = wb && posb < len && sb.w > 0 && tab_bits(sb.z) > 0;
+        const int32_t ta = acta ? __ldg(req + posa) : 0, tb = actb ? __ldg(req + posb) : 0;
+        int4 a0 = make_int4(0, 0, 0, 0), a1 = a0, b0 = a0, b1 = a0;
+        const int4* taba = nullptr;
+        const int4* tabb = nullptr;
+        if (acta) {
+          const int32_t bits = tab_bits(sa.z);
+          const uint32_t mask = (1u << bits) - 1, h = slot_hash(ta, bits);
+          taba = trees[pa].child + sa.y;
+          a0 = __ldg(taba + h);
+          a1 = __ldg(taba + ((h + 1) & mask));
         }
-        for (unsigned needm = __ballot_sync(kFull, need); needm;) {
-          const int j = __ffs(needm) - 1;
-          const unsigned long long la = __shfl_sync(kFull, (unsigned long long)(uintptr_t)(lab + from2), j);
-          const int32_t rp = __shfl_sync(kFull, pos + from2, j);
-          const bool mine = need && (unsigned long long)(uintptr_t)(lab + from2) == la && pos + from2 == rp;
-          const unsigned grp = __ballot_sync(kFull, mine);
-          int32_t cmax = mine ? lim - from2 : 0;
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) cmax = max(cmax, __shfl_xor_sync(kFull, cmax, o));
-          const int32_t kk = compare_range<8, true>(reinterpret_cast<const int32_t*>(la), req + rp, 0, cmax, lane);
-          if (mine) {
-            k = from2 + min(kk < 0 ? cmax : kk, lim - from2);
-            need = false;
-          }
-          needm &= ~grp;
+        if (actb) {
+          const int32_t bits = tab_bits(sb.z);
+          const uint32_t mask = (1u << bits) - 1, h = slot_hash(tb, bits);
+          tabb = trees[pb].child + sb.y;
+          b0 = __ldg(tabb + h);
+          b1 = __ldg(tabb + ((h + 1) & mask));
         }
-        if (act) {
-          pos += k;
-          m = pos;
-          if (kLeader && ck && k == ce.w && pos <= climit) *ck = make_int4(pos, nn.x, nn.y, nn.z);
-          act = k == ce.w && pos < len && nn.z > 0 &&
-                find_child_1(trees[p].child + nn.x, tab_bits(nn.y), __ldg(req + pos), ce);
+        int4 cea = make_int4(0, 0, 0, 0), ceb = cea;
+        if (acta) {
+          const int r = probe_first2(a0, a1, ta, cea);
+          acta = r > 0 || (r < 0 && find_child_1(taba, tab_bits(sa.z), ta, cea));
         }
-      }
-      if (p < P) {
-        out_match[frow + p] = m;
-        const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
-        best = key > best ? key : best;
+        if (actb) {
+          const int r = probe_first2(b0, b1, tb, ceb);
+          actb = r > 0 || (r < 0 && find_child_1(tabb, tab_bits(sb.z), tb, ceb));
+        }
+        lane_walks<false>(trees, pa, req, len, c, acta, cea, posa, ma, nullptr, -1, lane, err);
+        lane_walks<false>(trees, pb, req, len, c, actb, ceb, posb, mb, nullptr, -1, lane, err);
+        if (pa < P) {
+          out_match[frow + pa] = ma;
+          const unsigned long long key = route_key(ma, __ldg(load + pa), pa, alpha);
+          best = key > best ? key : best;
+        }
+        if (pb < P) {
+          out_match[frow + pb] = mb;
+          const unsigned long long key = route_key(mb, __ldg(load + pb), pb, alpha);
+          best = key > best ? key : best;
+        }
       }
     }
 #pragma unroll
