@@ -461,6 +461,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
 constexpr int kFollowThreads = 256;
 constexpr int kFollowCtasPerSm = 4;
 constexpr int kThreadSpan = 64;
+constexpr int kFollowIlp = 2;  // trees a follower's lane takes per iteration (their first loads overlap; 3 or 4 spill)
 
 // One thread: the child with first token tok in a table of 2^bits (>= 4, even) slots, two slots per step of
 // the linear probe.  Returns false if there is none.
@@ -588,7 +589,7 @@ __device__ __forceinline__ int probe_first2(const int4& a, const int4& b, int32_
 //   leader with a checkpoint row records the checkpoints its followers resume from.
 //   !kLeader: the request follows leader lead[f] with common prefix c = cpre[f]: match(f, T) = match(lead,
 //   T) if that is < c, else a walk resumed at the leader's checkpoint that does not compare f's first c
-//   tokens.  A lane takes two trees at a time (p and p + 32): the leader's matches, the checkpoints and the
+//   tokens.  A lane takes kFollowIlp trees at a time (p, p + 32, ...): the leader's matches, the checkpoints and the
 //   first probe step of both are loaded before either is looked at.
 template <bool kLeader>
 __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
@@ -656,58 +657,54 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
       const int32_t row = __ldg(gid + l);
       const int64_t lrow = (int64_t)l * P;  // the leaders' pass has finished: the leader's row is final
       const int4* ckrow = ckpt + (int64_t)(row >= 0 ? row : 0) * P;
-      for (int32_t p0 = 0; p0 < P; p0 += 64) {
-        const int32_t pa = p0 + lane, pb = p0 + 32 + lane;
-        const int32_t mla = pa < P ? out_match[lrow + pa] : 0;
-        const int32_t mlb = pb < P ? out_match[lrow + pb] : 0;
-        const bool wa = pa < P && len > 0 && mla >= c && c < len;
-        const bool wb = pb < P && len > 0 && mlb >= c && c < len;
-        int4 sa = make_int4(0, 0, 0, 0), sb = make_int4(0, 0, 0, 0);
-        if (wa) sa = row >= 0 ? ckrow[pa] : root_checkpoint(trees[pa]);
-        if (wb) sb = row >= 0 ? ckrow[pb] : root_checkpoint(trees[pb]);
-        int32_t posa = min(sa.x, len), posb = min(sb.x, len);
-        int32_t ma = wa ? posa : len == 0 ? 0 : mla < c ? mla : len;
-        int32_t mb = wb ? posb : len == 0 ? 0 : mlb < c ? mlb : len;
-        bool acta = wa && posa < len && sa.w > 0 && tab_bits(sa.z) > 0;
-        bool actb = wb && posb < len && sb.w > 0 && tab_bits(sb.z) > 0;
-        const int32_t ta = acta ? __ldg(req + posa) : 0, tb = actb ? __ldg(req + posb) : 0;
-        int4 a0 = make_int4(0, 0, 0, 0), a1 = a0, b0 = a0, b1 = a0;
-        const int4* taba = nullptr;
-        const int4* tabb = nullptr;
-        if (acta) {
-          const int32_t bits = tab_bits(sa.z);
-          const uint32_t mask = (1u << bits) - 1, h = slot_hash(ta, bits);
-          taba = trees[pa].child + sa.y;
-          a0 = __ldg(taba + h);
-          a1 = __ldg(taba + ((h + 1) & mask));
+      for (int32_t p0 = 0; p0 < P; p0 += 32 * kFollowIlp) {
+        int32_t pt[kFollowIlp], ml[kFollowIlp], pos[kFollowIlp], m[kFollowIlp], tk[kFollowIlp];
+        bool act[kFollowIlp];
+        int4 st[kFollowIlp], e0[kFollowIlp], e1[kFollowIlp], ce[kFollowIlp];
+        const int4* tab[kFollowIlp];
+#pragma unroll
+        for (int g = 0; g < kFollowIlp; ++g) {
+          pt[g] = p0 + 32 * g + lane;
+          ml[g] = pt[g] < P ? out_match[lrow + pt[g]] : 0;
         }
-        if (actb) {
-          const int32_t bits = tab_bits(sb.z);
-          const uint32_t mask = (1u << bits) - 1, h = slot_hash(tb, bits);
-          tabb = trees[pb].child + sb.y;
-          b0 = __ldg(tabb + h);
-          b1 = __ldg(tabb + ((h + 1) & mask));
+#pragma unroll
+        for (int g = 0; g < kFollowIlp; ++g) {
+          const bool w = pt[g] < P && len > 0 && ml[g] >= c && c < len;
+          st[g] = make_int4(0, 0, 0, 0);
+          if (w) st[g] = row >= 0 ? ckrow[pt[g]] : root_checkpoint(trees[pt[g]]);
+          pos[g] = min(st[g].x, len);
+          m[g] = w ? pos[g] : len == 0 ? 0 : ml[g] < c ? ml[g] : len;
+          act[g] = w && pos[g] < len && st[g].w > 0 && tab_bits(st[g].z) > 0;
         }
-        int4 cea = make_int4(0, 0, 0, 0), ceb = cea;
-        if (acta) {
-          const int r = probe_first2(a0, a1, ta, cea);
-          acta = r > 0 || (r < 0 && find_child_1(taba, tab_bits(sa.z), ta, cea));
+#pragma unroll
+        for (int g = 0; g < kFollowIlp; ++g) tk[g] = act[g] ? __ldg(req + pos[g]) : 0;
+#pragma unroll
+        for (int g = 0; g < kFollowIlp; ++g) {
+          e0[g] = e1[g] = ce[g] = make_int4(0, 0, 0, 0);
+          tab[g] = nullptr;
+          if (act[g]) {
+            const int32_t bits = tab_bits(st[g].z);
+            const uint32_t mask = (1u << bits) - 1, h = slot_hash(tk[g], bits);
+            tab[g] = trees[pt[g]].child + st[g].y;
+            e0[g] = __ldg(tab[g] + h);
+            e1[g] = __ldg(tab[g] + ((h + 1) & mask));
+          }
         }
-        if (actb) {
-          const int r = probe_first2(b0, b1, tb, ceb);
-          actb = r > 0 || (r < 0 && find_child_1(tabb, tab_bits(sb.z), tb, ceb));
+#pragma unroll
+        for (int g = 0; g < kFollowIlp; ++g) {
+          if (act[g]) {
+            const int r = probe_first2(e0[g], e1[g], tk[g], ce[g]);
+            act[g] = r > 0 || (r < 0 && find_child_1(tab[g], tab_bits(st[g].z), tk[g], ce[g]));
+          }
         }
-        lane_walks<false>(trees, pa, req, len, c, acta, cea, posa, ma, nullptr, -1, lane, err);
-        lane_walks<false>(trees, pb, req, len, c, actb, ceb, posb, mb, nullptr, -1, lane, err);
-        if (pa < P) {
-          out_match[frow + pa] = ma;
-          const unsigned long long key = route_key(ma, __ldg(load + pa), pa, alpha);
-          best = key > best ? key : best;
-        }
-        if (pb < P) {
-          out_match[frow + pb] = mb;
-          const unsigned long long key = route_key(mb, __ldg(load + pb), pb, alpha);
-          best = key > best ? key : best;
+#pragma unroll
+        for (int g = 0; g < kFollowIlp; ++g) {
+          lane_walks<false>(trees, pt[g], req, len, c, act[g], ce[g], pos[g], m[g], nullptr, -1, lane, err);
+          if (pt[g] < P) {
+            out_match[frow + pt[g]] = m[g];
+            const unsigned long long key = route_key(m[g], __ldg(load + pt[g]), pt[g], alpha);
+            best = key > best ? key : best;
+          }
         }
       }
     }
