@@ -589,8 +589,8 @@ __device__ __forceinline__ int probe_first2(const int4& a, const int4& b, int32_
 //   leader with a checkpoint row records the checkpoints its followers resume from.
 //   !kLeader: the request follows leader lead[f] with common prefix c = cpre[f]: match(f, T) = match(lead,
 //   T) if that is < c, else a walk resumed at the leader's checkpoint that does not compare f's first c
-//   tokens.  A lane takes kFollowIlp trees at a time (p, p + 32, ...): the leader's matches, the checkpoints and the
-//   first probe step of both are loaded before either is looked at.
+//   tokens.  A lane takes kFollowIlp trees at a time (p, p + 32, ...): the leader's matches, the
+//   checkpoints and the first probe step of each are loaded before any of them is looked at.
 template <bool kLeader>
 __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
