@@ -1271,10 +1271,11 @@ __global__ void __launch_bounds__(kCompactThreads) compact_kernel(CompactJob* jo
 
 // Moves the own-arena labels of every compacted tree, after compact_kernel: a warp takes 32 consecutive
 // new ids of one job, whose scratch entries give each label's old and new offsets and length, and copies
-// their labels as one run of `total` tokens.  Token i of the run belongs to the first lane whose inclusive
-// prefix sum of lengths exceeds i (a binary search over the lanes, every lane taking part in the shuffles);
-// lanes move 8 tokens each per step, loads before stores.  Items are (job, group of 32 ids), grid-strided,
-// so one big tree's labels spread over the whole GPU.
+// the labels with all 32 lanes, kLabelsInFlight labels at a time, kLabelSteps coalesced loads per lane
+// and label in flight (most own-arena labels are under 128 tokens: one round).  Items are (job, group
+// of 32 ids), grid-strided, so one big tree's labels spread over the whole GPU.
+constexpr int kLabelSteps = 4;
+constexpr int kLabelsInFlight = 4;
 __global__ void __launch_bounds__(kLabelThreads) compact_labels_kernel(const CompactJob* __restrict__ jobs,
                                                                        int64_t n_items, int32_t groups_per_job) {
   const int lane = threadIdx.x & 31;
@@ -1285,34 +1286,35 @@ __global__ void __launch_bounds__(kLabelThreads) compact_labels_kernel(const Com
     if (J.status != 0 || c0 >= J.n_node) continue;
     const int32_t c = c0 + lane;
     const int4 s = c < J.n_node ? J.queue[c] : make_int4(0, 0, 0, 0);
-    int32_t incl = s.w;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int32_t y = __shfl_up_sync(kFull, incl, o);
-      if (lane >= o) incl += y;
-    }
-    const int32_t total = __shfl_sync(kFull, incl, 31);
-    // Token i of the run, owned by lane k, is old token sbase[k] + i and new token dbase[k] + i.
-    const int32_t sbase = s.y - (incl - s.w), dbase = s.z - (incl - s.w);
     const int32_t* __restrict__ src = J.label;
     int32_t* __restrict__ dst = J.nlabel;
-    for (int32_t i0 = 0; i0 < total; i0 += 256) {
-      int32_t x[8], to[8];
+    for (int k = 0; k < 32; k += kLabelsInFlight) {
+      int32_t y[kLabelsInFlight], z[kLabelsInFlight], w[kLabelsInFlight];
+      int32_t wmax = 0;
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int32_t i = i0 + u * 32 + lane;
-        int lo = 0;
-#pragma unroll
-        for (int step = 16; step > 0; step >>= 1)
-          if (__shfl_sync(kFull, incl, lo + step - 1) <= i) lo += step;
-        const int32_t k_src = __shfl_sync(kFull, sbase, lo & 31), k_dst = __shfl_sync(kFull, dbase, lo & 31);
-        const bool ok = i < total;
-        x[u] = ok ? __ldg(src + k_src + i) : 0;
-        to[u] = ok ? k_dst + i : -1;
+      for (int q = 0; q < kLabelsInFlight; ++q) {
+        y[q] = __shfl_sync(kFull, s.y, k + q);
+        z[q] = __shfl_sync(kFull, s.z, k + q);
+        w[q] = __shfl_sync(kFull, s.w, k + q);
+        wmax = max(wmax, w[q]);
       }
+      for (int32_t b0 = 0; b0 < wmax; b0 += 32 * kLabelSteps) {
+        int32_t x[kLabelsInFlight][kLabelSteps];
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (to[u] >= 0) dst[to[u]] = x[u];
+        for (int q = 0; q < kLabelsInFlight; ++q)
+#pragma unroll
+          for (int u = 0; u < kLabelSteps; ++u) {
+            const int32_t t = b0 + u * 32 + lane;
+            x[q][u] = t < w[q] ? __ldg(src + y[q] + t) : 0;
+          }
+#pragma unroll
+        for (int q = 0; q < kLabelsInFlight; ++q)
+#pragma unroll
+          for (int u = 0; u < kLabelSteps; ++u) {
+            const int32_t t = b0 + u * 32 + lane;
+            if (t < w[q]) dst[z[q] + t] = x[q][u];
+          }
+      }
     }
   }
 }
