@@ -231,3 +231,42 @@ def test_device_compaction_keeps_every_tree_canonical():
         om, op, _ = oracle.route(trees, tok, off, W.load(), W.alpha)
         assert_same_route(gm, gp, om, op, f"round {step}")
     assert compacted >= W.P
+
+
+def test_compaction_takes_trees_near_the_threshold_along():
+    """Once some tree's stale label tokens pass half of its label arena, apply_delta compacts it on the
+    device, and in the same call every tree at least 70% of the way there (replicas that receive deltas at
+    the same rate reach the threshold within a few calls of one another).  A tree further away keeps its
+    stale space.  Each tree holds 2,000 sequences of 100 tokens with distinct first tokens, one leaf edge
+    under the root each, so deleting a sequence leaves exactly its 100 label tokens stale."""
+    rng = random.Random(11)
+    n, L = 2000, 100
+    seqs = [[[1 + i] + [rng.randrange(1, 1 << 20) for _ in range(L - 1)] for i in range(n)] for _ in range(3)]
+    r = router_from_seqlists([seqlist_from_lists(s) for s in seqs])
+    ots = [_oracle_tree(s) for s in seqs]
+    done = [0, 0, 0]
+
+    def delete(counts):
+        ops, dl, pb = [], [], [0]
+        for p, k in enumerate(counts):
+            for s in seqs[p][done[p]:done[p] + k]:
+                ops.append(1)
+                dl.append(s)
+                assert ots[p].remove(s)
+            done[p] += k
+            pb.append(len(ops))
+        assert r.apply_delta(-1, np.array(ops, np.int32), seqlist_from_lists(dl), np.array(pb, np.int64)) == 0
+
+    ratio = lambda p: r.stats(p)["stale_label"] / r.stats(p)["label_tokens"]
+    # Tree 1 ends at 42% stale, tree 2 at 20%: neither passes half, nothing is compacted.
+    delete([0, 840, 400])
+    assert 0.35 < ratio(1) < 0.5 and 0 < ratio(2) < 0.35 and ratio(0) == 0
+    stale2 = r.stats(2)["stale_label"]
+    assert stale2 == 400 * L
+    # Tree 0 passes half: it is compacted, and tree 1 with it although this call gave it no ops.
+    delete([1200, 0, 0])
+    assert r.stats(0)["stale_label"] == 0 and r.stats(1)["stale_label"] == 0
+    assert r.stats(2)["stale_label"] == stale2
+    assert r.stats(0)["label_tokens"] == (n - 1200) * L and r.stats(1)["label_tokens"] == (n - 840) * L
+    for p in range(3):
+        assert same_snapshot(r.download(p), ots[p].export()), p

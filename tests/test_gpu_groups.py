@@ -102,6 +102,29 @@ def test_small_vocabulary_deep_trees_grouped(seed):
     _check(trees, reqs, load, rng.choice([0, 2]), f"seed {seed}")
 
 
+@pytest.mark.parametrize("P", [45, 97])
+def test_followers_with_tree_counts_off_the_lane_groups(P):
+    """Followers take trees 64 at a time (two per lane); P = 45 and 97 leave the last pair of 32-tree
+    groups partly empty.  Many trees hold the shared stems, so followers resume at checkpoints in most of
+    them."""
+    rng = random.Random(P)
+    V = 500
+    stems = [[rng.randrange(V) for _ in range(rng.randint(HEAD, 600))] for _ in range(6)]
+    trees = []
+    for _ in range(P):
+        t = []
+        for _ in range(rng.randint(0, 30)):
+            s = rng.choice(stems)
+            t.append(s[:rng.randint(len(s) // 2, len(s))] + [rng.randrange(V) for _ in range(rng.randint(0, 40))])
+        trees.append(t)
+    reqs = []
+    for _ in range(1500):
+        s = rng.choice(stems)
+        reqs.append(s[:rng.randint(HEAD, len(s))] + [rng.randrange(V) for _ in range(rng.randint(0, 50))])
+    load = [rng.randrange(8) for _ in range(P)]
+    _check(trees, reqs, load, 1, f"P={P}")
+
+
 def test_route_launch_count():
     """A grouped batch of short requests is routed by two grouping kernels, a leader pass and a follower
     pass."""
