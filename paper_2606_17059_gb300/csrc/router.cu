@@ -853,35 +853,10 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   const int32_t* d_op = d->op;
   const int64_t *d_sb = S.seg_begin, *d_so = S.seg_off, *d_pb = d->peer_begin;
   const int32_t *d_sl = S.seg_len, *d_pool = S.pool;
-  if (d->mem == P2P_MEM_DEVICE) {
-    // Validate on the device; only the 16-byte result comes back.
-    CK(p2p::launch_validate(r->d_hdr, d, peer, r->P, r->stream));
-    r->launches += 1;
-    int32_t h[4] = {0, 0, 0, 0};
-    CK(d2h(r, h, r->d_hdr, sizeof(h)));
-    unsigned long long ml = 0;
-    std::memcpy(&ml, h, sizeof(ml));
-    max_len = (int64_t)ml;
-    max_runs = h[3];
-    if (h[2] & p2p::STATIC_BAD_OP) return fail(r, P2P_E_INVAL, "bad op code in the delta");
-    if (h[2] & p2p::STATIC_BAD_SEGMENT) return fail(r, P2P_E_INVAL, "seg_begin or a segment is malformed or outside the pool");
-    if (h[2] & p2p::STATIC_TOO_LONG) return fail(r, P2P_E_INVAL, "a sequence is longer than 2^31-1 tokens");
-    if (h[2] & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
-  } else {
-    std::string err;
-    if (!p2p::check_seqs(&S, err, &max_len, nullptr)) return fail(r, P2P_E_INVAL, err);
-    for (int64_t i = 0; i < n; ++i) {
-      if (d->op[i] != P2P_OP_INSERT && d->op[i] != P2P_OP_DELETE)
-        return fail(r, P2P_E_INVAL, "bad op code at " + std::to_string(i));
-      max_runs = std::max(max_runs, S.seg_begin[i + 1] - S.seg_begin[i]);
-    }
-    if (peer == -1) {
-      const int64_t* pb = d->peer_begin;
-      if (pb[0] != 0 || pb[r->P] != n) return fail(r, P2P_E_INVAL, "peer_begin must run from 0 to n");
-      for (int32_t p = 0; p < r->P; ++p)
-        if (pb[p + 1] < pb[p]) return fail(r, P2P_E_INVAL, "peer_begin not non-decreasing");
-    }
-    // Device copies of the delta.
+  p2p_delta dv = *d;  // the delta as the device reads it
+  if (d->mem == P2P_MEM_HOST) {
+    // Host arrays are copied as they are into device buffers and validated there like a device-resident
+    // delta: one pass over millions of ops on the GPU instead of a scan on the host.
     CK(ensure(r, r->d_op, (size_t)n * sizeof(int32_t)));
     CK(ensure(r, r->d_seg_begin, (size_t)(n + 1) * sizeof(int64_t)));
     CK(ensure(r, r->d_seg_off, (size_t)std::max<int64_t>(S.n_segs, 1) * sizeof(int64_t)));
@@ -898,13 +873,35 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
       CK(ensure(r, r->d_peer_begin, (size_t)(r->P + 1) * sizeof(int64_t)));
       CK(cudaMemcpyAsync(r->d_peer_begin.p, d->peer_begin, (size_t)(r->P + 1) * sizeof(int64_t), cudaMemcpyHostToDevice,
                          r->stream));
-      d_pb = (const int64_t*)r->d_peer_begin.p;
+      dv.peer_begin = (const int64_t*)r->d_peer_begin.p;
     }
-    d_op = (const int32_t*)r->d_op.p;
-    d_sb = (const int64_t*)r->d_seg_begin.p;
-    d_so = (const int64_t*)r->d_seg_off.p;
-    d_sl = (const int32_t*)r->d_seg_len.p;
-    d_pool = (const int32_t*)r->d_pool.p;
+    dv.op = (const int32_t*)r->d_op.p;
+    dv.seqs.seg_begin = (const int64_t*)r->d_seg_begin.p;
+    dv.seqs.seg_off = (const int64_t*)r->d_seg_off.p;
+    dv.seqs.seg_len = (const int32_t*)r->d_seg_len.p;
+    dv.seqs.pool = (const int32_t*)r->d_pool.p;
+    dv.mem = P2P_MEM_DEVICE;
+    d_op = dv.op;
+    d_sb = dv.seqs.seg_begin;
+    d_so = dv.seqs.seg_off;
+    d_sl = dv.seqs.seg_len;
+    d_pool = dv.seqs.pool;
+    d_pb = dv.peer_begin;
+  }
+  {
+    // Validate on the device; only the 16-byte result comes back.
+    CK(p2p::launch_validate(r->d_hdr, &dv, peer, r->P, r->stream));
+    r->launches += 1;
+    int32_t h[4] = {0, 0, 0, 0};
+    CK(d2h(r, h, r->d_hdr, sizeof(h)));
+    unsigned long long ml = 0;
+    std::memcpy(&ml, h, sizeof(ml));
+    max_len = (int64_t)ml;
+    max_runs = h[3];
+    if (h[2] & p2p::STATIC_BAD_OP) return fail(r, P2P_E_INVAL, "bad op code in the delta");
+    if (h[2] & p2p::STATIC_BAD_SEGMENT) return fail(r, P2P_E_INVAL, "seg_begin or a segment is malformed or outside the pool");
+    if (h[2] & p2p::STATIC_TOO_LONG) return fail(r, P2P_E_INVAL, "a sequence is longer than 2^31-1 tokens");
+    if (h[2] & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
   }
   CK(ensure(r, r->d_done, (size_t)std::max<int64_t>(n, 1)));
   int32_t* gather = nullptr;
