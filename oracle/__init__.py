@@ -14,6 +14,10 @@ What it computes, and the passages it follows:
   ``match - alpha*load``, ties to the lower load, then to the lower tree index.
 * ``brute`` (pure Python) -- the same quantities written as their plain definitions, used to pin the
   C++ oracle on tiny inputs.
+* ``decide`` (pure Python) -- the route decision with excluded peers and a fallback target: a peer that
+  pushes back (Section 4.1, hot specialist push-back) or is suspected to have failed (Section 4.2,
+  in-flight forwarded request failure) is not a candidate, and the next-best candidate is where a request
+  goes when forwarding to the best one times out.
 """
 from __future__ import annotations
 
@@ -173,6 +177,30 @@ def route(trees, tokens: np.ndarray, offsets: np.ndarray, load, alpha: int, n_th
     ctr = np.zeros(4, np.int64)
     lib.oracle_route(arr, P, _p(tokens), _p(offsets), B, _p(ld), alpha, _p(match), _p(peer), n_threads, _p(ctr))
     return match, peer, ctr
+
+
+def decide(match, load, alpha: int, excluded=None):
+    """Best and next-best target of every request from its match row, skipping excluded peers.
+
+    For row b of ``match`` [B, P], the candidates are the peers p with ``excluded[p]`` false, ordered by
+    the tuple (match[b, p] - alpha*load[p], -load[p], -p): Algorithm 1's argmax with the load term and the
+    tie-breaks of ``route``.  Returns (best int32[B], next int32[B]), the first and second candidate of that
+    order, -1 where there are fewer candidates.  Section 4.1 takes a pushed-back peer out of routing and
+    Section 4.2 a suspected-failed one; on a forwarding timeout Section 4.2 falls back to the next-best
+    target.  Plain Python over the tuples."""
+    match = np.asarray(match)
+    B, P = match.shape
+    ex = np.zeros(P, bool) if excluded is None else np.asarray(excluded).astype(bool)
+    best = np.full(B, -1, np.int32)
+    nxt = np.full(B, -1, np.int32)
+    for b in range(B):
+        cand = sorted(((int(match[b, p]) - alpha * int(load[p]), -int(load[p]), -p) for p in range(P) if not ex[p]),
+                      reverse=True)
+        if cand:
+            best[b] = -cand[0][2]
+        if len(cand) > 1:
+            nxt[b] = -cand[1][2]
+    return best, nxt
 
 
 def touched_bytes(counters: np.ndarray) -> int:

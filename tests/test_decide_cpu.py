@@ -1,0 +1,46 @@
+"""Pins of the oracle's route decision with excluded peers and a fallback target (``oracle.decide``):
+hand-worked rows, agreement with the C++ oracle's route argmax when nothing is excluded, and the
+invariants that excluding the best candidate promotes the next-best one and that the two differ."""
+import random
+
+import numpy as np
+
+import oracle
+import workload as wl
+
+
+def test_hand_worked_rows():
+    # Scores with alpha = 1: 5-1, 5-0, 3-0 = 4, 5, 3.
+    best, nxt = oracle.decide([[5, 5, 3]], [1, 0, 0], 1)
+    assert (best[0], nxt[0]) == (1, 0)
+    best, nxt = oracle.decide([[5, 5, 3]], [1, 0, 0], 1, excluded=[0, 1, 0])
+    assert (best[0], nxt[0]) == (0, 2)
+    best, nxt = oracle.decide([[5, 5, 3]], [1, 0, 0], 1, excluded=[1, 1, 0])
+    assert (best[0], nxt[0]) == (2, -1)
+    best, nxt = oracle.decide([[5, 5, 3]], [1, 0, 0], 1, excluded=[1, 1, 1])
+    assert (best[0], nxt[0]) == (-1, -1)
+    # Equal scores: the lower load wins (4-1 = 3-0), then the lower index.
+    best, nxt = oracle.decide([[4, 3], [3, 3]], [1, 0], 1)
+    assert best.tolist() == [1, 1] and nxt.tolist() == [0, 0]
+    best, nxt = oracle.decide([[3, 3]], [0, 0], 0)
+    assert (best[0], nxt[0]) == (0, 1)
+
+
+def test_best_is_the_route_argmax_and_exclusion_promotes_the_next():
+    prm = wl.preset(0)
+    prm.update(P=6, n_seq=200, n_prefix=12, B=300)
+    W = wl.Workload(params=prm, seed=9)
+    trees = oracle.build_trees([W.tree(p) for p in range(W.P)])
+    tok, off = W.requests()
+    load = W.load()
+    match, peer, _ = oracle.route(trees, tok, off, load, W.alpha)
+    best, nxt = oracle.decide(match, load, W.alpha)
+    assert np.array_equal(best, peer)
+    assert (best != nxt).all() and (nxt >= 0).all()
+    rng = random.Random(4)
+    for b in rng.sample(range(W.B), 40):
+        ex = np.zeros(W.P, np.uint8)
+        ex[best[b]] = 1
+        b2, n2 = oracle.decide(match[b:b + 1], load, W.alpha, excluded=ex)
+        assert b2[0] == nxt[b]
+        assert n2[0] not in (best[b], nxt[b])
