@@ -364,6 +364,9 @@ def run_ours(args):
                     "bytes_per_launch": bytes_per_launch, "route_ms": route_avg_ms,
                     "bytes_basis": f"oracle touched-byte counters over {n_acc} requests x {P} trees, "
                                    f"scaled to {B} requests per launch"}
+        # ---- optional: the route decision with excluded peers on this batch's match matrix ----
+        if args.decide:
+            res["decide"] = time_decide(router, out_match, load, alpha, P, B, hbm, src)
         # ---- end to end through the host-pointer C-ABI call ----
         e2e = run_e2e(args, W, router, tok_np, h_off.numpy(), load, alpha, has_delta, n_cpu)
         res.update({
@@ -382,6 +385,31 @@ def run_ours(args):
     router.close()
     if dist:
         dist.destroy_process_group()
+
+
+def time_decide(router, out_match, load, alpha, P, B, hbm, src, reps: int = 10):
+    """p2p_route_decide on the routed batch's match matrix with 5% of the trees excluded (seeded): mean
+    time of `reps` calls after 3 warm-up calls (CUDA events on the router stream), and the read rate of
+    the B x P int32 matrix against the HBM copy bandwidth."""
+    import torch
+    ex = (np.random.default_rng(5).random(P) < 0.05).astype(np.uint8)
+    peer = torch.empty(B, dtype=torch.int32, device="cuda")
+    nxt = torch.empty(B, dtype=torch.int32, device="cuda")
+    for _ in range(3):
+        router.decide(out_match, load, alpha, ex, peer, nxt)
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        router.decide(out_match, load, alpha, ex, peer, nxt)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    gbs = B * P * 4 / (ms / 1e3) / 1e9
+    return {"kernel": "decide_kernel", "ms": ms, "excluded": int(ex.sum()), "bytes_per_launch": B * P * 4,
+            "achieved_gbs": gbs, "peak_gbs": hbm, "frac": gbs / hbm, "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
+            "note": "the match matrix is read once per call; it may partly sit in L2 from the route step"}
 
 
 def run_e2e(args, W, router, tok_np, off_np, load, alpha, has_delta, n_cpu):
@@ -470,6 +498,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--decide", action="store_true",
+                    help="also time p2p_route_decide (excluded peers, next-best target) on the routed batch")
     ap.add_argument("--ref-requests", type=int, default=65536)
     ap.add_argument("--ref-seconds", type=float, default=4.0, help="oracle time per reference step")
     ap.add_argument("--trees", type=int, default=0, help="override P (a scaled-down variant, not a bench line)")

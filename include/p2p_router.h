@@ -223,6 +223,23 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
 int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* offsets, int64_t B,
                          const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
 
+/* Route decision with excluded peers and a fallback target, from a batch's match matrix.  Section 4.1
+ * (hot specialist push-back) stops routing to a peer that advertised back-pressure; Section 4.2
+ * (in-flight forwarded request failure) marks a peer that missed its broadcasts as suspected-failed, and on
+ * a forwarding timeout sends the request to the next-best target, which may be the node itself.
+ *   match       DEVICE int32[B*P] row-major, as p2p_route_batch writes it (values below 0 count as 0)
+ *   load        HOST int32[P], alpha: as for p2p_route_batch; copied before return
+ *   excluded    HOST uint8[P] (nullable = none): excluded[p] != 0 takes tree p out of the candidates;
+ *               copied before return
+ *   out_peer    DEVICE int32[B]: the first candidate of the route order (match - alpha*load, then the lower
+ *               load, then the lower index), -1 if every tree is excluded
+ *   out_next    DEVICE int32[B]: the second candidate of that order, -1 if there is none
+ * With nothing excluded, out_peer equals p2p_route_batch's out_peer.  Asynchronous on the router stream;
+ * one kernel launch.  B = 0 is a no-op.  Errors: P2P_E_INVAL (B < 0, NULL pointers, load or alpha out of
+ * range), P2P_E_CUDA. */
+int p2p_route_decide(p2p_router* r, const int32_t* match, int64_t B, const int32_t* load, int32_t alpha,
+                     const uint8_t* excluded, int32_t* out_peer, int32_t* out_next);
+
 #ifdef __cplusplus
 }
 #endif

@@ -20,7 +20,7 @@ __all__ = [
     "p2p_router_create", "p2p_router_destroy", "p2p_router_set_stream", "p2p_router_sync", "p2p_last_error",
     "p2p_router_num_trees", "p2p_router_launch_count", "p2p_snapshot_build", "p2p_snapshot_view", "p2p_snapshot_free",
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
-    "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host",
+    "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host", "p2p_route_decide",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -92,6 +92,7 @@ def _load():
             "p2p_tree_stats": (ctypes.c_int, [_vp, _i32, P(_i64 * 9)]),
             "p2p_route_batch": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, _i32, _vp, _vp]),
             "p2p_route_batch_host": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _i32, _vp, _vp]),
+            "p2p_route_decide": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -292,6 +293,20 @@ def p2p_route_batch(r, tokens, n_tokens: int, offsets, B: int, load, alpha: int,
                                    _addr(out_match), _addr(out_peer)), r)
 
 
+def p2p_route_decide(r, match, B: int, load, alpha: int, excluded, out_peer, out_next) -> None:
+    """Best and next-best non-excluded tree per request from a device match matrix [B, P] (CUDA tensors or
+    addresses); load and excluded (uint8 per tree, or None) are host arrays."""
+    ld = _host_i32(load)
+    n = p2p_router_num_trees(r)
+    ex = None
+    if excluded is not None:
+        ex = np.ascontiguousarray(np.asarray(excluded), dtype=np.uint8)
+    if ld.size != n or (ex is not None and ex.size != n):
+        raise ValueError(f"load and excluded must have one entry per tree ({n})")
+    _check(_load().p2p_route_decide(r, _addr(match), B, ld.ctypes.data, alpha,
+                                    ex.ctypes.data if ex is not None else None, _addr(out_peer), _addr(out_next)), r)
+
+
 def p2p_route_batch_host(r, tokens: np.ndarray, offsets: np.ndarray, B: int, load, alpha: int,
                          out_match: np.ndarray, out_peer: np.ndarray) -> None:
     """Host routing: every array is a host numpy array (pinned memory copies faster)."""
@@ -358,6 +373,17 @@ class Router:
             out_peer = torch.empty(B, dtype=torch.int32, device=tokens.device)
         p2p_route_batch(self._h, tokens, tokens.numel(), offsets, B, load, alpha, out_match, out_peer)
         return out_match, out_peer
+
+    def decide(self, match, load, alpha: int, excluded=None, out_peer=None, out_next=None):
+        """match is a CUDA int32 tensor [B, P]; returns (peer [B], next [B]) CUDA tensors."""
+        import torch
+        B = match.shape[0]
+        if out_peer is None:
+            out_peer = torch.empty(B, dtype=torch.int32, device=match.device)
+        if out_next is None:
+            out_next = torch.empty(B, dtype=torch.int32, device=match.device)
+        p2p_route_decide(self._h, match, B, load, alpha, excluded, out_peer, out_next)
+        return out_peer, out_next
 
     def route_host(self, tokens: np.ndarray, offsets: np.ndarray, load, alpha: int, out_match=None, out_peer=None):
         B = len(offsets) - 1

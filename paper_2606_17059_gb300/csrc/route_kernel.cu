@@ -717,6 +717,56 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
   }
 }
 
+// Route decision from a match matrix with excluded peers (one warp per request): the best and the next-best
+// candidate by the route order of route_key, skipping peers with excluded[p] != 0 (Section 4.1: a peer that
+// pushes back; Section 4.2: a suspected-failed peer, and the next-best target a request falls back to when
+// forwarding times out).  Each lane keeps the two largest keys of its peers, and five butterfly steps merge
+// the lanes' pairs.  A key is never 0 (score + 2^31 >= 1), so 0 marks "no candidate" (-1 out).  Match values
+// below 0 count as 0.
+constexpr int kDecideUnroll = 8;  // columns a lane loads per stretch (a 256-tree row in one stretch)
+__global__ void __launch_bounds__(256) decide_kernel(const int32_t* __restrict__ match, int64_t B, int32_t P,
+                                                     const int32_t* __restrict__ load, int32_t alpha,
+                                                     const uint8_t* __restrict__ excluded,
+                                                     int32_t* __restrict__ out_peer, int32_t* __restrict__ out_next) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
+  for (int64_t b = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; b < B; b += warps) {
+    const int32_t* row = match + b * P;
+    unsigned long long k1 = 0, k2 = 0;
+    for (int32_t p0 = 0; p0 < P; p0 += 32 * kDecideUnroll) {
+      int32_t v[kDecideUnroll];  // a lane's columns of this stretch, loaded before any is looked at
+#pragma unroll
+      for (int u = 0; u < kDecideUnroll; ++u) {
+        const int32_t p = p0 + 32 * u + lane;
+        v[u] = p < P ? __ldg(row + p) : 0;
+      }
+#pragma unroll
+      for (int u = 0; u < kDecideUnroll; ++u) {
+        const int32_t p = p0 + 32 * u + lane;
+        if (p >= P || (excluded && excluded[p])) continue;
+        const unsigned long long k = route_key(max(v[u], 0), __ldg(load + p), p, alpha);
+        if (k > k1) {
+          k2 = k1;
+          k1 = k;
+        } else if (k > k2) {
+          k2 = k;
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long o1 = __shfl_xor_sync(kFull, k1, o), o2 = __shfl_xor_sync(kFull, k2, o);
+      const unsigned long long lo = k1 < o1 ? k1 : o1, hi = k1 < o1 ? o1 : k1, r2 = k2 < o2 ? o2 : k2;
+      k1 = hi;
+      k2 = lo < r2 ? r2 : lo;
+    }
+    if (lane == 0) {
+      out_peer[b] = k1 ? 0xFFFF - (int32_t)(k1 & 0xFFFFull) : -1;
+      out_next[b] = k2 ? 0xFFFF - (int32_t)(k2 & 0xFFFFull) : -1;
+    }
+  }
+}
+
 }  // namespace
 
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
@@ -763,6 +813,15 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                                                        g->counts + 1, g->lead, g->cpre, g->gid, nullptr, g->ckpt, d_load,
                                                        alpha, out_match, out_peer, d_err, nullptr);
   *launched += 1;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,
+                          const uint8_t* d_excluded, int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st) {
+  if (B <= 0) return cudaSuccess;
+  const int64_t want = (B + 7) / 8;
+  const int grid = (int)std::min<int64_t>(want, (int64_t)std::max(num_sms, 1) * 8);
+  decide_kernel<<<grid, 256, 0, st>>>(match, B, P, d_load, alpha, d_excluded, out_peer, out_next);
   return cudaGetLastError();
 }
 

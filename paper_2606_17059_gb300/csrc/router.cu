@@ -91,6 +91,8 @@ struct p2p_router {
   int32_t* d_err = nullptr;
   int32_t* d_hdr = nullptr;  // validation result of device-resident deltas
   int32_t* h_load = nullptr;  // pinned, kLoadRing slots of P values
+  uint8_t* d_mask = nullptr;  // excluded peers of p2p_route_decide
+  uint8_t* h_mask = nullptr;  // pinned, kLoadRing slots of P bytes (staged with the load of the same slot)
   cudaEvent_t load_ev[kLoadRing] = {};
   // Copy streams of p2p_route_batch_host (inputs in, results out) and the events that order them.
   cudaStream_t cp_in = nullptr, cp_out = nullptr;
@@ -274,14 +276,20 @@ int check_load(p2p_router* r, const int32_t* load, int32_t alpha) {
   return P2P_OK;
 }
 
-// Stages load[P] through a pinned ring slot (the slot's previous copy has finished once its event has).
-int stage_load(p2p_router* r, const int32_t* load) {
+// Stages load[P] (and, if given, the excluded-peer bytes mask[P]) through a pinned ring slot; the slot's
+// previous copies have finished once its event has.
+int stage_load(p2p_router* r, const int32_t* load, const uint8_t* mask = nullptr) {
   const int s = r->load_slot;
   r->load_slot = (s + 1) % kLoadRing;
   CK(cudaEventSynchronize(r->load_ev[s]));
   int32_t* slot = r->h_load + (size_t)s * r->P;
   std::memcpy(slot, load, (size_t)r->P * sizeof(int32_t));
   CK(cudaMemcpyAsync(r->d_load, slot, (size_t)r->P * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
+  if (mask) {
+    uint8_t* ms = r->h_mask + (size_t)s * r->P;
+    std::memcpy(ms, mask, (size_t)r->P);
+    CK(cudaMemcpyAsync(r->d_mask, ms, (size_t)r->P, cudaMemcpyHostToDevice, r->stream));
+  }
   CK(cudaEventRecord(r->load_ev[s], r->stream));
   return P2P_OK;
 }
@@ -695,9 +703,11 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   e = dalloc(r, (void**)&r->d_views, (size_t)P * sizeof(TreeView));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_states, (size_t)P * sizeof(TreeState));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_load, (size_t)P * sizeof(int32_t));
+  if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_mask, (size_t)P);
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_err, sizeof(int32_t));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_hdr, p2p::kStaticHeaderInts * sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_load, (size_t)kLoadRing * P * sizeof(int32_t));
+  if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_mask, (size_t)kLoadRing * P);
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_err, sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_states, (size_t)P * sizeof(TreeState));
   for (int i = 0; i < kLoadRing && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&r->load_ev[i], cudaEventDisableTiming);
@@ -741,6 +751,7 @@ void p2p_router_destroy(p2p_router* r) {
     dfree(r, r->d_views);
     dfree(r, r->d_states);
     dfree(r, r->d_load);
+    dfree(r, r->d_mask);
     dfree(r, r->d_err);
     dfree(r, r->d_hdr);
     dfree(r, r->d_shared);
@@ -761,6 +772,7 @@ void p2p_router_destroy(p2p_router* r) {
     if (r->ev_routed[i]) cudaEventDestroy(r->ev_routed[i]);
   }
   if (r->h_load) cudaFreeHost(r->h_load);
+  if (r->h_mask) cudaFreeHost(r->h_mask);
   if (r->h_err) cudaFreeHost(r->h_err);
   if (r->h_states) cudaFreeHost(r->h_states);
   delete r;
@@ -1063,6 +1075,21 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
   DeviceGuard g(r->device);
   if (int rc = stage_load(r, load)) return rc;
   return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer);
+}
+
+int p2p_route_decide(p2p_router* r, const int32_t* match, int64_t B, const int32_t* load, int32_t alpha,
+                     const uint8_t* excluded, int32_t* out_peer, int32_t* out_next) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (B < 0) return fail(r, P2P_E_INVAL, "negative B");
+  if (int rc = check_load(r, load, alpha)) return rc;
+  if (B == 0) return P2P_OK;
+  if (!match || !out_peer || !out_next) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r->device);
+  if (int rc = stage_load(r, load, excluded)) return rc;
+  CK(p2p::launch_decide(match, B, r->P, r->d_load, alpha, excluded ? r->d_mask : nullptr, out_peer, out_next,
+                        r->num_sms, r->stream));
+  r->launches += 1;
+  return P2P_OK;
 }
 
 int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* offsets, int64_t B, const int32_t* load,
