@@ -134,6 +134,15 @@ def _host_i32(a) -> np.ndarray:
     return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
 
 
+def _load_vec(r, load) -> np.ndarray:
+    """The per-tree load as a host int32 array; the library reads one entry per tree."""
+    ld = _host_i32(load)
+    n = p2p_router_num_trees(r)
+    if ld.ndim != 1 or ld.size != n:
+        raise ValueError(f"load must have one entry per tree ({n}), got shape {ld.shape}")
+    return ld
+
+
 def _seqs_struct(sl, keep: list) -> Seqs:
     """Seqs struct from an object with seg_begin/seg_off/seg_len/pool (numpy arrays or CUDA tensors)."""
     arrs = []
@@ -288,7 +297,7 @@ def p2p_tree_stats(r, peer: int) -> dict:
 
 def p2p_route_batch(r, tokens, n_tokens: int, offsets, B: int, load, alpha: int, out_match, out_peer) -> None:
     """Device routing: tokens/offsets/out_match/out_peer are CUDA tensors (or addresses), load is host."""
-    ld = _host_i32(load)
+    ld = _load_vec(r, load)
     _check(_load().p2p_route_batch(r, _addr(tokens), n_tokens, _addr(offsets), B, ld.ctypes.data, alpha,
                                    _addr(out_match), _addr(out_peer)), r)
 
@@ -296,13 +305,13 @@ def p2p_route_batch(r, tokens, n_tokens: int, offsets, B: int, load, alpha: int,
 def p2p_route_decide(r, match, B: int, load, alpha: int, excluded, out_peer, out_next) -> None:
     """Best and next-best non-excluded tree per request from a device match matrix [B, P] (CUDA tensors or
     addresses); load and excluded (uint8 per tree, or None) are host arrays."""
-    ld = _host_i32(load)
-    n = p2p_router_num_trees(r)
+    ld = _load_vec(r, load)
+    n = ld.size
     ex = None
     if excluded is not None:
         ex = np.ascontiguousarray(np.asarray(excluded), dtype=np.uint8)
-    if ld.size != n or (ex is not None and ex.size != n):
-        raise ValueError(f"load and excluded must have one entry per tree ({n})")
+    if ex is not None and ex.size != n:
+        raise ValueError(f"excluded must have one entry per tree ({n})")
     _check(_load().p2p_route_decide(r, _addr(match), B, ld.ctypes.data, alpha,
                                     ex.ctypes.data if ex is not None else None, _addr(out_peer), _addr(out_next)), r)
 
@@ -310,10 +319,13 @@ def p2p_route_decide(r, match, B: int, load, alpha: int, excluded, out_peer, out
 def p2p_route_batch_host(r, tokens: np.ndarray, offsets: np.ndarray, B: int, load, alpha: int,
                          out_match: np.ndarray, out_peer: np.ndarray) -> None:
     """Host routing: every array is a host numpy array (pinned memory copies faster)."""
-    ld = _host_i32(load)
+    ld = _load_vec(r, load)
     for a, dt in ((tokens, np.int32), (offsets, np.int64), (out_match, np.int32), (out_peer, np.int32)):
         if not isinstance(a, np.ndarray) or a.dtype != dt or not a.flags["C_CONTIGUOUS"]:
             raise TypeError("host routing needs C-contiguous numpy arrays (int32 tokens/outputs, int64 offsets)")
+    if B > 0 and (offsets.size < B + 1 or out_match.size < B * ld.size or out_peer.size < B
+                  or tokens.size < int(offsets[B])):
+        raise ValueError("host routing arrays are smaller than B requests need")
     _check(_load().p2p_route_batch_host(r, _addr(tokens), _addr(offsets), B, ld.ctypes.data, alpha,
                                         _addr(out_match), _addr(out_peer)), r)
 
