@@ -26,17 +26,22 @@
 //   root's table) and the warps take these buckets, heaviest first.
 // Ops on the same sequence share an anchor and a next token, or a first token, so every bucket applies
 // them in op order.  Inside an op the warp cooperates: a child lookup probes 32 table slots at once, labels
-// are compared 128 tokens per step and copied 128 per step; lane 0 performs scalar stores and __syncwarp()
+// are compared 256 tokens per step and copied 256 per step; lane 0 performs scalar stores and __syncwarp()
 // orders them before later reads.  Adding or removing a child touches one slot (a table is doubled and
 // rehashed when it passes 1/2 occupancy), so the cost of an op does not grow with the fan-out of the nodes
 // it passes.
 //
-// Space.  Node, child-entry and label arenas are bump-allocated with compare-and-swap on the tree's
-// counters; an op reserves everything it may need before it mutates anything.  If an arena is full the op
+// Space.  Node, child-entry and label arenas are bump-allocated: each warp takes slabs from the tree's
+// counters by compare-and-swap and hands out its ops' room from them; an op reserves everything it may
+// need before it mutates anything.  If an arena is full the op
 // is left undone, its bucket stops (as do, for the rest of the launch, the first-token buckets of every op
 // it holds back, so no later op on the same sequence overtakes it) and the tree is flagged; the host grows
 // the arenas and relaunches.  A per-op done flag records what is applied, so every op is applied whole,
 // once.  Every loop is bounded by a sequence length, a list size or an iteration cap.
+//
+// Compaction (after the delta, when stale space passes live space): compact_kernel copies each tree's
+// structure breadth-first into fresh arrays (one CTA per tree), then compact_labels_kernel moves the labels
+// of all compacted trees over the whole GPU.
 #include "internal.h"
 
 namespace p2p {

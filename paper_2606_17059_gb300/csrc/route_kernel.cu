@@ -20,7 +20,8 @@
 // coalesced load, whatever the fan-out), and an edge label is compared 32 consecutive tokens per warp load,
 // up to kUnroll loads in flight per lane, folded into one vote per block; the first mismatch is searched
 // only inside the block that holds it.  The route decision keeps the max of a packed 64-bit key per
-// request.  Integer work only: no tensor cores.
+// request.  decide_kernel (p2p_route_decide) makes the decision again from a match matrix with some trees
+// excluded and also returns the next-best tree (Sections 4.1 and 4.2).  Integer work only: no tensor cores.
 #include "internal.h"
 
 namespace p2p {

@@ -2,7 +2,9 @@
 //
 // The router owns P trees in HBM (layout in internal.h), allocated from a router-private stream-ordered
 // memory pool so that replacing a tree (snapshot upload, arena growth) frees the old arrays in stream
-// order, after any route still reading them.  All device work goes to the router's stream.
+// order, after any route still reading them.  Each tree also keeps a spare set of arrays that device
+// compaction copies it into (the old set becomes the next spare).  All device work goes to the router's
+// stream.
 #include <algorithm>
 #include <cstring>
 #include <string>
