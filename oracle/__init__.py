@@ -14,6 +14,8 @@ What it computes, and the passages it follows:
   ``match - alpha*load``, ties to the lower load, then to the lower tree index.
 * ``brute`` (pure Python) -- the same quantities written as their plain definitions, used to pin the
   C++ oracle on tiny inputs.
+* ``update_estimates`` -- UpdateTrieEstimate of Algorithm 1 over a routed batch: request b is inserted
+  into the tree it was routed to (the node's estimate of that peer's cache after a successful send).
 * ``decide`` (pure Python) -- the route decision with excluded peers and a fallback target: a peer that
   pushes back (Section 4.1, hot specialist push-back) or is suspected to have failed (Section 4.2,
   in-flight forwarded request failure) is not a candidate, and the next-best candidate is where a request
@@ -177,6 +179,17 @@ def route(trees, tokens: np.ndarray, offsets: np.ndarray, load, alpha: int, n_th
     ctr = np.zeros(4, np.int64)
     lib.oracle_route(arr, P, _p(tokens), _p(offsets), B, _p(ld), alpha, _p(match), _p(peer), n_threads, _p(ctr))
     return match, peer, ctr
+
+
+def update_estimates(trees, tokens: np.ndarray, offsets: np.ndarray, peer) -> None:
+    """Algorithm 1, after a request is sent to node k and acknowledged: UpdateTrieEstimate(r, k) inserts r
+    into the sender's estimate of k's trie (Section 2 primitive list).  For a routed batch: request b,
+    tokens[offsets[b] .. offsets[b+1]), is inserted into trees[peer[b]]; a request with peer[b] < 0 (no
+    target) is skipped.  One plain insert per request, in batch order."""
+    for b in range(len(offsets) - 1):
+        k = int(peer[b])
+        if k >= 0:
+            trees[k].insert(tokens[int(offsets[b]):int(offsets[b + 1])])
 
 
 def decide(match, load, alpha: int, excluded=None):
