@@ -223,8 +223,8 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
 int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* offsets, int64_t B,
                          const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
 
-/* Route decision with excluded peers and a fallback target, from a batch's match matrix.  Section 4.1
- * (hot specialist push-back) stops routing to a peer that advertised back-pressure; Section 4.2
+/* Route decision with excluded peers and a fallback target, from a batch's match matrix.  Section 3.2
+ * (hot specialist push-back) stops routing to a peer that advertised back-pressure; Section 3.3
  * (in-flight forwarded request failure) marks a peer that missed its broadcasts as suspected-failed, and on
  * a forwarding timeout sends the request to the next-best target, which may be the node itself.
  *   match       DEVICE int32[B*P] row-major, as p2p_route_batch writes it (values below 0 count as 0)

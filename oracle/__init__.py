@@ -14,10 +14,12 @@ What it computes, and the passages it follows:
   ``match - alpha*load``, ties to the lower load, then to the lower tree index.
 * ``brute`` (pure Python) -- the same quantities written as their plain definitions, used to pin the
   C++ oracle on tiny inputs.
+* ``lru`` (pure Python) -- a node's own trie with EvictLRUTrie (one least-recently-used leaf token at a
+  time, Section 2 primitive list and Algorithm 1) and the expected hit rate of Section 5.
 * ``update_estimates`` -- UpdateTrieEstimate of Algorithm 1 over a routed batch: request b is inserted
   into the tree it was routed to (the node's estimate of that peer's cache after a successful send).
 * ``decide`` (pure Python) -- the route decision with excluded peers and a fallback target: a peer that
-  pushes back (Section 4.1, hot specialist push-back) or is suspected to have failed (Section 4.2,
+  pushes back (Section 3.2, hot specialist push-back) or is suspected to have failed (Section 3.3,
   in-flight forwarded request failure) is not a candidate, and the next-best candidate is where a request
   goes when forwarding to the best one times out.
 """
@@ -198,8 +200,8 @@ def decide(match, load, alpha: int, excluded=None):
     For row b of ``match`` [B, P], the candidates are the peers p with ``excluded[p]`` false, ordered by
     the tuple (match[b, p] - alpha*load[p], -load[p], -p): Algorithm 1's argmax with the load term and the
     tie-breaks of ``route``.  Returns (best int32[B], next int32[B]), the first and second candidate of that
-    order, -1 where there are fewer candidates.  Section 4.1 takes a pushed-back peer out of routing and
-    Section 4.2 a suspected-failed one; on a forwarding timeout Section 4.2 falls back to the next-best
+    order, -1 where there are fewer candidates.  Section 3.2 takes a pushed-back peer out of routing and
+    Section 3.3 a suspected-failed one; on a forwarding timeout Section 3.3 falls back to the next-best
     target.  Plain Python over the tuples."""
     match = np.asarray(match)
     B, P = match.shape

@@ -21,7 +21,7 @@
 // up to kUnroll loads in flight per lane, folded into one vote per block; the first mismatch is searched
 // only inside the block that holds it.  The route decision keeps the max of a packed 64-bit key per
 // request.  decide_kernel (p2p_route_decide) makes the decision again from a match matrix with some trees
-// excluded and also returns the next-best tree (Sections 4.1 and 4.2).  Integer work only: no tensor cores.
+// excluded and also returns the next-best tree (Sections 3.2 and 3.3).  Integer work only: no tensor cores.
 #include "internal.h"
 
 namespace p2p {
@@ -719,8 +719,8 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
 }
 
 // Route decision from a match matrix with excluded peers (one warp per request): the best and the next-best
-// candidate by the route order of route_key, skipping peers with excluded[p] != 0 (Section 4.1: a peer that
-// pushes back; Section 4.2: a suspected-failed peer, and the next-best target a request falls back to when
+// candidate by the route order of route_key, skipping peers with excluded[p] != 0 (Section 3.2: a peer that
+// pushes back; Section 3.3: a suspected-failed peer, and the next-best target a request falls back to when
 // forwarding times out).  Each lane keeps the two largest keys of its peers, and five butterfly steps merge
 // the lanes' pairs.  A key is never 0 (score + 2^31 >= 1), so 0 marks "no candidate" (-1 out).  Match values
 // below 0 count as 0.
