@@ -44,3 +44,17 @@ def test_best_is_the_route_argmax_and_exclusion_promotes_the_next():
         b2, n2 = oracle.decide(match[b:b + 1], load, W.alpha, excluded=ex)
         assert b2[0] == nxt[b]
         assert n2[0] not in (best[b], nxt[b])
+
+
+def test_random_rows_agree_with_the_cpp_argmax():
+    """With nothing excluded, the first candidate is the C++ oracle's argmax (oracle_argmax) on random rows
+    full of ties (small match values and loads)."""
+    rng = np.random.default_rng(17)
+    for _ in range(300):
+        P = int(rng.integers(1, 40))
+        row = rng.integers(0, 6, size=P).astype(np.int32)
+        load = rng.integers(0, 4, size=P).astype(np.int32)
+        alpha = int(rng.integers(0, 3))
+        best, nxt = oracle.decide(row[None, :], load, alpha)
+        assert best[0] == oracle.argmax_peer(row, load, alpha)
+        assert (nxt[0] == -1) == (P == 1)
