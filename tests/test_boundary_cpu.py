@@ -35,6 +35,27 @@ def test_library_builds_and_exports_every_declared_symbol():
         assert hasattr(lib, name)
 
 
+def _declared_parameter_counts():
+    """Entry point -> number of parameters, from the prototypes in include/p2p_router.h."""
+    src = open(os.path.join(ROOT, "include", "p2p_router.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    out = {}
+    for name, params in re.findall(r"\b(p2p_[a-z_]+)\s*\(([^;{]*?)\)\s*;", src, flags=re.S):
+        params = params.strip()
+        out[name] = 0 if params in ("", "void") else len(params.split(","))
+    return out
+
+
+def test_binding_signatures_match_the_header():
+    """The ctypes binding passes as many arguments to each entry point as its prototype declares."""
+    counts = _declared_parameter_counts()
+    assert set(counts) == set(_declared_functions())
+    lib = g._load()
+    for name, n in counts.items():
+        fn = getattr(lib, name)
+        assert fn.argtypes is not None and len(fn.argtypes) == n, (name, n, fn.argtypes)
+
+
 def test_library_has_no_oracle_dependency():
     out = subprocess.run(["nm", "-D", g.build()], capture_output=True, text=True).stdout
     assert "otree" not in out and "oracle" not in out
