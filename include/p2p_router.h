@@ -18,7 +18,9 @@
  *     ties go to the lower load, then to the lower tree index.  Requires alpha >= 0, 0 <= load <= 65535,
  *     alpha * load <= 2^31 - 1 and P <= 65536.
  *   - Every call returns P2P_OK (0) or a negative error code; p2p_last_error() gives a message.  A call
- *     that fails leaves the router's trees unchanged.
+ *     that fails leaves the router's trees unchanged, with one exception: p2p_tree_apply_delta_static,
+ *     which may not grow a tree, returns P2P_E_NOMEM with the trees that ran out of room holding part of
+ *     their ops (each op applied whole or not at all).
  *   - Device work is enqueued on the router's stream (p2p_router_set_stream); calls that take device
  *     pointers return before the work finishes.  Asynchronous device-side errors are reported by the
  *     next p2p_router_sync() as P2P_E_DEVICE.
@@ -189,8 +191,9 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
  * per tree the call touches; a delta that needs more gets P2P_E_INVAL.  If a tree's arenas run out of room, the call returns P2P_E_NOMEM and that
  * tree holds only part of its ops (each op applied whole or not at all); p2p_tree_apply_delta, which may
  * allocate, grows trees.
- * The first call on a device looks up the static array's device address (cudaGetSymbolAddress, with
- * the router's device current) and caches it; make that first call before any stream capture.  Every
+ * Every call looks up the static array's device address (cudaGetSymbolAddress, with the router's device
+ * current; the lookup allocates nothing).  The first lookup on a device may load the library's module
+ * there, so make the first call before any stream capture.  Every
  * call shares the array, so calls whose device work overlaps (for example two routers on different
  * streams) race: order them.  The call returns when the delta is applied.  Other errors as
  * p2p_tree_apply_delta. */
@@ -210,7 +213,8 @@ int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]);
  *   load        HOST int32[P], copied before return; alpha >= 0 (see Conventions)
  *   out_match   DEVICE int32[B*P], row-major: out_match[b*P + p] = match(r_b, T_p)
  *   out_peer    DEVICE int32[B]: the chosen tree of request b
- * Asynchronous on the router stream.  B = 0 is a no-op.  Errors: P2P_E_INVAL, P2P_E_CUDA. */
+ * Asynchronous on the router stream.  B = 0 is a no-op; B may be at most 2^30 (split larger batches).
+ * Errors: P2P_E_INVAL, P2P_E_CUDA. */
 int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
                     const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
 

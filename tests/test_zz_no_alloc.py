@@ -92,7 +92,7 @@ def test_static_delta_rejects_host_memory_sizes_beyond_its_scratch_and_full_tree
     d = g.Delta(h_op.ctypes.data, g._seqs_struct(h, keep), None, g.P2P_MEM_HOST)
     rc = g._load().p2p_tree_apply_delta_static(r.handle, 0, ctypes.byref(d), None)
     assert rc == g.P2P_E_INVAL and "device memory" in g.p2p_last_error(r.handle)
-    # An op whose sequence is split into more than two pool runs is gathered into the scratch: 32 buckets x
+    # An op whose sequence is split into more than two pool runs is gathered into the scratch: 16 warps x
     # a 600,000-token sequence per tree cannot fit in the 8 MiB array.
     n = 600_000
     pool = _dev(np.arange(n, dtype=np.int32))
