@@ -202,15 +202,19 @@ def decide(match, load, alpha: int, excluded=None):
     tie-breaks of ``route``.  Returns (best int32[B], next int32[B]), the first and second candidate of that
     order, -1 where there are fewer candidates.  Section 3.2 takes a pushed-back peer out of routing and
     Section 3.3 a suspected-failed one; on a forwarding timeout Section 3.3 falls back to the next-best
-    target.  Plain Python over the tuples."""
+    target.  Plain Python over the tuples.
+
+    A match entry below 0 counts as 0: PrefixMatch is a count of tokens, so no route produces one, and a
+    negative entry in a caller's matrix is read as "nothing matched" (the reading the device decision
+    applies too)."""
     match = np.asarray(match)
     B, P = match.shape
     ex = np.zeros(P, bool) if excluded is None else np.asarray(excluded).astype(bool)
     best = np.full(B, -1, np.int32)
     nxt = np.full(B, -1, np.int32)
     for b in range(B):
-        cand = sorted(((int(match[b, p]) - alpha * int(load[p]), -int(load[p]), -p) for p in range(P) if not ex[p]),
-                      reverse=True)
+        cand = sorted(((max(int(match[b, p]), 0) - alpha * int(load[p]), -int(load[p]), -p)
+                       for p in range(P) if not ex[p]), reverse=True)
         if cand:
             best[b] = -cand[0][2]
         if len(cand) > 1:

@@ -1,6 +1,7 @@
 """Pins of the oracle's route decision with excluded peers and a fallback target (``oracle.decide``):
 hand-worked rows, agreement with the C++ oracle's route argmax when nothing is excluded, and the
-invariants that excluding the best candidate promotes the next-best one and that the two differ."""
+invariants that excluding the best candidate promotes the next-best one and that the two differ; a negative
+match entry counts as 0 (a prefix-match length is never negative)."""
 import random
 
 import numpy as np
@@ -58,3 +59,13 @@ def test_random_rows_agree_with_the_cpp_argmax():
         best, nxt = oracle.decide(row[None, :], load, alpha)
         assert best[0] == oracle.argmax_peer(row, load, alpha)
         assert (nxt[0] == -1) == (P == 1)
+
+
+def test_negative_match_entries_count_as_zero():
+    # Hand-worked: alpha = 1, loads 0 and 3.  Tree 0's entry -5 counts as 0, score 0; tree 1 scores 2 - 3 = -1.
+    # Taken literally, -5 would lose to -1.
+    best, nxt = oracle.decide([[-5, 2]], [0, 3], 1)
+    assert (best[0], nxt[0]) == (0, 1)
+    # A row of negative entries decides by load alone, like an empty tree's zeros: lower load, then index.
+    best, nxt = oracle.decide([[-1, -7, -2**31]], [2, 1, 1], 3)
+    assert (best[0], nxt[0]) == (1, 2)

@@ -1,7 +1,7 @@
 """GPU parity of the route decision with excluded peers and a fallback target (p2p_route_decide) against
 the oracle's plain tuple ordering, through the C ABI: random match matrices with ties and masks (none,
-some, all but one, all), tree counts on and off the warp width, and a routed batch whose decision with
-nothing excluded must equal the route's own choice."""
+some, all but one, all), tree counts on and off the warp width, negative entries (read as 0 on both sides),
+and a routed batch whose decision with nothing excluded must equal the route's own choice."""
 import random
 
 import numpy as np
@@ -46,6 +46,21 @@ def test_random_matrices_and_masks(P):
             gp, gn = _decide(r, match, load, alpha, ex)
             op, on = oracle.decide(match, load, alpha, ex)
             assert np.array_equal(gp, op) and np.array_equal(gn, on), (P, alpha, None if ex is None else ex.sum())
+
+
+@pytest.mark.parametrize("P", [3, 40])
+def test_negative_entries_count_as_zero(P):
+    rng = np.random.default_rng(100 + P)
+    B = 1500
+    r = g.Router(P)
+    match = rng.integers(-6, 6, size=(B, P), dtype=np.int32)
+    match[::7, 0] = np.iinfo(np.int32).min  # the most negative entry too
+    load = rng.integers(0, 4, size=P).astype(np.int32)
+    for alpha in (0, 1, 5):
+        for ex in (None, (rng.random(P) < 0.3).astype(np.uint8)):
+            gp, gn = _decide(r, match, load, alpha, ex)
+            op, on = oracle.decide(match, load, alpha, ex)
+            assert np.array_equal(gp, op) and np.array_equal(gn, on), (P, alpha)
 
 
 def test_decision_of_a_routed_batch():
