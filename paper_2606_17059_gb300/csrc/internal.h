@@ -109,12 +109,11 @@ struct GroupScratch {
 cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
                          const GroupScratch& g, int num_sms, cudaStream_t st);
 
-// Route kernels (lookup + route decision), see route_kernel.cu.  Without groups (g == nullptr) one launch
-// routes every request; with groups, a leader pass and a follower pass.  *launched is set to the number of
-// kernels launched.
 // Best and next-best non-excluded peer of every row of match [B x P] (route_key order); -1 where none.
 cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,
                           const uint8_t* d_excluded, int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st);
+// Route kernels (lookup + route decision) of a grouped batch, see route_kernel.cu: a leader pass and a
+// follower pass (g is required).  *launched is set to the number of kernels launched.
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens,
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
                          int32_t* out_match, int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms,

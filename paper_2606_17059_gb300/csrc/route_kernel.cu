@@ -6,7 +6,7 @@
 //
 // Passes.  A grouped batch (group_kernel.cu) is routed by a leader pass and a follower pass.  Leaders of
 // short requests, and all followers, are walked by lane_kernel (a lane per tree; below).  Leaders whose
-// requests are longer than a staging window on average, and batches too large to group, go to route_kernel:
+// requests are longer than a staging window on average go to route_kernel:
 //
 // route_kernel schedule.  A CTA takes requests b = list[blockIdx.x], list[blockIdx.x + gridDim.x], ...; its
 // work items are (request, group of G consecutive trees) in that order, handed to warps from a shared
@@ -255,7 +255,7 @@ __device__ __forceinline__ unsigned long long route_key(int32_t m, int32_t ld, i
          (unsigned long long)(0xFFFF - p);
 }
 
-// Routes requests list[0 .. *count) (every request b < B if list is NULL) with full walks.
+// Routes the leaders list[0 .. *count) of a grouped batch with full walks.
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ list,
@@ -277,7 +277,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
   }
   if (threadIdx.x == 0) s_next = 0;
   __syncthreads();
-  const int64_t n_all = count ? (int64_t)*count : B;  // requests of this launch
+  const int64_t n_all = *count;  // requests of this launch
   const int64_t n_req = n_all > blockIdx.x ? (n_all - blockIdx.x + gridDim.x - 1) / gridDim.x : 0;
   // A work item is (request k, trees p0 .. p0 + G - 1): G grows with P so that the per-item costs (the
   // shared counter, the staging waits, the route-key merge) are shared by several walks while every warp of
@@ -303,7 +303,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     }
     const int s = (int)(k % kSlots);
     const int64_t kb = blockIdx.x + k * gridDim.x;
-    const int64_t b = list ? (int64_t)__ldg(list + kb) : kb;
+    const int64_t b = __ldg(list + kb);
     Slot& sl = s_slot[s];
     int32_t* st = s_tok + s * kSlotTokens;
     if (c == 0) {
@@ -350,8 +350,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
         sl.shift = shift;
         sl.best = 0;
         sl.done = 0;
-        sl.row = gid ? __ldg(gid + b) : -1;
-        sl.climit = gid ? __ldg(cmin + b) : -1;
+        sl.row = __ldg(gid + b);
+        sl.climit = __ldg(cmin + b);
         __threadfence_block();
         *(volatile int*)&sl.ready = (int)k;
       }
@@ -776,17 +776,7 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          int* launched) {
   *launched = 0;
   if (B <= 0) return cudaSuccess;
-  if (!g) {  // ungrouped: the staged kernel over every request
-    const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
-    cudaError_t e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
-    const int grid = (int)(B < max_ctas ? B : max_ctas);
-    route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, nullptr, nullptr,
-                                               nullptr, nullptr, nullptr, d_load, alpha, out_match, out_peer, d_err);
-    *launched = 1;
-    return cudaGetLastError();
-  }
+  if (!g) return cudaErrorInvalidValue;  // every batch is grouped first
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
   cudaError_t e;

@@ -23,6 +23,8 @@ constexpr int kLoadRing = 8;
 // kPipeRequests requests each.
 constexpr int kPipe = 8;
 constexpr int64_t kPipeRequests = 131072;
+// Largest batch of one routing call: the grouping kernels and the pass lists index requests with int32.
+constexpr int64_t kMaxBatch = (int64_t)1 << 30;
 
 struct DevBuf {
   void* p = nullptr;
@@ -193,17 +195,10 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
   return cudaSuccess;
 }
 
-// Groups the batch by shared prefix and routes it (leaders, then followers); batches too large for 32-bit
-// request indices are routed in one ungrouped pass.
+// Groups the batch by shared prefix and routes it (leaders, then followers).  The callers check B <= kMaxBatch
+// (request indices and list positions are 32-bit).
 int route(p2p_router* r, const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
           int32_t alpha, int32_t* out_match, int32_t* out_peer) {
-  if (B > ((int64_t)1 << 30)) {
-    int launched = 0;
-    CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
-                         r->d_err, nullptr, r->num_sms, r->stream, &launched));
-    r->launches += launched;
-    return P2P_OK;
-  }
   p2p::GroupScratch g;
   CK(group_scratch(r, B, g));
   CK(p2p::launch_group(tokens, n_tokens, tok_base, offsets, B, g, r->num_sms, r->stream));
@@ -1071,6 +1066,7 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
                     const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
   if (B < 0 || n_tokens < 0) return fail(r, P2P_E_INVAL, "negative B or n_tokens");
+  if (B > kMaxBatch) return fail(r, P2P_E_INVAL, "B exceeds 2^30 requests per call: split the batch");
   if (int rc = check_load(r, load, alpha)) return rc;
   if (B == 0) return P2P_OK;
   if (!offsets || !out_match || !out_peer || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
@@ -1098,6 +1094,7 @@ int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* of
                          int32_t alpha, int32_t* out_match, int32_t* out_peer) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
   if (B < 0) return fail(r, P2P_E_INVAL, "negative B");
+  if (B > kMaxBatch) return fail(r, P2P_E_INVAL, "B exceeds 2^30 requests per call: split the batch");
   if (int rc = check_load(r, load, alpha)) return rc;
   if (B == 0) return P2P_OK;
   if (!offsets || !out_match || !out_peer) return fail(r, P2P_E_INVAL, "NULL host pointer");
