@@ -202,6 +202,11 @@ def test_invalid_arguments_are_rejected():
         r.upload(0, bad)
     assert e.value.code == g.P2P_E_FORMAT
     assert np.all(r.download(0)["label_off"] == 0)  # unchanged (still empty)
+    # More than 2^30 requests in one call: rejected before any device pointer is read.
+    big = (1 << 30) + 1
+    with pytest.raises(g.P2PError) as e:
+        g.p2p_route_batch(r.handle, tok, 4, off, big, [0, 0], 1, tok, tok)
+    assert e.value.code == g.P2P_E_INVAL and "2^30" in str(e.value)
 
 
 def test_route_on_a_side_stream():
