@@ -1,9 +1,12 @@
 """GPU parity at the full sizes of the stale-replica workload (P=64, 262,144 requests) and the scale workload
-(P=256 trees of 100,000 sequences, 1,048,576 requests, a 5% + 5% delta per replica), in the launch
-configuration the bench times.  The stale-replica workload is compared in full; for the scale workload the
-oracle cannot hold all 256 trees in a test, so outputs are sampled: match columns of sampled trees for
-sampled requests, the route of every sampled request recomputed from its GPU match row, and the patched
-trees of sampled replicas byte for byte."""
+(P=256 trees of 100,000 sequences, 1,048,576 requests, a 5% + 5% delta per replica per batch), in the launch
+configuration the bench times.  Both are compared in full: every match value, every chosen peer, and every
+patched tree byte for byte against the oracle.  The scale workload first runs anti-entropy rounds until the
+delta call compacts the replicas in one wave (and one round after it), so the compaction path is compared
+at full size too."""
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 import pytest
 
@@ -53,40 +56,66 @@ def test_stale_replica_workload_full_size():
     assert_same_route(hm, hp, gm, gp, "host-pointer call in chunks")
 
 
-def test_scale_workload_sampled_outputs():
+def _build_router(W, n_threads):
+    """Snapshots built on host threads, uploaded in order (as the bench does)."""
+    r = g.Router(W.P)
+
+    def make(p):
+        return g.p2p_snapshot_build(W.tree(p))
+
+    with ThreadPoolExecutor(max_workers=n_threads) as ex:
+        for p, snap in enumerate(ex.map(make, range(W.P))):
+            flat = g.FlatTree()
+            g._load().p2p_snapshot_view(snap, flat)
+            g._check(g._load().p2p_tree_upload(r.handle, p, flat), r.handle)
+            g.p2p_snapshot_free(snap)
+    r.sync()
+    return r
+
+
+def test_scale_workload_full_after_a_compaction_wave():
+    import torch
     W = wl.Workload(4)
     P, B = W.P, W.B
-    r = g.Router(P)
-    for p in range(P):
-        r.build(p, W.tree(p))
-    rng = np.random.default_rng(4)
-    sample_trees = sorted(rng.choice(P, size=6, replace=False).tolist())
-    otrees = {p: t for p, t in zip(sample_trees, oracle.build_trees([W.tree(p) for p in sample_trees], n_threads=16))}
-    # One anti-entropy round on every replica (device), the same ops on the sampled oracle trees.
-    W.delta_make(0, W.params["delta_frac"], W.params["delta_frac"], n_threads=16)
-    d = W.delta(n_threads=16)
-    assert r.apply_delta(-1, d.op, d.seqs, d.peer_begin) == 0
-    for p in sample_trees:
-        assert otrees[p].apply_ops(d.op, d.seqs, int(d.peer_begin[p]), int(d.peer_begin[p + 1])) == 0
-    for p in sample_trees[:3]:
-        assert same_snapshot(r.download(p), otrees[p].export()), p
-    # The full batch on the device.
-    tok, off = W.requests(n_threads=16)
+    nt = os.cpu_count() or 8
+    r = _build_router(W, nt)
+    otrees = oracle.build_trees([W.tree(p) for p in range(P)], n_threads=nt)
+    frac = W.params["delta_frac"]
+
+    def stale_labels():
+        return np.array([r.stats(p)["stale_label"] for p in range(P)])
+
+    wave = None
+    for s in range(40):
+        W.delta_make(s, frac, frac, n_threads=nt)
+        d = W.delta(n_threads=nt)
+        before = stale_labels()
+        if s % 2:  # odd rounds from device arrays (the bench's path), even rounds from host arrays
+            dev = lambda a: torch.from_numpy(np.ascontiguousarray(a)).cuda()
+            sl = wl.SeqList(dev(d.seqs.seg_begin), dev(d.seqs.seg_off), dev(d.seqs.seg_len), dev(d.seqs.pool))
+            assert r.apply_delta(-1, dev(d.op), sl, dev(d.peer_begin), on_device=True) == 0
+        else:
+            assert r.apply_delta(-1, d.op, d.seqs, d.peer_begin) == 0
+
+        def apply(p):
+            return otrees[p].apply_ops(d.op, d.seqs, int(d.peer_begin[p]), int(d.peer_begin[p + 1]))
+
+        with ThreadPoolExecutor(max_workers=nt) as ex:
+            assert sum(ex.map(apply, range(P))) == 0
+        compacted = int((stale_labels() < before).sum())
+        if wave is not None:
+            break  # one more round on the compacted trees
+        if compacted >= P // 2:
+            wave = (s, compacted)
+    assert wave is not None, "no compaction wave in 40 anti-entropy rounds"
+    # The full batch on the device, and the oracle over all 256 trees.
+    tok, off = W.requests(n_threads=nt)
     load = W.load()
     gm, gp = _route_full(r, tok, off, load, W.alpha)
-    assert gm.shape == (B, P) and gp.min() >= 0 and gp.max() < P
-    lens = np.diff(off)
-    assert np.all(gm <= lens[:, None]) and gm.max() > 1000
-    # Sampled requests: match columns of the sampled trees, and the route from each full GPU match row.
-    reqs = np.sort(rng.choice(B, size=20000, replace=False))
-    sub_tok = np.concatenate([tok[off[b]:off[b + 1]] for b in reqs])
-    sub_off = np.zeros(len(reqs) + 1, np.int64)
-    np.cumsum(lens[reqs], out=sub_off[1:])
-    om, _, _ = oracle.route([otrees[p] for p in sample_trees], sub_tok, sub_off, load[sample_trees], W.alpha,
-                            n_threads=16)
-    got = gm[reqs][:, sample_trees]
-    bad = np.argwhere(got != om)
-    assert len(bad) == 0, f"{len(bad)} sampled match mismatches, first {bad[:3].tolist()}"
-    for i in range(0, len(reqs), 7):
-        b = reqs[i]
-        assert oracle.argmax_peer(gm[b], load, W.alpha) == gp[b], b
+    om, op, _ = oracle.route(otrees, tok, off, load, W.alpha, n_threads=nt)
+    assert gm.max() > 1000
+    assert_same_route(gm, gp, om, op, f"scale workload, full size, after the compaction wave of round {wave[0]}")
+    del gm, om
+    # Every patched replica byte for byte.
+    for p in range(P):
+        assert same_snapshot(r.download(p), otrees[p].export()), p
