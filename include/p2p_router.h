@@ -133,6 +133,18 @@ int32_t p2p_router_num_trees(const p2p_router* r);
  * lets a caller count the device work a region of code issued.  Not part of the paper's method. */
 int64_t p2p_router_launch_count(const p2p_router* r);
 
+/* Kernel clock, a measurement aid (not part of the paper's method).  With on != 0 the router records a CUDA
+ * event pair on its stream around each of its kernel launches and sums the device time per kernel; the
+ * totals start from zero.  on = 0 switches the clock off and drops the totals.  Waits for queued work.
+ * Each pair adds an event record before and after the launch, a few microseconds of stream work. */
+int p2p_router_kernel_clock(p2p_router* r, int32_t on);
+
+/* Totals of kernel i (0 <= i < 16, an index into the library's list of kernels) since the clock was
+ * switched on: *name (nullable) receives the kernel's name (a static string), *launches and *ms (nullable)
+ * the timed launches and their summed device time in milliseconds; 0 and 0.0 while the clock is off.
+ * Waits for queued work.  Errors: P2P_E_INVAL (i out of range), P2P_E_CUDA. */
+int p2p_router_kernel_time(p2p_router* r, int32_t i, const char** name, int64_t* launches, double* ms);
+
 /* ---- snapshots (host only; no GPU needed) ---------------------------------------------------------- */
 
 /* Builds the canonical snapshot of the multiset `seqs` (host pointers), i.e. the radix tree a node would

@@ -21,6 +21,7 @@ __all__ = [
     "p2p_router_num_trees", "p2p_router_launch_count", "p2p_snapshot_build", "p2p_snapshot_view", "p2p_snapshot_free",
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
     "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host", "p2p_route_decide",
+    "p2p_router_kernel_clock", "p2p_router_kernel_time",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -93,6 +94,8 @@ def _load():
             "p2p_route_batch": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, _i32, _vp, _vp]),
             "p2p_route_batch_host": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _i32, _vp, _vp]),
             "p2p_route_decide": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp]),
+            "p2p_router_kernel_clock": (ctypes.c_int, [_vp, _i32]),
+            "p2p_router_kernel_time": (ctypes.c_int, [_vp, _i32, P(ctypes.c_char_p), P(_i64), P(ctypes.c_double)]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(lib, name)
@@ -190,6 +193,22 @@ def p2p_router_num_trees(r) -> int:
 
 def p2p_router_launch_count(r) -> int:
     return int(_load().p2p_router_launch_count(r))
+
+
+KERNEL_COUNT = 16  # kernels the kernel clock keeps totals for (indices 0 .. 15)
+
+
+def p2p_router_kernel_clock(r, on: bool) -> None:
+    _check(_load().p2p_router_kernel_clock(r, 1 if on else 0), r)
+
+
+def p2p_router_kernel_time(r, i: int) -> tuple[str, int, float]:
+    """(kernel name, timed launches, summed device ms) of kernel i since the clock was switched on."""
+    name = ctypes.c_char_p()
+    n = _i64()
+    ms = ctypes.c_double()
+    _check(_load().p2p_router_kernel_time(r, i, ctypes.byref(name), ctypes.byref(n), ctypes.byref(ms)), r)
+    return (name.value.decode() if name.value else ""), int(n.value), float(ms.value)
 
 
 def p2p_snapshot_build(seqlist):
@@ -374,6 +393,18 @@ class Router:
 
     def launch_count(self) -> int:
         return p2p_router_launch_count(self._h)
+
+    def kernel_clock(self, on: bool) -> None:
+        p2p_router_kernel_clock(self._h, on)
+
+    def kernel_times(self) -> dict:
+        """{kernel name: (launches, summed device ms)} of the kernels launched since the clock was switched on."""
+        out = {}
+        for i in range(KERNEL_COUNT):
+            name, n, ms = p2p_router_kernel_time(self._h, i)
+            if n:
+                out[name] = (n, ms)
+        return out
 
     def route(self, tokens, offsets, load, alpha: int, out_match=None, out_peer=None):
         """tokens (int32) and offsets (int64) are CUDA tensors; returns (match [B,P], peer [B]) tensors."""

@@ -1343,16 +1343,17 @@ __global__ void refresh_views_kernel(const TreeState* st, TreeView* view, int32_
 cudaError_t launch_refresh_views(const TreeState* d_states, TreeView* d_views, int32_t n, const int32_t* shared,
                                  cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
-  refresh_views_kernel<<<(n + 127) / 128, 128, 0, st>>>(d_states, d_views, n, shared);
+  P2P_TIMED(K_REFRESH_VIEWS, st, (refresh_views_kernel<<<(n + 127) / 128, 128, 0, st>>>(d_states, d_views, n, shared)));
   return cudaGetLastError();
 }
 
 cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, int32_t max_cap_node, int num_sms, cudaStream_t st) {
   if (n_jobs <= 0) return cudaSuccess;
-  compact_kernel<<<n_jobs, kCompactThreads, 0, st>>>(d_jobs);
+  P2P_TIMED(K_COMPACT, st, (compact_kernel<<<n_jobs, kCompactThreads, 0, st>>>(d_jobs)));
   const int32_t groups = (max_cap_node + 31) / 32;
-  compact_labels_kernel<<<std::max(num_sms, 1) * kLabelCtasPerSm, kLabelThreads, 0, st>>>(
-      d_jobs, (int64_t)n_jobs * groups, groups);
+  P2P_TIMED(K_COMPACT_LABELS, st,
+            (compact_labels_kernel<<<std::max(num_sms, 1) * kLabelCtasPerSm, kLabelThreads, 0, st>>>(
+                d_jobs, (int64_t)n_jobs * groups, groups)));
   return cudaGetLastError();
 }
 
@@ -1363,8 +1364,9 @@ cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, co
   const int dyn = delta_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
   if (e != cudaSuccess) return e;
-  delta_kernel<<<n_trees, kDeltaWarps * 32, dyn, st>>>(d_states, done, op, seg_begin, seg_off, seg_len, pool, gather,
-                                                       gather_stride, shared);
+  P2P_TIMED(K_DELTA, st,
+            (delta_kernel<<<n_trees, kDeltaWarps * 32, dyn, st>>>(d_states, done, op, seg_begin, seg_off, seg_len, pool,
+                                                                  gather, gather_stride, shared)));
   return cudaGetLastError();
 }
 
@@ -1373,20 +1375,21 @@ cudaError_t launch_validate(int32_t* header, const p2p_delta* d, int32_t peer, i
   if (e != cudaSuccess) return e;
   const p2p_seqs& S = d->seqs;
   const int64_t blocks = std::min<int64_t>((S.n + 255) / 256, 4096);
-  validate_kernel<<<(int)std::max<int64_t>(blocks, 1), 256, 0, st>>>(header, d->op, S.seg_begin, S.seg_off, S.seg_len,
-                                                                    S.n, S.n_segs, S.n_pool,
-                                                                    peer == -1 ? d->peer_begin : nullptr, P);
+  P2P_TIMED(K_VALIDATE, st,
+            (validate_kernel<<<(int)std::max<int64_t>(blocks, 1), 256, 0, st>>>(
+                header, d->op, S.seg_begin, S.seg_off, S.seg_len, S.n, S.n_segs, S.n_pool,
+                peer == -1 ? d->peer_begin : nullptr, P)));
   return cudaGetLastError();
 }
 
 cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* peer_begin, int64_t n, cudaStream_t st) {
-  init_ranges_kernel<<<(nt + 127) / 128, 128, 0, st>>>(d_states, nt, peer_begin, n);
+  P2P_TIMED(K_INIT_RANGES, st, (init_ranges_kernel<<<(nt + 127) / 128, 128, 0, st>>>(d_states, nt, peer_begin, n)));
   return cudaGetLastError();
 }
 
 cudaError_t launch_set_tree(TreeState* d_state, TreeView* d_view, TreeState value, const int32_t* shared,
                             cudaStream_t st) {
-  set_tree_kernel<<<1, 1, 0, st>>>(d_state, d_view, value, shared);
+  P2P_TIMED(K_SET_TREE, st, (set_tree_kernel<<<1, 1, 0, st>>>(d_state, d_view, value, shared)));
   return cudaGetLastError();
 }
 

@@ -240,19 +240,24 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   const int64_t resolve_ctas = (B + kGroupThreads / 32 - 1) / (kGroupThreads / 32);            // a warp per request
   const int grid = (int)std::min<int64_t>(hash_ctas, (int64_t)num_sms * 8);
   const int grid2 = (int)std::min<int64_t>(resolve_ctas, (int64_t)num_sms * 8);
-  group_hash_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.keys, g.vals, g.bits,
-                                                    g.slot_of);
+  P2P_TIMED(K_GROUP_HASH, st,
+            (group_hash_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.keys, g.vals,
+                                                               g.bits, g.slot_of)));
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   // Large batches: a warp per 32 requests (at least 32 warps per SM still busy; fewest atomics).  Smaller
   // ones: a warp per request, so that the common-prefix compares spread over as many warps as there are
   // requests.
   if (B >= (int64_t)num_sms * 32 * 32) {
-    group_resolve32_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
-                                                           g.lead, g.cpre, g.lists, g.counts, g.gid, g.cmin, g.gcap);
+    P2P_TIMED(K_GROUP_RESOLVE32, st,
+              (group_resolve32_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals,
+                                                                      g.slot_of, g.lead, g.cpre, g.lists, g.counts,
+                                                                      g.gid, g.cmin, g.gcap)));
   } else {
-    group_resolve_kernel<<<grid2, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals, g.slot_of,
-                                                          g.lead, g.cpre, g.lists, g.counts, g.gid, g.cmin, g.gcap);
+    P2P_TIMED(K_GROUP_RESOLVE, st,
+              (group_resolve_kernel<<<grid2, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals,
+                                                                     g.slot_of, g.lead, g.cpre, g.lists, g.counts,
+                                                                     g.gid, g.cmin, g.gcap)));
   }
   return cudaGetLastError();
 }

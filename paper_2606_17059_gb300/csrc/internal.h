@@ -85,6 +85,31 @@ inline __host__ __device__ bool tab_full(int32_t bits, int64_t used_after) {
 }
 constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits of meta
 
+// Kernel clock: per-kernel device time of a router's launches, a measurement aid (not part of the method).
+// Launchers bracket every launch with clock_mark(id, ...); a router whose clock is on installs it in
+// t_clock for the duration of an API call on the calling thread (one router per host thread at a time).
+enum KernelId {
+  K_GROUP_HASH, K_GROUP_RESOLVE, K_GROUP_RESOLVE32, K_ROUTE_STAGED, K_LANE_LEADER, K_LANE_FOLLOWER, K_DECIDE,
+  K_VALIDATE, K_INIT_RANGES, K_DELTA, K_COMPACT, K_COMPACT_LABELS, K_REFRESH_VIEWS, K_SET_TREE,
+  K_UPDATE_COUNT, K_UPDATE_SCATTER, K_COUNT_
+};
+const char* kernel_name(int id);
+struct KernelClock {
+  virtual void mark(int id, bool end, cudaStream_t st) = 0;
+  virtual ~KernelClock() = default;
+};
+extern thread_local KernelClock* t_clock;
+inline void clock_mark(int id, bool end, cudaStream_t st) {
+  if (t_clock) t_clock->mark(id, end, st);
+}
+// One timed launch: the variadic part is the kernel<<<...>>>(...) expression.
+#define P2P_TIMED(id, st, ...)          \
+  do {                                  \
+    ::p2p::clock_mark(id, false, st);   \
+    __VA_ARGS__;                        \
+    ::p2p::clock_mark(id, true, st);    \
+  } while (0)
+
 // Bits of the router's device error word.
 enum { ERR_BAD_OFFSETS = 1, ERR_CORRUPT_TREE = 2, ERR_STALL = 4 };
 

@@ -788,21 +788,27 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
     if (e != cudaSuccess) return e;
     const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
     const int grid = (int)(B < max_ctas ? B : max_ctas);
-    route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists, g->counts,
-                                               g->gid, g->cmin, g->ckpt, d_load, alpha, out_match, out_peer, d_err);
+    P2P_TIMED(K_ROUTE_STAGED, st,
+              (route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists,
+                                                          g->counts, g->gid, g->cmin, g->ckpt, d_load, alpha, out_match,
+                                                          out_peer, d_err)));
     *launched = 1;
   } else {
     // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
-    lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists,
-                                                        g->counts, nullptr, nullptr, g->gid, g->cmin, g->ckpt, d_load,
-                                                        alpha, out_match, out_peer, d_err, g->counts + 3);
+    P2P_TIMED(K_LANE_LEADER, st,
+              (lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
+                                                                   g->lists, g->counts, nullptr, nullptr, g->gid,
+                                                                   g->cmin, g->ckpt, d_load, alpha, out_match, out_peer,
+                                                                   d_err, g->counts + 3)));
     *launched = 1;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B,
-                                                       g->counts + 1, g->lead, g->cpre, g->gid, nullptr, g->ckpt, d_load,
-                                                       alpha, out_match, out_peer, d_err, nullptr);
+  P2P_TIMED(K_LANE_FOLLOWER, st,
+            (lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
+                                                                  g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
+                                                                  nullptr, g->ckpt, d_load, alpha, out_match, out_peer,
+                                                                  d_err, nullptr)));
   *launched += 1;
   return cudaGetLastError();
 }
@@ -812,7 +818,7 @@ cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int3
   if (B <= 0) return cudaSuccess;
   const int64_t want = (B + 7) / 8;
   const int grid = (int)std::min<int64_t>(want, (int64_t)std::max(num_sms, 1) * 8);
-  decide_kernel<<<grid, 256, 0, st>>>(match, B, P, d_load, alpha, d_excluded, out_peer, out_next);
+  P2P_TIMED(K_DECIDE, st, (decide_kernel<<<grid, 256, 0, st>>>(match, B, P, d_load, alpha, d_excluded, out_peer, out_next)));
   return cudaGetLastError();
 }
 

@@ -79,6 +79,96 @@ void table_put(int4* tab, int32_t bits, const int4& e) {
 
 }  // namespace
 
+namespace p2p {
+
+thread_local KernelClock* t_clock = nullptr;
+
+const char* kernel_name(int id) {
+  static const char* const names[K_COUNT_] = {
+      "group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel", "route_kernel", "lane_kernel<true>",
+      "lane_kernel<false>", "decide_kernel", "validate_kernel", "init_ranges_kernel", "delta_kernel",
+      "compact_kernel", "compact_labels_kernel", "refresh_views_kernel", "set_tree_kernel", "update_count_kernel",
+      "update_scatter_kernel"};
+  return id >= 0 && id < K_COUNT_ ? names[id] : "";
+}
+
+}  // namespace p2p
+
+namespace {
+
+// The router's kernel clock: an event pair recorded around each launch on the launch stream; the pairs are
+// resolved into per-kernel totals when the totals are read (or when many are pending).
+struct RouterClock final : p2p::KernelClock {
+  struct Pending {
+    int id;
+    cudaEvent_t a, b;
+  };
+  std::vector<cudaEvent_t> spare;
+  std::vector<Pending> pending;
+  int open_id = -1;
+  cudaEvent_t open_ev = nullptr;
+  double ms[p2p::K_COUNT_] = {};
+  int64_t n[p2p::K_COUNT_] = {};
+  cudaError_t err = cudaSuccess;
+
+  cudaEvent_t get() {
+    if (!spare.empty()) {
+      cudaEvent_t e = spare.back();
+      spare.pop_back();
+      return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+      err = cudaErrorMemoryAllocation;
+      return nullptr;
+    }
+    return e;
+  }
+  void mark(int id, bool end, cudaStream_t st) override {
+    if (!end) {
+      open_id = id;
+      open_ev = get();
+      if (open_ev) cudaEventRecord(open_ev, st);
+      return;
+    }
+    cudaEvent_t b = get();
+    if (open_ev && b && open_id == id) {
+      cudaEventRecord(b, st);
+      pending.push_back(Pending{id, open_ev, b});
+    } else {
+      if (open_ev) spare.push_back(open_ev);
+      if (b) spare.push_back(b);
+    }
+    open_ev = nullptr;
+    open_id = -1;
+    if (pending.size() >= 65536) resolve();
+  }
+  // Waits for the pending pairs and adds them to the totals.
+  void resolve() {
+    for (const Pending& q : pending) {
+      float t = 0.f;
+      if (cudaEventSynchronize(q.b) == cudaSuccess && cudaEventElapsedTime(&t, q.a, q.b) == cudaSuccess) {
+        ms[q.id] += t;
+        n[q.id] += 1;
+      }
+      spare.push_back(q.a);
+      spare.push_back(q.b);
+    }
+    pending.clear();
+  }
+  void reset() {
+    resolve();
+    std::fill(ms, ms + p2p::K_COUNT_, 0.0);
+    std::fill(n, n + p2p::K_COUNT_, 0);
+  }
+  ~RouterClock() override {
+    resolve();
+    for (cudaEvent_t e : spare) cudaEventDestroy(e);
+  }
+};
+
+}  // namespace
+
 struct p2p_router {
   int32_t P = 0;
   int device = 0;
@@ -109,6 +199,7 @@ struct p2p_router {
   DevBuf grp_keys, grp_vals, grp_req, grp_ckpt;  // shared-prefix grouping of a batch
   DevBuf cmp_jobs, cmp_queue;          // device compaction
   int64_t launches = 0;  // kernels this router has launched
+  RouterClock* clock = nullptr;  // per-kernel device time, while switched on
   // Shared label pool: long labels interned across trees (device array, host mirror, content index).
   int32_t* d_shared = nullptr;
   int64_t shared_cap = 0;
@@ -119,14 +210,22 @@ struct p2p_router {
 
 namespace {
 
-// Makes the router's device current for the duration of a call.
+// Makes the router's device current for the duration of a call, and installs its kernel clock (if on) on
+// the calling thread.
 struct DeviceGuard {
   int prev = -1;
   bool changed = false;
+  p2p::KernelClock* prev_clock = nullptr;
+  explicit DeviceGuard(const p2p_router* r) : DeviceGuard(r->device) {
+    prev_clock = p2p::t_clock;
+    p2p::t_clock = r->clock;
+  }
   explicit DeviceGuard(int dev) {
+    prev_clock = p2p::t_clock;
     if (cudaGetDevice(&prev) == cudaSuccess && prev != dev) changed = cudaSetDevice(dev) == cudaSuccess;
   }
   ~DeviceGuard() {
+    p2p::t_clock = prev_clock;
     if (changed) cudaSetDevice(prev);
   }
 };
@@ -736,7 +835,7 @@ int p2p_router_create(int32_t P, p2p_router** out) {
 
 void p2p_router_destroy(p2p_router* r) {
   if (!r) return;
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   cudaStreamSynchronize(r->stream);
   if (r->pool) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
@@ -772,12 +871,13 @@ void p2p_router_destroy(p2p_router* r) {
   if (r->h_mask) cudaFreeHost(r->h_mask);
   if (r->h_err) cudaFreeHost(r->h_err);
   if (r->h_states) cudaFreeHost(r->h_states);
+  delete r->clock;
   delete r;
 }
 
 int p2p_router_set_stream(p2p_router* r, void* stream) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   CK(cudaStreamSynchronize(r->stream));
   r->stream = (cudaStream_t)stream;
   return P2P_OK;
@@ -785,7 +885,7 @@ int p2p_router_set_stream(p2p_router* r, void* stream) {
 
 int p2p_router_sync(p2p_router* r) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   return do_sync(r);
 }
 
@@ -795,9 +895,43 @@ int32_t p2p_router_num_trees(const p2p_router* r) { return r ? r->P : 0; }
 
 int64_t p2p_router_launch_count(const p2p_router* r) { return r ? r->launches : 0; }
 
+int p2p_router_kernel_clock(p2p_router* r, int32_t on) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  DeviceGuard g(r->device);
+  CK(cudaStreamSynchronize(r->stream));
+  if (on) {
+    if (!r->clock) r->clock = new RouterClock();
+    r->clock->reset();
+  } else if (r->clock) {
+    r->clock->resolve();
+    delete r->clock;
+    r->clock = nullptr;
+  }
+  return P2P_OK;
+}
+
+int p2p_router_kernel_time(p2p_router* r, int32_t i, const char** name, int64_t* launches, double* ms) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (i < 0 || i >= p2p::K_COUNT_) return fail(r, P2P_E_INVAL, "kernel index out of range");
+  if (name) *name = p2p::kernel_name(i);
+  int64_t n = 0;
+  double t = 0.0;
+  if (r->clock) {
+    DeviceGuard g(r->device);
+    CK(cudaStreamSynchronize(r->stream));
+    r->clock->resolve();
+    if (r->clock->err != cudaSuccess) return cuda_fail(r, r->clock->err, "kernel clock");
+    n = r->clock->n[i];
+    t = r->clock->ms[i];
+  }
+  if (launches) *launches = n;
+  if (ms) *ms = t;
+  return P2P_OK;
+}
+
 int p2p_tree_upload(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   if (int rc = check_peer(r, peer)) return rc;
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   return upload_flat(r, peer, t);
 }
 
@@ -809,7 +943,7 @@ int p2p_tree_build(p2p_router* r, int32_t peer, const p2p_seqs* seqs) {
   if (!p2p::build_snapshot(*seqs, snap, err)) return fail(r, P2P_E_NOMEM, err);
   p2p_flat_tree v;
   p2p_snapshot_view(&snap, &v);
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   return upload_flat(r, peer, &v);
 }
 
@@ -817,7 +951,7 @@ int p2p_tree_download(p2p_router* r, int32_t peer, p2p_snapshot** out) {
   if (int rc = check_peer(r, peer)) return rc;
   if (!out) return fail(r, P2P_E_INVAL, "out is NULL");
   *out = nullptr;
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   p2p_snapshot* s = new p2p_snapshot();
   const int rc = download(r, peer, s);
   if (rc != P2P_OK) {
@@ -831,7 +965,7 @@ int p2p_tree_download(p2p_router* r, int32_t peer, p2p_snapshot** out) {
 int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]) {
   if (int rc = check_peer(r, peer)) return rc;
   if (!out) return fail(r, P2P_E_INVAL, "out is NULL");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   CK(cudaStreamSynchronize(r->stream));
   const TreeState& t = r->hs[(size_t)peer];
   const int64_t v[9] = {(int64_t)t.n_node - t.dead_nodes, t.n_node, t.n_child, t.n_label, t.stale_child,
@@ -845,7 +979,7 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   if (peer < -1 || peer >= r->P) return fail(r, P2P_E_INVAL, "peer out of range");
   if (!d) return fail(r, P2P_E_INVAL, "delta is NULL");
   if (d->mem != P2P_MEM_HOST && d->mem != P2P_MEM_DEVICE) return fail(r, P2P_E_INVAL, "delta.mem must be HOST or DEVICE");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   const p2p_seqs& S = d->seqs;
   const int64_t n = S.n;
   if (n < 0 || S.n_segs < 0 || S.n_pool < 0) return fail(r, P2P_E_INVAL, "negative size in delta");
@@ -1005,7 +1139,7 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
   if (S.n > 0 && (!d->op || !S.seg_begin || (S.n_segs > 0 && (!S.seg_off || !S.seg_len)) || (S.n_pool > 0 && !S.pool)))
     return fail(r, P2P_E_INVAL, "NULL array in delta");
   if (peer == -1 && S.n > 0 && !d->peer_begin) return fail(r, P2P_E_INVAL, "peer = -1 needs peer_begin");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   int32_t* header = nullptr;
   int32_t* tokens = nullptr;
   CK(p2p::static_scratch(r->device, &header, &tokens));
@@ -1070,7 +1204,7 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
   if (int rc = check_load(r, load, alpha)) return rc;
   if (B == 0) return P2P_OK;
   if (!offsets || !out_match || !out_peer || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   if (int rc = stage_load(r, load)) return rc;
   return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer);
 }
@@ -1082,7 +1216,7 @@ int p2p_route_decide(p2p_router* r, const int32_t* match, int64_t B, const int32
   if (int rc = check_load(r, load, alpha)) return rc;
   if (B == 0) return P2P_OK;
   if (!match || !out_peer || !out_next) return fail(r, P2P_E_INVAL, "NULL device pointer");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   if (int rc = stage_load(r, load, excluded)) return rc;
   CK(p2p::launch_decide(match, B, r->P, r->d_load, alpha, excluded ? r->d_mask : nullptr, out_peer, out_next,
                         r->num_sms, r->stream));
@@ -1103,7 +1237,7 @@ int p2p_route_batch_host(p2p_router* r, const int32_t* tokens, const int64_t* of
     if (offsets[b + 1] < offsets[b]) return fail(r, P2P_E_INVAL, "offsets decrease at " + std::to_string(b));
   const int64_t n_tok = offsets[B] - offsets[0];
   if (n_tok > 0 && !tokens) return fail(r, P2P_E_INVAL, "tokens is NULL");
-  DeviceGuard g(r->device);
+  DeviceGuard g(r);
   CK(ensure(r, r->req_tok, (size_t)std::max<int64_t>(n_tok, 1) * sizeof(int32_t)));
   CK(ensure(r, r->req_off, (size_t)(B + 1) * sizeof(int64_t)));
   CK(ensure(r, r->out_match, (size_t)B * r->P * sizeof(int32_t)));

@@ -223,3 +223,30 @@ def test_route_on_a_side_stream():
     r.sync()
     om, op = oracle_route(sls, tok, off, W.load(), W.alpha)
     assert_same_route(m.cpu().numpy(), p.cpu().numpy(), om, op, "side stream")
+
+
+def test_kernel_clock_counts_every_launch():
+    import torch
+    W = wl.Workload(0)
+    sls = [W.tree(p) for p in range(W.P)]
+    r = router_from_seqlists(sls)
+    tok, off = W.requests(0, 1000)
+    t = torch.from_numpy(tok).cuda()
+    o = torch.from_numpy(off).cuda()
+    assert r.kernel_times() == {}  # off
+    r.kernel_clock(True)
+    n0 = r.launch_count()
+    for _ in range(3):
+        r.route(t, o, W.load(), W.alpha)
+    W.delta_make(0, 0.05, 0.05)
+    d = W.delta()
+    r.apply_delta(-1, d.op, d.seqs, d.peer_begin)
+    times = r.kernel_times()
+    assert sum(n for n, _ in times.values()) == r.launch_count() - n0
+    assert times["lane_kernel<false>"][0] == 3 and times["group_hash_kernel"][0] == 3
+    assert times["delta_kernel"][0] >= 1 and times["validate_kernel"][0] == 1
+    assert all(ms > 0 for _, ms in times.values())
+    r.kernel_clock(False)
+    assert r.kernel_times() == {}
+    with pytest.raises(g.P2PError):
+        g.p2p_router_kernel_time(r.handle, g.KERNEL_COUNT)
