@@ -65,6 +65,7 @@ def _load():
             "otree_match": (i64, [vp, vp, i64, vp]),
             "otree_insert_segmented": (None, [vp, vp, vp, vp, vp, i64, i64]),
             "otree_apply_ops": (i64, [vp, vp, vp, vp, vp, vp, i64, i64]),
+            "otree_apply_ops_counted": (i64, [vp, vp, vp, vp, vp, vp, i64, i64, vp]),
             "otree_stats": (None, [vp, vp]),
             "otree_export": (ctypes.c_int, [vp] + [vp] * 8),
             "oracle_argmax": (i32, [i32, vp, vp, i32]),
@@ -132,6 +133,16 @@ class OTree:
             i1 = len(op)
         return int(self._lib.otree_apply_ops(self._h, _p(op), _p(sl.seg_begin), _p(sl.seg_off), _p(sl.seg_len),
                                              _p(sl.pool), i0, i1))
+
+    def apply_ops_counted(self, op: np.ndarray, sl, counters: np.ndarray, i0: int = 0, i1: int | None = None) -> int:
+        """As ``apply_ops``, adding each op's touched-byte counters to ``counters`` (int64[8]): the read-only
+        PrefixMatch walk of its sequence before the op (tokens compared, nodes visited, child-search bytes),
+        then sequence tokens, pool runs, INSERTs, label tokens the INSERTs add, DELETEs."""
+        if i1 is None:
+            i1 = len(op)
+        assert counters.dtype == np.int64 and counters.size >= 8
+        return int(self._lib.otree_apply_ops_counted(self._h, _p(op), _p(sl.seg_begin), _p(sl.seg_off),
+                                                     _p(sl.seg_len), _p(sl.pool), i0, i1, _p(counters)))
 
     def stats(self) -> tuple[int, int, int]:
         """(nodes including the root, label tokens, stored sequences)."""
@@ -220,6 +231,16 @@ def decide(match, load, alpha: int, excluded=None):
         if len(cand) > 1:
             nxt[b] = -cand[1][2]
     return best, nxt
+
+
+def delta_touched_bytes(counters: np.ndarray) -> int:
+    """Algorithmic bytes of anti-entropy ops from ``apply_ops_counted``'s counters: per op, its input (4 B op
+    code, 8 B sequence start, 12 B per pool run, 4 B per sequence token), its walk (4 B per token compared,
+    20 B per node visited, the child-search bytes), and what it writes (an INSERT: 4 B per new label token
+    plus 36 B for a new node record and child entry; a DELETE: a 16 B node record)."""
+    c = [int(x) for x in counters]
+    n_ops = c[5] + c[7]
+    return (12 * n_ops + 12 * c[4] + 4 * c[3]) + (4 * c[0] + 20 * c[1] + c[2]) + (4 * c[6] + 36 * c[5] + 16 * c[7])
 
 
 def touched_bytes(counters: np.ndarray) -> int:

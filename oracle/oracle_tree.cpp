@@ -256,6 +256,32 @@ int64_t otree_apply_ops(otree* t, const int32_t* op, const int64_t* seg_begin, c
   return absent;
 }
 
+// As otree_apply_ops, with the touched-byte counters of an anti-entropy delta: before each op, the read-only
+// PrefixMatch walk of its sequence adds to ctr[0..2] (tokens compared, nodes visited, child-search bytes,
+// as for a lookup); then ctr[3] += sequence tokens, ctr[4] += pool runs, ctr[5] += INSERTs, ctr[6] += label
+// tokens an INSERT adds (sequence length - match), ctr[7] += DELETEs.
+int64_t otree_apply_ops_counted(otree* t, const int32_t* op, const int64_t* seg_begin, const int64_t* seg_off,
+                                const int32_t* seg_len, const int32_t* pool, int64_t i0, int64_t i1, int64_t* ctr) {
+  Tree& T = *reinterpret_cast<Tree*>(t);
+  int64_t absent = 0;
+  for (int64_t i = i0; i < i1; ++i) {
+    const std::vector<int32_t> s = gather(seg_begin, seg_off, seg_len, pool, i);
+    const int64_t n = (int64_t)s.size();
+    const int64_t m = match(T, s.data(), n, ctr);
+    ctr[3] += n;
+    ctr[4] += seg_begin[i + 1] - seg_begin[i];
+    if (op[i] == 0) {
+      ctr[5] += 1;
+      ctr[6] += n - m;
+      insert(T, s.data(), n);
+    } else {
+      ctr[7] += 1;
+      if (remove(T, s.data(), n) == 0) ++absent;
+    }
+  }
+  return absent;
+}
+
 // out[0] = nodes (root included), out[1] = label tokens, out[2] = stored sequences (sum of term counts).
 void otree_stats(const otree* t, int64_t* out) {
   std::vector<const Node*> nodes;
