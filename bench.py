@@ -6,10 +6,19 @@ every replica (device INSERT/DELETE) followed by the route of the batch (longest
 P trees + route decision); for the other workloads the route alone.  Inputs are seeded synthetic
 stand-ins for the paper's few-shot-prompt workloads (see workload/wl.h), resident in HBM when the timed
 region starts.  The JSON line also carries:
-  roofline      the route kernel's algorithmic bytes/s (per launch: the oracle's touched-byte accounting)
-                against the measured HBM copy bandwidth;
-  e2e           the same metric through the host-pointer C-ABI call (copies in the timed region);
-  cpu_baseline  the CPU oracle on the host cores over a bounded sample of the same workload.
+  kernels       every kernel launched in the timed region: launches, device ms per step (the library's kernel
+                clock, CUDA events on the router stream), share, and its DRAM traffic per launch where an ncu
+                capture of the same kernel source gave one;
+  roofline      the stage that takes the most time -- the delta kernel, or the route step's four launches --
+                against the measured HBM copy bandwidth: achieved = algorithmic bytes per launch / device time.
+                The delta kernel's algorithmic bytes are the oracle's per-op counters (input, walk, writes);
+                the route step's are its compulsory bytes (request tokens and offsets read once, the match
+                matrix and peers written once).  `traffic` is ncu's DRAM bytes for that kernel;
+  route         the route step's compulsory-byte rate and its touched-byte rate (the oracle's per-(request,
+                tree) walk bytes, which shared-prefix groups and L2 hits let the device exceed);
+  e2e           the same metric through the host-pointer C-ABI calls (copies in the timed region);
+  cpu_baseline  the CPU oracle on the host cores over a bounded sample of the same workload, on all cores and
+                on one thread, with the CPU model.
 --impl reference times that oracle as the reference arm.
 
 Multi-GPU (torchrun): every rank holds all P trees and routes its own batch (requests [rank*B, (rank+1)*B)
@@ -18,9 +27,11 @@ of the request stream); no data-path collective.  Timing is max over ranks.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import os
+import platform
 import statistics
 import subprocess
 import sys
@@ -43,6 +54,58 @@ WORKLOADS = {
                 "1,048,576 requests/batch, 5% DELETE + 5% INSERT per replica per batch"),
 }
 L2_BYTES = 126 * 2**20
+CSRC = os.path.join(ROOT, "paper_2606_17059_gb300", "csrc")
+# Source file of each kernel (with internal.h, the layout they share): a DRAM-traffic figure holds only for
+# the source it was captured on.
+KERNEL_SOURCE = {
+    "group_hash_kernel": "group_kernel.cu", "group_resolve_kernel": "group_kernel.cu",
+    "group_resolve32_kernel": "group_kernel.cu", "route_kernel": "route_kernel.cu",
+    "lane_kernel<true>": "route_kernel.cu", "lane_kernel<false>": "route_kernel.cu", "decide_kernel": "route_kernel.cu",
+    "validate_kernel": "delta_kernel.cu", "init_ranges_kernel": "delta_kernel.cu", "delta_kernel": "delta_kernel.cu",
+    "compact_kernel": "delta_kernel.cu", "compact_labels_kernel": "delta_kernel.cu",
+    "refresh_views_kernel": "delta_kernel.cu", "set_tree_kernel": "delta_kernel.cu",
+    "update_count_kernel": "update_kernel.cu", "update_scatter_kernel": "update_kernel.cu",
+}
+# DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum) per workload and kernel, with the
+# source hash of the capture and the profile summary that holds the command.  A figure whose source hash
+# differs from the current source is not reported (the kernel changed since it was taken).
+TRAFFIC: dict = {}
+
+
+def source_hash(kernel: str) -> str | None:
+    f = KERNEL_SOURCE.get(kernel)
+    if f is None or not os.path.exists(os.path.join(CSRC, f)):
+        return None
+    h = hashlib.sha256()
+    for name in (f, "internal.h"):
+        with open(os.path.join(CSRC, name), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_of(workload: str, kernel: str):
+    t = TRAFFIC.get(workload, {}).get(kernel)
+    if t is None or t["source"] != source_hash(kernel):
+        return None
+    return t
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().startswith("Model name:"):
+                return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                if ln.lower().startswith("model name"):
+                    return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    return platform.processor() or platform.machine()
 
 
 def log(*a):
@@ -235,6 +298,43 @@ def oracle_sample(W, otrees, tok, off, load, alpha, target_s: float, n_threads: 
     return n / secs, secs, n, ctr, desc, (m, peer)
 
 
+def oracle_single_thread(otrees, tok, off, load, alpha, target_s: float):
+    """The oracle's route on one host thread over the first requests of the batch (about target_s of CPU
+    work).  Returns (requests/s, requests)."""
+    import oracle as orc
+    B = len(off) - 1
+    pilot = min(B, 16)
+    t0 = time.perf_counter()
+    orc.route(otrees, tok, off[: pilot + 1], load, alpha, n_threads=1)
+    per_req = (time.perf_counter() - t0) / pilot
+    n = int(min(B, max(pilot, target_s / max(per_req, 1e-9))))
+    t0 = time.perf_counter()
+    orc.route(otrees, tok, off[: n + 1], load, alpha, n_threads=1)
+    return n / (time.perf_counter() - t0), n
+
+
+def delta_op_bytes(otrees, delta, share: float, n_threads: int):
+    """Mean algorithmic bytes per op of a delta (oracle counters: input, walk, writes) over the ops that
+    follow the timed share in every tree (those trees have applied the ops before them).  Returns (bytes per
+    op, ops counted)."""
+    import oracle as orc
+    pb = delta.peer_begin
+
+    def count(p):
+        lo, hi = int(pb[p]), int(pb[p + 1])
+        a = lo + int(math.ceil(share * (hi - lo)))
+        b = min(hi, a + max(1, (hi - lo) // 50))
+        c = np.zeros(8, np.int64)
+        if a < b:
+            otrees[p].apply_ops_counted(delta.op, delta.seqs, c, a, b)
+        return c
+
+    with ThreadPoolExecutor(max_workers=n_threads) as ex:
+        tot = sum(ex.map(count, range(len(otrees))))
+    n_ops = int(tot[5] + tot[7])
+    return (orc.delta_touched_bytes(tot) / n_ops if n_ops else 0.0), n_ops
+
+
 # ---- our arm --------------------------------------------------------------------------------------------
 
 def run_ours(args):
@@ -308,6 +408,7 @@ def run_ours(args):
     torch.cuda.synchronize()
     clocks = ClockSampler(local)
     clocks.start()
+    router.kernel_clock(True)  # per-kernel device time over the timed steps
     launches0 = router.launch_count()
     evs = []
     t_begin = torch.cuda.Event(enable_timing=True)
@@ -323,6 +424,8 @@ def run_ours(args):
     t_end.record(stream)
     torch.cuda.synchronize()
     launches = router.launch_count() - launches0
+    ktimes = router.kernel_times()
+    router.kernel_clock(False)
     clk = clocks.stop()
     if dist:
         dist.barrier()
@@ -342,28 +445,82 @@ def run_ours(args):
         # (For the delta workload the oracle trees are the initial replicas, before the GPU's deltas: they
         # differ from the device trees by a few percent of their edges, so they give the byte accounting
         # but no parity check; the tests check that workload's parity.)
-        ctr, n_acc, cpu = None, 0, None
+        ctr, n_acc, cpu, counted_share = None, 0, None, 0.0
         if want_oracle:
             rate, secs, n_acc, ctr, desc, (om, op) = oracle_sample(
                 W, otrees, tok_np, off_np, load, alpha, args.cpu_seconds, n_cpu,
                 delta=host_delta0 if has_delta else None, B_total=B)
+            counted_share = n_acc / B
+            rate1, n1 = oracle_single_thread(otrees, tok_np, off_np, load, alpha, args.cpu1_seconds)
             cpu = {"value": rate, "unit": "requests/s", "cores": n_cpu, "kind": "oracle",
-                   "sample": desc + f" ({secs:.1f} s on {n_cpu} host threads)"}
+                   "sample": desc + f" ({secs:.1f} s on {n_cpu} host threads)", "cpu_model": cpu_model(),
+                   "single_thread": {"value": rate1, "unit": "requests/s", "cores": 1,
+                                     "sample": f"route of the first {n1} requests x all {P} trees on one thread"}}
             if not has_delta:
                 same = bool(np.array_equal(gm[:n_acc], om) and np.array_equal(gp[:n_acc], op))
                 res["parity_spot_check"] = {"requests": n_acc, "bit_exact": same}
         hbm, src = peaks()
+        peak_source = f"{src} (MEASURED_PEAKS.json hbm_gbs, STREAM-style copy)"
         route_avg_ms = statistics.mean(route_ms)
-        roof = None
+        tkey = None if (args.trees or args.batch) else args.workload
+        # ---- every kernel of the timed region (the library's kernel clock) ----
+        k_total = sum(ms for _, ms in ktimes.values()) or 1.0
+        kernels = []
+        for name, (n, ms) in sorted(ktimes.items(), key=lambda kv: -kv[1][1]):
+            t = traffic_of(tkey, name) if tkey else None
+            row = {"kernel": name, "launches_per_step": n / args.steps, "ms_per_step": ms / args.steps,
+                   "ms_per_launch": ms / n, "share": ms / k_total, "traffic_per_launch": t["bytes"] if t else None}
+            if t:
+                row["dram_gbs"] = t["bytes"] / (ms / n / 1e3) / 1e9
+                row["dram_frac"] = row["dram_gbs"] / hbm
+                row["traffic_profile"] = t["profile"]
+            kernels.append(row)
+        kt = {k["kernel"]: k for k in kernels}
+        # ---- the route step: compulsory bytes, and the oracle's touched bytes ----
+        compulsory = 4 * int(n_tok) + 8 * (B + 1) + 4 * B * P + 4 * B
+        route = {"kernels": [k for k in ("group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel",
+                                         "route_kernel", "lane_kernel<true>", "lane_kernel<false>") if k in kt],
+                 "ms": route_avg_ms, "compulsory_bytes": compulsory,
+                 "compulsory_gbs": compulsory / (route_avg_ms / 1e3) / 1e9}
+        route["compulsory_frac"] = route["compulsory_gbs"] / hbm
+        tr = [traffic_of(tkey, k) if tkey else None for k in route["kernels"]]
+        route["traffic"] = sum(t["bytes"] for t in tr) if tr and all(tr) else None
+        if route["traffic"]:
+            route["dram_gbs"] = route["traffic"] / (route_avg_ms / 1e3) / 1e9
         if ctr is not None:
-            bytes_per_launch = orc.touched_bytes(ctr) / n_acc * B
-            achieved = bytes_per_launch / (route_avg_ms / 1e3) / 1e9
-            roof = {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s", "frac": achieved / hbm,
-                    "traffic": None,
-                    "kernel": "route step: group_hash + group_resolve + lane_kernel (leaders, followers)", "peak_source": f"{src} (MEASURED_PEAKS.json hbm_gbs)",
-                    "bytes_per_launch": bytes_per_launch, "route_ms": route_avg_ms,
-                    "bytes_basis": f"oracle touched-byte counters over {n_acc} requests x {P} trees, "
-                                   f"scaled to {B} requests per launch"}
+            touched = orc.touched_bytes(ctr) / n_acc * B
+            route.update({"touched_bytes": touched, "effective_gbs": touched / (route_avg_ms / 1e3) / 1e9,
+                          "touched_basis": f"oracle per-(request, tree) walk counters over {n_acc} requests x {P} "
+                                           f"trees, scaled to {B} requests; groups and L2 hits let the device "
+                                           "exceed HBM by this measure"})
+        # ---- the roofline of the stage that takes the most time ----
+        roof = None
+        delta_k = kt.get("delta_kernel")
+        if delta_k and delta_k["ms_per_step"] >= route_avg_ms and has_delta:
+            n_ops_step = len(host_delta0.op)
+            per_op, counted = delta_op_bytes(otrees, host_delta0, counted_share, n_cpu) if want_oracle else (0.0, 0)
+            if counted:
+                alg = per_op * n_ops_step / delta_k["launches_per_step"]
+                achieved = alg / (delta_k["ms_per_launch"] / 1e3) / 1e9
+                t = traffic_of(tkey, "delta_kernel") if tkey else None
+                roof = {"bound": "hbm", "kernel": "delta_kernel", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                        "frac": achieved / hbm, "traffic": t["bytes"] if t else None, "peak_source": peak_source,
+                        "bytes_per_launch": alg, "ms_per_launch": delta_k["ms_per_launch"],
+                        "bytes_basis": f"oracle per-op counters (input, PrefixMatch walk, writes) over {counted} ops, "
+                                       f"{per_op:.0f} B per op x {n_ops_step} ops per step"}
+                if t:
+                    roof["dram_gbs"] = t["bytes"] / (delta_k["ms_per_launch"] / 1e3) / 1e9
+                    roof["dram_frac"] = roof["dram_gbs"] / hbm
+        if roof is None:
+            roof = {"bound": "hbm", "kernel": "route step: " + " + ".join(route["kernels"]),
+                    "achieved": route["compulsory_gbs"], "peak": hbm, "unit": "GB/s", "frac": route["compulsory_frac"],
+                    "traffic": route["traffic"], "peak_source": peak_source, "bytes_per_launch": compulsory,
+                    "ms_per_launch": route_avg_ms,
+                    "bytes_basis": "compulsory bytes: request tokens and offsets read once, match matrix and peers "
+                                   "written once (tree bytes left out: a lower bound)"}
+            if route["traffic"]:
+                roof["dram_gbs"] = route["dram_gbs"]
+                roof["dram_frac"] = route["dram_gbs"] / hbm
         # ---- optional: the route decision with excluded peers on this batch's match matrix ----
         if args.decide:
             res["decide"] = time_decide(router, out_match, load, alpha, P, B, hbm, src)
@@ -379,7 +536,8 @@ def run_ours(args):
                        "step": "delta on every replica + route" if has_delta else "route"},
             "lookups_per_s": value * P, "route_ms": route_avg_ms,
             "delta_ms": statistics.mean(delta_ms) if has_delta else None,
-            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": int(launches), "clocks": clk,
+            "roofline": roof, "route": route, "kernels": kernels, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": int(launches), "clocks": clk,
         })
         print(json.dumps(res), flush=True)
     router.close()
@@ -423,10 +581,20 @@ def run_e2e(args, W, router, tok_np, off_np, load, alpha, has_delta, n_cpu):
     k = max(1, min(args.steps, args.e2e_steps))
     hds = []
     if has_delta:
+        import workload as wl
         base = args.warmup + args.steps
+
+        def pinned(a):  # the delta's host arrays in pinned memory, as a serving process would keep them
+            t = torch.empty(a.shape, dtype=getattr(torch, a.dtype.name), pin_memory=True).numpy()
+            t[...] = a
+            return t
+
         for s in range(k + 1):
             W.delta_make(base + s, W.params["delta_frac"], W.params["delta_frac"], n_threads=n_cpu)
-            hds.append(W.delta(n_threads=n_cpu))
+            d = W.delta(n_threads=n_cpu)
+            sl = d.seqs
+            hds.append(type(d)(pinned(d.op), wl.SeqList(pinned(sl.seg_begin), pinned(sl.seg_off), pinned(sl.seg_len),
+                                                        pinned(sl.pool)), pinned(d.peer_begin)))
 
     def one(i):
         if has_delta:
@@ -442,8 +610,10 @@ def run_e2e(args, W, router, tok_np, off_np, load, alpha, has_delta, n_cpu):
     h2d = tok_np.nbytes + off_np.nbytes + 4 * P
     if has_delta:
         h2d += delta_bytes(hds[1])
+    d2h = h_match.nbytes + h_peer.nbytes
     return {"value": k * B / secs, "unit": "requests/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(h_match.nbytes + h_peer.nbytes), "steps": k,
+            "d2h_bytes_per_step": int(d2h), "steps": k, "host_link_gbs": (h2d + d2h) * k / secs / 1e9,
+            "host_buffers": "pinned",
             "call": "p2p_tree_apply_delta (host arrays) + p2p_route_batch_host" if has_delta else "p2p_route_batch_host"}
 
 
@@ -497,6 +667,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
+    ap.add_argument("--cpu1-seconds", type=float, default=4.0, help="target time of the single-thread oracle sample")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--decide", action="store_true",
                     help="also time p2p_route_decide (excluded peers, next-best target) on the routed batch")
