@@ -64,7 +64,8 @@ KERNEL_SOURCE = {
     "validate_kernel": "delta_kernel.cu", "init_ranges_kernel": "delta_kernel.cu", "delta_kernel": "delta_kernel.cu",
     "compact_kernel": "delta_kernel.cu", "compact_labels_kernel": "delta_kernel.cu",
     "refresh_views_kernel": "delta_kernel.cu", "set_tree_kernel": "delta_kernel.cu",
-    "update_count_kernel": "update_kernel.cu", "update_scatter_kernel": "update_kernel.cu",
+    "update_count_kernel": "update_kernel.cu", "update_scan_kernel": "update_kernel.cu",
+    "update_scatter_kernel": "update_kernel.cu",
 }
 # DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum) per workload and kernel, with the
 # source hash of the capture and the profile summary that holds the command.  A figure whose source hash

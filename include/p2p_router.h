@@ -46,6 +46,7 @@ enum {
 };
 
 enum { P2P_OP_INSERT = 0, P2P_OP_DELETE = 1 };
+enum { P2P_KERNEL_COUNT = 17 }; /* kernels the kernel clock keeps totals for */
 enum { P2P_MEM_HOST = 0, P2P_MEM_DEVICE = 1 };
 
 typedef struct p2p_router p2p_router;
@@ -139,7 +140,7 @@ int64_t p2p_router_launch_count(const p2p_router* r);
  * Each pair adds an event record before and after the launch, a few microseconds of stream work. */
 int p2p_router_kernel_clock(p2p_router* r, int32_t on);
 
-/* Totals of kernel i (0 <= i < 16, an index into the library's list of kernels) since the clock was
+/* Totals of kernel i (0 <= i < P2P_KERNEL_COUNT, an index into the library's list of kernels) since the clock was
  * switched on: *name (nullable) receives the kernel's name (a static string), *launches and *ms (nullable)
  * the timed launches and their summed device time in milliseconds; 0 and 0.0 while the clock is off.
  * Waits for queued work.  Errors: P2P_E_INVAL (i out of range), P2P_E_CUDA. */
@@ -210,6 +211,23 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
  * streams) race: order them.  The call returns when the delta is applied.  Other errors as
  * p2p_tree_apply_delta. */
 int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent);
+
+/* Own-tree and estimate maintenance after routing (Algorithm 1): once request r has been sent to node k and
+ * acknowledged, the sender inserts r into its estimate of k's trie (UpdateTrieEstimate(r, k)); a request the
+ * node serves itself, k = its own tree (index 0 by convention), goes into its own trie (UpdateTrie; the
+ * request's tokens stand in for the result, whose generated tokens are not known here).  For a routed batch:
+ * request b is inserted once into tree peer[b]; requests with peer[b] < 0 (no route) are skipped.
+ *   tokens      DEVICE int32[n_tokens]; request b is tokens[offsets[b] .. offsets[b+1]) (read, never copied)
+ *   offsets     DEVICE int64[B+1]
+ *   peer        DEVICE int32[B], as p2p_route_batch writes it (any values < P)
+ *   n_inserted  (nullable) receives the number of requests inserted
+ * The batch is counting-sorted by tree on the device into an INSERT delta held in router buffers and applied
+ * like p2p_tree_apply_delta (arena growth and compaction included); inserts commute, so the trees equal those
+ * of inserting the requests one by one in batch order.  Waits for the work.  B = 0 is a no-op; B <= 2^30.
+ * Errors: P2P_E_INVAL (a peer >= P, or a routed request with offsets outside [0, n_tokens] or decreasing:
+ * nothing changes), P2P_E_NOMEM, P2P_E_CUDA, P2P_E_DEVICE. */
+int p2p_update_estimates(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
+                         const int32_t* peer, int64_t* n_inserted);
 
 /* Sizes of tree `peer`: out[0] live nodes (root included), out[1] node slots in use, out[2] child
  * entries in use, out[3] label tokens in use, out[4] stale child entries, out[5] stale label tokens,

@@ -21,7 +21,7 @@ __all__ = [
     "p2p_router_num_trees", "p2p_router_launch_count", "p2p_snapshot_build", "p2p_snapshot_view", "p2p_snapshot_free",
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
     "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host", "p2p_route_decide",
-    "p2p_router_kernel_clock", "p2p_router_kernel_time",
+    "p2p_router_kernel_clock", "p2p_router_kernel_time", "p2p_update_estimates",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -95,6 +95,7 @@ def _load():
             "p2p_route_batch_host": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _i32, _vp, _vp]),
             "p2p_route_decide": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp]),
             "p2p_router_kernel_clock": (ctypes.c_int, [_vp, _i32]),
+            "p2p_update_estimates": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, P(_i64)]),
             "p2p_router_kernel_time": (ctypes.c_int, [_vp, _i32, P(ctypes.c_char_p), P(_i64), P(ctypes.c_double)]),
         }
         for name, (res, args) in sig.items():
@@ -195,7 +196,7 @@ def p2p_router_launch_count(r) -> int:
     return int(_load().p2p_router_launch_count(r))
 
 
-KERNEL_COUNT = 16  # kernels the kernel clock keeps totals for (indices 0 .. 15)
+KERNEL_COUNT = 17  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 16)
 
 
 def p2p_router_kernel_clock(r, on: bool) -> None:
@@ -304,6 +305,14 @@ def p2p_tree_apply_delta_static(r, peer: int, op, seqlist, peer_begin=None) -> i
     return int(absent.value)
 
 
+def p2p_update_estimates(r, tokens, n_tokens: int, offsets, B: int, peer) -> int:
+    """Inserts request b into tree peer[b] for every routed request (UpdateTrieEstimate / UpdateTrie of
+    Algorithm 1); tokens, offsets and peer are CUDA tensors (or addresses).  Returns the requests inserted."""
+    n = _i64()
+    _check(_load().p2p_update_estimates(r, _addr(tokens), n_tokens, _addr(offsets), B, _addr(peer), ctypes.byref(n)), r)
+    return int(n.value)
+
+
 STAT_NAMES = ("live_nodes", "node_slots", "child_entries", "label_tokens", "stale_child", "stale_label",
               "cap_node", "cap_child", "cap_label")
 
@@ -390,6 +399,10 @@ class Router:
 
     def sync(self) -> None:
         p2p_router_sync(self._h)
+
+    def update_estimates(self, tokens, offsets, peer) -> int:
+        """After routing: request b (CUDA tensors tokens/offsets) goes into tree peer[b]; returns the count."""
+        return p2p_update_estimates(self._h, tokens, tokens.numel(), offsets, offsets.numel() - 1, peer)
 
     def launch_count(self) -> int:
         return p2p_router_launch_count(self._h)

@@ -91,8 +91,9 @@ constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits 
 enum KernelId {
   K_GROUP_HASH, K_GROUP_RESOLVE, K_GROUP_RESOLVE32, K_ROUTE_STAGED, K_LANE_LEADER, K_LANE_FOLLOWER, K_DECIDE,
   K_VALIDATE, K_INIT_RANGES, K_DELTA, K_COMPACT, K_COMPACT_LABELS, K_REFRESH_VIEWS, K_SET_TREE,
-  K_UPDATE_COUNT, K_UPDATE_SCATTER, K_COUNT_
+  K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_COUNT_
 };
+static_assert(K_COUNT_ == P2P_KERNEL_COUNT, "the header's kernel count");
 const char* kernel_name(int id);
 struct KernelClock {
   virtual void mark(int id, bool end, cudaStream_t st) = 0;
@@ -196,6 +197,18 @@ cudaError_t static_scratch(int device, int32_t** header, int32_t** tokens);
 cudaError_t launch_validate(int32_t* header, const p2p_delta* d, int32_t peer, int32_t P, cudaStream_t st);
 cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* peer_begin, int64_t n, cudaStream_t st);
 constexpr int kStaticHeaderInts = 64;
+
+// A routed batch as a device-resident INSERT delta (update_kernel.cu).  counts [P] must be zero and bad [1]
+// zero before the count launch; bad receives 1 (a peer >= P) | 2 (a routed request with invalid offsets).
+// The scan writes peer_begin [P+1], the scatter cursors [P], seg_begin[n] = n and *total = n; the scatter
+// fills op, seg_begin, seg_off and seg_len [n] (each op one run of the request's tokens).
+cudaError_t launch_update_count(const int32_t* peer, const int64_t* offsets, int64_t B, int64_t n_tokens, int32_t P,
+                                int32_t* counts, int32_t* bad, int num_sms, cudaStream_t st);
+cudaError_t launch_update_scan(const int32_t* counts, int32_t P, int64_t* peer_begin, int32_t* cursor,
+                               int64_t* seg_begin_end, int64_t* total, cudaStream_t st);
+cudaError_t launch_update_scatter(const int32_t* peer, const int64_t* offsets, int64_t B, int64_t n_tokens, int32_t P,
+                                  int32_t* cursor, int32_t* op, int64_t* seg_begin, int64_t* seg_off, int32_t* seg_len,
+                                  int num_sms, cudaStream_t st);
 
 // Host-side helpers in snapshot.cpp.
 void set_global_error(const std::string& msg);

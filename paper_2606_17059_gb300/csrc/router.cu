@@ -88,7 +88,7 @@ const char* kernel_name(int id) {
       "group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel", "route_kernel", "lane_kernel<true>",
       "lane_kernel<false>", "decide_kernel", "validate_kernel", "init_ranges_kernel", "delta_kernel",
       "compact_kernel", "compact_labels_kernel", "refresh_views_kernel", "set_tree_kernel", "update_count_kernel",
-      "update_scatter_kernel"};
+      "update_scan_kernel", "update_scatter_kernel"};
   return id >= 0 && id < K_COUNT_ ? names[id] : "";
 }
 
@@ -198,6 +198,7 @@ struct p2p_router {
   DevBuf d_op, d_seg_begin, d_seg_off, d_seg_len, d_pool, d_peer_begin, d_done, d_gather;
   DevBuf grp_keys, grp_vals, grp_req, grp_ckpt;  // shared-prefix grouping of a batch
   DevBuf cmp_jobs, cmp_queue;          // device compaction
+  DevBuf upd_cnt, upd_op, upd_sb, upd_so, upd_sl;  // a routed batch as an INSERT delta (p2p_update_estimates)
   int64_t launches = 0;  // kernels this router has launched
   RouterClock* clock = nullptr;  // per-kernel device time, while switched on
   // Shared label pool: long labels interned across trees (device array, host mirror, content index).
@@ -842,7 +843,8 @@ void p2p_router_destroy(p2p_router* r) {
     for (TreeState& t : r->spare) free_tree_arrays(r, t);
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
-                      &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue})
+                      &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue,
+                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -1193,6 +1195,71 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
                                     " ran out of arena room: some of its ops were not applied (p2p_tree_apply_delta grows trees)");
   }
   if (n_absent) *n_absent = absent;
+  return rc;
+}
+
+// UpdateTrieEstimate / UpdateTrie of Algorithm 1 over a routed batch: the batch is counting-sorted by its
+// chosen tree into an INSERT delta in router buffers (update_kernel.cu), whose ops are runs of the request
+// tokens, and applied by the delta path.
+int p2p_update_estimates(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
+                         const int32_t* peer, int64_t* n_inserted) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (n_inserted) *n_inserted = 0;
+  if (B < 0 || n_tokens < 0) return fail(r, P2P_E_INVAL, "negative B or n_tokens");
+  if (B > kMaxBatch) return fail(r, P2P_E_INVAL, "B exceeds 2^30 requests per call: split the batch");
+  if (B == 0) return P2P_OK;
+  if (!offsets || !peer || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r);
+  const int32_t P = r->P;
+  // counts [P] int32 | cursor [P] int32 | bad [2] int32 | peer_begin [P+1] int64 | total [1] int64
+  const size_t cnt_bytes = ((size_t)2 * P + 2) * sizeof(int32_t);
+  CK(ensure(r, r->upd_cnt, cnt_bytes + (size_t)(P + 2) * sizeof(int64_t)));
+  int32_t* counts = static_cast<int32_t*>(r->upd_cnt.p);
+  int32_t* cursor = counts + P;
+  int32_t* bad = cursor + P;
+  int64_t* peer_begin = reinterpret_cast<int64_t*>(static_cast<char*>(r->upd_cnt.p) + cnt_bytes);
+  int64_t* total = peer_begin + P + 1;
+  CK(ensure(r, r->upd_sb, (size_t)(B + 1) * sizeof(int64_t)));
+  int64_t* seg_begin = static_cast<int64_t*>(r->upd_sb.p);
+  CK(cudaMemsetAsync(counts, 0, cnt_bytes, r->stream));
+  CK(p2p::launch_update_count(peer, offsets, B, n_tokens, P, counts, bad, r->num_sms, r->stream));
+  CK(p2p::launch_update_scan(counts, P, peer_begin, cursor, seg_begin + B, total, r->stream));
+  r->launches += 2;
+  struct {
+    int32_t bad[2];
+    int64_t total;
+  } h = {};
+  CK(cudaMemcpyAsync(h.bad, bad, sizeof(h.bad), cudaMemcpyDeviceToHost, r->stream));
+  CK(cudaMemcpyAsync(&h.total, total, sizeof(h.total), cudaMemcpyDeviceToHost, r->stream));
+  CK(cudaStreamSynchronize(r->stream));
+  if (h.bad[0] & 1) return fail(r, P2P_E_INVAL, "a peer index is >= P");
+  if (h.bad[0] & 2) return fail(r, P2P_E_INVAL, "a routed request has offsets outside [0, n_tokens] or decreasing");
+  const int64_t n = h.total;
+  if (n == 0) return P2P_OK;
+  CK(ensure(r, r->upd_op, (size_t)n * sizeof(int32_t)));
+  CK(ensure(r, r->upd_so, (size_t)n * sizeof(int64_t)));
+  CK(ensure(r, r->upd_sl, (size_t)n * sizeof(int32_t)));
+  int32_t* op = static_cast<int32_t*>(r->upd_op.p);
+  int64_t* seg_off = static_cast<int64_t*>(r->upd_so.p);
+  int32_t* seg_len = static_cast<int32_t*>(r->upd_sl.p);
+  // seg_begin[n] = n was written by the scan at seg_begin + B: move it to its place when n < B.
+  if (n < B) CK(cudaMemcpyAsync(seg_begin + n, seg_begin + B, sizeof(int64_t), cudaMemcpyDeviceToDevice, r->stream));
+  CK(p2p::launch_update_scatter(peer, offsets, B, n_tokens, P, cursor, op, seg_begin, seg_off, seg_len, r->num_sms,
+                                r->stream));
+  r->launches += 1;
+  p2p_delta d = {};
+  d.op = op;
+  d.seqs.n = n;
+  d.seqs.seg_begin = seg_begin;
+  d.seqs.seg_off = seg_off;
+  d.seqs.seg_len = seg_len;
+  d.seqs.pool = tokens;
+  d.seqs.n_segs = n;
+  d.seqs.n_pool = n_tokens;
+  d.peer_begin = peer_begin;
+  d.mem = P2P_MEM_DEVICE;
+  const int rc = p2p_tree_apply_delta(r, -1, &d, nullptr);
+  if (rc == P2P_OK && n_inserted) *n_inserted = n;
   return rc;
 }
 
