@@ -77,17 +77,17 @@ def test_unrouted_requests_are_skipped_and_bad_input_changes_nothing():
         r.update_estimates(t, o, _dev(bad))
     assert e.value.code == g.P2P_E_INVAL
     off_bad = off.copy()
-    off_bad[7] = off_bad[8] + 1  # request 6 ends before it starts ... and request 7 starts after it ends
+    off_bad[7] = off_bad[8] + 1  # request 7 now starts after it ends (request 6 grows by one token)
     routed = peer.copy()
-    routed[6] = 0
+    routed[7] = 0
     with pytest.raises(g.P2PError) as e:
         r.update_estimates(t, _dev(off_bad), _dev(routed))
     assert e.value.code == g.P2P_E_INVAL
     for p in range(W.P):
         assert same_snapshot(r.download(p), before[p]), p
-    # Unrouted requests with invalid offsets are not looked at.
+    # An unrouted request with invalid offsets is not looked at.
     unrouted = peer.copy()
-    unrouted[6] = unrouted[7] = -1
+    unrouted[7] = -1
     assert g.p2p_update_estimates(r.handle, t, t.numel(), _dev(off_bad), W.B, _dev(unrouted)) == int((unrouted >= 0).sum())
     oracle.update_estimates(otrees, tok, off_bad, unrouted)
     _check_trees(r, otrees)
