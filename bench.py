@@ -527,6 +527,9 @@ def run_ours(args):
             res["decide"] = time_decide(router, out_match, load, alpha, P, B, hbm, src)
         # ---- end to end through the host-pointer C-ABI call ----
         e2e = run_e2e(args, W, router, tok_np, h_off.numpy(), load, alpha, has_delta, n_cpu)
+        # ---- UpdateTrieEstimate / UpdateTrie of Algorithm 1 on the last timed batch (changes the trees) ----
+        if not args.no_update:
+            res["update_estimates"] = time_update(router, d_tok, d_off, out_peer, route_avg_ms)
         res.update({
             "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -544,6 +547,30 @@ def run_ours(args):
     router.close()
     if dist:
         dist.destroy_process_group()
+
+
+def time_update(router, d_tok, d_off, out_peer, route_ms):
+    """One p2p_update_estimates call on the last timed batch (every request inserted into the tree it was routed
+    to): CUDA events on the router stream around the call (the call waits for its work, so host-side steps
+    between its launches count too), and the device time of its kernels from the kernel clock."""
+    import torch
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    router.kernel_clock(True)
+    t0 = time.perf_counter()
+    e0.record(stream)
+    n = router.update_estimates(d_tok, d_off, out_peer)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    wall = (time.perf_counter() - t0) * 1e3
+    kt = router.kernel_times()
+    router.kernel_clock(False)
+    ms = e0.elapsed_time(e1)
+    return {"inserted": n, "ms": ms, "wall_ms": wall, "kernel_ms": {k: v[1] for k, v in kt.items()},
+            "route_plus_update_ms": route_ms + ms,
+            "note": "one call after the timed steps on the last routed batch; the first call on fresh trees also "
+                    "grows their arenas"}
 
 
 def time_decide(router, out_match, load, alpha, P, B, hbm, src, reps: int = 10):
@@ -670,6 +697,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle sample")
     ap.add_argument("--cpu1-seconds", type=float, default=4.0, help="target time of the single-thread oracle sample")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-update", action="store_true",
+                    help="skip the timing of p2p_update_estimates (UpdateTrieEstimate) on the last routed batch")
     ap.add_argument("--decide", action="store_true",
                     help="also time p2p_route_decide (excluded peers, next-best target) on the routed batch")
     ap.add_argument("--ref-requests", type=int, default=65536)
