@@ -248,6 +248,21 @@ int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]);
 int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
                     const int32_t* load, int32_t alpha, int32_t* out_match, int32_t* out_peer);
 
+/* p2p_route_batch with the route decision of p2p_route_decide made in the same pass: the walk kernels keep
+ * the two largest route keys of the trees not excluded while they write the match row, so the match matrix
+ * is not read again (Section 3.2, hot specialist push-back: no routing to a peer that pushed back; Section
+ * 3.3, in-flight forwarded request failure: no routing to a suspected-failed peer, and the next-best target
+ * for a forwarding timeout).
+ *   excluded    HOST uint8[P] (nullable = none), copied before return: excluded[p] != 0 takes tree p out of
+ *               the candidates (its match column is still written)
+ *   out_peer    DEVICE int32[B]: the first candidate of the route order, -1 if every tree is excluded
+ *   out_next    DEVICE int32[B] (nullable): the second candidate, -1 if there is none
+ * Other arguments, limits and errors as p2p_route_batch; out_match is the same.  With excluded and out_next
+ * both NULL this is p2p_route_batch.  Asynchronous on the router stream. */
+int p2p_route_batch_decide(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
+                           const int32_t* load, int32_t alpha, const uint8_t* excluded, int32_t* out_match,
+                           int32_t* out_peer, int32_t* out_next);
+
 /* As p2p_route_batch with every pointer in HOST memory: copies the requests to the device, routes,
  * copies both outputs back and waits.  Large batches go in up to 8 chunks of at least 131,072 requests:
  * a chunk's inputs are copied in while the chunk before it is routed and the one before that is copied

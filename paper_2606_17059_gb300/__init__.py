@@ -21,7 +21,7 @@ __all__ = [
     "p2p_router_num_trees", "p2p_router_launch_count", "p2p_snapshot_build", "p2p_snapshot_view", "p2p_snapshot_free",
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
     "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host", "p2p_route_decide",
-    "p2p_router_kernel_clock", "p2p_router_kernel_time", "p2p_update_estimates",
+    "p2p_router_kernel_clock", "p2p_router_kernel_time", "p2p_update_estimates", "p2p_route_batch_decide",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -96,6 +96,7 @@ def _load():
             "p2p_route_decide": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i32, _vp, _vp, _vp]),
             "p2p_router_kernel_clock": (ctypes.c_int, [_vp, _i32]),
             "p2p_update_estimates": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, P(_i64)]),
+            "p2p_route_batch_decide": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp]),
             "p2p_router_kernel_time": (ctypes.c_int, [_vp, _i32, P(ctypes.c_char_p), P(_i64), P(ctypes.c_double)]),
         }
         for name, (res, args) in sig.items():
@@ -330,6 +331,27 @@ def p2p_route_batch(r, tokens, n_tokens: int, offsets, B: int, load, alpha: int,
                                    _addr(out_match), _addr(out_peer)), r)
 
 
+def _mask(r, excluded, n: int):
+    if excluded is None:
+        return None
+    ex = np.ascontiguousarray(np.asarray(excluded), dtype=np.uint8)
+    if ex.size != n:
+        raise ValueError(f"excluded must have one entry per tree ({n})")
+    return ex
+
+
+def p2p_route_batch_decide(r, tokens, n_tokens: int, offsets, B: int, load, alpha: int, excluded, out_match, out_peer,
+                           out_next=None) -> None:
+    """Device routing with excluded trees and the next-best target decided in the walk kernels; tokens, offsets,
+    out_match, out_peer and out_next (or None) are CUDA tensors, load and excluded (uint8 per tree, or None)
+    host arrays."""
+    ld = _load_vec(r, load)
+    ex = _mask(r, excluded, ld.size)
+    _check(_load().p2p_route_batch_decide(r, _addr(tokens), n_tokens, _addr(offsets), B, ld.ctypes.data, alpha,
+                                          ex.ctypes.data if ex is not None else None, _addr(out_match),
+                                          _addr(out_peer), _addr(out_next)), r)
+
+
 def p2p_route_decide(r, match, B: int, load, alpha: int, excluded, out_peer, out_next) -> None:
     """Best and next-best non-excluded tree per request from a device match matrix [B, P] (CUDA tensors or
     addresses); load and excluded (uint8 per tree, or None) are host arrays."""
@@ -429,6 +451,17 @@ class Router:
             out_peer = torch.empty(B, dtype=torch.int32, device=tokens.device)
         p2p_route_batch(self._h, tokens, tokens.numel(), offsets, B, load, alpha, out_match, out_peer)
         return out_match, out_peer
+
+    def route_decide(self, tokens, offsets, load, alpha: int, excluded=None, want_next: bool = True):
+        """Routing with excluded trees and the next-best target in one pass; returns (match [B,P], peer [B],
+        next [B] or None) CUDA tensors."""
+        import torch
+        B = offsets.numel() - 1
+        m = torch.empty((B, self.P), dtype=torch.int32, device=tokens.device)
+        p = torch.empty(B, dtype=torch.int32, device=tokens.device)
+        n = torch.empty(B, dtype=torch.int32, device=tokens.device) if want_next else None
+        p2p_route_batch_decide(self._h, tokens, tokens.numel(), offsets, B, load, alpha, excluded, m, p, n)
+        return m, p, n
 
     def decide(self, match, load, alpha: int, excluded=None, out_peer=None, out_next=None):
         """match is a CUDA int32 tensor [B, P]; returns (peer [B], next [B]) CUDA tensors."""

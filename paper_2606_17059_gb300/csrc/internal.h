@@ -139,11 +139,14 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
 cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,
                           const uint8_t* d_excluded, int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st);
 // Route kernels (lookup + route decision) of a grouped batch, see route_kernel.cu: a leader pass and a
-// follower pass (g is required).  *launched is set to the number of kernels launched.
+// follower pass (g is required).  *launched is set to the number of kernels launched.  With d_excluded
+// (device bytes [P]) or out_next (device [B]) the passes make the decision with excluded trees and the
+// next-best target instead of the plain argmax.
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens,
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
                          int32_t* out_match, int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms,
-                         cudaStream_t st, int* launched);
+                         cudaStream_t st, int* launched, const uint8_t* d_excluded = nullptr,
+                         int32_t* out_next = nullptr);
 
 // Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaWarps warps
 // per tree.  done[i] (one byte per op of the call, zero before the first launch, kept across relaunches)

@@ -255,13 +255,66 @@ __device__ __forceinline__ unsigned long long route_key(int32_t m, int32_t ld, i
          (unsigned long long)(0xFFFF - p);
 }
 
-// Routes the leaders list[0 .. *count) of a grouped batch with full walks.
+// The route decision of one request, accumulated over its trees by one lane and merged over the warp.
+//   kDecide = false: the max packed key (the route of Algorithm 1's argmax with the load term).
+//   kDecide = true: the two largest keys of the trees not excluded (excl[p] != 0 takes tree p out; Section 3.2,
+//   a peer that pushes back; Section 3.3, a suspected-failed peer), i.e. the best target and the next-best one
+//   that a request falls back to when forwarding times out.  A key is never 0 (score + 2^31 >= 1), so 0 marks
+//   "no candidate" (-1 out).
+template <bool kDecide>
+struct RouteAcc;
+template <>
+struct RouteAcc<false> {
+  unsigned long long k1 = 0;
+  __device__ __forceinline__ void add(unsigned long long key, int32_t, const uint8_t*) { k1 = key > k1 ? key : k1; }
+  __device__ __forceinline__ void warp_merge() {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(kFull, k1, o);
+      k1 = other > k1 ? other : k1;
+    }
+  }
+  __device__ __forceinline__ void write(int64_t b, int32_t* out_peer, int32_t*) const {
+    out_peer[b] = 0xFFFF - (int32_t)(k1 & 0xFFFFull);
+  }
+};
+template <>
+struct RouteAcc<true> {
+  unsigned long long k1 = 0, k2 = 0;
+  __device__ __forceinline__ void add(unsigned long long key, int32_t p, const uint8_t* excl) {
+    if (excl && __ldg(excl + p)) return;
+    if (key > k1) {
+      k2 = k1;
+      k1 = key;
+    } else if (key > k2) {
+      k2 = key;
+    }
+  }
+  __device__ __forceinline__ void warp_merge() {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long o1 = __shfl_xor_sync(kFull, k1, o), o2 = __shfl_xor_sync(kFull, k2, o);
+      const unsigned long long lo = k1 < o1 ? k1 : o1, hi = k1 < o1 ? o1 : k1, r2 = k2 < o2 ? o2 : k2;
+      k1 = hi;
+      k2 = lo < r2 ? r2 : lo;
+    }
+  }
+  __device__ __forceinline__ void write(int64_t b, int32_t* out_peer, int32_t* out_next) const {
+    out_peer[b] = k1 ? 0xFFFF - (int32_t)(k1 & 0xFFFFull) : -1;
+    if (out_next) out_next[b] = k2 ? 0xFFFF - (int32_t)(k2 & 0xFFFFull) : -1;
+  }
+};
+
+// Routes the leaders list[0 .. *count) of a grouped batch with full walks.  kDecide: the decision with
+// excluded trees and the next-best target (RouteAcc<true>), made by the request's last warp from its match
+// row once every item of the request has written its part.
+template <bool kDecide>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ list,
     const int32_t* __restrict__ count, const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin,
     int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match,
-    int32_t* __restrict__ out_peer, int32_t* err) {
+    int32_t* __restrict__ out_peer, int32_t* err, const uint8_t* __restrict__ excl, int32_t* __restrict__ out_next) {
   extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
   __shared__ int4 s_root[kWarps][32];  // per warp: the item's root-table windows
@@ -429,18 +482,32 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
         best = key > best ? key : best;
       }
     }
+    int last = 0;
     if (lane == 0) {
-      atomicMax(&sl.best, best);
+      if (!kDecide) atomicMax(&sl.best, best);
       __threadfence_block();
-      if (atomicAdd(&sl.done, 1) == C - 1) {  // last item of request k: route it, free the slot
-        __threadfence_block();
-        const unsigned long long bk = *(volatile unsigned long long*)&sl.best;
-        if (len < 0) {
+      last = atomicAdd(&sl.done, 1) == C - 1;  // last item of request k: route it, free the slot
+    }
+    if (__shfl_sync(kFull, last, 0)) {
+      __threadfence_block();
+      if (len < 0) {
+        if (lane == 0) {
           out_peer[b] = -1;
+          if (kDecide && out_next) out_next[b] = -1;
           atomicOr(err, ERR_BAD_OFFSETS);
-        } else {
-          out_peer[b] = 0xFFFF - (int32_t)(bk & 0xFFFFull);
         }
+      } else if constexpr (kDecide) {
+        // The row was written by this CTA's warps before their (fenced) item counts: read it past L1.
+        RouteAcc<true> acc;
+        for (int32_t p = lane; p < P; p += 32) acc.add(route_key(__ldcg(out_match + b * P + p), __ldg(load + p), p, alpha), p, excl);
+        acc.warp_merge();
+        if (lane == 0) acc.write(b, out_peer, out_next);
+      } else if (lane == 0) {
+        const unsigned long long bk = *(volatile unsigned long long*)&sl.best;
+        out_peer[b] = 0xFFFF - (int32_t)(bk & 0xFFFFull);
+      }
+      __syncwarp();
+      if (lane == 0) {
         __threadfence_block();
         *(volatile int*)&sl.free_for = (int)(k + kSlots);
       }
@@ -592,14 +659,14 @@ __device__ __forceinline__ int probe_first2(const int4& a, const int4& b, int32_
 //   T) if that is < c, else a walk resumed at the leader's checkpoint that does not compare f's first c
 //   tokens.  A lane takes kFollowIlp trees at a time (p, p + 32, ...): the leader's matches, the
 //   checkpoints and the first probe step of each are loaded before any of them is looked at.
-template <bool kLeader>
+template <bool kLeader, bool kDecide>
 __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, const int32_t* __restrict__ list,
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
     const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
     const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int32_t* err, int32_t* cursor) {
+    int32_t* err, int32_t* cursor, const uint8_t* __restrict__ excl, int32_t* __restrict__ out_next) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
@@ -621,13 +688,14 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
       for (int32_t p = lane; p < P; p += 32) out_match[frow + p] = 0;
       if (lane == 0) {
         out_peer[f] = -1;
+        if (kDecide && out_next) out_next[f] = -1;
         atomicOr(err, ERR_BAD_OFFSETS);
       }
       continue;
     }
     const int32_t* req = tokens + start;
     const int32_t len = (int32_t)min(end - start, (int64_t)INT32_MAX);
-    unsigned long long best = 0;
+    RouteAcc<kDecide> acc;
     if constexpr (kLeader) {
       const int32_t row = __ldg(gid + f);
       const int32_t climit = row >= 0 ? __ldg(cmin + f) : -1;
@@ -648,8 +716,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
         lane_walks<true>(trees, p, req, len, 0, act, ce, pos, m, ck, climit, lane, err);
         if (p < P) {
           out_match[frow + p] = m;
-          const unsigned long long key = route_key(m, __ldg(load + p), p, alpha);
-          best = key > best ? key : best;
+          acc.add(route_key(m, __ldg(load + p), p, alpha), p, excl);
         }
       }
     } else {
@@ -703,18 +770,13 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
           lane_walks<false>(trees, pt[g], req, len, c, act[g], ce[g], pos[g], m[g], nullptr, -1, lane, err);
           if (pt[g] < P) {
             out_match[frow + pt[g]] = m[g];
-            const unsigned long long key = route_key(m[g], __ldg(load + pt[g]), pt[g], alpha);
-            best = key > best ? key : best;
+            acc.add(route_key(m[g], __ldg(load + pt[g]), pt[g], alpha), pt[g], excl);
           }
         }
       }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const unsigned long long other = __shfl_xor_sync(kFull, best, o);
-      best = other > best ? other : best;
-    }
-    if (lane == 0) out_peer[f] = 0xFFFF - (int32_t)(best & 0xFFFFull);
+    acc.warp_merge();
+    if (lane == 0) acc.write(f, out_peer, out_next);
   }
 }
 
@@ -770,13 +832,14 @@ __global__ void __launch_bounds__(256) decide_kernel(const int32_t* __restrict__
 
 }  // namespace
 
-cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
-                         const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
-                         int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st,
-                         int* launched) {
-  *launched = 0;
-  if (B <= 0) return cudaSuccess;
-  if (!g) return cudaErrorInvalidValue;  // every batch is grouped first
+namespace {
+
+// The leader and follower passes with the decision of RouteAcc<kDecide>.
+template <bool kDecide>
+cudaError_t launch_passes(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
+                          const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
+                          int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st,
+                          const uint8_t* excl, int32_t* out_next, int* launched) {
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
   cudaError_t e;
@@ -784,33 +847,47 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
     // Requests of a staging window or longer on average: the leaders' walks are long compares, which the
     // staged kernel's warps do from shared memory.
     const size_t smem = (size_t)kSlots * kSlotTokens * sizeof(int32_t);
-    e = cudaFuncSetAttribute(route_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    e = cudaFuncSetAttribute(route_kernel<kDecide>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const int64_t max_ctas = (int64_t)num_sms * kCtasPerSm;
     const int grid = (int)(B < max_ctas ? B : max_ctas);
     P2P_TIMED(K_ROUTE_STAGED, st,
-              (route_kernel<<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, g->lists,
-                                                          g->counts, g->gid, g->cmin, g->ckpt, d_load, alpha, out_match,
-                                                          out_peer, d_err)));
+              (route_kernel<kDecide><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B,
+                                                                   g->lists, g->counts, g->gid, g->cmin, g->ckpt, d_load,
+                                                                   alpha, out_match, out_peer, d_err, excl, out_next)));
     *launched = 1;
   } else {
     // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
     P2P_TIMED(K_LANE_LEADER, st,
-              (lane_kernel<true><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
-                                                                   g->lists, g->counts, nullptr, nullptr, g->gid,
-                                                                   g->cmin, g->ckpt, d_load, alpha, out_match, out_peer,
-                                                                   d_err, g->counts + 3)));
+              (lane_kernel<true, kDecide><<<grid2, kFollowThreads, 0, st>>>(
+                  d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists, g->counts, nullptr, nullptr, g->gid,
+                  g->cmin, g->ckpt, d_load, alpha, out_match, out_peer, d_err, g->counts + 3, excl, out_next)));
     *launched = 1;
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   P2P_TIMED(K_LANE_FOLLOWER, st,
-            (lane_kernel<false><<<grid2, kFollowThreads, 0, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets,
-                                                                  g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
-                                                                  nullptr, g->ckpt, d_load, alpha, out_match, out_peer,
-                                                                  d_err, nullptr)));
+            (lane_kernel<false, kDecide><<<grid2, kFollowThreads, 0, st>>>(
+                d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
+                nullptr, g->ckpt, d_load, alpha, out_match, out_peer, d_err, nullptr, excl, out_next)));
   *launched += 1;
   return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
+                         const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
+                         int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st,
+                         int* launched, const uint8_t* d_excluded, int32_t* out_next) {
+  *launched = 0;
+  if (B <= 0) return cudaSuccess;
+  if (!g) return cudaErrorInvalidValue;  // every batch is grouped first
+  if (d_excluded || out_next)
+    return launch_passes<true>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, d_load, alpha, out_match, out_peer,
+                               d_err, g, num_sms, st, d_excluded, out_next, launched);
+  return launch_passes<false>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, d_load, alpha, out_match, out_peer,
+                              d_err, g, num_sms, st, nullptr, nullptr, launched);
 }
 
 cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,

@@ -297,14 +297,17 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
 
 // Groups the batch by shared prefix and routes it (leaders, then followers).  The callers check B <= kMaxBatch
 // (request indices and list positions are 32-bit).
+// With d_excl (the staged mask) or out_next, the passes make the decision with excluded trees and the next-best
+// target.
 int route(p2p_router* r, const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
-          int32_t alpha, int32_t* out_match, int32_t* out_peer) {
+          int32_t alpha, int32_t* out_match, int32_t* out_peer, const uint8_t* d_excl = nullptr,
+          int32_t* out_next = nullptr) {
   p2p::GroupScratch g;
   CK(group_scratch(r, B, g));
   CK(p2p::launch_group(tokens, n_tokens, tok_base, offsets, B, g, r->num_sms, r->stream));
   int launched = 0;
   CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
-                       r->d_err, &g, r->num_sms, r->stream, &launched));
+                       r->d_err, &g, r->num_sms, r->stream, &launched, d_excl, out_next));
   r->launches += 2 + launched;
   return P2P_OK;
 }
@@ -1274,6 +1277,21 @@ int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, cons
   DeviceGuard g(r);
   if (int rc = stage_load(r, load)) return rc;
   return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer);
+}
+
+int p2p_route_batch_decide(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
+                           const int32_t* load, int32_t alpha, const uint8_t* excluded, int32_t* out_match,
+                           int32_t* out_peer, int32_t* out_next) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (B < 0 || n_tokens < 0) return fail(r, P2P_E_INVAL, "negative B or n_tokens");
+  if (B > kMaxBatch) return fail(r, P2P_E_INVAL, "B exceeds 2^30 requests per call: split the batch");
+  if (int rc = check_load(r, load, alpha)) return rc;
+  if (B == 0) return P2P_OK;
+  if (!offsets || !out_match || !out_peer || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r);
+  if (int rc = stage_load(r, load, excluded)) return rc;
+  return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer, excluded ? r->d_mask : nullptr,
+               out_next);
 }
 
 int p2p_route_decide(p2p_router* r, const int32_t* match, int64_t B, const int32_t* load, int32_t alpha,

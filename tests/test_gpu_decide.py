@@ -103,3 +103,62 @@ def test_invalid_arguments_and_empty_batch():
     with pytest.raises(ValueError):
         g.p2p_route_decide(r.handle, m, 4, [0, 0, 0], 1, [1, 0], out, out.clone())
     g.p2p_route_decide(r.handle, m, 0, [0, 0, 0], 1, None, out, out.clone())  # B = 0: nothing happens
+
+
+def _fused(r, tok, off, load, alpha, ex, want_next=True):
+    import torch
+    m, p, n = r.route_decide(torch.from_numpy(tok).cuda(), torch.from_numpy(off).cuda(), load, alpha, ex, want_next)
+    r.sync()
+    return m.cpu().numpy(), p.cpu().numpy(), (n.cpu().numpy() if n is not None else None)
+
+
+@pytest.mark.parametrize("cfg", [0, 3])
+def test_decision_fused_into_the_walks_matches_the_oracle(cfg):
+    """p2p_route_batch_decide on workload 0 (lane-walk leaders) and workload 3 (staged leaders of long
+    requests), with masks none, some, all but one and all: the match matrix is the oracle's and (peer, next)
+    is oracle.decide of it."""
+    W = wl.Workload(cfg)
+    sls = [W.tree(p) for p in range(W.P)]
+    r = router_from_seqlists(sls)
+    trees = oracle.build_trees(sls, n_threads=16)
+    B = 2000 if cfg == 3 else W.B
+    tok, off = W.requests(0, B)
+    load = W.load()
+    om, opeer, _ = oracle.route(trees, tok, off, load, W.alpha, n_threads=16)
+    rng = np.random.default_rng(cfg)
+    one = np.ones(W.P, np.uint8)
+    one[rng.integers(W.P)] = 0
+    for ex in (None, (rng.random(W.P) < 0.3).astype(np.uint8), one, np.ones(W.P, np.uint8)):
+        gm, gp, gn = _fused(r, tok, off, load, W.alpha, ex)
+        assert np.array_equal(gm, om)
+        bp, bn = oracle.decide(om, load, W.alpha, ex)
+        assert np.array_equal(gp, bp) and np.array_equal(gn, bn), None if ex is None else int(ex.sum())
+        if ex is None:
+            assert np.array_equal(gp, opeer)
+    # Without a mask or a next-best output it is the plain route.
+    gm, gp, gn = _fused(r, tok, off, load, W.alpha, None, want_next=False)
+    assert gn is None and np.array_equal(gm, om) and np.array_equal(gp, opeer)
+
+
+@pytest.mark.parametrize("seed", [1, 2])
+def test_decision_fused_ties_and_groups(seed):
+    """Vocabularies of 2-4 tokens (deep sharing, many equal scores) and tree counts off the warp width."""
+    rng = random.Random(seed)
+    P = 37 + seed
+    V = 2 + seed
+    seqlists = []
+    for _ in range(P):
+        seqs = [[rng.randrange(V) for _ in range(rng.randint(1, 90))] for _ in range(rng.randint(0, 40))]
+        from gpu_util import seqlist_from_lists
+        seqlists.append(seqlist_from_lists(seqs))
+    reqs = [[rng.randrange(V) for _ in range(rng.randint(0, 120))] for _ in range(700)]
+    from gpu_util import csr_from_lists
+    tok, off = csr_from_lists(reqs)
+    load = np.array([rng.randrange(4) for _ in range(P)], np.int32)
+    r = router_from_seqlists(seqlists)
+    trees = oracle.build_trees(seqlists)
+    om, _, _ = oracle.route(trees, tok, off, load, 1)
+    ex = np.array([rng.random() < 0.25 for _ in range(P)], np.uint8)
+    gm, gp, gn = _fused(r, tok, off, load, 1, ex)
+    bp, bn = oracle.decide(om, load, 1, ex)
+    assert np.array_equal(gm, om) and np.array_equal(gp, bp) and np.array_equal(gn, bn)
