@@ -523,8 +523,9 @@ def run_ours(args):
                 roof["dram_gbs"] = route["dram_gbs"]
                 roof["dram_frac"] = route["dram_gbs"] / hbm
         # ---- optional: the route decision with excluded peers on this batch's match matrix ----
-        if args.decide:
+        if not args.no_decide:
             res["decide"] = time_decide(router, out_match, load, alpha, P, B, hbm, src)
+            res["route_decide"] = time_route_decide(router, d_tok, n_tok, d_off, B, load, alpha, P, route_avg_ms)
         # ---- end to end through the host-pointer C-ABI call ----
         e2e = run_e2e(args, W, router, tok_np, h_off.numpy(), load, alpha, has_delta, n_cpu)
         # ---- UpdateTrieEstimate / UpdateTrie of Algorithm 1 on the last timed batch (changes the trees) ----
@@ -571,6 +572,36 @@ def time_update(router, d_tok, d_off, out_peer, route_ms):
             "route_plus_update_ms": route_ms + ms,
             "note": "one call after the timed steps on the last routed batch; the first call on fresh trees also "
                     "grows their arenas"}
+
+
+def time_route_decide(router, d_tok, n_tok, d_off, B, load, alpha, P, route_ms, reps: int = 5):
+    """p2p_route_batch_decide (the route with 5% of the trees excluded and the next-best target, decided in the
+    walk kernels) against p2p_route_batch on the same batch: mean route time of `reps` calls of each, after
+    one warm-up call, CUDA events on the router stream."""
+    import torch
+    import paper_2606_17059_gb300 as g
+    ex = (np.random.default_rng(5).random(P) < 0.05).astype(np.uint8)
+    m = torch.empty((B, P), dtype=torch.int32, device="cuda")
+    peer = torch.empty(B, dtype=torch.int32, device="cuda")
+    nxt = torch.empty(B, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        fn()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(reps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    plain = timed(lambda: g.p2p_route_batch(router.handle, d_tok, n_tok, d_off, B, load, alpha, m, peer))
+    fused = timed(lambda: g.p2p_route_batch_decide(router.handle, d_tok, n_tok, d_off, B, load, alpha, ex, m, peer, nxt))
+    return {"call": "p2p_route_batch_decide", "excluded": int(ex.sum()), "ms": fused, "plain_route_ms": plain,
+            "cost": fused / plain - 1.0, "timed_step_route_ms": route_ms,
+            "note": "back-to-back calls on the timed batch (no L2 flush between them)"}
 
 
 def time_decide(router, out_match, load, alpha, P, B, hbm, src, reps: int = 10):
@@ -699,8 +730,9 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-update", action="store_true",
                     help="skip the timing of p2p_update_estimates (UpdateTrieEstimate) on the last routed batch")
-    ap.add_argument("--decide", action="store_true",
-                    help="also time p2p_route_decide (excluded peers, next-best target) on the routed batch")
+    ap.add_argument("--no-decide", action="store_true",
+                    help="skip the timing of p2p_route_decide and p2p_route_batch_decide (excluded peers, next-best "
+                         "target) on the routed batch")
     ap.add_argument("--ref-requests", type=int, default=65536)
     ap.add_argument("--ref-seconds", type=float, default=4.0, help="oracle time per reference step")
     ap.add_argument("--trees", type=int, default=0, help="override P (a scaled-down variant, not a bench line)")
