@@ -65,7 +65,8 @@ KERNEL_SOURCE = {
     "compact_kernel": "delta_kernel.cu", "compact_labels_kernel": "delta_kernel.cu",
     "refresh_views_kernel": "delta_kernel.cu", "set_tree_kernel": "delta_kernel.cu",
     "update_count_kernel": "update_kernel.cu", "update_scan_kernel": "update_kernel.cu",
-    "update_scatter_kernel": "update_kernel.cu",
+    "update_scatter_kernel": "update_kernel.cu", "group_ranges_kernel": "group_kernel.cu",
+    "group_place_kernel": "group_kernel.cu",
 }
 # DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum) per workload and kernel, with the
 # source hash of the capture and the profile summary that holds the command.  A figure whose source hash
@@ -480,7 +481,8 @@ def run_ours(args):
         # ---- the route step: compulsory bytes, and the oracle's touched bytes ----
         compulsory = 4 * int(n_tok) + 8 * (B + 1) + 4 * B * P + 4 * B
         route = {"kernels": [k for k in ("group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel",
-                                         "route_kernel", "lane_kernel<true>", "lane_kernel<false>") if k in kt],
+                                         "group_ranges_kernel", "group_place_kernel", "route_kernel",
+                                         "lane_kernel<true>", "lane_kernel<false>") if k in kt],
                  "ms": route_avg_ms, "compulsory_bytes": compulsory,
                  "compulsory_gbs": compulsory / (route_avg_ms / 1e3) / 1e9}
         route["compulsory_frac"] = route["compulsory_gbs"] / hbm

@@ -197,7 +197,7 @@ def p2p_router_launch_count(r) -> int:
     return int(_load().p2p_router_launch_count(r))
 
 
-KERNEL_COUNT = 17  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 16)
+KERNEL_COUNT = 19  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 18)
 
 
 def p2p_router_kernel_clock(r, on: bool) -> None:

@@ -533,6 +533,10 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
       if (lane == 0) t.node[n0] = make_int4(0, 0, 0, 1);
       __syncwarp();
       if (st == 0 && (slot = claim(t, nd.x, tab_bits(nd.y), tok, slot, lane)) < 0) return OP_CORRUPT;
+      if (cur == 0 && lane == 0) {  // a new first token at the root: the route kernels' filter must know it
+        const uint32_t h = root_filter_bit(tok);
+        atomicOr(t.g->rfilter + (h >> 5), 1u << (h & 31));
+      }
       publish(t, slot, n0, l0, (int32_t)L, lane);
       if (lane == 0) atomicAdd(&t.node[cur].z, 1);
       __syncwarp();
@@ -1327,14 +1331,14 @@ __global__ void __launch_bounds__(kLabelThreads) compact_labels_kernel(const Com
 __global__ void set_tree_kernel(TreeState* st, TreeView* view, TreeState v, const int32_t* shared) {
   *st = v;
   const int4 root = v.node[0];
-  *view = TreeView{v.node, v.child, v.label, shared, root.x, tab_bits(root.y)};
+  *view = TreeView{v.node, v.child, v.label, shared, v.rfilter, root.x, tab_bits(root.y)};
 }
 
 __global__ void refresh_views_kernel(const TreeState* st, TreeView* view, int32_t n, const int32_t* shared) {
   const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) {
     const int4 root = st[i].node[0];
-    view[i] = TreeView{st[i].node, st[i].child, st[i].label, shared, root.x, tab_bits(root.y)};
+    view[i] = TreeView{st[i].node, st[i].child, st[i].label, shared, st[i].rfilter, root.x, tab_bits(root.y)};
   }
 }
 

@@ -13,7 +13,9 @@
 // and inserted into an open-addressing table; the smallest request index with that key leads the group.
 // A follower whose exact common prefix with its leader is shorter than kGroupHead (a hash collision) routes
 // as a leader instead.  The leader choice is deterministic (smallest index); the order of the two request
-// lists is not, and only affects scheduling.
+// lists is not, and only affects scheduling.  Each group's followers take a contiguous range of the follower
+// list (group_ranges_kernel, group_place_kernel): the warps that route them at the same time then read the
+// leader's match row, its checkpoints and the tables at the checkpoint nodes once, from cache.
 #include "internal.h"
 
 namespace p2p {
@@ -110,14 +112,14 @@ __device__ int64_t lcp_warp(const int32_t* __restrict__ a, const int32_t* __rest
 
 // One warp per 32 consecutive requests (lane i owns request base + i): each request's leader; for each
 // follower in turn, the exact common prefix with its leader (the whole warp compares); then the warp's
-// leaders and followers are appended to lists[0 ..) and lists[B ..) with one counter update each.  counts
-// must start at zero, gid at -1 and cmin at INT32_MAX.  A leader with followers gets the smallest of their
-// common prefixes in cmin and, while rows last, a checkpoint row in gid (one update per distinct leader of
-// the warp's followers).
+// leaders are appended to lists[0 ..) with one counter update, and each follower takes its rank in its group
+// (fcnt[leader] counts them; the rank goes to slot_of[b]).  counts and fcnt must start at zero, gid at -1 and
+// cmin at INT32_MAX.  A leader with followers gets the smallest of their common prefixes in cmin and, while
+// rows last, a checkpoint row in gid (one update per distinct leader of the warp's followers).
 __global__ void __launch_bounds__(kGroupThreads) group_resolve32_kernel(
     const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
-    int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
-    int32_t* lists, int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap) {
+    int64_t B, const int32_t* __restrict__ vals, int32_t* slot_of, int32_t* lead, int32_t* cpre, int32_t* lists,
+    int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap, int32_t* fcnt) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
   for (int64_t base = (((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5) * 32; base < B; base += warps * 32) {
@@ -150,32 +152,37 @@ __global__ void __launch_bounds__(kGroupThreads) group_resolve32_kernel(
       lead[b] = (int32_t)b;
       lists[lbase + __popc(lm & below)] = (int32_t)b;
     }
+    (void)fbase;
     const unsigned same = __match_any_sync(kFull, is_f ? l : -1);
     if (is_f) {
       lead[b] = l;
       cpre[b] = my_c;
-      lists[B + fbase + __popc(fm & below)] = (int32_t)b;
       const int32_t c_min = (int32_t)__reduce_min_sync(same, (unsigned)my_c);
-      if (lane == __ffs(same) - 1) {
+      const int first = __ffs(same) - 1;
+      int32_t rbase = 0;
+      if (lane == first) {
         atomicMin(&cmin[l], c_min);
+        rbase = atomicAdd(&fcnt[l], __popc(same));
         if (atomicCAS(&gid[l], -1, -2) == -1) {  // the leader's first follower gives it a row
           const int32_t row = atomicAdd(&counts[2], 1);
           atomicExch(&gid[l], row < gcap ? row : -1);
         }
       }
+      slot_of[b] = __shfl_sync(same, rbase, first) + __popc(same & below);  // rank in the group
     }
   }
 }
 
-// One warp per request: its leader and the exact common prefix with it; the CTA's 8 requests of a round are
-// then appended to lists[0 ..) (leaders) or lists[B ..) (followers) with one counter update per list and
-// round.  counts must start at zero, gid at -1 and cmin at INT32_MAX.  A leader with followers gets the
-// smallest of their common prefixes in cmin (updated only when a follower lowers it, so popular groups
-// make few atomics) and, while rows last, a checkpoint row in gid.
+// One warp per request: its leader and the exact common prefix with it; the CTA's leaders of a round are
+// then appended to lists[0 ..) with one counter update per round, and the followers counted (one update per
+// round) and ranked in their groups as in group_resolve32_kernel.  counts and fcnt must start at zero, gid at
+// -1 and cmin at INT32_MAX.  A leader with followers gets the smallest of their common prefixes in cmin
+// (updated only when a follower lowers it, so popular groups make few atomics) and, while rows last, a
+// checkpoint row in gid.
 __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
     const int32_t* __restrict__ tokens, int64_t n_tokens, int64_t tok_base, const int64_t* __restrict__ offsets,
-    int64_t B, const int32_t* __restrict__ vals, const int32_t* __restrict__ slot_of, int32_t* lead, int32_t* cpre,
-    int32_t* lists, int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap) {
+    int64_t B, const int32_t* __restrict__ vals, int32_t* slot_of, int32_t* lead, int32_t* cpre, int32_t* lists,
+    int32_t* counts, int32_t* gid, int32_t* cmin, int32_t gcap, int32_t* fcnt) {
   constexpr int kWarps = kGroupThreads / 32;
   __shared__ int s_kind[kWarps];  // 0: none, 1: leader, 2: follower
   __shared__ int s_pos[kWarps];   // the request's index in its list
@@ -213,7 +220,7 @@ __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
     } else if (lane == 0 && kind == 2) {
       lead[b] = l;
       cpre[b] = c32;
-      lists[B + s_pos[warp]] = (int32_t)b;
+      slot_of[b] = atomicAdd(&fcnt[l], 1);  // rank in the group (slot_of[b] was read above)
       if (c32 < *(volatile int32_t*)&cmin[l]) atomicMin(&cmin[l], c32);
       if (*(volatile int32_t*)&gid[l] == -1 && atomicCAS(&gid[l], -1, -2) == -1) {
         const int32_t row = atomicAdd(&counts[2], 1);  // the leader's first follower gives it a row
@@ -221,6 +228,39 @@ __global__ void __launch_bounds__(kGroupThreads) group_resolve_kernel(
       }
     }
     __syncthreads();  // s_kind and s_pos are reused next round
+  }
+}
+
+// Gives every leader with followers a contiguous range of the follower list: fcnt[l] (its follower count)
+// becomes the start of the range.  One warp per 32 consecutive requests: an inclusive scan of their counts
+// and one counter update per warp (counts[4]).
+__global__ void __launch_bounds__(kGroupThreads) group_ranges_kernel(int64_t B, int32_t* fcnt, int32_t* counts) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = (int64_t)gridDim.x * (kGroupThreads / 32);
+  for (int64_t base = (((int64_t)blockIdx.x * kGroupThreads + threadIdx.x) >> 5) * 32; base < B; base += warps * 32) {
+    const int64_t b = base + lane;
+    const int32_t c = b < B ? fcnt[b] : 0;  // zero for every request that leads no follower
+    int32_t incl = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int32_t v = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += v;
+    }
+    int32_t off = 0;
+    if (lane == 31 && incl) off = atomicAdd(&counts[4], incl);
+    off = __shfl_sync(kFull, off, 31);
+    if (c) fcnt[b] = off + incl - c;
+  }
+}
+
+// Places follower b at lists[B + start of its leader's range + its rank in the group].
+__global__ void __launch_bounds__(kGroupThreads) group_place_kernel(int64_t B, const int32_t* __restrict__ lead,
+                                                                    const int32_t* __restrict__ rank,
+                                                                    const int32_t* __restrict__ fcnt, int32_t* lists) {
+  const int64_t stride = (int64_t)gridDim.x * kGroupThreads;
+  for (int64_t b = (int64_t)blockIdx.x * kGroupThreads + threadIdx.x; b < B; b += stride) {
+    const int32_t l = lead[b];
+    if (l != (int32_t)b) lists[B + fcnt[l] + rank[b]] = (int32_t)b;
   }
 }
 
@@ -232,7 +272,8 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   const size_t slots = (size_t)1 << g.bits;
   cudaError_t e = cudaMemsetAsync(g.keys, 0, slots * sizeof(unsigned long long), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g.vals, 0x7f, slots * sizeof(int32_t), st);  // 0x7f7f7f7f > any index
-  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 4 * sizeof(int32_t), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.counts, 0, 8 * sizeof(int32_t), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g.fcnt, 0, (size_t)B * sizeof(int32_t), st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g.gid, 0xff, (size_t)B * sizeof(int32_t), st);   // -1
   if (e == cudaSuccess) e = cudaMemsetAsync(g.cmin, 0x7f, (size_t)B * sizeof(int32_t), st);  // > any prefix
   if (e != cudaSuccess) return e;
@@ -252,13 +293,21 @@ cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
     P2P_TIMED(K_GROUP_RESOLVE32, st,
               (group_resolve32_kernel<<<grid, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals,
                                                                       g.slot_of, g.lead, g.cpre, g.lists, g.counts,
-                                                                      g.gid, g.cmin, g.gcap)));
+                                                                      g.gid, g.cmin, g.gcap, g.fcnt)));
   } else {
     P2P_TIMED(K_GROUP_RESOLVE, st,
               (group_resolve_kernel<<<grid2, kGroupThreads, 0, st>>>(tokens, n_tokens, tok_base, offsets, B, g.vals,
                                                                      g.slot_of, g.lead, g.cpre, g.lists, g.counts,
-                                                                     g.gid, g.cmin, g.gcap)));
+                                                                     g.gid, g.cmin, g.gcap, g.fcnt)));
   }
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  // Each group's followers side by side in the follower list.
+  const int64_t place_ctas = (B + kGroupThreads - 1) / kGroupThreads;
+  const int grid3 = (int)std::min<int64_t>(place_ctas, (int64_t)num_sms * 8);
+  P2P_TIMED(K_GROUP_RANGES, st, (group_ranges_kernel<<<grid, kGroupThreads, 0, st>>>(B, g.fcnt, g.counts)));
+  P2P_TIMED(K_GROUP_PLACE, st,
+            (group_place_kernel<<<grid3, kGroupThreads, 0, st>>>(B, g.lead, g.slot_of, g.fcnt, g.lists)));
   return cudaGetLastError();
 }
 

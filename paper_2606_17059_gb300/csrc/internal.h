@@ -38,8 +38,22 @@ struct TreeView {
   const int4* child;
   const int32_t* label;
   const int32_t* shared;        // the router's shared label pool
+  const uint32_t* rfilter;      // the root's first-token filter (see below)
   int32_t root_off, root_bits;  // the root's children table (copied from node[0] when the view is set)
 };
+
+// Root first-token filter, one per tree: a bit per 16-bit hash of a token, set for the first token of every
+// child the root has had since the tree was uploaded (bits are never cleared, so a clear bit proves the token
+// starts no child; a set bit may be stale).  A request whose first token is absent matches nothing in the
+// tree; the filter (8 KB a tree, 2 MB for 256 trees) stays in L2, while the root tables it spares (~1 MB a
+// tree at the scale workload) do not.  Fresh prompts, a fifth of the scale workload's requests, are such
+// requests in most trees.
+constexpr int kRootFilterWords = 2048;
+inline __host__ __device__ uint32_t root_filter_bit(int32_t tok) { return ((uint32_t)tok * 0xC2B2AE3Du) >> 16; }
+inline __host__ __device__ bool root_filter_has(const uint32_t* f, int32_t tok) {
+  const uint32_t h = root_filter_bit(tok);
+  return (f[h >> 5] >> (h & 31)) & 1u;
+}
 
 // Start of the label of an edge whose label_off is `off` (see the layout above).
 inline __host__ __device__ const int32_t* label_ptr(const int32_t* label, const int32_t* shared, int32_t off) {
@@ -54,6 +68,7 @@ struct TreeState {
   int4* node;
   int4* child;
   int32_t* label;
+  uint32_t* rfilter;           // the root's first-token filter (kRootFilterWords words; the router's array)
   int32_t n_node, cap_node;    // node slots used (bump arena) / capacity
   int32_t n_child, cap_child;  // child-table slots used (bump arena) / capacity
   int32_t n_label, cap_label;  // label tokens used (bump arena) / capacity
@@ -91,7 +106,7 @@ constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits 
 enum KernelId {
   K_GROUP_HASH, K_GROUP_RESOLVE, K_GROUP_RESOLVE32, K_ROUTE_STAGED, K_LANE_LEADER, K_LANE_FOLLOWER, K_DECIDE,
   K_VALIDATE, K_INIT_RANGES, K_DELTA, K_COMPACT, K_COMPACT_LABELS, K_REFRESH_VIEWS, K_SET_TREE,
-  K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_COUNT_
+  K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_GROUP_RANGES, K_GROUP_PLACE, K_COUNT_
 };
 static_assert(K_COUNT_ == P2P_KERNEL_COUNT, "the header's kernel count");
 const char* kernel_name(int id);
@@ -116,7 +131,9 @@ enum { ERR_BAD_OFFSETS = 1, ERR_CORRUPT_TREE = 2, ERR_STALL = 4 };
 
 // Shared-prefix groups of a batch (group_kernel.cu): requests of at least kGroupHead tokens are grouped by
 // their first kGroupHead tokens; lead[b] is b's group leader, cpre[b] its exact common prefix with the
-// leader (followers only); lists[0 .. counts[0]) are the leaders, lists[B .. B + counts[1]) the followers.
+// leader (followers only); lists[0 .. counts[0]) are the leaders, lists[B .. B + counts[1]) the followers,
+// each group's followers side by side (so the warps routing them at the same time share the leader's row,
+// checkpoints and tables in cache).
 constexpr int kGroupHead = 64;
 struct GroupScratch {
   unsigned long long* keys;  // 2^bits slots
@@ -126,7 +143,9 @@ struct GroupScratch {
   int32_t* lead;     // [B]
   int32_t* cpre;     // [B]
   int32_t* lists;    // [2B]
-  int32_t* counts;   // [4]: leaders, followers, groups with a checkpoint row, the leader pass's work cursor
+  int32_t* counts;   // [8]: leaders, followers, groups with a checkpoint row, the leader pass's work cursor,
+                     //      the follower ranges handed out
+  int32_t* fcnt;     // [B]: a leader's follower count, then the start of its followers' range
   int32_t* gid;      // [B]: a leader's checkpoint row (-1: none)
   int32_t* cmin;     // [B]: a leader's smallest common prefix with its followers
   int4* ckpt;        // [gcap * P]: per (row, tree) the leader's walk state to resume from (see route_kernel.cu)

@@ -443,13 +443,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
       bool hit = false, empty = false;
       if (tp < p1) {
         const int32_t bits = trees[tp].root_bits;
-        if (bits > 0) {
+        if (bits > 0 && root_filter_has(trees[tp].rfilter, tok0)) {
           const uint32_t mask = (1u << bits) - 1;
           re = __ldg(trees[tp].child + trees[tp].root_off + ((slot_hash(tok0, bits) + (lane & 3)) & mask));
           hit = re.y >= 1 && re.x == tok0;
           empty = re.y == 0;
         } else {
-          empty = true;  // an empty root table holds nothing
+          empty = true;  // an empty root table, or a first token the root filter rules out
         }
       }
       s_re[lane] = re;
@@ -699,6 +699,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     if constexpr (kLeader) {
       const int32_t row = __ldg(gid + f);
       const int32_t climit = row >= 0 ? __ldg(cmin + f) : -1;
+      const int32_t tok0 = len > 0 ? __ldg(req) : 0;
       for (int32_t p0 = 0; p0 < P; p0 += 32) {
         const int32_t p = p0 + lane;
         int32_t m = 0, pos = 0;
@@ -711,7 +712,10 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
             ck = ckpt + (int64_t)row * P + p;
             *ck = st;
           }
-          act = st.w > 0 && find_child_1(trees[p].child + st.y, tab_bits(st.z), __ldg(req), ce);
+          // The root filter answers most absent first tokens (fresh prompts) from L2; the root table only
+          // when the token may be there.
+          act = st.w > 0 && root_filter_has(trees[p].rfilter, tok0) &&
+                find_child_1(trees[p].child + st.y, tab_bits(st.z), tok0, ce);
         }
         lane_walks<true>(trees, p, req, len, 0, act, ce, pos, m, ck, climit, lane, err);
         if (p < P) {

@@ -88,7 +88,7 @@ const char* kernel_name(int id) {
       "group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel", "route_kernel", "lane_kernel<true>",
       "lane_kernel<false>", "decide_kernel", "validate_kernel", "init_ranges_kernel", "delta_kernel",
       "compact_kernel", "compact_labels_kernel", "refresh_views_kernel", "set_tree_kernel", "update_count_kernel",
-      "update_scan_kernel", "update_scatter_kernel"};
+      "update_scan_kernel", "update_scatter_kernel", "group_ranges_kernel", "group_place_kernel"};
   return id >= 0 && id < K_COUNT_ ? names[id] : "";
 }
 
@@ -181,6 +181,7 @@ struct p2p_router {
   std::vector<TreeState> spare;
   TreeView* d_views = nullptr;
   TreeState* d_states = nullptr;
+  uint32_t* d_rfilter = nullptr;  // P root first-token filters of kRootFilterWords words
   int32_t* d_load = nullptr;
   int32_t* d_err = nullptr;
   int32_t* d_hdr = nullptr;  // validation result of device-resident deltas
@@ -269,14 +270,14 @@ cudaError_t ensure(p2p_router* r, DevBuf& b, size_t bytes) {
 }
 
 // Scratch of the shared-prefix grouping for a batch of B requests (B <= 2^30): a key table of at least 2B
-// slots; slot_of, lead, cpre (B each), the two request lists (2B), gid and cmin (B each) and four counts;
+// slots; slot_of, lead, cpre (B each), the two request lists (2B), gid, cmin and fcnt (B each) and eight counts;
 // and checkpoint rows, as many as fit in 256 MB (and at most B/2 + 1, one per leader with followers).
 cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
   const int64_t slots = std::max<int64_t>(next_pow2(2 * B), 1024);
   const int64_t gcap = std::max<int64_t>(1, std::min<int64_t>(B / 2 + 1, ((int64_t)256 << 20) / ((int64_t)r->P * 16)));
   cudaError_t e = ensure(r, r->grp_keys, (size_t)slots * sizeof(unsigned long long));
   if (e == cudaSuccess) e = ensure(r, r->grp_vals, (size_t)slots * sizeof(int32_t));
-  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(7 * B + 4) * sizeof(int32_t));
+  if (e == cudaSuccess) e = ensure(r, r->grp_req, (size_t)(8 * B + 8) * sizeof(int32_t));
   if (e == cudaSuccess) e = ensure(r, r->grp_ckpt, (size_t)gcap * r->P * sizeof(int4));
   if (e != cudaSuccess) return e;
   int32_t* q = static_cast<int32_t*>(r->grp_req.p);
@@ -289,7 +290,8 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
   g.lists = q + 3 * B;
   g.gid = q + 5 * B;
   g.cmin = q + 6 * B;
-  g.counts = q + 7 * B;
+  g.fcnt = q + 7 * B;
+  g.counts = q + 8 * B;
   g.ckpt = static_cast<int4*>(r->grp_ckpt.p);
   g.gcap = (int32_t)gcap;
   return cudaSuccess;
@@ -308,7 +310,7 @@ int route(p2p_router* r, const int32_t* tokens, int64_t n_tokens, int64_t tok_ba
   int launched = 0;
   CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
                        r->d_err, &g, r->num_sms, r->stream, &launched, d_excl, out_next));
-  r->launches += 2 + launched;
+  r->launches += 4 + launched;
   return P2P_OK;
 }
 
@@ -350,6 +352,8 @@ int install_empty_tree(p2p_router* r, int32_t p) {
   if (e != cudaSuccess) return cuda_fail(r, e, "allocating an empty tree");
   const int4 root = make_int4(0, p2p::make_meta(rb, 0), 0, 0);
   CK(cudaMemsetAsync(t.child, 0, ((size_t)1 << rb) * sizeof(int4), r->stream));
+  t.rfilter = r->d_rfilter + (size_t)p * p2p::kRootFilterWords;
+  CK(cudaMemsetAsync(t.rfilter, 0, p2p::kRootFilterWords * sizeof(uint32_t), r->stream));
   CK(cudaMemcpyAsync(t.node, &root, sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   CK(cudaStreamSynchronize(r->stream));  // `root` is a host temporary
   t.n_node = 1;
@@ -518,6 +522,14 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   nt.n_node = (int32_t)N;
   nt.n_child = (int32_t)slots;
   nt.n_label = (int32_t)n_own;
+  // The root's first-token filter: exactly the root's children now.
+  std::vector<uint32_t> filt(p2p::kRootFilterWords, 0u);
+  for (int64_t e = t->child_begin[0]; e < (int64_t)t->child_begin[0] + t->child_count[0]; ++e) {
+    const uint32_t h = p2p::root_filter_bit(t->child_first_tok[e]);
+    filt[h >> 5] |= 1u << (h & 31);
+  }
+  nt.rfilter = r->d_rfilter + (size_t)peer * p2p::kRootFilterWords;
+  CK(cudaMemcpyAsync(nt.rfilter, filt.data(), filt.size() * sizeof(uint32_t), cudaMemcpyHostToDevice, r->stream));
   TreeState& old = r->hs[(size_t)peer];
   free_tree_arrays(r, old);
   old = nt;
@@ -749,6 +761,7 @@ bool nears_compaction(const TreeState& t) {
 
 // Resets the per-call fields of trees [p0, p1) and copies their states to the device.
 int push_states(p2p_router* r, int32_t p0, int32_t p1) {
+  for (int32_t p = p0; p < p1; ++p) r->hs[(size_t)p].rfilter = r->d_rfilter + (size_t)p * p2p::kRootFilterWords;
   std::memcpy(r->h_states, r->hs.data() + p0, (size_t)(p1 - p0) * sizeof(TreeState));
   CK(cudaMemcpyAsync(r->d_states + p0, r->h_states, (size_t)(p1 - p0) * sizeof(TreeState), cudaMemcpyHostToDevice,
                      r->stream));
@@ -802,6 +815,7 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   r->spare.assign((size_t)P, TreeState{});
   e = dalloc(r, (void**)&r->d_views, (size_t)P * sizeof(TreeView));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_states, (size_t)P * sizeof(TreeState));
+  if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_rfilter, (size_t)P * p2p::kRootFilterWords * sizeof(uint32_t));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_load, (size_t)P * sizeof(int32_t));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_mask, (size_t)P);
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_err, sizeof(int32_t));
@@ -851,6 +865,7 @@ void p2p_router_destroy(p2p_router* r) {
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
+    dfree(r, r->d_rfilter);
     dfree(r, r->d_load);
     dfree(r, r->d_mask);
     dfree(r, r->d_err);

@@ -250,3 +250,35 @@ def test_kernel_clock_counts_every_launch():
     assert r.kernel_times() == {}
     with pytest.raises(g.P2PError):
         g.p2p_router_kernel_time(r.handle, g.KERNEL_COUNT)
+
+
+def test_root_first_tokens_added_and_removed_by_deltas():
+    """A first token that a delta adds at the root is found by the next route (the root filter learns it on
+    the device); one whose sequences are all deleted matches nothing again (its filter bit stays set)."""
+    import torch
+    rng = np.random.default_rng(12)
+    base = [[int(t)] + rng.integers(0, 50, size=20).tolist() for t in range(0, 4000, 7)]
+    r = router_from_seqlists([seqlist_from_lists(base)])
+    otree = oracle.build_trees([seqlist_from_lists(base)])[0]
+    new = [[int(t)] + rng.integers(0, 50, size=12).tolist() for t in range(3, 4000, 7)]
+    gone = base[::3]
+    ops = np.array([0] * len(new) + [1] * len(gone), np.int32)
+    sl = seqlist_from_lists(new + gone)
+    assert r.apply_delta(0, _dev_arr(ops), _dev_seqlist(sl), None, on_device=True) == 0
+    otree.apply_ops(ops, sl)
+    reqs = [s[:15] for s in new] + [s[:15] for s in base] + [[t, 1, 2] for t in range(1, 4000, 7)]
+    tok, off = csr_from_lists(reqs)
+    gm, gp = route_device(r, tok, off, [0], 0)
+    om, op, _ = oracle.route([otree], tok, off, [0], 0)
+    assert_same_route(gm, gp, om, op, "root filter after a delta")
+    assert (gm[: len(new), 0] == 15).all()
+    del torch
+
+
+def _dev_arr(a):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _dev_seqlist(sl):
+    return wl.SeqList(_dev_arr(sl.seg_begin), _dev_arr(sl.seg_off), _dev_arr(sl.seg_len), _dev_arr(sl.pool))
