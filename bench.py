@@ -9,7 +9,7 @@ region starts.  The JSON line also carries:
   kernels       every kernel launched in the timed region: launches, device ms per step (the library's kernel
                 clock, CUDA events on the router stream), share, and its DRAM traffic per launch where an ncu
                 capture of the same kernel source gave one;
-  roofline      the stage that takes the most time -- the delta kernel, or the route step's four launches --
+  roofline      the stage that takes the most time -- the delta kernel, or the route step's launches --
                 against the measured HBM copy bandwidth: achieved = algorithmic bytes per launch / device time.
                 The delta kernel's algorithmic bytes are the oracle's per-op counters (input, walk, writes);
                 the route step's are its compulsory bytes (request tokens and offsets read once, the match

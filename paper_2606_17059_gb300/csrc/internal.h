@@ -154,18 +154,20 @@ struct GroupScratch {
 cudaError_t launch_group(const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
                          const GroupScratch& g, int num_sms, cudaStream_t st);
 
+// Staged load words (d_load) carry the load in the low 16 bits and kLoadExcluded for a tree that the
+// decision with excluded trees takes out.
+constexpr int32_t kLoadExcluded = 1 << 16;
 // Best and next-best non-excluded peer of every row of match [B x P] (route_key order); -1 where none.
 cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,
-                          const uint8_t* d_excluded, int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st);
+                          int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st);
 // Route kernels (lookup + route decision) of a grouped batch, see route_kernel.cu: a leader pass and a
-// follower pass (g is required).  *launched is set to the number of kernels launched.  With d_excluded
-// (device bytes [P]) or out_next (device [B]) the passes make the decision with excluded trees and the
-// next-best target instead of the plain argmax.
+// follower pass (g is required).  *launched is set to the number of kernels launched.  With decide (load
+// words carrying kLoadExcluded) or out_next (device [B]) the passes make the decision with excluded trees
+// and the next-best target instead of the plain argmax.
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens,
                          int64_t tok_base, const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha,
                          int32_t* out_match, int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms,
-                         cudaStream_t st, int* launched, const uint8_t* d_excluded = nullptr,
-                         int32_t* out_next = nullptr);
+                         cudaStream_t st, int* launched, bool decide = false, int32_t* out_next = nullptr);
 
 // Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaWarps warps
 // per tree.  done[i] (one byte per op of the call, zero before the first launch, kept across relaunches)

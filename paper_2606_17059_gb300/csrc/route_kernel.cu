@@ -248,7 +248,9 @@ __device__ __forceinline__ bool wait_for(const int* flag, int v, int lane) {
 
 // Packed route key: (score + 2^31) << 32 | (0xFFFF - load) << 16 | (0xFFFF - p); a larger key is a better
 // route (higher score, then lower load, then lower index).  The host guarantees alpha * load <= 2^31 - 1,
-// load <= 65535 and P <= 65536, so every field fits.
+// load <= 65535 and P <= 65536, so every field fits.  The staged load word of tree p carries kExcluded when
+// the decision with excluded trees takes p out (the load itself is the low 16 bits).
+constexpr int32_t kExcluded = kLoadExcluded;
 __device__ __forceinline__ unsigned long long route_key(int32_t m, int32_t ld, int32_t p, int32_t alpha) {
   const long long score = (long long)m - (long long)alpha * ld;
   return ((unsigned long long)(score + 2147483648LL) << 32) | ((unsigned long long)(0xFFFF - ld) << 16) |
@@ -257,7 +259,7 @@ __device__ __forceinline__ unsigned long long route_key(int32_t m, int32_t ld, i
 
 // The route decision of one request, accumulated over its trees by one lane and merged over the warp.
 //   kDecide = false: the max packed key (the route of Algorithm 1's argmax with the load term).
-//   kDecide = true: the two largest keys of the trees not excluded (excl[p] != 0 takes tree p out; Section 3.2,
+//   kDecide = true: the two largest keys of the trees not excluded (kExcluded in the load word; Section 3.2,
 //   a peer that pushes back; Section 3.3, a suspected-failed peer), i.e. the best target and the next-best one
 //   that a request falls back to when forwarding times out.  A key is never 0 (score + 2^31 >= 1), so 0 marks
 //   "no candidate" (-1 out).
@@ -266,7 +268,10 @@ struct RouteAcc;
 template <>
 struct RouteAcc<false> {
   unsigned long long k1 = 0;
-  __device__ __forceinline__ void add(unsigned long long key, int32_t, const uint8_t*) { k1 = key > k1 ? key : k1; }
+  __device__ __forceinline__ void add(int32_t m, int32_t ldw, int32_t p, int32_t alpha) {
+    const unsigned long long key = route_key(m, ldw, p, alpha);
+    k1 = key > k1 ? key : k1;
+  }
   __device__ __forceinline__ void warp_merge() {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -281,8 +286,9 @@ struct RouteAcc<false> {
 template <>
 struct RouteAcc<true> {
   unsigned long long k1 = 0, k2 = 0;
-  __device__ __forceinline__ void add(unsigned long long key, int32_t p, const uint8_t* excl) {
-    if (excl && __ldg(excl + p)) return;
+  __device__ __forceinline__ void add(int32_t m, int32_t ldw, int32_t p, int32_t alpha) {
+    if (ldw & kExcluded) return;
+    const unsigned long long key = route_key(m, ldw, p, alpha);
     if (key > k1) {
       k2 = k1;
       k1 = key;
@@ -314,7 +320,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
     int64_t tok_base, const int64_t* __restrict__ offsets, int64_t B, const int32_t* __restrict__ list,
     const int32_t* __restrict__ count, const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin,
     int4* __restrict__ ckpt, const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match,
-    int32_t* __restrict__ out_peer, int32_t* err, const uint8_t* __restrict__ excl, int32_t* __restrict__ out_next) {
+    int32_t* __restrict__ out_peer, int32_t* err, int32_t* __restrict__ out_next) {
   extern __shared__ __align__(128) int32_t s_tok[];  // kSlots x kSlotTokens
   __shared__ Slot s_slot[kSlots];
   __shared__ int4 s_root[kWarps][32];  // per warp: the item's root-table windows
@@ -499,7 +505,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) route_kernel(
       } else if constexpr (kDecide) {
         // The row was written by this CTA's warps before their (fenced) item counts: read it past L1.
         RouteAcc<true> acc;
-        for (int32_t p = lane; p < P; p += 32) acc.add(route_key(__ldcg(out_match + b * P + p), __ldg(load + p), p, alpha), p, excl);
+        for (int32_t p = lane; p < P; p += 32) acc.add(__ldcg(out_match + b * P + p), __ldg(load + p), p, alpha);
         acc.warp_merge();
         if (lane == 0) acc.write(b, out_peer, out_next);
       } else if (lane == 0) {
@@ -666,7 +672,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const int32_t* __restrict__ count, const int32_t* __restrict__ lead, const int32_t* __restrict__ cpre,
     const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
     const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
-    int32_t* err, int32_t* cursor, const uint8_t* __restrict__ excl, int32_t* __restrict__ out_next) {
+    int32_t* err, int32_t* cursor, int32_t* __restrict__ out_next) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
@@ -720,7 +726,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
         lane_walks<true>(trees, p, req, len, 0, act, ce, pos, m, ck, climit, lane, err);
         if (p < P) {
           out_match[frow + p] = m;
-          acc.add(route_key(m, __ldg(load + p), p, alpha), p, excl);
+          acc.add(m, __ldg(load + p), p, alpha);
         }
       }
     } else {
@@ -774,7 +780,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
           lane_walks<false>(trees, pt[g], req, len, c, act[g], ce[g], pos[g], m[g], nullptr, -1, lane, err);
           if (pt[g] < P) {
             out_match[frow + pt[g]] = m[g];
-            acc.add(route_key(m[g], __ldg(load + pt[g]), pt[g], alpha), pt[g], excl);
+            acc.add(m[g], __ldg(load + pt[g]), pt[g], alpha);
           }
         }
       }
@@ -785,21 +791,18 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
 }
 
 // Route decision from a match matrix with excluded peers (one warp per request): the best and the next-best
-// candidate by the route order of route_key, skipping peers with excluded[p] != 0 (Section 3.2: a peer that
-// pushes back; Section 3.3: a suspected-failed peer, and the next-best target a request falls back to when
-// forwarding times out).  Each lane keeps the two largest keys of its peers, and five butterfly steps merge
-// the lanes' pairs.  A key is never 0 (score + 2^31 >= 1), so 0 marks "no candidate" (-1 out).  Match values
-// below 0 count as 0.
+// candidate by the route order of route_key, skipping trees whose staged load word carries kExcluded
+// (Section 3.2: a peer that pushes back; Section 3.3: a suspected-failed peer, and the next-best target a
+// request falls back to when forwarding times out), with RouteAcc<true>.  Match values below 0 count as 0.
 constexpr int kDecideUnroll = 8;  // columns a lane loads per stretch (a 256-tree row in one stretch)
 __global__ void __launch_bounds__(256) decide_kernel(const int32_t* __restrict__ match, int64_t B, int32_t P,
                                                      const int32_t* __restrict__ load, int32_t alpha,
-                                                     const uint8_t* __restrict__ excluded,
                                                      int32_t* __restrict__ out_peer, int32_t* __restrict__ out_next) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
   for (int64_t b = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; b < B; b += warps) {
     const int32_t* row = match + b * P;
-    unsigned long long k1 = 0, k2 = 0;
+    RouteAcc<true> acc;
     for (int32_t p0 = 0; p0 < P; p0 += 32 * kDecideUnroll) {
       int32_t v[kDecideUnroll];  // a lane's columns of this stretch, loaded before any is looked at
 #pragma unroll
@@ -810,27 +813,11 @@ __global__ void __launch_bounds__(256) decide_kernel(const int32_t* __restrict__
 #pragma unroll
       for (int u = 0; u < kDecideUnroll; ++u) {
         const int32_t p = p0 + 32 * u + lane;
-        if (p >= P || (excluded && excluded[p])) continue;
-        const unsigned long long k = route_key(max(v[u], 0), __ldg(load + p), p, alpha);
-        if (k > k1) {
-          k2 = k1;
-          k1 = k;
-        } else if (k > k2) {
-          k2 = k;
-        }
+        if (p < P) acc.add(max(v[u], 0), __ldg(load + p), p, alpha);
       }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const unsigned long long o1 = __shfl_xor_sync(kFull, k1, o), o2 = __shfl_xor_sync(kFull, k2, o);
-      const unsigned long long lo = k1 < o1 ? k1 : o1, hi = k1 < o1 ? o1 : k1, r2 = k2 < o2 ? o2 : k2;
-      k1 = hi;
-      k2 = lo < r2 ? r2 : lo;
-    }
-    if (lane == 0) {
-      out_peer[b] = k1 ? 0xFFFF - (int32_t)(k1 & 0xFFFFull) : -1;
-      out_next[b] = k2 ? 0xFFFF - (int32_t)(k2 & 0xFFFFull) : -1;
-    }
+    acc.warp_merge();
+    if (lane == 0) acc.write(b, out_peer, out_next);
   }
 }
 
@@ -843,7 +830,7 @@ template <bool kDecide>
 cudaError_t launch_passes(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
                           const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
                           int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st,
-                          const uint8_t* excl, int32_t* out_next, int* launched) {
+                          int32_t* out_next, int* launched) {
   const int64_t want = (B + kFollowThreads / 32 - 1) / (kFollowThreads / 32);
   const int grid2 = (int)std::min<int64_t>(want, (int64_t)num_sms * kFollowCtasPerSm);
   cudaError_t e;
@@ -858,14 +845,14 @@ cudaError_t launch_passes(const TreeView* d_trees, int32_t P, const int32_t* tok
     P2P_TIMED(K_ROUTE_STAGED, st,
               (route_kernel<kDecide><<<grid, kThreads, smem, st>>>(d_trees, P, tokens, n_tokens, tok_base, offsets, B,
                                                                    g->lists, g->counts, g->gid, g->cmin, g->ckpt, d_load,
-                                                                   alpha, out_match, out_peer, d_err, excl, out_next)));
+                                                                   alpha, out_match, out_peer, d_err, out_next)));
     *launched = 1;
   } else {
     // Shorter requests: most leader walks end within a few tokens, so each lane walks its own tree.
     P2P_TIMED(K_LANE_LEADER, st,
               (lane_kernel<true, kDecide><<<grid2, kFollowThreads, 0, st>>>(
                   d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists, g->counts, nullptr, nullptr, g->gid,
-                  g->cmin, g->ckpt, d_load, alpha, out_match, out_peer, d_err, g->counts + 3, excl, out_next)));
+                  g->cmin, g->ckpt, d_load, alpha, out_match, out_peer, d_err, g->counts + 3, out_next)));
     *launched = 1;
   }
   e = cudaGetLastError();
@@ -873,7 +860,7 @@ cudaError_t launch_passes(const TreeView* d_trees, int32_t P, const int32_t* tok
   P2P_TIMED(K_LANE_FOLLOWER, st,
             (lane_kernel<false, kDecide><<<grid2, kFollowThreads, 0, st>>>(
                 d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
-                nullptr, g->ckpt, d_load, alpha, out_match, out_peer, d_err, nullptr, excl, out_next)));
+                nullptr, g->ckpt, d_load, alpha, out_match, out_peer, d_err, nullptr, out_next)));
   *launched += 1;
   return cudaGetLastError();
 }
@@ -883,23 +870,23 @@ cudaError_t launch_passes(const TreeView* d_trees, int32_t P, const int32_t* tok
 cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* tokens, int64_t n_tokens, int64_t tok_base,
                          const int64_t* offsets, int64_t B, const int32_t* d_load, int32_t alpha, int32_t* out_match,
                          int32_t* out_peer, int32_t* d_err, const GroupScratch* g, int num_sms, cudaStream_t st,
-                         int* launched, const uint8_t* d_excluded, int32_t* out_next) {
+                         int* launched, bool decide, int32_t* out_next) {
   *launched = 0;
   if (B <= 0) return cudaSuccess;
   if (!g) return cudaErrorInvalidValue;  // every batch is grouped first
-  if (d_excluded || out_next)
+  if (decide || out_next)
     return launch_passes<true>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, d_load, alpha, out_match, out_peer,
-                               d_err, g, num_sms, st, d_excluded, out_next, launched);
+                               d_err, g, num_sms, st, out_next, launched);
   return launch_passes<false>(d_trees, P, tokens, n_tokens, tok_base, offsets, B, d_load, alpha, out_match, out_peer,
-                              d_err, g, num_sms, st, nullptr, nullptr, launched);
+                              d_err, g, num_sms, st, nullptr, launched);
 }
 
 cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,
-                          const uint8_t* d_excluded, int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st) {
+                          int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
   const int64_t want = (B + 7) / 8;
   const int grid = (int)std::min<int64_t>(want, (int64_t)std::max(num_sms, 1) * 8);
-  P2P_TIMED(K_DECIDE, st, (decide_kernel<<<grid, 256, 0, st>>>(match, B, P, d_load, alpha, d_excluded, out_peer, out_next)));
+  P2P_TIMED(K_DECIDE, st, (decide_kernel<<<grid, 256, 0, st>>>(match, B, P, d_load, alpha, out_peer, out_next)));
   return cudaGetLastError();
 }
 

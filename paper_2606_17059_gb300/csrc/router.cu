@@ -186,8 +186,6 @@ struct p2p_router {
   int32_t* d_err = nullptr;
   int32_t* d_hdr = nullptr;  // validation result of device-resident deltas
   int32_t* h_load = nullptr;  // pinned, kLoadRing slots of P values
-  uint8_t* d_mask = nullptr;  // excluded peers of p2p_route_decide
-  uint8_t* h_mask = nullptr;  // pinned, kLoadRing slots of P bytes (staged with the load of the same slot)
   cudaEvent_t load_ev[kLoadRing] = {};
   // Copy streams of p2p_route_batch_host (inputs in, results out) and the events that order them.
   cudaStream_t cp_in = nullptr, cp_out = nullptr;
@@ -299,17 +297,16 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
 
 // Groups the batch by shared prefix and routes it (leaders, then followers).  The callers check B <= kMaxBatch
 // (request indices and list positions are 32-bit).
-// With d_excl (the staged mask) or out_next, the passes make the decision with excluded trees and the next-best
-// target.
+// With decide (an excluded-peer mask staged with the load) or out_next, the passes make the decision with
+// excluded trees and the next-best target.
 int route(p2p_router* r, const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
-          int32_t alpha, int32_t* out_match, int32_t* out_peer, const uint8_t* d_excl = nullptr,
-          int32_t* out_next = nullptr) {
+          int32_t alpha, int32_t* out_match, int32_t* out_peer, bool decide = false, int32_t* out_next = nullptr) {
   p2p::GroupScratch g;
   CK(group_scratch(r, B, g));
   CK(p2p::launch_group(tokens, n_tokens, tok_base, offsets, B, g, r->num_sms, r->stream));
   int launched = 0;
   CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
-                       r->d_err, &g, r->num_sms, r->stream, &launched, d_excl, out_next));
+                       r->d_err, &g, r->num_sms, r->stream, &launched, decide, out_next));
   r->launches += 4 + launched;
   return P2P_OK;
 }
@@ -380,20 +377,18 @@ int check_load(p2p_router* r, const int32_t* load, int32_t alpha) {
   return P2P_OK;
 }
 
-// Stages load[P] (and, if given, the excluded-peer bytes mask[P]) through a pinned ring slot; the slot's
-// previous copies have finished once its event has.
+// Stages load[P] through a pinned ring slot; with an excluded-peer mask (mask[p] != 0), tree p's load word
+// also carries kLoadExcluded.  The slot's previous copy has finished once its event has.
 int stage_load(p2p_router* r, const int32_t* load, const uint8_t* mask = nullptr) {
   const int s = r->load_slot;
   r->load_slot = (s + 1) % kLoadRing;
   CK(cudaEventSynchronize(r->load_ev[s]));
   int32_t* slot = r->h_load + (size_t)s * r->P;
   std::memcpy(slot, load, (size_t)r->P * sizeof(int32_t));
+  if (mask)
+    for (int32_t p = 0; p < r->P; ++p)
+      if (mask[p]) slot[p] |= p2p::kLoadExcluded;
   CK(cudaMemcpyAsync(r->d_load, slot, (size_t)r->P * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
-  if (mask) {
-    uint8_t* ms = r->h_mask + (size_t)s * r->P;
-    std::memcpy(ms, mask, (size_t)r->P);
-    CK(cudaMemcpyAsync(r->d_mask, ms, (size_t)r->P, cudaMemcpyHostToDevice, r->stream));
-  }
   CK(cudaEventRecord(r->load_ev[s], r->stream));
   return P2P_OK;
 }
@@ -817,11 +812,9 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_states, (size_t)P * sizeof(TreeState));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_rfilter, (size_t)P * p2p::kRootFilterWords * sizeof(uint32_t));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_load, (size_t)P * sizeof(int32_t));
-  if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_mask, (size_t)P);
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_err, sizeof(int32_t));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_hdr, p2p::kStaticHeaderInts * sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_load, (size_t)kLoadRing * P * sizeof(int32_t));
-  if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_mask, (size_t)kLoadRing * P);
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_err, sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_states, (size_t)P * sizeof(TreeState));
   for (int i = 0; i < kLoadRing && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&r->load_ev[i], cudaEventDisableTiming);
@@ -867,7 +860,6 @@ void p2p_router_destroy(p2p_router* r) {
     dfree(r, r->d_states);
     dfree(r, r->d_rfilter);
     dfree(r, r->d_load);
-    dfree(r, r->d_mask);
     dfree(r, r->d_err);
     dfree(r, r->d_hdr);
     dfree(r, r->d_shared);
@@ -888,7 +880,6 @@ void p2p_router_destroy(p2p_router* r) {
     if (r->ev_routed[i]) cudaEventDestroy(r->ev_routed[i]);
   }
   if (r->h_load) cudaFreeHost(r->h_load);
-  if (r->h_mask) cudaFreeHost(r->h_mask);
   if (r->h_err) cudaFreeHost(r->h_err);
   if (r->h_states) cudaFreeHost(r->h_states);
   delete r->clock;
@@ -1305,8 +1296,7 @@ int p2p_route_batch_decide(p2p_router* r, const int32_t* tokens, int64_t n_token
   if (!offsets || !out_match || !out_peer || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
   DeviceGuard g(r);
   if (int rc = stage_load(r, load, excluded)) return rc;
-  return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer, excluded ? r->d_mask : nullptr,
-               out_next);
+  return route(r, tokens, n_tokens, 0, offsets, B, alpha, out_match, out_peer, excluded != nullptr, out_next);
 }
 
 int p2p_route_decide(p2p_router* r, const int32_t* match, int64_t B, const int32_t* load, int32_t alpha,
@@ -1318,7 +1308,7 @@ int p2p_route_decide(p2p_router* r, const int32_t* match, int64_t B, const int32
   if (!match || !out_peer || !out_next) return fail(r, P2P_E_INVAL, "NULL device pointer");
   DeviceGuard g(r);
   if (int rc = stage_load(r, load, excluded)) return rc;
-  CK(p2p::launch_decide(match, B, r->P, r->d_load, alpha, excluded ? r->d_mask : nullptr, out_peer, out_next,
+  CK(p2p::launch_decide(match, B, r->P, r->d_load, alpha, out_peer, out_next,
                         r->num_sms, r->stream));
   r->launches += 1;
   return P2P_OK;
