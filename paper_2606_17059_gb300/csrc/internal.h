@@ -108,7 +108,7 @@ enum KernelId {
   K_VALIDATE, K_INIT_RANGES, K_DELTA, K_COMPACT, K_COMPACT_LABELS, K_REFRESH_VIEWS, K_SET_TREE,
   K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_GROUP_RANGES, K_GROUP_PLACE, K_COUNT_
 };
-static_assert(K_COUNT_ == P2P_KERNEL_COUNT, "the header's kernel count");
+static_assert((int)K_COUNT_ == (int)P2P_KERNEL_COUNT, "the header's kernel count");
 const char* kernel_name(int id);
 struct KernelClock {
   virtual void mark(int id, bool end, cudaStream_t st) = 0;

@@ -126,12 +126,12 @@ def test_followers_with_tree_counts_off_the_lane_groups(P):
 
 
 def test_route_launch_count():
-    """A grouped batch of short requests is routed by two grouping kernels, a leader pass and a follower
-    pass."""
+    """A grouped batch of short requests is routed by four grouping kernels (hash, resolve, follower ranges,
+    follower placement), a leader pass and a follower pass."""
     rng = random.Random(3)
     trees = [[[rng.randrange(10) for _ in range(100)] for _ in range(5)]]
     r = router_from_seqlists([seqlist_from_lists(t) for t in trees])
     tok, off = csr_from_lists([trees[0][0], trees[0][0][:80], [1, 2, 3]])
     n0 = r.launch_count()
     route_device(r, tok, off, [0], 0)
-    assert r.launch_count() - n0 == 4
+    assert r.launch_count() - n0 == 6
