@@ -549,9 +549,10 @@ int download(p2p_router* r, int32_t peer, p2p_snapshot* out) {
   return P2P_OK;
 }
 
-// Rebuilds tree p's root table (node 0's children) in fresh slots of the child arena, doubled and without
-// tombstones.  Only the host does this: during a delta every warp of the tree shares the root table.
-int regrow_root(p2p_router* r, int32_t p) {
+// Rebuilds tree p's root table (node 0's children) in fresh slots of the child arena, doubled (or, with
+// extra > 0, sized for `extra` more children) and without tombstones.  Only the host does this: during a delta
+// every warp of the tree shares the root table.
+int regrow_root(p2p_router* r, int32_t p, int64_t extra = 0) {
   TreeState& t = r->hs[(size_t)p];
   int4 root;
   CK(d2h(r, &root, t.node, sizeof(int4)));
@@ -561,7 +562,7 @@ int regrow_root(p2p_router* r, int32_t p) {
   std::vector<int4> kids;
   for (const int4& s : tab)
     if (s.y >= 1) kids.push_back(s);
-  const int32_t nb = std::max(bits + 1, table_bits_for((int64_t)kids.size(), true));
+  const int32_t nb = std::max(bits + 1, table_bits_for((int64_t)kids.size() + extra, true));
   if (nb > p2p::kMaxTabBits) return fail(r, P2P_E_NOMEM, "root table too large");
   const int64_t n_slots = (int64_t)1 << nb;
   if ((int64_t)t.cap_child - t.n_child < n_slots) {
@@ -640,6 +641,35 @@ int grow_tree(p2p_router* r, int32_t p) {
   t.status = p2p::DELTA_OK;
   t.need_node = t.need_child = t.need_label = t.need_root = 0;
   return P2P_OK;
+}
+
+// Before a delta of many INSERTs: a tree whose root table would pass 1/2 claimed with `ins[p - p0]` more
+// children gets a root table sized for them now (growing its child arena first if needed), so the delta kernel
+// does not stop and relaunch once per doubling.  Reads the roots of those trees (one copy each, one wait).
+int presize_roots(p2p_router* r, int32_t p0, int32_t p1, const int64_t* ins) {
+  std::vector<int32_t> ps;
+  for (int32_t p = p0; p < p1; ++p)
+    if (ins[p - p0] >= 1024) ps.push_back(p);
+  if (ps.empty()) return P2P_OK;
+  std::vector<int4> roots(ps.size());
+  for (size_t i = 0; i < ps.size(); ++i)
+    CK(cudaMemcpyAsync(&roots[i], r->hs[(size_t)ps[i]].node, sizeof(int4), cudaMemcpyDeviceToHost, r->stream));
+  CK(cudaStreamSynchronize(r->stream));
+  for (size_t i = 0; i < ps.size(); ++i) {
+    const int32_t p = ps[i];
+    const int64_t extra = ins[p - p0];
+    if (!p2p::tab_full(p2p::tab_bits(roots[i].y), (int64_t)p2p::tab_used(roots[i].y) + extra)) continue;
+    int rc = regrow_root(r, p, extra);
+    if (rc == 1) {  // the child arena has no room for the new table: grow it first
+      TreeState& t = r->hs[(size_t)p];
+      t.need_node = t.need_label = 0;
+      t.need_root = 0;
+      rc = grow_tree(r, p);
+      if (rc == P2P_OK) rc = regrow_root(r, p, extra);
+    }
+    if (rc != P2P_OK) return rc == 1 ? fail(r, P2P_E_NOMEM, "no room for a root table") : rc;
+  }
+  return push_states(r, p0, p1);
 }
 
 // Rebuilds a tree whose arenas are mostly stale entries: canonical export, then a fresh upload.
@@ -1238,13 +1268,20 @@ int p2p_update_estimates(p2p_router* r, const int32_t* tokens, int64_t n_tokens,
     int32_t bad[2];
     int64_t total;
   } h = {};
+  std::vector<int64_t> pb((size_t)P + 1);
   CK(cudaMemcpyAsync(h.bad, bad, sizeof(h.bad), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaMemcpyAsync(&h.total, total, sizeof(h.total), cudaMemcpyDeviceToHost, r->stream));
+  CK(cudaMemcpyAsync(pb.data(), peer_begin, pb.size() * sizeof(int64_t), cudaMemcpyDeviceToHost, r->stream));
   CK(cudaStreamSynchronize(r->stream));
   if (h.bad[0] & 1) return fail(r, P2P_E_INVAL, "a peer index is >= P");
   if (h.bad[0] & 2) return fail(r, P2P_E_INVAL, "a routed request has offsets outside [0, n_tokens] or decreasing");
   const int64_t n = h.total;
   if (n == 0) return P2P_OK;
+  // Every op is an INSERT: a tree that takes many (the fresh prompts of a batch all go to its least-loaded
+  // tree) gets its root table sized for them before the delta kernel runs.
+  std::vector<int64_t> ins((size_t)P);
+  for (int32_t p = 0; p < P; ++p) ins[(size_t)p] = pb[(size_t)p + 1] - pb[(size_t)p];
+  if (int rc = presize_roots(r, 0, P, ins.data())) return rc;
   CK(ensure(r, r->upd_op, (size_t)n * sizeof(int32_t)));
   CK(ensure(r, r->upd_so, (size_t)n * sizeof(int64_t)));
   CK(ensure(r, r->upd_sl, (size_t)n * sizeof(int32_t)));
