@@ -271,7 +271,7 @@ def test_root_first_tokens_added_and_removed_by_deltas():
     gm, gp = route_device(r, tok, off, [0], 0)
     om, op, _ = oracle.route([otree], tok, off, [0], 0)
     assert_same_route(gm, gp, om, op, "root filter after a delta")
-    assert (gm[: len(new), 0] == 15).all()
+    assert (gm[: len(new), 0] == 13).all()  # each new sequence is 13 tokens long
     del torch
 
 
