@@ -311,6 +311,43 @@ struct RouteAcc<true> {
   }
 };
 
+// The lane walks' accumulator.  The plain argmax keeps its key in a register; the decision with excluded
+// trees keeps a lane's two keys in shared memory, so the walk loops (at their register limit) do not lose
+// loads in flight to it.  finish() merges over the warp and lane 0 writes the decision.
+template <bool kDecide>
+struct LaneAcc : RouteAcc<false> {
+  __device__ explicit LaneAcc(unsigned long long*) {}
+  __device__ __forceinline__ void finish(int lane, int64_t b, int32_t* out_peer, int32_t* out_next) {
+    warp_merge();
+    if (lane == 0) write(b, out_peer, out_next);
+  }
+};
+template <>
+struct LaneAcc<true> {
+  unsigned long long* s;  // s[0] and s[32]: this lane's largest and second-largest key
+  __device__ explicit LaneAcc(unsigned long long* p) : s(p) {
+    s[0] = 0;
+    s[32] = 0;
+  }
+  __device__ __forceinline__ void add(int32_t m, int32_t ldw, int32_t p, int32_t alpha) {
+    if (ldw & kExcluded) return;
+    const unsigned long long key = route_key(m, ldw, p, alpha), k1 = s[0];
+    if (key > k1) {
+      s[32] = k1;
+      s[0] = key;
+    } else if (key > s[32]) {
+      s[32] = key;
+    }
+  }
+  __device__ __forceinline__ void finish(int lane, int64_t b, int32_t* out_peer, int32_t* out_next) {
+    RouteAcc<true> r;
+    r.k1 = s[0];
+    r.k2 = s[32];
+    r.warp_merge();
+    if (lane == 0) r.write(b, out_peer, out_next);
+  }
+};
+
 // Routes the leaders list[0 .. *count) of a grouped batch with full walks.  kDecide: the decision with
 // excluded trees and the next-best target (RouteAcc<true>), made by the request's last warp from its match
 // row once every item of the request has written its part.
@@ -673,6 +710,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const int32_t* __restrict__ gid, const int32_t* __restrict__ cmin, int4* __restrict__ ckpt,
     const int32_t* __restrict__ load, int32_t alpha, int32_t* __restrict__ out_match, int32_t* __restrict__ out_peer,
     int32_t* err, int32_t* cursor, int32_t* __restrict__ out_next) {
+  __shared__ unsigned long long s_top[kDecide ? kFollowThreads / 32 : 1][kDecide ? 64 : 1];
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kFollowThreads / 32);
   const int64_t n = *count;
@@ -701,7 +739,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     }
     const int32_t* req = tokens + start;
     const int32_t len = (int32_t)min(end - start, (int64_t)INT32_MAX);
-    RouteAcc<kDecide> acc;
+    LaneAcc<kDecide> acc(kDecide ? &s_top[threadIdx.x >> 5][lane] : nullptr);
     if constexpr (kLeader) {
       const int32_t row = __ldg(gid + f);
       const int32_t climit = row >= 0 ? __ldg(cmin + f) : -1;
@@ -785,8 +823,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
         }
       }
     }
-    acc.warp_merge();
-    if (lane == 0) acc.write(f, out_peer, out_next);
+    acc.finish(lane, f, out_peer, out_next);
   }
 }
 

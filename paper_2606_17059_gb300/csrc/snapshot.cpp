@@ -277,33 +277,48 @@ bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* c
       if (k[i - 1].x == k[i].x) return false;
     return (int64_t)k.size() == nd.z;
   };
-  // Preorder DFS; each stacked item carries the slot through which the node was reached.
-  std::vector<int64_t> order;
-  std::vector<int4> via;
+  // Preorder DFS; each stacked item carries the slot through which the node was reached.  A non-root node
+  // with one child and no sequence (an LRU tree keeps such nodes where an access ended inside an edge) is
+  // merged with its child, so the export is canonical whatever the device layout: an exported node carries
+  // the chain of slots whose labels it concatenates, and `order` holds the chain's last node.
+  std::vector<int64_t> order, first;  // an exported node's last and first device node
+  std::vector<std::vector<int4>> via;
   std::vector<std::vector<int4>> children;
   std::vector<std::pair<int64_t, int4>> st{{0, make_int4(0, 0, 0, 0)}};
   std::vector<int4> k;
-  int64_t total_label = 0;
+  int64_t total_label = 0, visited = 0;
+  auto check_label = [&](const int4& e) {
+    const bool own = e.z >= 0;
+    const int64_t start = own ? e.z : ~(int64_t)e.z;
+    return e.w >= 1 && start + e.w <= (own ? n_label : n_shared);
+  };
   while (!st.empty()) {
     auto [v, e] = st.back();
     st.pop_back();
-    if (v < 0 || v >= n_node || (int64_t)order.size() >= n_node) return err = "corrupt device tree (node index)", false;
-    if (v != 0) {
-      const bool own = e.z >= 0;
-      const int64_t start = own ? e.z : ~(int64_t)e.z;
-      if (e.w < 1 || start + e.w > (own ? n_label : n_shared)) return err = "corrupt device tree (label)", false;
-      total_label += e.w;
+    const int64_t v0 = v;
+    std::vector<int4> chain;
+    for (;;) {
+      if (v < 0 || v >= n_node || ++visited > n_node) return err = "corrupt device tree (node index)", false;
+      if (v != 0) {
+        if (!check_label(e)) return err = "corrupt device tree (label)", false;
+        total_label += e.w;
+        chain.push_back(e);
+      }
+      if (!kids(v, k)) return err = "corrupt device tree (children table)", false;
+      if (v == 0 || k.size() != 1 || node[v].w != 0) break;
+      e = k[0];
+      v = e.y;
     }
-    if (!kids(v, k)) return err = "corrupt device tree (children table)", false;
     order.push_back(v);
-    via.push_back(e);
+    first.push_back(v0);
+    via.push_back(chain);
     children.push_back(k);
     for (auto it = k.rbegin(); it != k.rend(); ++it) st.push_back({it->y, *it});
   }
   if (total_label > INT32_MAX) return err = "tree has more than 2^31-1 label tokens", false;
   const size_t N = order.size();
   std::vector<int32_t> id((size_t)n_node, -1);
-  for (size_t j = 0; j < N; ++j) id[(size_t)order[j]] = (int32_t)j;
+  for (size_t j = 0; j < N; ++j) id[(size_t)first[j]] = (int32_t)j;  // child entries name a chain's first node
   out.n_nodes = (int32_t)N;
   out.n_labels = (int32_t)total_label;
   out.label_off.assign(N, 0);
@@ -319,10 +334,13 @@ bool snapshot_from_device_layout(const int4* node, int64_t n_node, const int4* c
     const int64_t v = order[j];
     out.label_off[j] = (int32_t)lab;
     if (v != 0) {
-      const int4 ce = via[j];
-      std::memcpy(out.labels.data() + lab, label_ptr(label, shared, ce.z), (size_t)ce.w * sizeof(int32_t));
-      out.label_len[j] = ce.w;
-      lab += ce.w;
+      int32_t len = 0;
+      for (const int4& ce : via[j]) {
+        std::memcpy(out.labels.data() + lab, label_ptr(label, shared, ce.z), (size_t)ce.w * sizeof(int32_t));
+        lab += ce.w;
+        len += ce.w;
+      }
+      out.label_len[j] = len;
     }
     const std::vector<int4>& kk = children[j];
     out.child_begin[j] = (int32_t)ch;
