@@ -46,7 +46,7 @@ enum {
 };
 
 enum { P2P_OP_INSERT = 0, P2P_OP_DELETE = 1 };
-enum { P2P_KERNEL_COUNT = 19 }; /* kernels the kernel clock keeps totals for */
+enum { P2P_KERNEL_COUNT = 26 }; /* kernels the kernel clock keeps totals for */
 enum { P2P_MEM_HOST = 0, P2P_MEM_DEVICE = 1 };
 
 typedef struct p2p_router p2p_router;
@@ -228,6 +228,51 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
  * nothing changes), P2P_E_NOMEM, P2P_E_CUDA, P2P_E_DEVICE. */
 int p2p_update_estimates(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
                          const int32_t* peer, int64_t* n_inserted);
+
+/* ---- LRU cache trie (EvictLRUTrie of Algorithm 1) --------------------------------------------------------
+ *
+ * A node's own trie is its KV cache: Algorithm 1 inserts what the node serves (UpdateTrie) and, while a
+ * request needs more memory than is free, evicts the least recently used leaf token, one token at a time
+ * (Section 2 primitive list: evictLRUTrie).  A tree made an LRU tree keeps a last-access time per token
+ * (stored per node: an access that ends inside an edge splits the edge there, so every edge's tokens share
+ * one time).  Times are caller-given integers that never decrease, at most 2^32 - 2.  Semantics, per token:
+ *   - an insert at time t touches every token of the sequence's path; an access at time t touches the
+ *     request's matched tokens;
+ *   - an eviction removes the leaf token with the oldest last access, ties to the lexicographically smallest
+ *     token path (signed token order); sequences that ended at it now end one token earlier.
+ * An LRU tree changes only through these calls: uploads, deltas and p2p_update_estimates that would change it
+ * are rejected (P2P_E_INVAL).  It is routed like any tree, and its export is canonical.  It is not compacted
+ * (evicted nodes stay in its arenas as stale space).
+ */
+
+/* Makes tree `tree` an LRU tree; its current tokens get time 0.  A no-op if it is one already. */
+int p2p_lru_enable(p2p_router* r, int32_t tree);
+
+/* UpdateTrie of a batch at time `time`: each request (DEVICE tokens/offsets as for p2p_route_batch) is
+ * inserted once, then every token of its path is touched.  Waits for the work.  Errors: P2P_E_INVAL (not an
+ * LRU tree, time out of order, invalid offsets: nothing changes), P2P_E_NOMEM, P2P_E_CUDA. */
+int p2p_lru_insert(p2p_router* r, int32_t tree, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets,
+                   int64_t B, int64_t time);
+
+/* Requests served from the cache at time `time`: each request's matched tokens are touched, and
+ * out_match (DEVICE int32[B], nullable) receives PrefixMatch(r_b, tree).  Waits for the work.  Requests with
+ * invalid offsets match 0, touch nothing and make the next p2p_router_sync return P2P_E_DEVICE.  Errors:
+ * P2P_E_INVAL, P2P_E_NOMEM (no room to split edges), P2P_E_CUDA. */
+int p2p_lru_access(p2p_router* r, int32_t tree, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets,
+                   int64_t B, int64_t time, int32_t* out_match);
+
+/* EvictLRUTrie n_tokens times: removes the n_tokens least recently used leaf tokens in the order above (all
+ * of them if the tree holds fewer); *n_evicted (nullable) receives how many.  The removal is done at once on
+ * the device (the order is that of one-token evictions; see lru_kernel.cu).  Waits for the work.  Errors:
+ * P2P_E_INVAL, P2P_E_CUDA, P2P_E_DEVICE. */
+int p2p_lru_evict(p2p_router* r, int32_t tree, int64_t n_tokens, int64_t* n_evicted);
+
+/* Section 5's expected cache hit rate of routed requests: out[b] = match[b*P + peer[b]] / |r_b| in single
+ * precision (IEEE division, rounded to nearest), 0 for an empty request or peer[b] < 0.  match (DEVICE
+ * int32[B*P]), offsets (DEVICE int64[B+1]), peer (DEVICE int32[B]) as p2p_route_batch writes and reads them;
+ * out DEVICE float[B].  Asynchronous on the router stream.  Errors: P2P_E_INVAL. */
+int p2p_hit_rate(p2p_router* r, const int32_t* match, const int64_t* offsets, int64_t B, const int32_t* peer,
+                 float* out);
 
 /* Sizes of tree `peer`: out[0] live nodes (root included), out[1] node slots in use, out[2] child
  * entries in use, out[3] label tokens in use, out[4] stale child entries, out[5] stale label tokens,

@@ -22,6 +22,7 @@ __all__ = [
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
     "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host", "p2p_route_decide",
     "p2p_router_kernel_clock", "p2p_router_kernel_time", "p2p_update_estimates", "p2p_route_batch_decide",
+    "p2p_lru_enable", "p2p_lru_insert", "p2p_lru_access", "p2p_lru_evict", "p2p_hit_rate",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -97,6 +98,11 @@ def _load():
             "p2p_router_kernel_clock": (ctypes.c_int, [_vp, _i32]),
             "p2p_update_estimates": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, P(_i64)]),
             "p2p_route_batch_decide": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64, _vp, _i32, _vp, _vp, _vp, _vp]),
+            "p2p_lru_enable": (ctypes.c_int, [_vp, _i32]),
+            "p2p_lru_insert": (ctypes.c_int, [_vp, _i32, _vp, _i64, _vp, _i64, _i64]),
+            "p2p_lru_access": (ctypes.c_int, [_vp, _i32, _vp, _i64, _vp, _i64, _i64, _vp]),
+            "p2p_lru_evict": (ctypes.c_int, [_vp, _i32, _i64, P(_i64)]),
+            "p2p_hit_rate": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _vp]),
             "p2p_router_kernel_time": (ctypes.c_int, [_vp, _i32, P(ctypes.c_char_p), P(_i64), P(ctypes.c_double)]),
         }
         for name, (res, args) in sig.items():
@@ -197,7 +203,7 @@ def p2p_router_launch_count(r) -> int:
     return int(_load().p2p_router_launch_count(r))
 
 
-KERNEL_COUNT = 19  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 18)
+KERNEL_COUNT = 26  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 25)
 
 
 def p2p_router_kernel_clock(r, on: bool) -> None:
@@ -312,6 +318,32 @@ def p2p_update_estimates(r, tokens, n_tokens: int, offsets, B: int, peer) -> int
     n = _i64()
     _check(_load().p2p_update_estimates(r, _addr(tokens), n_tokens, _addr(offsets), B, _addr(peer), ctypes.byref(n)), r)
     return int(n.value)
+
+
+def p2p_lru_enable(r, tree: int) -> None:
+    _check(_load().p2p_lru_enable(r, tree), r)
+
+
+def p2p_lru_insert(r, tree: int, tokens, n_tokens: int, offsets, B: int, time: int) -> None:
+    """UpdateTrie of a batch at `time` (CUDA tensors tokens/offsets)."""
+    _check(_load().p2p_lru_insert(r, tree, _addr(tokens), n_tokens, _addr(offsets), B, time), r)
+
+
+def p2p_lru_access(r, tree: int, tokens, n_tokens: int, offsets, B: int, time: int, out_match=None) -> None:
+    """Requests served at `time`: their matched tokens are touched; out_match (CUDA int32 [B] or None)."""
+    _check(_load().p2p_lru_access(r, tree, _addr(tokens), n_tokens, _addr(offsets), B, time, _addr(out_match)), r)
+
+
+def p2p_lru_evict(r, tree: int, n_tokens: int) -> int:
+    """Evicts the n_tokens least recently used leaf tokens; returns how many were evicted."""
+    n = _i64()
+    _check(_load().p2p_lru_evict(r, tree, n_tokens, ctypes.byref(n)), r)
+    return int(n.value)
+
+
+def p2p_hit_rate(r, match, offsets, B: int, peer, out) -> None:
+    """Expected hit rate match[b, peer[b]] / len(b) of routed requests (CUDA tensors; out float32 [B])."""
+    _check(_load().p2p_hit_rate(r, _addr(match), _addr(offsets), B, _addr(peer), _addr(out)), r)
 
 
 STAT_NAMES = ("live_nodes", "node_slots", "child_entries", "label_tokens", "stale_child", "stale_label",

@@ -18,8 +18,8 @@ BUILD_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libp2prouter.so")
 NVCC = os.environ.get("NVCC", "/usr/local/cuda/bin/nvcc" if os.path.exists("/usr/local/cuda/bin/nvcc") else "nvcc")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["route_kernel.cu", "group_kernel.cu", "delta_kernel.cu", "delta_static.cu", "update_kernel.cu", "router.cu",
-           "snapshot.cpp"]
+SOURCES = ["route_kernel.cu", "group_kernel.cu", "delta_kernel.cu", "delta_static.cu", "update_kernel.cu",
+           "lru_kernel.cu", "router.cu", "snapshot.cpp"]
 
 
 def _flags(extra=()):

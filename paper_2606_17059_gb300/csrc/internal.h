@@ -69,6 +69,7 @@ struct TreeState {
   int4* child;
   int32_t* label;
   uint32_t* rfilter;           // the root's first-token filter (kRootFilterWords words; the router's array)
+  uint32_t* stamp;             // LRU trees only (else NULL): per node slot, the last access of its edge's tokens
   int32_t n_node, cap_node;    // node slots used (bump arena) / capacity
   int32_t n_child, cap_child;  // child-table slots used (bump arena) / capacity
   int32_t n_label, cap_label;  // label tokens used (bump arena) / capacity
@@ -106,7 +107,8 @@ constexpr int32_t kMaxTabBits = 26;  // slots ever claimed must fit the 27 bits 
 enum KernelId {
   K_GROUP_HASH, K_GROUP_RESOLVE, K_GROUP_RESOLVE32, K_ROUTE_STAGED, K_LANE_LEADER, K_LANE_FOLLOWER, K_DECIDE,
   K_VALIDATE, K_INIT_RANGES, K_DELTA, K_COMPACT, K_COMPACT_LABELS, K_REFRESH_VIEWS, K_SET_TREE,
-  K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_GROUP_RANGES, K_GROUP_PLACE, K_COUNT_
+  K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_GROUP_RANGES, K_GROUP_PLACE, K_LRU_WALK, K_LRU_STAMP,
+  K_LRU_ORDER, K_LRU_SELECT, K_LRU_EVICT, K_LRU_OPS, K_HIT_RATE, K_COUNT_
 };
 static_assert((int)K_COUNT_ == (int)P2P_KERNEL_COUNT, "the header's kernel count");
 const char* kernel_name(int id);
@@ -233,6 +235,32 @@ cudaError_t launch_update_scan(const int32_t* counts, int32_t P, int64_t* peer_b
 cudaError_t launch_update_scatter(const int32_t* peer, const int64_t* offsets, int64_t B, int64_t n_tokens, int32_t P,
                                   int32_t* cursor, int32_t* op, int64_t* seg_begin, int64_t* seg_off, int32_t* seg_len,
                                   int num_sms, cudaStream_t st);
+
+// LRU trees (lru_kernel.cu): walk + stamp (an access), BFS order, the level passes, the selection counts and
+// the eviction; see that file for the method.  lvl_begin (host) holds n_levels + 1 offsets into order.
+cudaError_t launch_lru_walk(const TreeState& s, const int32_t* shared, const int32_t* tokens, int64_t n_tokens,
+                            const int64_t* offsets, int64_t B, int32_t* touch, int32_t* pslot, int32_t* out_match,
+                            int32_t* err, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_stamp(const TreeState& s, TreeState* d_state, const int32_t* shared, const int32_t* touch,
+                             const int32_t* pslot, int32_t n_node, uint32_t time, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_bfs(const TreeState& s, const int32_t* front, int32_t n_front, int32_t* next, int32_t* n_next,
+                           int32_t* parent, int32_t* cslot, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_init(const int32_t* order, int32_t n, int64_t* size, int64_t* off, int64_t* rank,
+                            unsigned long long* best, uint8_t* gone, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_levels(const TreeState& s, const int32_t* order, const int32_t* lvl_begin, int32_t n_levels,
+                              const int32_t* parent, const int32_t* cslot, int64_t* size, int64_t* off, int64_t* rank,
+                              unsigned long long* best, int32_t* end, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_count(const TreeState& s, const int32_t* nodes, int32_t n, const int32_t* cslot,
+                             const int64_t* rank, const int32_t* end, int mode, uint32_t S, unsigned long long K,
+                             unsigned long long* out, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_evict(const TreeState& s, TreeState* d_state, const int32_t* order, const int32_t* lvl_begin,
+                             int32_t n_levels, const int32_t* parent, const int32_t* cslot, const int64_t* rank,
+                             const int32_t* end, uint32_t S, unsigned long long K, int32_t cut, uint8_t* gone,
+                             int32_t* surv, int num_sms, cudaStream_t st);
+cudaError_t launch_lru_ops(const int64_t* offsets, int64_t B, int64_t n_tokens, int32_t* op, int64_t* seg_begin,
+                           int64_t* seg_off, int32_t* seg_len, int num_sms, cudaStream_t st);
+cudaError_t launch_hit_rate(const int32_t* match, int32_t P, const int64_t* offsets, int64_t B, const int32_t* peer,
+                            float* out, int num_sms, cudaStream_t st);
 
 // Host-side helpers in snapshot.cpp.
 void set_global_error(const std::string& msg);

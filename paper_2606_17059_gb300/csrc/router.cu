@@ -88,7 +88,9 @@ const char* kernel_name(int id) {
       "group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel", "route_kernel", "lane_kernel<true>",
       "lane_kernel<false>", "decide_kernel", "validate_kernel", "init_ranges_kernel", "delta_kernel",
       "compact_kernel", "compact_labels_kernel", "refresh_views_kernel", "set_tree_kernel", "update_count_kernel",
-      "update_scan_kernel", "update_scatter_kernel", "group_ranges_kernel", "group_place_kernel"};
+      "update_scan_kernel", "update_scatter_kernel", "group_ranges_kernel", "group_place_kernel", "lru_walk_kernel",
+      "lru_stamp_kernel", "lru_order_kernels", "lru_count_kernel", "lru_evict_kernel", "lru_ops_kernel",
+      "hit_rate_kernel"};
   return id >= 0 && id < K_COUNT_ ? names[id] : "";
 }
 
@@ -198,6 +200,9 @@ struct p2p_router {
   DevBuf grp_keys, grp_vals, grp_req, grp_ckpt;  // shared-prefix grouping of a batch
   DevBuf cmp_jobs, cmp_queue;          // device compaction
   DevBuf upd_cnt, upd_op, upd_sb, upd_so, upd_sl;  // a routed batch as an INSERT delta (p2p_update_estimates)
+  DevBuf lru_buf;                                   // scratch of the LRU calls
+  std::vector<uint8_t> lru;                         // per tree: kept as an LRU cache (p2p_lru_enable)
+  std::vector<int64_t> lru_time;                    // per LRU tree: the time of its last insert or access
   int64_t launches = 0;  // kernels this router has launched
   RouterClock* clock = nullptr;  // per-kernel device time, while switched on
   // Shared label pool: long labels interned across trees (device array, host mirror, content index).
@@ -321,9 +326,11 @@ void free_tree_arrays(p2p_router* r, TreeState& t) {
   dfree(r, t.node);
   dfree(r, t.child);
   dfree(r, t.label);
+  dfree(r, t.stamp);
   t.node = nullptr;
   t.child = nullptr;
   t.label = nullptr;
+  t.stamp = nullptr;
 }
 
 // Allocates the arrays of a tree with the given capacities; on failure frees what it got.
@@ -614,6 +621,14 @@ int grow_tree(p2p_router* r, int32_t p) {
   if (grow_n) {
     CK(cudaMemcpyAsync(nn, t.node, (size_t)t.n_node * sizeof(int4), cudaMemcpyDeviceToDevice, r->stream));
     dfree(r, t.node);
+    if (t.stamp) {  // an LRU tree's stamps follow its node slots; new slots start at time 0
+      uint32_t* ns = nullptr;
+      CK(dalloc(r, (void**)&ns, (size_t)cn * sizeof(uint32_t)));
+      CK(cudaMemcpyAsync(ns, t.stamp, (size_t)t.n_node * sizeof(uint32_t), cudaMemcpyDeviceToDevice, r->stream));
+      CK(cudaMemsetAsync(ns + t.n_node, 0, (size_t)(cn - t.n_node) * sizeof(uint32_t), r->stream));
+      dfree(r, t.stamp);
+      t.stamp = ns;
+    }
   }
   if (grow_c) {
     CK(cudaMemcpyAsync(nc, t.child, (size_t)t.n_child * sizeof(int4), cudaMemcpyDeviceToDevice, r->stream));
@@ -770,6 +785,7 @@ int compact_trees(p2p_router* r, const std::vector<int32_t>& ps, int32_t p0, int
 }
 
 bool needs_compaction(const TreeState& t) {
+  if (t.stamp) return false;  // LRU trees are not compacted (their stamps are indexed by node slot)
   return (t.stale_label > 65536 && 2 * t.stale_label > t.n_label) ||
          (t.stale_child > 65536 && 2 * t.stale_child > t.n_child) ||
          (t.dead_nodes > 16384 && 2 * t.dead_nodes > t.n_node);
@@ -779,6 +795,7 @@ bool needs_compaction(const TreeState& t) {
 // along in the same launch: replicas that receive deltas at the same rate reach the threshold within a few
 // calls of one another, and one compaction wave costs about as much as one of a handful of trees.
 bool nears_compaction(const TreeState& t) {
+  if (t.stamp) return false;
   return (t.stale_label > 45875 && 20 * t.stale_label > 7 * (int64_t)t.n_label) ||
          (t.stale_child > 45875 && 20 * t.stale_child > 7 * (int64_t)t.n_child) ||
          (t.dead_nodes > 11468 && 20 * t.dead_nodes > 7 * (int64_t)t.n_node);
@@ -799,6 +816,30 @@ int pull_states(p2p_router* r, int32_t p0, int32_t p1) {
                      r->stream));
   CK(cudaStreamSynchronize(r->stream));
   std::memcpy(r->hs.data() + p0, r->h_states, (size_t)(p1 - p0) * sizeof(TreeState));
+  return P2P_OK;
+}
+
+// A delta may not give ops to an LRU tree (its stamps change only through the p2p_lru_* calls).  With
+// peer = -1, the ranges of the LRU trees are read from peer_begin (host, or two words copied back each).
+int reject_lru_ops(p2p_router* r, int32_t peer, const p2p_delta* d) {
+  const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
+  for (int32_t p = p0; p < p1; ++p) {
+    if (!r->lru[(size_t)p]) continue;
+    int64_t n = d->seqs.n;
+    if (peer == -1) {
+      int64_t pb[2] = {0, 0};
+      if (d->mem == P2P_MEM_HOST) {
+        pb[0] = d->peer_begin[p];
+        pb[1] = d->peer_begin[p + 1];
+      } else {
+        CK(cudaMemcpyAsync(pb, d->peer_begin + p, sizeof(pb), cudaMemcpyDeviceToHost, r->stream));
+        CK(cudaStreamSynchronize(r->stream));
+      }
+      n = pb[1] - pb[0];
+    }
+    if (n != 0)
+      return fail(r, P2P_E_INVAL, "tree " + std::to_string(p) + " is an LRU tree: it changes only through the p2p_lru_* calls");
+  }
   return P2P_OK;
 }
 
@@ -838,6 +879,8 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   }
   r->hs.assign((size_t)P, TreeState{});
   r->spare.assign((size_t)P, TreeState{});
+  r->lru.assign((size_t)P, 0);
+  r->lru_time.assign((size_t)P, 0);
   e = dalloc(r, (void**)&r->d_views, (size_t)P * sizeof(TreeView));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_states, (size_t)P * sizeof(TreeState));
   if (e == cudaSuccess) e = dalloc(r, (void**)&r->d_rfilter, (size_t)P * p2p::kRootFilterWords * sizeof(uint32_t));
@@ -884,7 +927,7 @@ void p2p_router_destroy(p2p_router* r) {
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
                       &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue,
-                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl})
+                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl, &r->lru_buf})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -972,12 +1015,14 @@ int p2p_router_kernel_time(p2p_router* r, int32_t i, const char** name, int64_t*
 
 int p2p_tree_upload(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   if (int rc = check_peer(r, peer)) return rc;
+  if (r->lru[(size_t)peer]) return fail(r, P2P_E_INVAL, "an LRU tree changes only through the p2p_lru_* calls");
   DeviceGuard g(r);
   return upload_flat(r, peer, t);
 }
 
 int p2p_tree_build(p2p_router* r, int32_t peer, const p2p_seqs* seqs) {
   if (int rc = check_peer(r, peer)) return rc;
+  if (r->lru[(size_t)peer]) return fail(r, P2P_E_INVAL, "an LRU tree changes only through the p2p_lru_* calls");
   std::string err;
   if (!seqs || !p2p::check_seqs(seqs, err, nullptr, nullptr)) return fail(r, P2P_E_INVAL, seqs ? err : "seqs is NULL");
   p2p_snapshot snap;
@@ -1015,7 +1060,13 @@ int p2p_tree_stats(p2p_router* r, int32_t peer, int64_t out[9]) {
   return P2P_OK;
 }
 
+static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent, bool lru_ok);
+
 int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent) {
+  return apply_delta_impl(r, peer, d, n_absent, false);
+}
+
+static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent, bool lru_ok) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
   if (peer < -1 || peer >= r->P) return fail(r, P2P_E_INVAL, "peer out of range");
   if (!d) return fail(r, P2P_E_INVAL, "delta is NULL");
@@ -1033,6 +1084,8 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   }
   const int32_t p0 = peer == -1 ? 0 : peer, p1 = peer == -1 ? r->P : peer + 1;
   const int32_t nt = p1 - p0;
+  if (!lru_ok)
+    if (int rc = reject_lru_ops(r, peer, d)) return rc;
   int64_t max_len = 0, max_runs = 0;
   const int32_t* d_op = d->op;
   const int64_t *d_sb = S.seg_begin, *d_so = S.seg_off, *d_pb = d->peer_begin;
@@ -1181,6 +1234,8 @@ int p2p_tree_apply_delta_static(p2p_router* r, int32_t peer, const p2p_delta* d,
     return fail(r, P2P_E_INVAL, "NULL array in delta");
   if (peer == -1 && S.n > 0 && !d->peer_begin) return fail(r, P2P_E_INVAL, "peer = -1 needs peer_begin");
   DeviceGuard g(r);
+  if (S.n > 0)
+    if (int rc = reject_lru_ops(r, peer, d)) return rc;
   int32_t* header = nullptr;
   int32_t* tokens = nullptr;
   CK(p2p::static_scratch(r->device, &header, &tokens));
@@ -1280,7 +1335,11 @@ int p2p_update_estimates(p2p_router* r, const int32_t* tokens, int64_t n_tokens,
   // Every op is an INSERT: a tree that takes many (the fresh prompts of a batch all go to its least-loaded
   // tree) gets its root table sized for them before the delta kernel runs.
   std::vector<int64_t> ins((size_t)P);
-  for (int32_t p = 0; p < P; ++p) ins[(size_t)p] = pb[(size_t)p + 1] - pb[(size_t)p];
+  for (int32_t p = 0; p < P; ++p) {
+    ins[(size_t)p] = pb[(size_t)p + 1] - pb[(size_t)p];
+    if (ins[(size_t)p] && r->lru[(size_t)p])
+      return fail(r, P2P_E_INVAL, "requests routed to LRU tree " + std::to_string(p) + " go in through p2p_lru_insert");
+  }
   if (int rc = presize_roots(r, 0, P, ins.data())) return rc;
   CK(ensure(r, r->upd_op, (size_t)n * sizeof(int32_t)));
   CK(ensure(r, r->upd_so, (size_t)n * sizeof(int64_t)));
@@ -1307,6 +1366,214 @@ int p2p_update_estimates(p2p_router* r, const int32_t* tokens, int64_t n_tokens,
   const int rc = p2p_tree_apply_delta(r, -1, &d, nullptr);
   if (rc == P2P_OK && n_inserted) *n_inserted = n;
   return rc;
+}
+
+// ---- LRU trees: EvictLRUTrie of Algorithm 1 with device stamps (lru_kernel.cu) ----------------------------
+
+static int check_lru(p2p_router* r, int32_t tree, int64_t time) {
+  if (int rc = check_peer(r, tree)) return rc;
+  if (!r->lru[(size_t)tree]) return fail(r, P2P_E_INVAL, "tree " + std::to_string(tree) + " is not an LRU tree");
+  if (time < r->lru_time[(size_t)tree] || time > (int64_t)0xFFFFFFFE)
+    return fail(r, P2P_E_INVAL, "time must not decrease and must be at most 2^32 - 2");
+  return P2P_OK;
+}
+
+// An access at `time`: PrefixMatch of every request, the touched nodes stamped, partially touched edges split.
+static int lru_access_impl(p2p_router* r, int32_t tree, const int32_t* tokens, int64_t n_tokens,
+                           const int64_t* offsets, int64_t B, int64_t time, int32_t* out_match) {
+  TreeState& t = r->hs[(size_t)tree];
+  // Room for one split (a node and a 4-slot table) per request.
+  const bool short_n = (int64_t)t.cap_node - t.n_node < B, short_c = (int64_t)t.cap_child - t.n_child < 4 * B;
+  if (short_n || short_c) {
+    if ((int64_t)t.n_node + B > INT32_MAX || (int64_t)t.n_child + 4 * B > INT32_MAX)
+      return fail(r, P2P_E_NOMEM, "the LRU tree would outgrow the int32 arena indices");
+    t.need_node = short_n ? clamp_i32(B) : 0;
+    t.need_child = short_c ? clamp_i32(4 * B) : 0;
+    t.need_label = 0;
+    t.need_root = 0;
+    if (int rc = grow_tree(r, tree)) return rc;
+  }
+  const int32_t n0 = t.n_node;
+  CK(ensure(r, r->lru_buf, (size_t)2 * n0 * sizeof(int32_t)));
+  int32_t* touch = static_cast<int32_t*>(r->lru_buf.p);
+  int32_t* pslot = touch + n0;
+  CK(cudaMemsetAsync(touch, 0, (size_t)n0 * sizeof(int32_t), r->stream));
+  if (int rc = push_states(r, tree, tree + 1)) return rc;
+  CK(p2p::launch_lru_walk(t, r->d_shared, tokens, n_tokens, offsets, B, touch, pslot, out_match, r->d_err, r->num_sms,
+                          r->stream));
+  CK(p2p::launch_lru_stamp(t, r->d_states + tree, r->d_shared, touch, pslot, n0, (uint32_t)time, r->num_sms,
+                           r->stream));
+  if (int rc = pull_states(r, tree, tree + 1)) return rc;
+  CK(p2p::launch_refresh_views(r->d_states + tree, r->d_views + tree, 1, r->d_shared, r->stream));
+  r->launches += 3;
+  r->lru_time[(size_t)tree] = time;
+  return P2P_OK;
+}
+
+int p2p_lru_enable(p2p_router* r, int32_t tree) {
+  if (int rc = check_peer(r, tree)) return rc;
+  if (r->lru[(size_t)tree]) return P2P_OK;
+  DeviceGuard g(r);
+  TreeState& t = r->hs[(size_t)tree];
+  CK(cudaStreamSynchronize(r->stream));
+  uint32_t* st = nullptr;
+  cudaError_t e = dalloc(r, (void**)&st, (size_t)std::max(t.cap_node, 1) * sizeof(uint32_t));
+  if (e != cudaSuccess) return fail(r, P2P_E_NOMEM, std::string("allocating stamps: ") + cudaGetErrorString(e));
+  CK(cudaMemsetAsync(st, 0, (size_t)std::max(t.cap_node, 1) * sizeof(uint32_t), r->stream));
+  t.stamp = st;
+  r->lru[(size_t)tree] = 1;
+  r->lru_time[(size_t)tree] = 0;
+  return push_states(r, tree, tree + 1);
+}
+
+int p2p_lru_access(p2p_router* r, int32_t tree, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets,
+                   int64_t B, int64_t time, int32_t* out_match) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (int rc = check_lru(r, tree, time)) return rc;
+  if (B < 0 || n_tokens < 0 || B > kMaxBatch) return fail(r, P2P_E_INVAL, "B or n_tokens out of range");
+  if (B == 0) return P2P_OK;
+  if (!offsets || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r);
+  return lru_access_impl(r, tree, tokens, n_tokens, offsets, B, time, out_match);
+}
+
+int p2p_lru_insert(p2p_router* r, int32_t tree, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets,
+                   int64_t B, int64_t time) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (int rc = check_lru(r, tree, time)) return rc;
+  if (B < 0 || n_tokens < 0 || B > kMaxBatch) return fail(r, P2P_E_INVAL, "B or n_tokens out of range");
+  if (B == 0) return P2P_OK;
+  if (!offsets || (n_tokens > 0 && !tokens)) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r);
+  CK(ensure(r, r->upd_op, (size_t)B * sizeof(int32_t)));
+  CK(ensure(r, r->upd_sb, (size_t)(B + 1) * sizeof(int64_t)));
+  CK(ensure(r, r->upd_so, (size_t)B * sizeof(int64_t)));
+  CK(ensure(r, r->upd_sl, (size_t)B * sizeof(int32_t)));
+  int32_t* op = static_cast<int32_t*>(r->upd_op.p);
+  int64_t* sb = static_cast<int64_t*>(r->upd_sb.p);
+  int64_t* so = static_cast<int64_t*>(r->upd_so.p);
+  int32_t* sl = static_cast<int32_t*>(r->upd_sl.p);
+  CK(p2p::launch_lru_ops(offsets, B, n_tokens, op, sb, so, sl, r->num_sms, r->stream));
+  r->launches += 1;
+  p2p_delta d = {};
+  d.op = op;
+  d.seqs.n = B;
+  d.seqs.seg_begin = sb;
+  d.seqs.seg_off = so;
+  d.seqs.seg_len = sl;
+  d.seqs.pool = tokens;
+  d.seqs.n_segs = B;
+  d.seqs.n_pool = n_tokens;
+  d.mem = P2P_MEM_DEVICE;
+  // UpdateTrie: the sequences go in (invalid offsets fail validation: nothing changes), then every token of
+  // their paths is touched at `time`.
+  if (int rc = apply_delta_impl(r, tree, &d, nullptr, true)) return rc;
+  return lru_access_impl(r, tree, tokens, n_tokens, offsets, B, time, nullptr);
+}
+
+int p2p_lru_evict(p2p_router* r, int32_t tree, int64_t n_tokens, int64_t* n_evicted) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (n_evicted) *n_evicted = 0;
+  if (int rc = check_peer(r, tree)) return rc;
+  if (!r->lru[(size_t)tree]) return fail(r, P2P_E_INVAL, "tree " + std::to_string(tree) + " is not an LRU tree");
+  if (n_tokens < 0) return fail(r, P2P_E_INVAL, "negative n_tokens");
+  if (n_tokens == 0) return P2P_OK;
+  DeviceGuard g(r);
+  const TreeState& t = r->hs[(size_t)tree];
+  const int64_t N = std::max<int32_t>(t.n_node, 1);
+  // Scratch, per node slot: order, parent, cslot, end, surv (int32); size, off, rank, best (64-bit); gone; and
+  // two counters.
+  const size_t bytes = (size_t)N * (5 * 4 + 4 * 8 + 1) + 64;
+  CK(ensure(r, r->lru_buf, bytes));
+  char* base = static_cast<char*>(r->lru_buf.p);
+  int64_t* size = reinterpret_cast<int64_t*>(base);
+  int64_t* off = size + N;
+  int64_t* rank = off + N;
+  unsigned long long* best = reinterpret_cast<unsigned long long*>(rank + N);
+  unsigned long long* ctr = best + N;                      // [0]: token count, [1]: the BFS frontier size
+  int32_t* order = reinterpret_cast<int32_t*>(ctr + 2);
+  int32_t* parent = order + N;
+  int32_t* cslot = parent + N;
+  int32_t* end = cslot + N;
+  int32_t* surv = end + N;
+  uint8_t* gone = reinterpret_cast<uint8_t*>(surv + N);
+  int32_t* n_next = reinterpret_cast<int32_t*>(ctr + 1);
+  // Breadth-first order of the live nodes, level by level (order[0] = the root).
+  CK(cudaMemsetAsync(order, 0, sizeof(int32_t), r->stream));
+  std::vector<int32_t> lvl{0, 1};
+  for (;;) {
+    const int32_t l = (int32_t)lvl.size() - 2;
+    CK(cudaMemsetAsync(n_next, 0, sizeof(int32_t), r->stream));
+    CK(p2p::launch_lru_bfs(t, order + lvl[(size_t)l], lvl[(size_t)l + 1] - lvl[(size_t)l], order + lvl[(size_t)l + 1],
+                           n_next, parent, cslot, r->num_sms, r->stream));
+    r->launches += 1;
+    int32_t h = 0;
+    CK(d2h(r, &h, n_next, sizeof(h)));
+    if (h == 0) break;
+    if ((int64_t)lvl.back() + h > N) return fail(r, P2P_E_DEVICE, "the LRU tree is inconsistent");
+    lvl.push_back(lvl.back() + h);
+  }
+  const int32_t n_levels = (int32_t)lvl.size() - 1, total = lvl.back();
+  CK(p2p::launch_lru_init(order, total, size, off, rank, best, gone, r->num_sms, r->stream));
+  CK(p2p::launch_lru_levels(t, order, lvl.data(), n_levels, parent, cslot, size, off, rank, best, end, r->num_sms,
+                            r->stream));
+  r->launches += 1 + 4 * (n_levels - 1);
+  auto count = [&](int mode, uint32_t S, unsigned long long K, unsigned long long& out) -> int {
+    CK(p2p::launch_lru_count(t, order + 1, total - 1, cslot, rank, end, mode, S, K, ctr, r->num_sms, r->stream));
+    r->launches += 1;
+    CK(d2h(r, &out, ctr, sizeof(out)));
+    return P2P_OK;
+  };
+  // The threshold: stamps first, then the (end rank, deeper first) key inside the boundary stamp.
+  unsigned long long all = 0, c = 0;
+  if (int rc = count(0, 0xFFFFFFFFu, 0, all)) return rc;
+  uint32_t S = 0xFFFFFFFFu;
+  unsigned long long K = 0;
+  int32_t cut = 0;
+  const unsigned long long want = (unsigned long long)n_tokens;
+  if (want < all) {
+    uint32_t lo = 0, hi = 0xFFFFFFFFu;  // count(stamp < lo) <= want < count(stamp < hi)
+    while (hi - lo > 1) {
+      const uint32_t mid = lo + (hi - lo) / 2;
+      if (int rc = count(0, mid, 0, c)) return rc;
+      if (c <= want) lo = mid; else hi = mid;
+    }
+    S = lo;
+    if (int rc = count(0, S, 0, c)) return rc;
+    const unsigned long long rest = want - c;
+    if (rest > 0) {
+      unsigned long long lo2 = 0, hi2 = ~0ull;
+      while (hi2 - lo2 > 1) {
+        const unsigned long long mid = lo2 + (hi2 - lo2) / 2;
+        if (int rc = count(1, S, mid, c)) return rc;
+        if (c <= rest) lo2 = mid; else hi2 = mid;
+      }
+      K = lo2;
+      if (int rc = count(1, S, K, c)) return rc;
+      cut = (int32_t)(rest - c);
+    }
+  }
+  if (int rc = push_states(r, tree, tree + 1)) return rc;
+  CK(p2p::launch_lru_evict(t, r->d_states + tree, order, lvl.data(), n_levels, parent, cslot, rank, end, S, K, cut, gone,
+                           surv, r->num_sms, r->stream));
+  r->launches += n_levels - 1;
+  if (int rc = pull_states(r, tree, tree + 1)) return rc;
+  CK(p2p::launch_refresh_views(r->d_states + tree, r->d_views + tree, 1, r->d_shared, r->stream));
+  r->launches += 1;
+  if (n_evicted) *n_evicted = (int64_t)std::min(want, all);
+  return P2P_OK;
+}
+
+int p2p_hit_rate(p2p_router* r, const int32_t* match, const int64_t* offsets, int64_t B, const int32_t* peer,
+                 float* out) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (B < 0) return fail(r, P2P_E_INVAL, "negative B");
+  if (B == 0) return P2P_OK;
+  if (!match || !offsets || !peer || !out) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r);
+  CK(p2p::launch_hit_rate(match, r->P, offsets, B, peer, out, r->num_sms, r->stream));
+  r->launches += 1;
+  return P2P_OK;
 }
 
 int p2p_route_batch(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B,
