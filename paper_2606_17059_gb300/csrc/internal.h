@@ -244,7 +244,7 @@ cudaError_t launch_lru_walk(const TreeState& s, const int32_t* shared, const int
 cudaError_t launch_lru_stamp(const TreeState& s, TreeState* d_state, const int32_t* shared, const int32_t* touch,
                              const int32_t* pslot, int32_t n_node, uint32_t time, int num_sms, cudaStream_t st);
 cudaError_t launch_lru_bfs(const TreeState& s, const int32_t* front, int32_t n_front, int32_t* next, int32_t* n_next,
-                           int32_t* parent, int32_t* cslot, int num_sms, cudaStream_t st);
+                           int32_t cap, int32_t* parent, int32_t* cslot, int num_sms, cudaStream_t st);
 cudaError_t launch_lru_init(const int32_t* order, int32_t n, int64_t* size, int64_t* off, int64_t* rank,
                             unsigned long long* best, uint8_t* gone, int num_sms, cudaStream_t st);
 cudaError_t launch_lru_levels(const TreeState& s, const int32_t* order, const int32_t* lvl_begin, int32_t n_levels,

@@ -153,10 +153,11 @@ __global__ void __launch_bounds__(kLruThreads) lru_stamp_kernel(LruTree t, TreeS
   }
 }
 
-// Warp per node of the frontier: its live children get parent and slot, and go to the next frontier.
+// Warp per node of the frontier: its live children get parent and slot, and go to the next frontier (at most
+// cap entries are written; the host checks the count against it).
 __global__ void __launch_bounds__(kLruThreads) lru_bfs_kernel(LruTree t, const int32_t* __restrict__ front,
                                                               int32_t n_front, int32_t* next, int32_t* n_next,
-                                                              int32_t* parent, int32_t* cslot) {
+                                                              int32_t cap, int32_t* parent, int32_t* cslot) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (kLruThreads / 32);
   for (int64_t i = ((int64_t)blockIdx.x * kLruThreads + threadIdx.x) >> 5; i < n_front; i += warps) {
@@ -173,8 +174,9 @@ __global__ void __launch_bounds__(kLruThreads) lru_bfs_kernel(LruTree t, const i
       int32_t base = 0;
       if (lane == 0) base = atomicAdd(n_next, __popc(m));
       base = __shfl_sync(kFull, base, 0);
-      if (live) {
-        next[base + __popc(m & ((1u << lane) - 1))] = x.y;
+      const int32_t at = base + __popc(m & ((1u << lane) - 1));
+      if (live && at < cap) {
+        next[at] = x.y;
         parent[x.y] = v;
         cslot[x.y] = nd.x + s;
       }
@@ -390,11 +392,11 @@ cudaError_t launch_lru_stamp(const TreeState& s, TreeState* d_state, const int32
 }
 
 cudaError_t launch_lru_bfs(const TreeState& s, const int32_t* front, int32_t n_front, int32_t* next, int32_t* n_next,
-                           int32_t* parent, int32_t* cslot, int num_sms, cudaStream_t st) {
+                           int32_t cap, int32_t* parent, int32_t* cslot, int num_sms, cudaStream_t st) {
   if (n_front <= 0) return cudaSuccess;
   P2P_TIMED(K_LRU_ORDER, st,
             (lru_bfs_kernel<<<grid_for(n_front, kLruThreads / 32, num_sms), kLruThreads, 0, st>>>(
-                lru_tree(s, nullptr), front, n_front, next, n_next, parent, cslot)));
+                lru_tree(s, nullptr), front, n_front, next, n_next, cap, parent, cslot)));
   return cudaGetLastError();
 }
 

@@ -1505,7 +1505,7 @@ int p2p_lru_evict(p2p_router* r, int32_t tree, int64_t n_tokens, int64_t* n_evic
     const int32_t l = (int32_t)lvl.size() - 2;
     CK(cudaMemsetAsync(n_next, 0, sizeof(int32_t), r->stream));
     CK(p2p::launch_lru_bfs(t, order + lvl[(size_t)l], lvl[(size_t)l + 1] - lvl[(size_t)l], order + lvl[(size_t)l + 1],
-                           n_next, parent, cslot, r->num_sms, r->stream));
+                           n_next, (int32_t)(N - lvl[(size_t)l + 1]), parent, cslot, r->num_sms, r->stream));
     r->launches += 1;
     int32_t h = 0;
     CK(d2h(r, &h, n_next, sizeof(h)));
