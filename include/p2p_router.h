@@ -308,6 +308,15 @@ int p2p_route_batch_decide(p2p_router* r, const int32_t* tokens, int64_t n_token
                            const int32_t* load, int32_t alpha, const uint8_t* excluded, int32_t* out_match,
                            int32_t* out_peer, int32_t* out_next);
 
+/* Announces the next batch to route (DEVICE tokens/offsets as for p2p_route_batch; B <= 2^30).  The route's
+ * first step, grouping requests by shared prefix, reads only the requests, so the next p2p_tree_apply_delta
+ * launches it on a low-priority side stream right after its delta kernel: it runs on the SM room the delta
+ * kernel leaves.  The next p2p_route_batch or p2p_route_batch_decide of the same batch (same pointers and
+ * sizes) waits for it instead of grouping; a route of another batch groups as usual.  The requests must not
+ * change between the two calls.  Not part of the paper's method: a scheduling aid for a step of delta +
+ * route.  Errors: P2P_E_INVAL. */
+int p2p_route_prepare(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B);
+
 /* As p2p_route_batch with every pointer in HOST memory: copies the requests to the device, routes,
  * copies both outputs back and waits.  Large batches go in up to 8 chunks of at least 131,072 requests:
  * a chunk's inputs are copied in while the chunk before it is routed and the one before that is copied

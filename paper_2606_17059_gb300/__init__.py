@@ -22,7 +22,7 @@ __all__ = [
     "p2p_flat_tree_validate", "p2p_tree_upload", "p2p_tree_build", "p2p_tree_download", "p2p_tree_apply_delta",
     "p2p_tree_apply_delta_static", "p2p_tree_stats", "p2p_route_batch", "p2p_route_batch_host", "p2p_route_decide",
     "p2p_router_kernel_clock", "p2p_router_kernel_time", "p2p_update_estimates", "p2p_route_batch_decide",
-    "p2p_lru_enable", "p2p_lru_insert", "p2p_lru_access", "p2p_lru_evict", "p2p_hit_rate",
+    "p2p_lru_enable", "p2p_lru_insert", "p2p_lru_access", "p2p_lru_evict", "p2p_hit_rate", "p2p_route_prepare",
 ]
 
 P2P_OK, P2P_E_INVAL, P2P_E_NOMEM, P2P_E_FORMAT, P2P_E_CUDA, P2P_E_DEVICE = 0, -1, -2, -3, -4, -5
@@ -103,6 +103,7 @@ def _load():
             "p2p_lru_access": (ctypes.c_int, [_vp, _i32, _vp, _i64, _vp, _i64, _i64, _vp]),
             "p2p_lru_evict": (ctypes.c_int, [_vp, _i32, _i64, P(_i64)]),
             "p2p_hit_rate": (ctypes.c_int, [_vp, _vp, _vp, _i64, _vp, _vp]),
+            "p2p_route_prepare": (ctypes.c_int, [_vp, _vp, _i64, _vp, _i64]),
             "p2p_router_kernel_time": (ctypes.c_int, [_vp, _i32, P(ctypes.c_char_p), P(_i64), P(ctypes.c_double)]),
         }
         for name, (res, args) in sig.items():
@@ -382,6 +383,11 @@ def p2p_route_batch_decide(r, tokens, n_tokens: int, offsets, B: int, load, alph
     _check(_load().p2p_route_batch_decide(r, _addr(tokens), n_tokens, _addr(offsets), B, ld.ctypes.data, alpha,
                                           ex.ctypes.data if ex is not None else None, _addr(out_match),
                                           _addr(out_peer), _addr(out_next)), r)
+
+
+def p2p_route_prepare(r, tokens, n_tokens: int, offsets, B: int) -> None:
+    """Announces the next batch (CUDA tensors): its grouping overlaps the next delta kernel."""
+    _check(_load().p2p_route_prepare(r, _addr(tokens), n_tokens, _addr(offsets), B), r)
 
 
 def p2p_route_decide(r, match, B: int, load, alpha: int, excluded, out_peer, out_next) -> None:

@@ -191,6 +191,16 @@ struct p2p_router {
   cudaEvent_t load_ev[kLoadRing] = {};
   // Copy streams of p2p_route_batch_host (inputs in, results out) and the events that order them.
   cudaStream_t cp_in = nullptr, cp_out = nullptr;
+  // p2p_route_prepare: a batch whose grouping runs on grp_stream (low priority) while the next delta kernel
+  // runs; the route of the same batch then waits for grp_done instead of grouping.
+  struct Prepared {
+    const int32_t* tokens = nullptr;
+    const int64_t* offsets = nullptr;
+    int64_t n_tokens = 0, B = 0;
+    int state = 0;  // 0 none, 1 staged (grouping not launched yet), 2 launched on grp_stream
+  } prep;
+  cudaStream_t grp_stream = nullptr;
+  cudaEvent_t grp_start = nullptr, grp_done = nullptr;
   cudaEvent_t ev_start = nullptr, ev_done = nullptr, ev_in[kPipe] = {}, ev_routed[kPipe] = {};
   int load_slot = 0;
   int32_t* h_err = nullptr;       // pinned
@@ -306,13 +316,48 @@ cudaError_t group_scratch(p2p_router* r, int64_t B, p2p::GroupScratch& g) {
 // excluded trees and the next-best target.
 int route(p2p_router* r, const int32_t* tokens, int64_t n_tokens, int64_t tok_base, const int64_t* offsets, int64_t B,
           int32_t alpha, int32_t* out_match, int32_t* out_peer, bool decide = false, int32_t* out_next = nullptr) {
+  const auto& pr = r->prep;
+  const bool same = pr.state != 0 && pr.tokens == tokens && pr.offsets == offsets && pr.n_tokens == n_tokens &&
+                    pr.B == B && tok_base == 0;
+  const bool grouped = same && pr.state == 2;
+  if (r->prep.state == 2) CK(cudaStreamWaitEvent(r->stream, r->grp_done, 0));  // its scratch is this call's
+  // (state 3, scratch taken but the grouping not launched, cannot outlive the delta call that took it)
+  r->prep.state = 0;
   p2p::GroupScratch g;
   CK(group_scratch(r, B, g));
-  CK(p2p::launch_group(tokens, n_tokens, tok_base, offsets, B, g, r->num_sms, r->stream));
+  if (!grouped) {
+    CK(p2p::launch_group(tokens, n_tokens, tok_base, offsets, B, g, r->num_sms, r->stream));
+    r->launches += 4;
+  }
   int launched = 0;
   CK(p2p::launch_route(r->d_views, r->P, tokens, n_tokens, tok_base, offsets, B, r->d_load, alpha, out_match, out_peer,
                        r->d_err, &g, r->num_sms, r->stream, &launched, decide, out_next));
-  r->launches += 4 + launched;
+  r->launches += launched;
+  return P2P_OK;
+}
+
+// A staged p2p_route_prepare grouping, in two steps around a delta kernel launch.  Before: its scratch is
+// allocated (router-stream order) and grp_start marks the router stream there, ahead of the delta kernel.
+// After: the grouping is launched on the side stream behind grp_start only, so it runs alongside the delta
+// kernel, whose CTAs are resident first; the grouping uses the room they leave.
+int prepare_scratch(p2p_router* r) {
+  if (r->prep.state != 1) return P2P_OK;
+  p2p::GroupScratch g;
+  CK(group_scratch(r, r->prep.B, g));
+  CK(cudaEventRecord(r->grp_start, r->stream));
+  r->prep.state = 3;
+  return P2P_OK;
+}
+
+int launch_prepared(p2p_router* r) {
+  if (r->prep.state != 3) return P2P_OK;
+  p2p::GroupScratch g;
+  CK(group_scratch(r, r->prep.B, g));  // the buffers of prepare_scratch (no allocation)
+  CK(cudaStreamWaitEvent(r->grp_stream, r->grp_start, 0));
+  CK(p2p::launch_group(r->prep.tokens, r->prep.n_tokens, 0, r->prep.offsets, r->prep.B, g, r->num_sms, r->grp_stream));
+  CK(cudaEventRecord(r->grp_done, r->grp_stream));
+  r->launches += 4;
+  r->prep.state = 2;
   return P2P_OK;
 }
 
@@ -891,6 +936,13 @@ int p2p_router_create(int32_t P, p2p_router** out) {
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_err, sizeof(int32_t));
   if (e == cudaSuccess) e = cudaMallocHost((void**)&r->h_states, (size_t)P * sizeof(TreeState));
   for (int i = 0; i < kLoadRing && e == cudaSuccess; ++i) e = cudaEventCreateWithFlags(&r->load_ev[i], cudaEventDisableTiming);
+  if (e == cudaSuccess) {
+    int lo = 0, hi = 0;  // the side stream of prepared groupings yields to the router's kernels
+    e = cudaDeviceGetStreamPriorityRange(&lo, &hi);
+    if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&r->grp_stream, cudaStreamNonBlocking, lo);
+  }
+  for (cudaEvent_t* ev : {&r->grp_start, &r->grp_done})
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(ev, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&r->cp_in, cudaStreamNonBlocking);
   if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&r->cp_out, cudaStreamNonBlocking);
   for (cudaEvent_t* ev : {&r->ev_start, &r->ev_done})
@@ -941,11 +993,13 @@ void p2p_router_destroy(p2p_router* r) {
   }
   for (cudaEvent_t ev : r->load_ev)
     if (ev) cudaEventDestroy(ev);
-  for (cudaStream_t s : {r->cp_in, r->cp_out})
+  for (cudaStream_t s : {r->cp_in, r->cp_out, r->grp_stream})
     if (s) {
       cudaStreamSynchronize(s);
       cudaStreamDestroy(s);
     }
+  for (cudaEvent_t ev : {r->grp_start, r->grp_done})
+    if (ev) cudaEventDestroy(ev);
   for (cudaEvent_t ev : {r->ev_start, r->ev_done})
     if (ev) cudaEventDestroy(ev);
   for (int i = 0; i < kPipe; ++i) {
@@ -1164,8 +1218,12 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
       rc = fail(r, P2P_E_NOMEM, "delta did not fit after 64 arena growths");
       break;
     }
+    if (round == 0)
+      if (int rc = prepare_scratch(r)) return rc;
     CK(p2p::launch_delta(r->d_states + p0, done, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->d_shared,
                          r->stream));
+    if (round == 0)
+      if (int rc = launch_prepared(r)) return rc;  // a prepared batch's grouping overlaps the delta kernel
     r->launches += 1;
     if (int e = pull_states(r, p0, p1)) return e;
     bool again = false;
@@ -1573,6 +1631,22 @@ int p2p_hit_rate(p2p_router* r, const int32_t* match, const int64_t* offsets, in
   DeviceGuard g(r);
   CK(p2p::launch_hit_rate(match, r->P, offsets, B, peer, out, r->num_sms, r->stream));
   r->launches += 1;
+  return P2P_OK;
+}
+
+int p2p_route_prepare(p2p_router* r, const int32_t* tokens, int64_t n_tokens, const int64_t* offsets, int64_t B) {
+  if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
+  if (B < 0 || n_tokens < 0 || B > kMaxBatch) return fail(r, P2P_E_INVAL, "B or n_tokens out of range");
+  if (B > 0 && (!offsets || (n_tokens > 0 && !tokens))) return fail(r, P2P_E_INVAL, "NULL device pointer");
+  DeviceGuard g(r);
+  if (r->prep.state == 2) CK(cudaStreamWaitEvent(r->stream, r->grp_done, 0));  // the scratch is free again
+  r->prep.state = 0;
+  if (B == 0) return P2P_OK;
+  r->prep.tokens = tokens;
+  r->prep.offsets = offsets;
+  r->prep.n_tokens = n_tokens;
+  r->prep.B = B;
+  r->prep.state = 1;
   return P2P_OK;
 }
 

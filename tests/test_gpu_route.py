@@ -282,3 +282,37 @@ def _dev_arr(a):
 
 def _dev_seqlist(sl):
     return wl.SeqList(_dev_arr(sl.seg_begin), _dev_arr(sl.seg_off), _dev_arr(sl.seg_len), _dev_arr(sl.pool))
+
+
+def test_prepared_grouping_overlapping_a_delta():
+    """p2p_route_prepare: the batch's grouping runs alongside the next delta kernel, and the route of the same
+    batch uses it; results equal a plain route after the same delta, and a route of another batch (or one
+    without a delta in between) groups as usual."""
+    import torch
+    W = wl.Workload(0)
+    sls = [W.tree(p) for p in range(W.P)]
+    ra, rb = router_from_seqlists(sls), router_from_seqlists(sls)
+    tok, off = W.requests()
+    t, o = torch.from_numpy(tok).cuda(), torch.from_numpy(off).cuda()
+    t2, o2 = t[: int(off[1000])].clone(), o[:1001].clone()
+    load = W.load()
+    for step in range(3):
+        W.delta_make(step, 0.05, 0.05)
+        d = W.delta()
+        g.p2p_route_prepare(ra.handle, t, t.numel(), o, W.B)
+        assert ra.apply_delta(-1, d.op, d.seqs, d.peer_begin) == 0
+        assert rb.apply_delta(-1, d.op, d.seqs, d.peer_begin) == 0
+        ma, pa = ra.route(t, o, load, W.alpha)
+        mb, pb = rb.route(t, o, load, W.alpha)
+        ra.sync()
+        rb.sync()
+        assert torch.equal(ma, mb) and torch.equal(pa, pb), step
+    # Prepared, then another batch routed (and no delta): both group on their own.
+    g.p2p_route_prepare(ra.handle, t, t.numel(), o, W.B)
+    g.p2p_route_prepare(ra.handle, t, t.numel(), o, W.B)  # twice: the later one stands
+    m2a, p2a = ra.route(t2, o2, load, W.alpha)
+    m2b, p2b = rb.route(t2, o2, load, W.alpha)
+    ma, pa = ra.route(t, o, load, W.alpha)
+    ra.sync()
+    rb.sync()
+    assert torch.equal(m2a, m2b) and torch.equal(p2a, p2b) and torch.equal(ma, mb) and torch.equal(pa, pb)
