@@ -396,6 +396,8 @@ def run_ours(args):
         if has_delta:
             op, sl, pb = deltas[s]
             ev[0].record(stream)
+            # The batch's grouping (it reads only the requests) runs alongside the delta kernel.
+            g.p2p_route_prepare(router.handle, d_tok, n_tok, d_off, B)
             router.apply_delta(-1, op, sl, pb, on_device=True)
         ev[1].record(stream)
         g.p2p_route_batch(router.handle, d_tok, n_tok, d_off, B, load, alpha, out_match, out_peer)
@@ -485,23 +487,27 @@ def run_ours(args):
         route = {"kernels": [k for k in ("group_hash_kernel", "group_resolve_kernel", "group_resolve32_kernel",
                                          "group_ranges_kernel", "group_place_kernel", "route_kernel",
                                          "lane_kernel<true>", "lane_kernel<false>") if k in kt],
-                 "ms": route_avg_ms, "compulsory_bytes": compulsory,
-                 "compulsory_gbs": compulsory / (route_avg_ms / 1e3) / 1e9}
+                 "ms": route_avg_ms, "compulsory_bytes": compulsory}
+        # Device time of the route kernels (with p2p_route_prepare the grouping runs alongside the delta kernel,
+        # outside the route span), the time the route's bytes are measured against.
+        route_k_ms = sum(kt[k]["ms_per_step"] for k in route["kernels"]) or route_avg_ms
+        route["kernel_ms"] = route_k_ms
+        route["compulsory_gbs"] = compulsory / (route_k_ms / 1e3) / 1e9
         route["compulsory_frac"] = route["compulsory_gbs"] / hbm
         tr = [traffic_of(tkey, k) if tkey else None for k in route["kernels"]]
         route["traffic"] = sum(t["bytes"] for t in tr) if tr and all(tr) else None
         if route["traffic"]:
-            route["dram_gbs"] = route["traffic"] / (route_avg_ms / 1e3) / 1e9
+            route["dram_gbs"] = route["traffic"] / (route_k_ms / 1e3) / 1e9
         if ctr is not None:
             touched = orc.touched_bytes(ctr) / n_acc * B
-            route.update({"touched_bytes": touched, "effective_gbs": touched / (route_avg_ms / 1e3) / 1e9,
+            route.update({"touched_bytes": touched, "effective_gbs": touched / (route_k_ms / 1e3) / 1e9,
                           "touched_basis": f"oracle per-(request, tree) walk counters over {n_acc} requests x {P} "
                                            f"trees, scaled to {B} requests; groups and L2 hits let the device "
                                            "exceed HBM by this measure"})
         # ---- the roofline of the stage that takes the most time ----
         roof = None
         delta_k = kt.get("delta_kernel")
-        if delta_k and delta_k["ms_per_step"] >= route_avg_ms and has_delta:
+        if delta_k and delta_k["ms_per_step"] >= route_k_ms and has_delta:
             n_ops_step = len(host_delta0.op)
             per_op, counted = delta_op_bytes(otrees, host_delta0, counted_share, n_cpu) if want_oracle else (0.0, 0)
             if counted:
@@ -520,7 +526,7 @@ def run_ours(args):
             roof = {"bound": "hbm", "kernel": "route step: " + " + ".join(route["kernels"]),
                     "achieved": route["compulsory_gbs"], "peak": hbm, "unit": "GB/s", "frac": route["compulsory_frac"],
                     "traffic": route["traffic"], "peak_source": peak_source, "bytes_per_launch": compulsory,
-                    "ms_per_launch": route_avg_ms,
+                    "ms_per_launch": route_k_ms,
                     "bytes_basis": "compulsory bytes: request tokens and offsets read once, match matrix and peers "
                                    "written once (tree bytes left out: a lower bound)"}
             if route["traffic"]:
