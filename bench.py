@@ -202,16 +202,19 @@ def max_over_ranks(ms: float, dist, device=None) -> float:
 
 # ---- workload setup ---------------------------------------------------------------------------------
 
-def make_workload(cfg: int, trees: int = 0, batch: int = 0):
-    """The preset workload; trees/batch > 0 scale P and B down (smaller variants for profiling only)."""
+def make_workload(cfg: int, trees: int = 0, batch: int = 0, seqs: int = 0):
+    """The preset workload; trees/batch/seqs > 0 scale P, B and the sequences per tree down (smaller variants
+    for profiling only)."""
     import workload as wl
-    if not trees and not batch:
+    if not trees and not batch and not seqs:
         return wl.Workload(cfg)
     prm = wl.preset(cfg)
     if trees:
         prm["P"] = trees
     if batch:
         prm["B"] = batch
+    if seqs:
+        prm["n_seq"] = seqs
     return wl.Workload(params=prm, seed=wl.default_seed(cfg))
 
 
@@ -355,10 +358,10 @@ def run_ours(args):
     cfg, wdesc = WORKLOADS[args.workload]
     n_cpu = os.cpu_count() or 1
     t_setup = time.perf_counter()
-    W = make_workload(cfg, args.trees, args.batch)
+    W = make_workload(cfg, args.trees, args.batch, args.seqs)
     P, B, alpha = W.P, W.B, W.alpha
-    if args.trees or args.batch:
-        wdesc += f" [scaled down: P={P}, B={B}]"
+    if args.trees or args.batch or args.seqs:
+        wdesc += f" [scaled down: P={P}, B={B}, {W.params['n_seq']} sequences per tree]"
     router = g.Router(P)
     want_oracle = rank == 0 and not args.no_cpu_baseline
     otrees = build_trees(W, router, want_oracle, n_cpu)
@@ -468,7 +471,7 @@ def run_ours(args):
         hbm, src = peaks()
         peak_source = f"{src} (MEASURED_PEAKS.json hbm_gbs, STREAM-style copy)"
         route_avg_ms = statistics.mean(route_ms)
-        tkey = None if (args.trees or args.batch) else args.workload
+        tkey = None if (args.trees or args.batch or args.seqs) else args.workload
         # ---- every kernel of the timed region (the library's kernel clock) ----
         k_total = sum(ms for _, ms in ktimes.values()) or 1.0
         kernels = []
@@ -695,7 +698,7 @@ def run_reference(args):
     import oracle as orc
     cfg, wdesc = WORKLOADS[args.workload]
     n_cpu = os.cpu_count() or 1
-    W = make_workload(cfg, args.trees, args.batch)
+    W = make_workload(cfg, args.trees, args.batch, args.seqs)
     P, B, alpha = W.P, W.B, W.alpha
     otrees = orc.build_trees([W.tree(p) for p in range(P)], n_threads=n_cpu)
     has_delta = W.params["delta_frac"] > 0
@@ -747,6 +750,8 @@ def main():
     ap.add_argument("--ref-seconds", type=float, default=4.0, help="oracle time per reference step")
     ap.add_argument("--trees", type=int, default=0, help="override P (a scaled-down variant, not a bench line)")
     ap.add_argument("--batch", type=int, default=0, help="override B (a scaled-down variant, not a bench line)")
+    ap.add_argument("--seqs", type=int, default=0,
+                    help="override the sequences per tree (a scaled-down variant, not a bench line)")
     args = ap.parse_args()
     if args.warmup < 3:
         log("warmup < 3 is below the timing rules; using 3")
