@@ -106,8 +106,11 @@ def test_random_operation_sequences(seed):
 
 
 def test_workload_tree_made_lru_after_upload():
+    """A generator tree (shared prompt prefixes, Zipf requests) made an LRU tree after its upload: accesses,
+    inserts of new prompts, and evictions of a few tokens at a time (the oracle evicts one token per scan of its
+    trie, so the evicted amounts stay small); then everything, which leaves every stored sequence empty."""
     prm = wl.preset(0)
-    prm.update(P=2, n_seq=400, n_prefix=12, B=600)
+    prm.update(P=2, n_seq=60, n_prefix=6, B=160, pre_lo=64, pre_hi=256)
     W = wl.Workload(params=prm, seed=33)
     sl = W.tree(0)
     r = router_from_seqlists([sl, W.tree(1)])
@@ -117,19 +120,24 @@ def test_workload_tree_made_lru_after_upload():
         o.insert(sl.seq(i).tolist(), 0)
     tok, off = W.requests()
     reqs = [tok[off[b]:off[b + 1]].tolist() for b in range(len(off) - 1)]
-    got = _access(r, 0, reqs[:300], 3)
-    assert got.tolist() == [o.access(s, 3) for s in reqs[:300]]
-    _insert(r, 0, reqs[300:400], 5)
-    for s in reqs[300:400]:
+    got = _access(r, 0, reqs[:100], 3)
+    assert got.tolist() == [o.access(s, 3) for s in reqs[:100]]
+    _insert(r, 0, reqs[100:130], 5)
+    for s in reqs[100:130]:
         o.insert(s, 5)
-    total = o.n_tokens
-    for n in (1, 17, 1000, total // 3, 10**9):
+    for t, n in ((5, 1), (6, 17), (6, 150), (9, 400)):
+        got = _access(r, 0, reqs[130:160], t)
+        assert got.tolist() == [o.access(s, t) for s in reqs[130:160]]
         evicted = g.p2p_lru_evict(r.handle, 0, n)
         k = 0
         while k < n and o.evict() is not None:
             k += 1
         assert evicted == k
         assert same_snapshot(r.download(0), _oracle_export(o)), n
+    stored = sum(o.sequences().values())
+    assert g.p2p_lru_evict(r.handle, 0, 10**12) == o.n_tokens
+    d = r.download(0)
+    assert d["label_off"].tolist() == [0] and d["term_count"].tolist() == [stored]
 
 
 def test_lru_tree_rejects_other_changes_and_bad_times():
