@@ -782,12 +782,15 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
         for (int g = 0; g < kFollowIlp; ++g) {
           pt[g] = p0 + 32 * g + lane;
           ml[g] = pt[g] < P ? out_match[lrow + pt[g]] : 0;
+          // The checkpoint is loaded with the leader's match, before the match says whether it is needed:
+          // a group's followers are routed side by side, so its row is in cache, and one round trip is saved.
+          st[g] = pt[g] < P && row >= 0 ? ckrow[pt[g]] : make_int4(0, 0, 0, 0);
         }
 #pragma unroll
         for (int g = 0; g < kFollowIlp; ++g) {
           const bool w = pt[g] < P && len > 0 && ml[g] >= c && c < len;
-          st[g] = make_int4(0, 0, 0, 0);
-          if (w) st[g] = row >= 0 ? ckrow[pt[g]] : root_checkpoint(trees[pt[g]]);
+          if (!w) st[g] = make_int4(0, 0, 0, 0);
+          else if (row < 0) st[g] = root_checkpoint(trees[pt[g]]);
           pos[g] = min(st[g].x, len);
           m[g] = w ? pos[g] : len == 0 ? 0 : ml[g] < c ? ml[g] : len;
           act[g] = w && pos[g] < len && st[g].w > 0 && tab_bits(st[g].z) > 0;
