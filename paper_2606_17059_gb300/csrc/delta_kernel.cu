@@ -779,6 +779,20 @@ __device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcod
                                  : remove(t, q, root, anchor, lane, memo, ae);
 }
 
+// Lane 0 asks L1 for the op code and pool-run descriptors of the warp's next op (op jn of the chunk at c0)
+// while the current op runs: the next op's first loads then hit in L1.  Only ops with a pool run are
+// prefetched (their descriptor index is inside the arrays).
+__device__ __forceinline__ void prefetch_op(const int32_t* op, const int64_t* seg_off, const int32_t* seg_len,
+                                            const int64_t* s_run, int64_t c0, int jn, int lane) {
+  if (lane != 0) return;
+  const int64_t g0 = s_run[jn];
+  asm volatile("prefetch.global.L1 [%0];" :: "l"(op + c0 + jn));
+  if (s_run[jn + 1] > g0) {
+    asm volatile("prefetch.global.L1 [%0];" :: "l"(seg_off + g0));
+    asm volatile("prefetch.global.L1 [%0];" :: "l"(seg_len + g0));
+  }
+}
+
 // Ranks kDeltaBuckets buckets by count (heaviest first, ties to the lower bucket) into order; one warp.
 __device__ void rank_buckets(const int* count, int* order, int lane) {
   const int mine = count[lane];
@@ -945,6 +959,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
             continue;
           }
           const int64_t i = c0 + jj;
+          if (mine) prefetch_op(op, seg_off, seg_len, s_run, c0, j0 + (__ffs(mine) - 1), lane);
           const int r = apply_op(t, root, s_anchor[jj], op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool,
                                  buf, lane, memo, &s_aentry[s_aslot[jj]]);
           if (lane == 0) {
@@ -995,6 +1010,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
           const int jj = j0 + (__ffs(mine) - 1);
           mine &= mine - 1;
           const int64_t i = c0 + jj;
+          if (mine) prefetch_op(op, seg_off, seg_len, s_run, c0, j0 + (__ffs(mine) - 1), lane);
           const int r = apply_op(t, root, -1, op[i], s_run[jj], s_run[jj + 1], seg_off, seg_len, pool, buf, lane,
                                  memo, nullptr);
           if (lane == 0) {
