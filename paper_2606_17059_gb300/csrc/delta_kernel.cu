@@ -61,6 +61,7 @@ struct Seq {
   const int32_t* a;
   const int32_t* b;
   int64_t na, n;
+  bool pooled;  // a points into the delta's pool (not into gather scratch)
   __device__ int32_t at(int64_t i) const { return i < na ? a[i] : b[i - na]; }
 };
 
@@ -294,10 +295,31 @@ struct MemoEntry {
   int64_t n;
 };
 // A warp's memo: kMemoSlots entries in shared memory, so that the shared prefixes of the several anchors a
-// warp serves all stay remembered.
+// warp serves all stay remembered.  Behind it, a table in global memory shared by every warp of the launch
+// (all trees): runs verified from the start of an interned label (router-wide pool) against the start of a
+// pool run of the delta.  The same prompt prefix is interned once for all replicas and sent once in the
+// delta's pool, so it is compared once per launch instead of once per tree, chunk and anchor.  A key is
+// (1 << 63 | pool offset of the label << 32 | pool offset of the run), claimed by compare-and-swap; its value
+// only grows (atomicMax) and is always a verified length, so a reader that sees a key before its value
+// reads 0 and merely compares.
+constexpr int kGlobalMemoProbes = 8;
 struct Memo {
   MemoEntry* e;
+  unsigned long long* gkeys;  // NULL: no global table
+  int32_t* gvals;
+  uint32_t gmask;
+  const int32_t* pool;
 };
+
+__device__ __forceinline__ unsigned long long global_memo_key(const Memo& m, const Seq& q, int32_t loff, int64_t pos) {
+  if (!m.gkeys || loff >= 0 || !q.pooled) return 0ull;
+  const int64_t soff = (q.a + pos) - m.pool;
+  if (soff < 0 || soff > 0xffffffffll) return 0ull;
+  return (1ull << 63) | ((unsigned long long)(uint32_t)~loff << 32) | (unsigned long long)soff;
+}
+__device__ __forceinline__ uint32_t global_memo_slot(unsigned long long key, uint32_t mask) {
+  return (uint32_t)((key * 0x9E3779B97F4A7C15ull) >> 32) & mask;
+}
 
 // First j in [from, lim) with a[j] != b[j], or lim (one warp; both arrays contiguous in global memory).
 // kDiffUnroll loads of 32 tokens in flight per lane and side; a block is folded into one OR of XORs per
@@ -331,15 +353,20 @@ __device__ int64_t first_diff_arrays(const int32_t* a, const int32_t* b, int64_t
 // First j in [from, lim) with lab[j] != q[pos + j], or lim.  Lane k looks at memo entry k, so a lookup is
 // one step.  The sequence side is compared run by run (its first pool run, then the second), so both
 // sides of every compare are contiguous.
-__device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int64_t from, int64_t lim, int lane,
-                              Memo& memo) {
+__device__ int64_t first_diff(const int32_t* lab, int32_t loff, const Seq& q, int64_t pos, int64_t from, int64_t lim,
+                              int lane, Memo& memo) {
   const bool in_a = pos < q.na;  // q[pos ..] starts in the first pool run, which the memo can describe
+  const unsigned long long gkey = in_a ? global_memo_key(memo, q, loff, pos) : 0ull;
   if (in_a) {
     int32_t skip = 0;
     if (lane < kMemoSlots) {
       const MemoEntry m = memo.e[lane];
       const int64_t dl = lab - m.lab, ds = (q.a + pos) - m.seq;
       if (m.lab && dl == ds && dl >= 0 && dl < m.n) skip = (int32_t)min(lim, m.n - dl);
+    }
+    if (gkey && lane >= kMemoSlots && lane < kMemoSlots + kGlobalMemoProbes) {
+      const uint32_t s = (global_memo_slot(gkey, memo.gmask) + (uint32_t)(lane - kMemoSlots)) & memo.gmask;
+      if (__ldcg(memo.gkeys + s) == gkey) skip = (int32_t)min(lim, (int64_t)__ldcg(memo.gvals + s));
     }
     from = max(from, (int64_t)__reduce_max_sync(kFull, (unsigned)skip));
   }
@@ -351,8 +378,20 @@ __device__ int64_t first_diff(const int32_t* lab, const Seq& q, int64_t pos, int
   }
   if (in_a && k >= 64) {  // remember a long verified run (within the first pool run), slot by label address
     if (lane == 0) {
+      const int64_t nv = min(k, q.na - pos);
       const uint32_t h = (uint32_t)(((uintptr_t)lab >> 2) * 0x9E3779B97F4A7C15ull >> 32) & (kMemoSlots - 1);
-      memo.e[h] = MemoEntry{lab, q.a + pos, min(k, q.na - pos)};
+      memo.e[h] = MemoEntry{lab, q.a + pos, nv};
+      if (gkey) {
+        const uint32_t h0 = global_memo_slot(gkey, memo.gmask);
+        for (uint32_t i = 0; i < kGlobalMemoProbes; ++i) {
+          const uint32_t s = (h0 + i) & memo.gmask;
+          const unsigned long long prev = atomicCAS(memo.gkeys + s, 0ull, gkey);
+          if (prev == 0ull || prev == gkey) {
+            atomicMax(memo.gvals + s, (int32_t)min(nv, (int64_t)INT32_MAX));
+            break;
+          }
+        }
+      }
     }
     __syncwarp();
   }
@@ -546,7 +585,7 @@ __device__ int insert(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
     const int4 nn = t.node[ce.y];  // the child's record, fetched while the label is compared
     const int64_t lim = min((int64_t)ce.w, n - pos);
-    const int64_t k = first_diff(t.lab(ce.z), q, pos, 1, lim, lane, memo);
+    const int64_t k = first_diff(t.lab(ce.z), ce.z, q, pos, 1, lim, lane, memo);
     if (k == ce.w) {
       cur = ce.y;
       pos += k;
@@ -630,7 +669,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     int4* ent = t.child + slot;
     if (ce.w <= 0 || ce.y <= 0) return OP_CORRUPT;
     const int4 nn = t.node[ce.y];  // the child's record, fetched while the label is compared
-    if (pos + ce.w > n || first_diff(t.lab(ce.z), q, pos, 1, ce.w, lane, memo) < ce.w) {
+    if (pos + ce.w > n || first_diff(t.lab(ce.z), ce.z, q, pos, 1, ce.w, lane, memo) < ce.w) {
       if (!passed) return OP_DEFER;
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
@@ -759,6 +798,7 @@ __device__ int apply_op(Tree& t, const int4& root, int32_t anchor, int32_t opcod
                         const int32_t* __restrict__ pool, int32_t* buf, int lane, Memo& memo, AnchorEntry* ae) {
   // The op's sequence: up to two pool runs are read in place, more are gathered into scratch.
   Seq q;
+  q.pooled = g1 - g0 <= 2;
   if (g1 - g0 <= 2) {
     q.a = pool + (g1 > g0 ? seg_off[g0] : 0);
     q.na = g1 > g0 ? seg_len[g0] : 0;
@@ -814,7 +854,8 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     delta_kernel(TreeState* states, uint8_t* done, const int32_t* __restrict__ op,
                  const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
                  const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int32_t* gather,
-                 int64_t stride, const int32_t* shared) {
+                 int64_t stride, const int32_t* shared, unsigned long long* gmemo_keys, int32_t* gmemo_vals,
+                 uint32_t gmemo_mask) {
   // The chunk's per-op and per-anchor arrays, in dynamic shared memory (delta_smem_bytes()).
   extern __shared__ __align__(16) unsigned char s_dyn[];
   AnchorEntry* s_aentry = reinterpret_cast<AnchorEntry*>(s_dyn);        // per anchor: its shortcut
@@ -859,7 +900,8 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   t.slab = s_slab[warp];
   const int4 root = t.node[0];  // its table offset and size hold for the whole launch
   int32_t* buf = gather ? gather + ((int64_t)blockIdx.x * kDeltaWarps + warp) * stride : nullptr;
-  Memo memo{s_memo[warp]};  // facts about immutable labels: valid whichever bucket the warp works on
+  // Facts about immutable labels: valid whichever bucket the warp works on.
+  Memo memo{s_memo[warp], gmemo_keys, gmemo_vals, gmemo_mask, pool};
   for (int64_t c0 = op_begin; c0 < op_end; c0 += kChunk) {
     const int clen = (int)min((int64_t)kChunk, op_end - c0);
     // 1. Per op: first-token bucket, done flag, and (for ops still to apply) the anchor.
@@ -1379,14 +1421,16 @@ cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, int32_t max_cap_n
 
 cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
-                         int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st) {
+                         int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st,
+                         const GlobalMemo* gm) {
   if (n_trees <= 0) return cudaSuccess;
   const int dyn = delta_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
   if (e != cudaSuccess) return e;
   P2P_TIMED(K_DELTA, st,
-            (delta_kernel<<<n_trees, kDeltaWarps * 32, dyn, st>>>(d_states, done, op, seg_begin, seg_off, seg_len, pool,
-                                                                  gather, gather_stride, shared)));
+            (delta_kernel<<<n_trees, kDeltaWarps * 32, dyn, st>>>(
+                d_states, done, op, seg_begin, seg_off, seg_len, pool, gather, gather_stride, shared,
+                gm ? gm->keys : nullptr, gm ? gm->vals : nullptr, gm ? gm->mask : 0u)));
   return cudaGetLastError();
 }
 

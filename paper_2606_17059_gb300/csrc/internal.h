@@ -175,9 +175,18 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
 // per tree.  done[i] (one byte per op of the call, zero before the first launch, kept across relaunches)
 // marks the ops applied so far.  gather (n_trees * kDeltaWarps * gather_stride tokens) is needed only when
 // an op's sequence has more than two pool runs; otherwise it may be NULL.
+// A launch-wide table of verified (interned label, pool run) equalities (keys all zero before a call's first
+// launch; keys [mask + 1], vals [mask + 1]).  NULL: none (the allocation-free call).
+struct GlobalMemo {
+  unsigned long long* keys;
+  int32_t* vals;
+  uint32_t mask;
+};
+constexpr int kGlobalMemoBits = 16;
 cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
-                         int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st);
+                         int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st,
+                         const GlobalMemo* gm = nullptr);
 
 // Compaction: copies the live part of a tree (everything reachable from the root) into fresh arrays, with
 // nodes renumbered in breadth-first order, every live table rehashed at its size without tombstones, and

@@ -211,6 +211,7 @@ struct p2p_router {
   DevBuf cmp_jobs, cmp_queue;          // device compaction
   DevBuf upd_cnt, upd_op, upd_sb, upd_so, upd_sl;  // a routed batch as an INSERT delta (p2p_update_estimates)
   DevBuf lru_buf;                                   // scratch of the LRU calls
+  DevBuf gmemo;                                     // the delta kernel's launch-wide verified-run table
   std::vector<uint8_t> lru;                         // per tree: kept as an LRU cache (p2p_lru_enable)
   std::vector<int64_t> lru_time;                    // per LRU tree: the time of its last insert or access
   int64_t launches = 0;  // kernels this router has launched
@@ -979,7 +980,7 @@ void p2p_router_destroy(p2p_router* r) {
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
                       &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue,
-                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl, &r->lru_buf})
+                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl, &r->lru_buf, &r->gmemo})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -1212,6 +1213,13 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
   CK(p2p::launch_init_ranges(r->d_states + p0, nt, peer == -1 ? d_pb : nullptr, n, r->stream));
   if (n) CK(cudaMemsetAsync(done, 0, (size_t)n, r->stream));
   r->launches += 1;
+  // The launch-wide verified-run table, cleared for this call (labels and the pool do not change during it).
+  const size_t gslots = (size_t)1 << p2p::kGlobalMemoBits;
+  CK(ensure(r, r->gmemo, gslots * (sizeof(unsigned long long) + sizeof(int32_t))));
+  p2p::GlobalMemo gm{static_cast<unsigned long long*>(r->gmemo.p),
+                     reinterpret_cast<int32_t*>(static_cast<unsigned long long*>(r->gmemo.p) + gslots),
+                     (uint32_t)(gslots - 1)};
+  CK(cudaMemsetAsync(r->gmemo.p, 0, gslots * (sizeof(unsigned long long) + sizeof(int32_t)), r->stream));
   int rc = P2P_OK;
   for (int round = 0;; ++round) {
     if (round == 64) {
@@ -1221,7 +1229,7 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
     if (round == 0)
       if (int rc = prepare_scratch(r)) return rc;
     CK(p2p::launch_delta(r->d_states + p0, done, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->d_shared,
-                         r->stream));
+                         r->stream, &gm));
     if (round == 0)
       if (int rc = launch_prepared(r)) return rc;  // a prepared batch's grouping overlaps the delta kernel
     r->launches += 1;
