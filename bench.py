@@ -9,8 +9,9 @@ region starts.  The JSON line also carries:
   kernels       every kernel launched in the timed region: launches, device ms per step (the library's kernel
                 clock, CUDA events on the router stream), share, and its DRAM traffic per launch where an ncu
                 capture of the same kernel source gave one;
-  roofline      the stage that takes the most time -- the delta kernel, or the route step's launches --
-                against the measured HBM copy bandwidth: achieved = algorithmic bytes per launch / device time.
+  roofline      the delta kernel when it is the kernel with the most device time, else the route step's launches
+                taken together, against the measured HBM copy bandwidth: achieved = algorithmic bytes per launch /
+                device time.
                 The delta kernel's algorithmic bytes are the oracle's per-op counters (input, walk, writes);
                 the route step's are its compulsory bytes (request tokens and offsets read once, the match
                 matrix and peers written once).  `traffic` is ncu's DRAM bytes for that kernel;
@@ -510,7 +511,10 @@ def run_ours(args):
         # ---- the roofline of the stage that takes the most time ----
         roof = None
         delta_k = kt.get("delta_kernel")
-        if delta_k and delta_k["ms_per_step"] >= route_k_ms and has_delta:
+        # The kernel with the most device time per step.  With the grouping running alongside the delta kernel
+        # (scale workload), the route kernels' device times overlap it and are not summed against it.
+        dominant = max(kernels, key=lambda k: k["ms_per_step"])["kernel"] if kernels else None
+        if delta_k and has_delta and dominant == "delta_kernel":
             n_ops_step = len(host_delta0.op)
             per_op, counted = delta_op_bytes(otrees, host_delta0, counted_share, n_cpu) if want_oracle else (0.0, 0)
             if counted:
