@@ -645,7 +645,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     __syncwarp();
     return OP_DONE;
   }
-  int32_t cur = 0, par = -1;
+  int32_t cur = 0, par = -1, gpar = -1;
   int4 *e_cur = nullptr, *e_par = nullptr;
   int64_t pos = 0;
   int4 nd = root, pn = root;  // records of cur and par (below the root and the anchor only this warp writes them)
@@ -675,6 +675,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
       return OP_DONE;
     }
     e_par = e_cur;
+    gpar = par;
     par = cur;
     pn = nd;
     e_cur = ent;
@@ -707,7 +708,11 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     return OP_DONE;
   }
   // A leaf that stores nothing any more: tombstone its slot in the parent's table.  (pn is only read when
-  // par is not the root.)
+  // par is not the root.)  A parent that stores nothing and has this leaf as its only child (a node an upload
+  // put in front of a label's own rest, or an LRU access's split) would be left empty: it goes too, from its
+  // own parent's table.
+  const bool drop_parent = par != 0 && pn.w == 0 && pn.z == 1;
+  if (drop_parent && (gpar < 0 || !e_par)) return anchor >= 0 ? OP_DEFER : OP_CORRUPT;  // (cannot happen)
   const bool fold_parent = par != 0 && pn.w == 0 && pn.z == 2;
   if (fold_parent && par == anchor) return OP_DEFER;  // (cannot happen: an anchor keeps >= 3 children)
   int32_t other = -1;
@@ -726,6 +731,14 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   add_stat(&t.g->stale_label, leaf_label, lane);
   add_stat(&t.g->dead_nodes, 1, lane);
   add_stat(&t.g->stale_child, tab_bits(nd.y) ? (int64_t)1 << tab_bits(nd.y) : 0, lane);
+  if (drop_parent) {
+    if (lane == 0) {
+      atomicExch(&e_par->y, -1);
+      atomicAdd(&t.node[gpar].z, -1);
+    }
+    add_stat(&t.g->dead_nodes, 1, lane);
+    add_stat(&t.g->stale_child, tab_bits(pn.y) ? (int64_t)1 << tab_bits(pn.y) : 0, lane);
+  }
   __syncwarp();
   if (fold_parent) fold_child(t, par, e_par, other, l0, lane);
   return OP_DONE;

@@ -49,8 +49,11 @@ int32_t log2_exact(int64_t p) {
   return b;
 }
 // Labels at least this long are interned in the router's shared pool (shorter ones stay in the tree's
-// own arena): the long runs are the shared prompt prefixes that many replicas hold.
+// own arena): the long runs are the shared prompt prefixes that many replicas hold.  Interned runs are also
+// indexed by their first kHeadTokens tokens (a few per head), to find a run that a longer label starts with.
 constexpr int32_t kInternMin = 128;
+constexpr int32_t kHeadTokens = 64;
+constexpr size_t kHeadCandidates = 8;
 
 // 64-bit content hash of a token run (FNV-1a over the 32-bit tokens, then a final avalanche); interning
 // always verifies the content, so a collision only means a run is not shared.
@@ -221,6 +224,8 @@ struct p2p_router {
   int64_t shared_cap = 0;
   std::vector<int32_t> h_shared;
   std::unordered_map<uint64_t, int32_t> intern;
+  // Interned runs by a hash of their first kHeadTokens tokens: (pool offset, length), a few per head.
+  std::unordered_map<uint64_t, std::vector<std::pair<int32_t, int32_t>>> heads;
   std::string err;
 };
 
@@ -489,32 +494,85 @@ int sync_shared_pool(p2p_router* r, int64_t from) {
   return P2P_OK;
 }
 
+// Interns a label of at least kInternMin tokens: an identical run, or a new run (whose head is then indexed).
+// Returns its encoded offset, or 0 with ok = false (the pool is full).
+int32_t intern_label(p2p_router* r, const int32_t* src, int32_t len, bool& ok) {
+  ok = true;
+  const uint64_t h = run_hash(src, len);
+  auto it = r->intern.find(h);
+  if (it != r->intern.end() && (int64_t)it->second + len <= (int64_t)r->h_shared.size() &&
+      std::memcmp(r->h_shared.data() + it->second, src, (size_t)len * sizeof(int32_t)) == 0)
+    return ~it->second;
+  if ((int64_t)r->h_shared.size() + len >= INT32_MAX) {
+    ok = false;
+    return 0;
+  }
+  const int32_t at = (int32_t)r->h_shared.size();
+  r->h_shared.insert(r->h_shared.end(), src, src + len);
+  r->intern.emplace(h, at);
+  auto& hs = r->heads[run_hash(src, kHeadTokens)];
+  if (hs.size() < kHeadCandidates) hs.emplace_back(at, len);
+  return ~at;
+}
+
+// The interned run sharing the longest prefix with src[0 .. len) among those indexed under the same head;
+// k = that prefix's length (0: none).
+int32_t longest_head(const p2p_router* r, const int32_t* src, int32_t len, int32_t& k) {
+  k = 0;
+  int32_t best = 0;
+  auto it = r->heads.find(run_hash(src, kHeadTokens));
+  if (it == r->heads.end()) return 0;
+  for (const auto& [at, rl] : it->second) {
+    const int32_t m = std::min(len, rl);
+    const int32_t* a = r->h_shared.data() + at;
+    const int32_t lcp = (int32_t)(std::mismatch(a, a + m, src).first - a);
+    if (lcp > k) {
+      k = lcp;
+      best = at;
+    }
+  }
+  return best;
+}
+
 int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
   std::string err;
   if (!p2p::validate_flat(t, err)) return fail(r, P2P_E_FORMAT, err);
   const int64_t N = t->n_nodes, NL = t->n_labels;
   // Labels: long runs are interned in the shared pool (label_off < 0 encodes pool offset ~off), the rest
-  // go to the tree's own arena.
+  // go to the tree's own arena.  A long label whose first part (kInternMin tokens or more) starts an interned
+  // run of another tree -- a prompt prefix that this tree holds with a single suffix, while other trees hold
+  // it with several -- is split there: the edge takes the shared run's start, and a node with one child and
+  // no sequence continues with the rest.  Every tree holding the prefix then points at one copy, so a walk
+  // compares it once for all of them (and the export merges the node back).  A label that is a prefix of an
+  // interned run points at that run.
   const int64_t shared_before = (int64_t)r->h_shared.size();
-  std::vector<int32_t> enc((size_t)N, 0), own;
+  std::vector<int32_t> enc((size_t)N, 0), head_len((size_t)N, 0), tail_enc((size_t)N, 0), own;
   own.reserve((size_t)NL);
+  int64_t n_split = 0;
   for (int64_t v = 1; v < N; ++v) {
     const int32_t* src = t->labels + t->label_off[v];
     const int32_t len = t->label_len[v];
     bool interned = false;
-    if (len >= kInternMin && (int64_t)r->h_shared.size() + len < INT32_MAX) {
-      const uint64_t h = run_hash(src, len);
-      auto it = r->intern.find(h);
-      if (it == r->intern.end()) {
-        const int32_t at = (int32_t)r->h_shared.size();
-        r->h_shared.insert(r->h_shared.end(), src, src + len);
-        r->intern.emplace(h, at);
+    if (len >= kInternMin) {
+      int32_t k = 0;
+      const int32_t at = longest_head(r, src, len, k);
+      if (k == len) {
         enc[(size_t)v] = ~at;
         interned = true;
-      } else if ((int64_t)it->second + len <= (int64_t)r->h_shared.size() &&
-                 std::memcmp(r->h_shared.data() + it->second, src, (size_t)len * sizeof(int32_t)) == 0) {
-        enc[(size_t)v] = ~it->second;
+      } else if (k >= kInternMin) {
+        enc[(size_t)v] = ~at;
+        head_len[(size_t)v] = k;
+        ++n_split;
+        const int32_t rest = len - k;
+        bool ok = false;
+        if (rest >= kInternMin) tail_enc[(size_t)v] = intern_label(r, src + k, rest, ok);
+        if (!ok) {
+          tail_enc[(size_t)v] = (int32_t)own.size();
+          own.insert(own.end(), src + k, src + len);
+        }
         interned = true;
+      } else {
+        enc[(size_t)v] = intern_label(r, src, len, interned);
       }
     }
     if (!interned) {
@@ -523,8 +581,10 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
     }
   }
   if (int rc = sync_shared_pool(r, shared_before)) return rc;
-  // Children tables, laid out in node order in the child arena.
-  std::vector<int32_t> bits((size_t)N), off((size_t)N, 0);
+  // Children tables, laid out in node order in the child arena; the split nodes (ids N ..) after them.
+  const int64_t NN = N + n_split;
+  if (NN > INT32_MAX / 2) return fail(r, P2P_E_NOMEM, "too many nodes");
+  std::vector<int32_t> bits((size_t)NN), off((size_t)NN, 0), split_id((size_t)N, 0);
   int64_t slots = 0;
   for (int64_t v = 0; v < N; ++v) {
     bits[(size_t)v] = table_bits_for(t->child_count[v], v == 0);
@@ -533,18 +593,38 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
     slots += bits[(size_t)v] ? (int64_t)1 << bits[(size_t)v] : 0;
     if (slots > INT32_MAX / 2) return fail(r, P2P_E_NOMEM, "children tables exceed the int32 arena");
   }
-  std::vector<int4> node((size_t)N), child((size_t)slots, make_int4(0, 0, 0, 0));
+  for (int64_t v = 1, x = N; v < N; ++v)
+    if (head_len[(size_t)v]) {
+      split_id[(size_t)v] = (int32_t)x;
+      bits[(size_t)x] = p2p::kMinTabBits;
+      off[(size_t)x] = (int32_t)slots;
+      slots += (int64_t)1 << p2p::kMinTabBits;
+      if (slots > INT32_MAX / 2) return fail(r, P2P_E_NOMEM, "children tables exceed the int32 arena");
+      ++x;
+    }
+  std::vector<int4> node((size_t)NN), child((size_t)slots, make_int4(0, 0, 0, 0));
   for (int64_t v = 0; v < N; ++v) {
     const int32_t cnt = t->child_count[v], b = bits[(size_t)v];
     node[(size_t)v] = make_int4(b ? off[(size_t)v] : 0, p2p::make_meta(b, cnt), cnt, t->term_count[v]);
     for (int64_t e = t->child_begin[v]; e < (int64_t)t->child_begin[v] + cnt; ++e) {
       const int32_t c = t->child_idx[e];
-      table_put(child.data() + off[(size_t)v], b, make_int4(t->child_first_tok[e], c, enc[(size_t)c], t->label_len[c]));
+      const int32_t k = head_len[(size_t)c];
+      if (!k) {
+        table_put(child.data() + off[(size_t)v], b, make_int4(t->child_first_tok[e], c, enc[(size_t)c], t->label_len[c]));
+        continue;
+      }
+      // v -> x (the shared head) -> c (the rest of the label).
+      const int32_t x = split_id[(size_t)c];
+      table_put(child.data() + off[(size_t)v], b, make_int4(t->child_first_tok[e], x, enc[(size_t)c], k));
+      node[(size_t)x] = make_int4(off[(size_t)x], p2p::make_meta(p2p::kMinTabBits, 1), 1, 0);
+      const int32_t* src = t->labels + t->label_off[c];
+      table_put(child.data() + off[(size_t)x], p2p::kMinTabBits,
+                make_int4(src[k], c, tail_enc[(size_t)c], t->label_len[c] - k));
     }
   }
   const int64_t n_own = (int64_t)own.size();
   // Headroom for device deltas (no regrowth for a few anti-entropy rounds of a few percent each).
-  const int32_t cap_node = clamp_i32(2 * N + 1024);
+  const int32_t cap_node = clamp_i32(2 * NN + 1024);
   const int32_t cap_child = clamp_i32(2 * slots + 1024);
   const int32_t cap_label = std::max(label_cap(n_own), clamp_i32(n_own + NL / 2));
   TreeState nt;
@@ -564,10 +644,10 @@ int upload_flat(p2p_router* r, int32_t peer, const p2p_flat_tree* t) {
       (void)cudaGetLastError();
     }
   }
-  CK(cudaMemcpyAsync(nt.node, node.data(), (size_t)N * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
+  CK(cudaMemcpyAsync(nt.node, node.data(), (size_t)NN * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   if (slots) CK(cudaMemcpyAsync(nt.child, child.data(), (size_t)slots * sizeof(int4), cudaMemcpyHostToDevice, r->stream));
   if (n_own) CK(cudaMemcpyAsync(nt.label, own.data(), (size_t)n_own * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
-  nt.n_node = (int32_t)N;
+  nt.n_node = (int32_t)NN;
   nt.n_child = (int32_t)slots;
   nt.n_label = (int32_t)n_own;
   // The root's first-token filter: exactly the root's children now.

@@ -270,3 +270,36 @@ def test_compaction_takes_trees_near_the_threshold_along():
     assert r.stats(0)["label_tokens"] == (n - 1200) * L and r.stats(1)["label_tokens"] == (n - 840) * L
     for p in range(3):
         assert same_snapshot(r.download(p), ots[p].export()), p
+
+
+def test_shared_heads_split_at_upload_then_patched():
+    """A long label that starts with another tree's interned run (a prompt held with one suffix here and with
+    several there) is uploaded as that run's start plus a node with one child: the trees export canonically,
+    route like the oracle, and deltas that delete and re-insert through such nodes stay exact."""
+    rng = np.random.default_rng(41)
+    prompt = rng.integers(0, 30000, size=300).tolist()
+    a = [prompt + [1, 2, 3], prompt + [4, 5]]
+    b = [prompt + [7, 8, 9, 10]]
+    c = [prompt[:200] + [11] * 50, prompt + [7, 8]]
+    trees = [a, b, c]
+    r = router_from_seqlists([seqlist_from_lists(t) for t in trees])
+    o = oracle.build_trees([seqlist_from_lists(t) for t in trees])
+    assert r.stats(1)["live_nodes"] == 3  # root, the shared head's node, the leaf
+    for p in range(3):
+        assert same_snapshot(r.download(p), o[p].export()), p
+    reqs = [prompt + [7, 8, 9], prompt[:250], prompt + [4], prompt[:200] + [11, 11], [5]]
+    tok, off = csr_from_lists(reqs)
+    gm, gp = route_device(r, tok, off, [0, 0, 0], 0)
+    om, op_, _ = oracle.route(o, tok, off, [0, 0, 0], 0)
+    assert_same_route(gm, gp, om, op_, "shared heads")
+    # Delete the only sequence of tree 1 (its head node goes too), then insert through tree 2's heads.
+    for p, ops, seqs in ((1, [1], [b[0]]), (2, [0, 1, 0], [prompt + [7], prompt + [7, 8], prompt[:100]])):
+        sl = seqlist_from_lists(seqs)
+        opa = np.array(ops, np.int32)
+        assert r.apply_delta(p, opa, sl) == 0
+        o[p].apply_ops(opa, sl)
+        assert same_snapshot(r.download(p), o[p].export()), p
+    assert r.stats(1)["live_nodes"] == 1
+    gm, gp = route_device(r, tok, off, [0, 0, 0], 0)
+    om, op_, _ = oracle.route(o, tok, off, [0, 0, 0], 0)
+    assert_same_route(gm, gp, om, op_, "shared heads after deltas")
