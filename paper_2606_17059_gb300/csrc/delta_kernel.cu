@@ -645,7 +645,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     __syncwarp();
     return OP_DONE;
   }
-  int32_t cur = 0, par = -1, gpar = -1;
+  int32_t cur = 0, par = -1, gpar = -1, s_gpar = -1;  // s_gpar: gpar's slot in its parent's table
   int4 *e_cur = nullptr, *e_par = nullptr;
   int64_t pos = 0;
   int4 nd = root, pn = root;  // records of cur and par (below the root and the anchor only this warp writes them)
@@ -674,6 +674,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
       add_stat(&t.g->n_absent, 1, lane);
       return OP_DONE;
     }
+    s_gpar = e_par ? (int32_t)(e_par - t.child) : -1;
     e_par = e_cur;
     gpar = par;
     par = cur;
@@ -711,6 +712,10 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   // par is not the root.)  A parent that stores nothing and has this leaf as its only child (a node an upload
   // put in front of a label's own rest, or an LRU access's split) would be left empty: it goes too, from its
   // own parent's table.
+  // The parent goes too when it would be left empty: it stores nothing and this leaf is its only child (an
+  // upload's node in front of a label's own rest).  Its own parent gpar then loses a child, and like any node
+  // left with one child and no sequence it takes that child in (so no chain of such nodes ever forms, and a
+  // removal never has to climb more than this one level).
   const bool drop_parent = par != 0 && pn.w == 0 && pn.z == 1;
   if (drop_parent && (gpar < 0 || !e_par)) return anchor >= 0 ? OP_DEFER : OP_CORRUPT;  // (cannot happen)
   const bool fold_parent = par != 0 && pn.w == 0 && pn.z == 2;
@@ -721,6 +726,18 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
     if (other < 0) return OP_CORRUPT;
     const int4 oe = t.child[other];
     const int64_t need = adjacent(*e_par, oe) ? 0 : (int64_t)e_par->w + oe.w;
+    if (!take(t, 0, 0, need, n0, c0, l0, lane)) return OP_NEED;
+  }
+  // gpar below the anchor (or in the serial phase) is this warp's alone; an anchor keeps >= 3 children.
+  int4 gpn = make_int4(0, 0, 0, 0);
+  if (drop_parent && gpar != 0 && gpar != anchor) gpn = t.node[gpar];
+  const bool fold_gpar = drop_parent && gpar != 0 && gpar != anchor && gpn.w == 0 && gpn.z == 2;
+  if (fold_gpar) {
+    if (s_gpar < 0) return anchor >= 0 ? OP_DEFER : OP_CORRUPT;  // (cannot happen: gpar was reached by a slot)
+    other = only_child(t, gpn.x, tab_bits(gpn.y), (int32_t)(e_par - t.child), lane);
+    if (other < 0) return OP_CORRUPT;
+    const int4 oe = t.child[other], ge = t.child[s_gpar];
+    const int64_t need = adjacent(ge, oe) ? 0 : (int64_t)ge.w + oe.w;
     if (!take(t, 0, 0, need, n0, c0, l0, lane)) return OP_NEED;
   }
   const int32_t leaf_label = e_cur->w;
@@ -741,6 +758,7 @@ __device__ int remove(Tree& t, const Seq& q, const int4& root, int32_t anchor, i
   }
   __syncwarp();
   if (fold_parent) fold_child(t, par, e_par, other, l0, lane);
+  if (fold_gpar) fold_child(t, gpar, t.child + s_gpar, other, l0, lane);
   return OP_DONE;
 }
 

@@ -303,3 +303,26 @@ def test_shared_heads_split_at_upload_then_patched():
     gm, gp = route_device(r, tok, off, [0, 0, 0], 0)
     om, op_, _ = oracle.route(o, tok, off, [0, 0, 0], 0)
     assert_same_route(gm, gp, om, op_, "shared heads after deltas")
+
+
+def test_deleting_through_two_shared_heads_under_one_node():
+    """Two prompts with the same first token, each held with one suffix: the node of their common first token
+    has two upload-split children.  Deleting both sequences in one delta empties the tree (the node left with
+    one such child takes it in, then goes with the last deletion)."""
+    rng = np.random.default_rng(43)
+    p1 = [7] + rng.integers(0, 30000, size=299).tolist()
+    p2 = [7] + rng.integers(0, 30000, size=299).tolist()
+    a = [p1 + [1], p1 + [2], p2 + [3], p2 + [4]]
+    b = [p1 + [5, 6], p2 + [8, 9]]
+    r = router_from_seqlists([seqlist_from_lists(a), seqlist_from_lists(b)])
+    assert r.stats(1)["live_nodes"] == 6  # root, the first token's node, two head nodes, two leaves
+    for order in ([0, 1], [1, 0]):
+        sl = seqlist_from_lists([b[i] for i in order])
+        assert r.apply_delta(1, np.array([1, 1], np.int32), sl) == 0
+        d = r.download(1)
+        assert d["label_off"].tolist() == [0] and d["term_count"].tolist() == [0]
+        reqs = [p1 + [5], p2[:10], [7]]
+        tok, off = csr_from_lists(reqs)
+        gm, _ = route_device(r, tok, off, [0, 0], 0)
+        assert (gm[:, 1] == 0).all()
+        assert r.apply_delta(1, np.zeros(2, np.int32), seqlist_from_lists(b)) == 0  # back for the next order
