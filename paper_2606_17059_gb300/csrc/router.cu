@@ -1327,40 +1327,49 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
     if (rc != P2P_OK || !again) break;
     if (int e = push_states(r, p0, p1)) return e;
   }
-  // Room ahead of the next call: a tree (not about to be compacted) whose free room in an arena is below
-  // twice what this call used there is grown now, so the next call's kernel does not stop for room.
-  for (int32_t p = p0; p < p1 && rc == P2P_OK; ++p) {
-    TreeState& t = r->hs[(size_t)p];
-    if (needs_compaction(t)) continue;
+  // Room ahead of the next call: free room in an arena below twice what this call used there.  Such a tree is
+  // grown now, so the next call's kernel does not stop for room -- unless it is compacted in this call.
+  // A wave of compaction starts when a tree is past the threshold, or when a tree near it is short of room
+  // (compaction hands it arrays with headroom, where growth would copy its stale space only to be replaced by
+  // a compaction a call or two later); every tree near the threshold goes along.
+  std::vector<int4> short_of((size_t)nt, make_int4(0, 0, 0, 0));  // (node, child, label room wanted, any)
+  bool wave = false;
+  for (int32_t p = p0; p < p1; ++p) {
+    const TreeState& t = r->hs[(size_t)p];
     const int4 b = before[(size_t)(p - p0)];
     const int64_t dn = 2 * std::max<int64_t>((int64_t)t.n_node - b.x, 0);
     const int64_t dc = 2 * std::max<int64_t>((int64_t)t.n_child - b.y, 0);
     const int64_t dl = 2 * std::max<int64_t>((int64_t)t.n_label - b.z, 0);
     const bool short_n = (int64_t)t.cap_node - t.n_node < dn, short_c = (int64_t)t.cap_child - t.n_child < dc,
                short_l = (int64_t)t.cap_label - t.n_label < dl;
-    if (!short_n && !short_c && !short_l) continue;
-    t.need_node = short_n ? clamp_i32(dn) : 0;
-    t.need_child = short_c ? clamp_i32(dc) : 0;
-    t.need_label = short_l ? clamp_i32(dl) : 0;
+    const bool is_short = short_n || short_c || short_l;
+    short_of[(size_t)(p - p0)] = make_int4(short_n ? clamp_i32(dn) : 0, short_c ? clamp_i32(dc) : 0,
+                                           short_l ? clamp_i32(dl) : 0, is_short);
+    wave = wave || needs_compaction(t) || (is_short && nears_compaction(t));
+  }
+  std::vector<int32_t> stale;
+  for (int32_t p = p0; wave && p < p1; ++p)
+    if (nears_compaction(r->hs[(size_t)p])) stale.push_back(p);  // (a tree past the threshold is near it)
+  for (int32_t p = p0, k = 0; p < p1 && rc == P2P_OK; ++p) {
+    if (k < (int32_t)stale.size() && stale[(size_t)k] == p) {
+      ++k;
+      continue;
+    }
+    const int4 s = short_of[(size_t)(p - p0)];
+    if (!s.w) continue;
+    TreeState& t = r->hs[(size_t)p];
+    t.need_node = s.x;
+    t.need_child = s.y;
+    t.need_label = s.z;
     t.need_root = 0;
     rc = grow_tree(r, p);
   }
-  // Publish the (possibly moved) arrays to the route kernel's view table; compact very stale trees.
+  // Publish the (possibly moved) arrays to the route kernel's view table; compact the stale trees.
   if (int e = push_states(r, p0, p1)) return e;
   CK(p2p::launch_refresh_views(r->d_states + p0, r->d_views + p0, nt, r->d_shared, r->stream));
   r->launches += 1;
   int64_t absent = 0;
-  std::vector<int32_t> stale;
-  for (int32_t p = p0; p < p1; ++p) {
-    const TreeState& t = r->hs[(size_t)p];
-    absent += t.n_absent;
-    if (needs_compaction(t)) stale.push_back(p);
-  }
-  if (!stale.empty()) {
-    stale.clear();
-    for (int32_t p = p0; p < p1; ++p)
-      if (nears_compaction(r->hs[(size_t)p])) stale.push_back(p);
-  }
+  for (int32_t p = p0; p < p1; ++p) absent += r->hs[(size_t)p].n_absent;
   if (rc == P2P_OK) rc = compact_trees(r, stale, p0, p1);
   if (n_absent) *n_absent = absent;
   return rc;
