@@ -74,7 +74,20 @@ KERNEL_SOURCE = {
 # DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum) per workload and kernel, with the
 # source hash of the capture and the profile summary that holds the command.  A figure whose source hash
 # differs from the current source is not reported (the kernel changed since it was taken).
-TRAFFIC: dict = {}
+TRAFFIC: dict = {
+    "cfg4": {k: dict(v, profile="profiles/traffic_workload4.md") for k, v in {
+        "delta_kernel": {"bytes": 6722429107, "source": "0b558fa44276b221"},
+        "validate_kernel": {"bytes": 98813542, "source": "0b558fa44276b221"},
+        "compact_kernel": {"bytes": 10288611840, "source": "0b558fa44276b221"},
+        "compact_labels_kernel": {"bytes": 24294580224, "source": "0b558fa44276b221"},
+        "group_hash_kernel": {"bytes": 491260902, "source": "c540f29ec07fe042"},
+        "group_resolve32_kernel": {"bytes": 9457387801, "source": "c540f29ec07fe042"},
+        "group_ranges_kernel": {"bytes": 4005196, "source": "c540f29ec07fe042"},
+        "group_place_kernel": {"bytes": 8145356, "source": "c540f29ec07fe042"},
+        "lane_kernel<true>": {"bytes": 6160865945, "source": "78aca06860acc42f"},
+        "lane_kernel<false>": {"bytes": 17196897484, "source": "78aca06860acc42f"},
+    }.items()},
+}
 
 
 def source_hash(kernel: str) -> str | None:
