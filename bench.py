@@ -69,7 +69,7 @@ KERNEL_SOURCE = {
     "update_scatter_kernel": "update_kernel.cu", "group_ranges_kernel": "group_kernel.cu",
     "group_place_kernel": "group_kernel.cu", "lru_walk_kernel": "lru_kernel.cu", "lru_stamp_kernel": "lru_kernel.cu",
     "lru_order_kernels": "lru_kernel.cu", "lru_count_kernel": "lru_kernel.cu", "lru_evict_kernel": "lru_kernel.cu",
-    "lru_ops_kernel": "lru_kernel.cu", "hit_rate_kernel": "lru_kernel.cu",
+    "lru_ops_kernel": "lru_kernel.cu", "hit_rate_kernel": "lru_kernel.cu", "room_kernel": "delta_kernel.cu",
 }
 # DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum) per workload and kernel, with the
 # source hash of the capture and the profile summary that holds the command.  A figure whose source hash

@@ -46,7 +46,7 @@ enum {
 };
 
 enum { P2P_OP_INSERT = 0, P2P_OP_DELETE = 1 };
-enum { P2P_KERNEL_COUNT = 26 }; /* kernels the kernel clock keeps totals for */
+enum { P2P_KERNEL_COUNT = 27 }; /* kernels the kernel clock keeps totals for */
 enum { P2P_MEM_HOST = 0, P2P_MEM_DEVICE = 1 };
 
 typedef struct p2p_router p2p_router;

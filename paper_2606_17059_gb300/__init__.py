@@ -204,7 +204,7 @@ def p2p_router_launch_count(r) -> int:
     return int(_load().p2p_router_launch_count(r))
 
 
-KERNEL_COUNT = 26  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 25)
+KERNEL_COUNT = 27  # P2P_KERNEL_COUNT: kernels the kernel clock keeps totals for (indices 0 .. 26)
 
 
 def p2p_router_kernel_clock(r, on: bool) -> None:

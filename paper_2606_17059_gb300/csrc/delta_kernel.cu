@@ -1159,6 +1159,44 @@ __global__ void validate_kernel(int32_t* header, const int32_t* __restrict__ op,
   }
 }
 
+// After a launch that stopped for room: for each tree flagged DELTA_NEED_SPACE, the room its ops not yet
+// applied may take -- every remaining INSERT's whole sequence as new label tokens, and the number of those
+// INSERTs -- so that the host grows the tree once for the rest of the call instead of once per doubling.
+// room[2 * i] = tokens, room[2 * i + 1] = INSERTs (0 for a tree that did not stop).  One CTA per tree.
+__global__ void room_kernel(const TreeState* __restrict__ states, const uint8_t* __restrict__ done,
+                            const int32_t* __restrict__ op, const int64_t* __restrict__ seg_begin,
+                            const int32_t* __restrict__ seg_len, long long* room) {
+  const TreeState& s = states[blockIdx.x];
+  long long tokens = 0, inserts = 0;
+  if (s.status & DELTA_NEED_SPACE) {
+    for (int64_t i = s.op_begin + threadIdx.x; i < s.op_end; i += blockDim.x) {
+      if (done[i] || op[i] != P2P_OP_INSERT) continue;
+      for (int64_t g = seg_begin[i]; g < seg_begin[i + 1]; ++g) tokens += seg_len[g];
+      inserts += 1;
+    }
+  }
+  for (int o = 16; o > 0; o >>= 1) {
+    tokens += __shfl_xor_sync(kFull, tokens, o);
+    inserts += __shfl_xor_sync(kFull, inserts, o);
+  }
+  __shared__ long long s_sum[2][32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) {
+    s_sum[0][warp] = tokens;
+    s_sum[1][warp] = inserts;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    long long a = 0, b = 0;
+    for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+      a += s_sum[0][w];
+      b += s_sum[1][w];
+    }
+    room[2 * blockIdx.x] = a;
+    room[2 * blockIdx.x + 1] = b;
+  }
+}
+
 // Sets each tree's op range for this call on the device (peer_begin stays in device memory).
 __global__ void init_ranges_kernel(TreeState* states, int32_t nt, const int64_t* __restrict__ peer_begin, int64_t n) {
   const int32_t i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -1474,6 +1512,13 @@ cudaError_t launch_validate(int32_t* header, const p2p_delta* d, int32_t peer, i
             (validate_kernel<<<(int)std::max<int64_t>(blocks, 1), 256, 0, st>>>(
                 header, d->op, S.seg_begin, S.seg_off, S.seg_len, S.n, S.n_segs, S.n_pool,
                 peer == -1 ? d->peer_begin : nullptr, P)));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_room(const TreeState* d_states, int32_t nt, const uint8_t* done, const int32_t* op,
+                        const int64_t* seg_begin, const int32_t* seg_len, long long* room, cudaStream_t st) {
+  if (nt <= 0) return cudaSuccess;
+  P2P_TIMED(K_ROOM, st, (room_kernel<<<nt, 256, 0, st>>>(d_states, done, op, seg_begin, seg_len, room)));
   return cudaGetLastError();
 }
 

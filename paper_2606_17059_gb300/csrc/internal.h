@@ -108,7 +108,7 @@ enum KernelId {
   K_GROUP_HASH, K_GROUP_RESOLVE, K_GROUP_RESOLVE32, K_ROUTE_STAGED, K_LANE_LEADER, K_LANE_FOLLOWER, K_DECIDE,
   K_VALIDATE, K_INIT_RANGES, K_DELTA, K_COMPACT, K_COMPACT_LABELS, K_REFRESH_VIEWS, K_SET_TREE,
   K_UPDATE_COUNT, K_UPDATE_SCAN, K_UPDATE_SCATTER, K_GROUP_RANGES, K_GROUP_PLACE, K_LRU_WALK, K_LRU_STAMP,
-  K_LRU_ORDER, K_LRU_SELECT, K_LRU_EVICT, K_LRU_OPS, K_HIT_RATE, K_COUNT_
+  K_LRU_ORDER, K_LRU_SELECT, K_LRU_EVICT, K_LRU_OPS, K_HIT_RATE, K_ROOM, K_COUNT_
 };
 static_assert((int)K_COUNT_ == (int)P2P_KERNEL_COUNT, "the header's kernel count");
 const char* kernel_name(int id);
@@ -231,6 +231,10 @@ cudaError_t static_scratch(int device, int32_t** header, int32_t** tokens);
 // [0..1] longest sequence (u64), [2] STATIC_* error bits, [3] most pool runs of one op.
 cudaError_t launch_validate(int32_t* header, const p2p_delta* d, int32_t peer, int32_t P, cudaStream_t st);
 cudaError_t launch_init_ranges(TreeState* d_states, int32_t nt, const int64_t* peer_begin, int64_t n, cudaStream_t st);
+// Per tree that stopped for room (DELTA_NEED_SPACE): room[2i] = label tokens and room[2i + 1] = INSERTs of its ops
+// not yet applied (upper bounds of the room the rest of the call takes).
+cudaError_t launch_room(const TreeState* d_states, int32_t nt, const uint8_t* done, const int32_t* op,
+                        const int64_t* seg_begin, const int32_t* seg_len, long long* room, cudaStream_t st);
 constexpr int kStaticHeaderInts = 64;
 
 // A routed batch as a device-resident INSERT delta (update_kernel.cu).  counts [P] must be zero and bad [1]

@@ -93,7 +93,7 @@ const char* kernel_name(int id) {
       "compact_kernel", "compact_labels_kernel", "refresh_views_kernel", "set_tree_kernel", "update_count_kernel",
       "update_scan_kernel", "update_scatter_kernel", "group_ranges_kernel", "group_place_kernel", "lru_walk_kernel",
       "lru_stamp_kernel", "lru_order_kernels", "lru_count_kernel", "lru_evict_kernel", "lru_ops_kernel",
-      "hit_rate_kernel"};
+      "hit_rate_kernel", "room_kernel"};
   return id >= 0 && id < K_COUNT_ ? names[id] : "";
 }
 
@@ -215,6 +215,7 @@ struct p2p_router {
   DevBuf upd_cnt, upd_op, upd_sb, upd_so, upd_sl;  // a routed batch as an INSERT delta (p2p_update_estimates)
   DevBuf lru_buf;                                   // scratch of the LRU calls
   DevBuf gmemo;                                     // the delta kernel's launch-wide verified-run table
+  DevBuf d_room;                                    // room bounds of the trees that stopped (room_kernel)
   std::vector<uint8_t> lru;                         // per tree: kept as an LRU cache (p2p_lru_enable)
   std::vector<int64_t> lru_time;                    // per LRU tree: the time of its last insert or access
   int64_t launches = 0;  // kernels this router has launched
@@ -714,10 +715,12 @@ int regrow_root(p2p_router* r, int32_t p, int64_t extra = 0) {
   return P2P_OK;
 }
 
-// Grows the arenas of tree p so that the largest op that did not fit does.
-int grow_tree(p2p_router* r, int32_t p) {
+// Grows the arenas of tree p so that the largest op that did not fit does (at least doubling them), or, with
+// whole, so that need_* -- the room the rest of the call may take -- fits with an eighth to spare.
+int grow_tree(p2p_router* r, int32_t p, bool whole = false) {
   TreeState& t = r->hs[(size_t)p];
-  auto newcap = [](int64_t cap, int64_t used, int64_t need) -> int64_t {
+  auto newcap = [whole](int64_t cap, int64_t used, int64_t need) -> int64_t {
+    if (whole) return std::max<int64_t>(cap, used + need + std::max<int64_t>(need / 8, 1024));
     return std::max<int64_t>(cap * 2, used + 2 * need + 1024);
   };
   bool grow_n = (int64_t)t.cap_node - t.n_node < t.need_node;
@@ -1060,7 +1063,8 @@ void p2p_router_destroy(p2p_router* r) {
     for (DevBuf* b : {&r->req_tok, &r->req_off, &r->out_match, &r->out_peer, &r->d_op, &r->d_seg_begin,
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
                       &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue,
-                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl, &r->lru_buf, &r->gmemo})
+                      &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl, &r->lru_buf, &r->gmemo,
+                      &r->d_room})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -1301,6 +1305,7 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
                      (uint32_t)(gslots - 1)};
   CK(cudaMemsetAsync(r->gmemo.p, 0, gslots * (sizeof(unsigned long long) + sizeof(int32_t)), r->stream));
   int rc = P2P_OK;
+  bool sized = false;  // the room of the rest of the call was bounded once (room_kernel)
   for (int round = 0;; ++round) {
     if (round == 64) {
       rc = fail(r, P2P_E_NOMEM, "delta did not fit after 64 arena growths");
@@ -1314,13 +1319,39 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
       if (int rc = launch_prepared(r)) return rc;  // a prepared batch's grouping overlaps the delta kernel
     r->launches += 1;
     if (int e = pull_states(r, p0, p1)) return e;
-    bool again = false;
+    bool again = false, stopped = false;
+    for (int32_t p = p0; p < p1; ++p) stopped = stopped || (r->hs[(size_t)p].status & p2p::DELTA_NEED_SPACE);
+    // The first stop for room: the room every op not yet applied may take, per tree (room_kernel), so that a
+    // tree is grown once for the rest of the call (a delta that brings many new sequences to one tree would
+    // otherwise stop at every doubling).  The bound counts INSERTs only; a later stop (a DELETE's fold needs
+    // label room too) grows by the largest op that did not fit, as before.
+    std::vector<long long> room;
+    if (stopped && !sized) {
+      sized = true;
+      CK(ensure(r, r->d_room, (size_t)nt * 2 * sizeof(long long)));
+      CK(p2p::launch_room(r->d_states + p0, nt, done, d_op, d_sb, d_sl, static_cast<long long*>(r->d_room.p),
+                          r->stream));
+      r->launches += 1;
+      room.resize((size_t)nt * 2);
+      CK(d2h(r, room.data(), r->d_room.p, room.size() * sizeof(long long)));
+    }
     for (int32_t p = p0; p < p1 && rc == P2P_OK; ++p) {
       TreeState& t = r->hs[(size_t)p];
       if (t.status & p2p::DELTA_CORRUPT) {
         rc = fail(r, P2P_E_DEVICE, "tree " + std::to_string(p) + " is inconsistent");
       } else if (t.status & p2p::DELTA_NEED_SPACE) {
-        rc = grow_tree(r, p);
+        bool whole = false;
+        if (!room.empty()) {
+          const long long tok = room[(size_t)(p - p0) * 2], ins = room[(size_t)(p - p0) * 2 + 1];
+          const auto bound = [](long long want, int32_t used) {
+            return (int32_t)std::min<long long>(want, (long long)INT32_MAX / 2 - used);
+          };
+          if (t.need_label) t.need_label = std::max(t.need_label, bound(tok, t.n_label));
+          if (t.need_node) t.need_node = std::max(t.need_node, bound(2 * ins + 64, t.n_node));
+          if (t.need_child) t.need_child = std::max(t.need_child, bound(8 * ins + 1024, t.n_child));
+          whole = true;
+        }
+        rc = grow_tree(r, p, whole);
         again = true;
       }
     }
