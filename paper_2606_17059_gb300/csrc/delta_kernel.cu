@@ -886,7 +886,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
                  const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
                  const int32_t* __restrict__ seg_len, const int32_t* __restrict__ pool, int32_t* gather,
                  int64_t stride, const int32_t* shared, unsigned long long* gmemo_keys, int32_t* gmemo_vals,
-                 uint32_t gmemo_mask) {
+                 uint32_t gmemo_mask, const int32_t* __restrict__ parts) {
   // The chunk's per-op and per-anchor arrays, in dynamic shared memory (delta_smem_bytes()).
   extern __shared__ __align__(16) unsigned char s_dyn[];
   AnchorEntry* s_aentry = reinterpret_cast<AnchorEntry*>(s_dyn);        // per anchor: its shortcut
@@ -909,7 +909,13 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   __shared__ int2 s_slab[kDeltaWarps][3];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   if (lane < 3) s_slab[warp][lane] = make_int2(0, 0);
-  TreeState* gs = states + blockIdx.x;
+  // This CTA's tree, and its part of the tree's ops: the ops whose first-token bucket is `part` modulo
+  // `nparts` (kDeltaBuckets buckets).  Ops with different first tokens touch disjoint subtrees and, of the
+  // root, only its table, whose claims and counts are atomic; so the CTAs of one tree never touch the same
+  // node below the root, and all ops on one sequence stay in one CTA, in op order.
+  const int32_t pw = parts ? parts[blockIdx.x] : (int32_t)blockIdx.x;
+  const int32_t part = parts ? (pw >> kPartShift) & 31 : 0, nparts = parts ? (pw >> kNpartShift) & 63 : 1;
+  TreeState* gs = states + (parts ? (pw & kPartTreeMask) : pw);
   if (lane < kMemoSlots) s_memo[warp][lane] = MemoEntry{nullptr, nullptr, 0};
   const int64_t op_begin = gs->op_begin, op_end = gs->op_end;
   if (threadIdx.x == 0) s_any = 0;
@@ -960,7 +966,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
         n += seg_len[g];
       }
       s_bucket[j] = (int8_t)b;
-      uint8_t fl = done[i] ? F_DONE : 0;
+      uint8_t fl = done[i] || b % nparts != part ? F_DONE : 0;  // another CTA's op: done as far as this one goes
       if (!fl && !s_stop[b]) {
         int32_t anchor, next_tok;
         find_anchor(t, root, seg_off, seg_len, pool, g0, g1, n, anchor, next_tok);
@@ -1491,15 +1497,15 @@ cudaError_t launch_compact(CompactJob* d_jobs, int32_t n_jobs, int32_t max_cap_n
 cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st,
-                         const GlobalMemo* gm) {
+                         const GlobalMemo* gm, const int32_t* parts, int32_t n_blocks) {
   if (n_trees <= 0) return cudaSuccess;
   const int dyn = delta_smem_bytes();
   cudaError_t e = cudaFuncSetAttribute(delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
   if (e != cudaSuccess) return e;
   P2P_TIMED(K_DELTA, st,
-            (delta_kernel<<<n_trees, kDeltaWarps * 32, dyn, st>>>(
+            (delta_kernel<<<parts ? n_blocks : n_trees, kDeltaWarps * 32, dyn, st>>>(
                 d_states, done, op, seg_begin, seg_off, seg_len, pool, gather, gather_stride, shared,
-                gm ? gm->keys : nullptr, gm ? gm->vals : nullptr, gm ? gm->mask : 0u)));
+                gm ? gm->keys : nullptr, gm ? gm->vals : nullptr, gm ? gm->mask : 0u, parts)));
   return cudaGetLastError();
 }
 

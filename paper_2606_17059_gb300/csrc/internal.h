@@ -172,9 +172,11 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
                          cudaStream_t st, int* launched, bool decide = false, int32_t* out_next = nullptr);
 
 // Delta kernel: applies the ops [op_begin, op_end) of states[0 .. n_trees), one CTA of kDeltaWarps warps
-// per tree.  done[i] (one byte per op of the call, zero before the first launch, kept across relaunches)
-// marks the ops applied so far.  gather (n_trees * kDeltaWarps * gather_stride tokens) is needed only when
-// an op's sequence has more than two pool runs; otherwise it may be NULL.
+// per tree, or per part of a tree: with parts (n_blocks words, one per CTA: tree | part << kPartShift |
+// nparts << kNpartShift) a tree's ops are split among nparts CTAs by first-token bucket modulo nparts
+// (1 <= nparts <= kDeltaBuckets).  done[i] (one byte per op of the call, zero before the first launch, kept
+// across relaunches) marks the ops applied so far.  gather (CTAs * kDeltaWarps * gather_stride tokens) is
+// needed only when an op's sequence has more than two pool runs; otherwise it may be NULL.
 // A launch-wide table of verified (interned label, pool run) equalities (keys all zero before a call's first
 // launch; keys [mask + 1], vals [mask + 1]).  NULL: none (the allocation-free call).
 struct GlobalMemo {
@@ -186,7 +188,10 @@ constexpr int kGlobalMemoBits = 16;
 cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, const int32_t* op,
                          const int64_t* seg_begin, const int64_t* seg_off, const int32_t* seg_len, const int32_t* pool,
                          int32_t* gather, int64_t gather_stride, const int32_t* shared, cudaStream_t st,
-                         const GlobalMemo* gm = nullptr);
+                         const GlobalMemo* gm = nullptr, const int32_t* parts = nullptr, int32_t n_blocks = 0);
+constexpr int kPartShift = 16, kNpartShift = 21;
+constexpr int32_t kPartTreeMask = (1 << kPartShift) - 1;  // a tree index < 65,536 (P <= 65,536)
+static_assert(kDeltaBuckets <= 32, "a part index fits in 5 bits and nparts in 6");
 
 // Compaction: copies the live part of a tree (everything reachable from the root) into fresh arrays, with
 // nodes renumbered in breadth-first order, every live table rehashed at its size without tombstones, and

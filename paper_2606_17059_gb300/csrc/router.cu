@@ -216,6 +216,8 @@ struct p2p_router {
   DevBuf lru_buf;                                   // scratch of the LRU calls
   DevBuf gmemo;                                     // the delta kernel's launch-wide verified-run table
   DevBuf d_room;                                    // room bounds of the trees that stopped (room_kernel)
+  DevBuf d_parts;                                   // the delta launch's CTA parts (split_trees)
+  std::vector<int32_t> h_parts;                     // their host copy (kept until the next call)
   std::vector<uint8_t> lru;                         // per tree: kept as an LRU cache (p2p_lru_enable)
   std::vector<int64_t> lru_time;                    // per LRU tree: the time of its last insert or access
   int64_t launches = 0;  // kernels this router has launched
@@ -1064,7 +1066,7 @@ void p2p_router_destroy(p2p_router* r) {
                       &r->d_seg_off, &r->d_seg_len, &r->d_pool, &r->d_peer_begin, &r->d_done, &r->d_gather,
                       &r->grp_keys, &r->grp_vals, &r->grp_req, &r->grp_ckpt, &r->cmp_jobs, &r->cmp_queue,
                       &r->upd_cnt, &r->upd_op, &r->upd_sb, &r->upd_so, &r->upd_sl, &r->lru_buf, &r->gmemo,
-                      &r->d_room})
+                      &r->d_room, &r->d_parts})
       dfree(r, b->p);
     dfree(r, r->d_views);
     dfree(r, r->d_states);
@@ -1205,6 +1207,43 @@ int p2p_tree_apply_delta(p2p_router* r, int32_t peer, const p2p_delta* d, int64_
   return apply_delta_impl(r, peer, d, n_absent, false);
 }
 
+// The CTAs of a delta launch.  A CTA takes the ops of one tree, except that a tree with many more ops than a
+// CTA's share of the call -- the call's ops over the SMs, and at least kPartOps -- is split into up to
+// kDeltaBuckets parts by first-token bucket, so that it does not hold the whole launch on one SM (a batch
+// routed mostly to one tree and inserted with p2p_update_estimates, for one).  n_blocks = nt and
+// d_parts = NULL when no tree is split.
+constexpr int64_t kPartOps = 16384;
+static int split_trees(p2p_router* r, int32_t peer, const p2p_delta* d, const int64_t* d_pb, int32_t p0, int32_t nt,
+                int64_t n, int32_t& n_blocks, const int32_t*& d_parts) {
+  n_blocks = nt;
+  d_parts = nullptr;
+  const int64_t share = std::max<int64_t>((n + r->num_sms - 1) / std::max(r->num_sms, 1), kPartOps);
+  if (n <= share) return P2P_OK;
+  std::vector<int64_t> ops((size_t)nt, n);
+  if (peer == -1) {
+    std::vector<int64_t> pb((size_t)r->P + 1);
+    if (d->mem == P2P_MEM_HOST) {
+      std::memcpy(pb.data(), d->peer_begin, pb.size() * sizeof(int64_t));
+    } else {
+      CK(d2h(r, pb.data(), d_pb, pb.size() * sizeof(int64_t)));
+    }
+    for (int32_t i = 0; i < nt; ++i) ops[(size_t)i] = pb[(size_t)i + 1] - pb[(size_t)i];
+  }
+  std::vector<int32_t>& w = r->h_parts;
+  w.clear();
+  for (int32_t i = 0; i < nt; ++i) {
+    const int32_t np = (int32_t)std::min<int64_t>(p2p::kDeltaBuckets, (ops[(size_t)i] + share - 1) / share);
+    for (int32_t c = 0; c < std::max(np, 1); ++c)
+      w.push_back(i | c << p2p::kPartShift | std::max(np, 1) << p2p::kNpartShift);
+  }
+  if ((int32_t)w.size() == nt) return P2P_OK;
+  CK(ensure(r, r->d_parts, w.size() * sizeof(int32_t)));
+  CK(cudaMemcpyAsync(r->d_parts.p, w.data(), w.size() * sizeof(int32_t), cudaMemcpyHostToDevice, r->stream));
+  n_blocks = (int32_t)w.size();
+  d_parts = static_cast<const int32_t*>(r->d_parts.p);
+  return P2P_OK;
+}
+
 static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int64_t* n_absent, bool lru_ok) {
   if (!r) return fail(nullptr, P2P_E_INVAL, "router is NULL");
   if (peer < -1 || peer >= r->P) return fail(r, P2P_E_INVAL, "peer out of range");
@@ -1280,10 +1319,14 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
     if (h[2] & p2p::STATIC_BAD_PEER_BEGIN) return fail(r, P2P_E_INVAL, "peer_begin must run non-decreasing from 0 to n");
   }
   CK(ensure(r, r->d_done, (size_t)std::max<int64_t>(n, 1)));
+  // A tree with many more ops than a CTA's share of the call is split among CTAs (delta_kernel's parts).
+  int32_t n_blocks = nt;
+  const int32_t* d_parts = nullptr;
+  if (int e = split_trees(r, peer, d, d_pb, p0, nt, n, n_blocks, d_parts)) return e;
   int32_t* gather = nullptr;
   const int64_t stride = std::max<int64_t>(max_len, 1);
   if (max_runs > 2) {
-    CK(ensure(r, r->d_gather, (size_t)nt * p2p::kDeltaWarps * stride * sizeof(int32_t)));
+    CK(ensure(r, r->d_gather, (size_t)n_blocks * p2p::kDeltaWarps * stride * sizeof(int32_t)));
     gather = (int32_t*)r->d_gather.p;
   }
   uint8_t* done = (uint8_t*)r->d_done.p;
@@ -1314,7 +1357,7 @@ static int apply_delta_impl(p2p_router* r, int32_t peer, const p2p_delta* d, int
     if (round == 0)
       if (int rc = prepare_scratch(r)) return rc;
     CK(p2p::launch_delta(r->d_states + p0, done, nt, d_op, d_sb, d_so, d_sl, d_pool, gather, stride, r->d_shared,
-                         r->stream, &gm));
+                         r->stream, &gm, d_parts, n_blocks));
     if (round == 0)
       if (int rc = launch_prepared(r)) return rc;  // a prepared batch's grouping overlaps the delta kernel
     r->launches += 1;

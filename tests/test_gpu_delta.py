@@ -326,3 +326,36 @@ def test_deleting_through_two_shared_heads_under_one_node():
         gm, _ = route_device(r, tok, off, [0, 0], 0)
         assert (gm[:, 1] == 0).all()
         assert r.apply_delta(1, np.zeros(2, np.int32), seqlist_from_lists(b)) == 0  # back for the next order
+
+
+@pytest.mark.parametrize("single", [False, True])
+def test_heavy_tree_split_among_ctas(single):
+    """A tree that takes far more ops than a CTA's share of the call (here ~40,000 against 16,384) is split
+    among several CTAs by first-token bucket.  Its ops still apply in order per sequence (inserts, deletes and
+    re-inserts of the same sequences, duplicates, empty sequences) and the export equals the oracle's byte for
+    byte, through a call on every tree (the other tree takes a few ops) and through a call on that tree alone."""
+    rng = random.Random(4242 + single)
+    V = 3000
+    stored = [[rng.randrange(V) for _ in range(rng.randint(1, 40))] for _ in range(3000)]
+    small = [[rng.randrange(V) for _ in range(rng.randint(1, 40))] for _ in range(50)]
+    r = router_from_seqlists([seqlist_from_lists(stored), seqlist_from_lists(small)])
+    t0, t1 = _oracle_tree(stored), _oracle_tree(small)
+    for rnd in range(2):
+        op0, seqs0 = _random_ops(rng, stored, V, 40_000, 40)
+        # the same sequences again: deletes and re-inserts that must follow their first op
+        again = [rng.randrange(len(seqs0)) for _ in range(2_000)]
+        op0 = np.concatenate([op0, np.array([1 - int(op0[i]) for i in again], np.int32), np.zeros(3, np.int32)])
+        seqs0 = seqs0 + [seqs0[i] for i in again] + [[], [], []]
+        if single:
+            sl = seqlist_from_lists(seqs0)
+            assert r.apply_delta(0, op0, sl) == t0.apply_ops(op0, sl)
+        else:
+            op1, seqs1 = _random_ops(rng, small, V, 20, 40)
+            ops = np.concatenate([op0, op1])
+            sl = seqlist_from_lists(seqs0 + seqs1)
+            pb = np.array([0, len(op0), len(ops)], np.int64)
+            r.apply_delta(-1, ops, sl, pb)
+            t0.apply_ops(ops, sl, 0, len(op0))
+            t1.apply_ops(ops, sl, len(op0), len(ops))
+            assert same_snapshot(r.download(1), t1.export()), f"round {rnd}: small tree"
+        assert same_snapshot(r.download(0), t0.export()), f"round {rnd}: heavy tree"
