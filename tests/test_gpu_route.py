@@ -275,6 +275,52 @@ def test_root_first_tokens_added_and_removed_by_deltas():
     del torch
 
 
+@pytest.mark.parametrize("seed", range(4))
+def test_requests_that_leave_after_one_or_two_tokens(seed):
+    """Requests that leave a tree after one or two tokens: first tokens small and large (up to 2^30), root
+    children whose label is one token, one-token requests, and deltas that remove every sequence of some first
+    tokens, bring new ones and bring removed ones back (the root filter keeps stale bits); every match value
+    and route against the oracle."""
+    rng = np.random.default_rng(300 + seed)
+    big = [200_000, 300_000, 1 << 30]
+    firsts = list(range(40)) + big
+
+    def seq():
+        t0 = int(rng.choice(firsts))
+        return [t0] + rng.integers(0, 60, size=int(rng.integers(0, 6))).tolist()
+
+    base = [[seq() for _ in range(300)] for _ in range(2)]
+    r = router_from_seqlists([seqlist_from_lists(b) for b in base])
+    otrees = oracle.build_trees([seqlist_from_lists(b) for b in base])
+    stored = [list(b) for b in base]
+    for rnd in range(4):
+        reqs = [[int(rng.integers(0, 45))] + rng.integers(0, 60, size=int(rng.integers(0, 4))).tolist()
+                for _ in range(1500)]
+        reqs += [[int(rng.choice(big))] + rng.integers(0, 60, size=int(rng.integers(0, 3))).tolist() for _ in range(200)]
+        reqs += [list(s[: int(rng.integers(1, len(s) + 1))]) for s in stored[0][:200]]
+        tok, off = csr_from_lists(reqs)
+        load = [int(x) for x in rng.integers(0, 3, size=2)]
+        gm, gp = route_device(r, tok, off, load, 1)
+        om, op, _ = oracle.route(otrees, tok, off, load, 1)
+        assert_same_route(gm, gp, om, op, f"seed {seed} round {rnd}")
+        # The next delta: every sequence of a few first tokens goes, new first tokens come, old ones come back.
+        gone_t0 = set(int(x) for x in rng.choice(firsts, size=6, replace=False))
+        ops, seqs, pb = [], [], [0]
+        for p in range(2):
+            dels = [s for s in stored[p] if s[0] in gone_t0]
+            ins = [[int(rng.integers(40, 44))] + rng.integers(0, 60, size=int(rng.integers(0, 5))).tolist()
+                   for _ in range(20)] + [seq() for _ in range(20)]
+            ops += [1] * len(dels) + [0] * len(ins)
+            seqs += dels + ins
+            pb.append(len(ops))
+            stored[p] = [s for s in stored[p] if s[0] not in gone_t0] + ins
+        op_a = np.array(ops, np.int32)
+        sl = seqlist_from_lists(seqs)
+        r.apply_delta(-1, op_a, sl, np.array(pb, np.int64))
+        for p in range(2):
+            otrees[p].apply_ops(op_a, sl, pb[p], pb[p + 1])
+
+
 def _dev_arr(a):
     import torch
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
