@@ -881,6 +881,9 @@ constexpr int delta_smem_bytes() {
          kChunk * 2 + kChunk * 1 * 2;
 }
 
+// kParts: the launch splits heavy trees among CTAs (parts); a separate instantiation, so that the ordinary
+// launch keeps the code it had without the split.
+template <bool kParts>
 __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
     delta_kernel(TreeState* states, uint8_t* done, const int32_t* __restrict__ op,
                  const int64_t* __restrict__ seg_begin, const int64_t* __restrict__ seg_off,
@@ -913,9 +916,9 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
   // `nparts` (kDeltaBuckets buckets).  Ops with different first tokens touch disjoint subtrees and, of the
   // root, only its table, whose claims and counts are atomic; so the CTAs of one tree never touch the same
   // node below the root, and all ops on one sequence stay in one CTA, in op order.
-  const int32_t pw = parts ? parts[blockIdx.x] : (int32_t)blockIdx.x;
-  const int32_t part = parts ? (pw >> kPartShift) & 31 : 0, nparts = parts ? (pw >> kNpartShift) & 63 : 1;
-  TreeState* gs = states + (parts ? (pw & kPartTreeMask) : pw);
+  const int32_t pw = kParts ? parts[blockIdx.x] : (int32_t)blockIdx.x;
+  const int32_t part = kParts ? (pw >> kPartShift) & 31 : 0, nparts = kParts ? (pw >> kNpartShift) & 63 : 1;
+  TreeState* gs = states + (kParts ? (pw & kPartTreeMask) : pw);
   if (lane < kMemoSlots) s_memo[warp][lane] = MemoEntry{nullptr, nullptr, 0};
   const int64_t op_begin = gs->op_begin, op_end = gs->op_end;
   if (threadIdx.x == 0) s_any = 0;
@@ -966,7 +969,7 @@ __global__ void __launch_bounds__(kDeltaWarps * 32, 2)
         n += seg_len[g];
       }
       s_bucket[j] = (int8_t)b;
-      uint8_t fl = done[i] || b % nparts != part ? F_DONE : 0;  // another CTA's op: done as far as this one goes
+      uint8_t fl = done[i] || (kParts && b % nparts != part) ? F_DONE : 0;  // another CTA's op: done here
       if (!fl && !s_stop[b]) {
         int32_t anchor, next_tok;
         find_anchor(t, root, seg_off, seg_len, pool, g0, g1, n, anchor, next_tok);
@@ -1500,12 +1503,20 @@ cudaError_t launch_delta(TreeState* d_states, uint8_t* done, int32_t n_trees, co
                          const GlobalMemo* gm, const int32_t* parts, int32_t n_blocks) {
   if (n_trees <= 0) return cudaSuccess;
   const int dyn = delta_smem_bytes();
-  cudaError_t e = cudaFuncSetAttribute(delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
+  cudaError_t e = cudaFuncSetAttribute(parts ? delta_kernel<true> : delta_kernel<false>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, dyn);
   if (e != cudaSuccess) return e;
-  P2P_TIMED(K_DELTA, st,
-            (delta_kernel<<<parts ? n_blocks : n_trees, kDeltaWarps * 32, dyn, st>>>(
-                d_states, done, op, seg_begin, seg_off, seg_len, pool, gather, gather_stride, shared,
-                gm ? gm->keys : nullptr, gm ? gm->vals : nullptr, gm ? gm->mask : 0u, parts)));
+  if (parts) {
+    P2P_TIMED(K_DELTA, st,
+              (delta_kernel<true><<<n_blocks, kDeltaWarps * 32, dyn, st>>>(
+                  d_states, done, op, seg_begin, seg_off, seg_len, pool, gather, gather_stride, shared,
+                  gm ? gm->keys : nullptr, gm ? gm->vals : nullptr, gm ? gm->mask : 0u, parts)));
+  } else {
+    P2P_TIMED(K_DELTA, st,
+              (delta_kernel<false><<<n_trees, kDeltaWarps * 32, dyn, st>>>(
+                  d_states, done, op, seg_begin, seg_off, seg_len, pool, gather, gather_stride, shared,
+                  gm ? gm->keys : nullptr, gm ? gm->vals : nullptr, gm ? gm->mask : 0u, nullptr)));
+  }
   return cudaGetLastError();
 }
 
