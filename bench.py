@@ -561,6 +561,9 @@ def run_ours(args):
         # ---- UpdateTrieEstimate / UpdateTrie of Algorithm 1 on the last timed batch (changes the trees) ----
         if not args.no_update:
             res["update_estimates"] = time_update(router, d_tok, d_off, out_peer, route_avg_ms)
+        # ---- the own tree as an LRU cache trie (last: an LRU tree takes no more deltas) ----
+        if not args.no_lru:
+            res["lru"] = time_lru(router, d_tok, n_tok, d_off, B, out_match, out_peer)
         res.update({
             "metric": METRIC, "value": value, "unit": "requests/s", "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -602,6 +605,34 @@ def time_update(router, d_tok, d_off, out_peer, route_ms):
             "route_plus_update_ms": route_ms + ms,
             "note": "one call after the timed steps on the last routed batch; the first call on fresh trees also "
                     "grows their arenas"}
+
+
+def time_lru(router, d_tok, n_tok, d_off, B, out_match, out_peer):
+    """The own tree (tree 0) as Section 2's LRU cache trie, after every other leg (an LRU tree takes no deltas):
+    p2p_lru_enable (not timed), one p2p_lru_access of the whole batch at time 1 (each request's matched tokens
+    stamped: Algorithm 1's cache hits), one p2p_lru_evict of 1% of the tree's own label tokens (EvictLRUTrie),
+    and p2p_hit_rate of the routed batch (Section 5's expected hit rate).  Wall time around each call, which
+    waits for its work (the hit rate is synchronized)."""
+    import paper_2606_17059_gb300 as g
+    import torch
+    g.p2p_lru_enable(router.handle, 0)
+    n_ev = max(1, router.stats(0)["label_tokens"] // 100)
+
+    def timed(fn):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        out = fn()
+        torch.cuda.synchronize()
+        return out, (time.perf_counter() - t0) * 1e3
+
+    m0 = torch.empty(B, dtype=torch.int32, device="cuda")
+    _, acc_ms = timed(lambda: g.p2p_lru_access(router.handle, 0, d_tok, n_tok, d_off, B, 1, m0))
+    evicted, ev_ms = timed(lambda: g.p2p_lru_evict(router.handle, 0, n_ev))
+    hr = torch.empty(B, dtype=torch.float32, device="cuda")
+    _, hr_ms = timed(lambda: g.p2p_hit_rate(router.handle, out_match, d_off, B, out_peer, hr))
+    return {"tree": 0, "access_ms": acc_ms, "access_requests": B, "matched_tokens": int(m0.sum().item()),
+            "evict_ms": ev_ms, "evicted_tokens": evicted, "hit_rate_ms": hr_ms,
+            "mean_expected_hit_rate": float(hr.mean().item())}
 
 
 def time_route_decide(router, d_tok, n_tok, d_off, B, load, alpha, P, route_ms, reps: int = 5):
@@ -760,6 +791,9 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-update", action="store_true",
                     help="skip the timing of p2p_update_estimates (UpdateTrieEstimate) on the last routed batch")
+    ap.add_argument("--no-lru", action="store_true",
+                    help="skip the timing of the LRU calls on the own tree (p2p_lru_access, p2p_lru_evict) and of "
+                         "p2p_hit_rate after the other legs")
     ap.add_argument("--no-decide", action="store_true",
                     help="skip the timing of p2p_route_decide and p2p_route_batch_decide (excluded peers, next-best "
                          "target) on the routed batch")

@@ -265,9 +265,17 @@ cudaError_t launch_lru_bfs(const TreeState& s, const int32_t* front, int32_t n_f
                            int32_t cap, int32_t* parent, int32_t* cslot, int num_sms, cudaStream_t st);
 cudaError_t launch_lru_init(const int32_t* order, int32_t n, int64_t* size, int64_t* off, int64_t* rank,
                             unsigned long long* best, uint8_t* gone, int num_sms, cudaStream_t st);
+// Scratch of the sibling-offset sort (n2 = the live non-root nodes rounded up to a power of two; N = node slots).
+struct LruSortScratch {
+  unsigned long long* key;  // [n2]
+  int32_t* val;             // [n2]
+  int32_t* first;           // [N]
+  int64_t* scan;            // [n2]
+};
 cudaError_t launch_lru_levels(const TreeState& s, const int32_t* order, const int32_t* lvl_begin, int32_t n_levels,
                               const int32_t* parent, const int32_t* cslot, int64_t* size, int64_t* off, int64_t* rank,
-                              unsigned long long* best, int32_t* end, int num_sms, cudaStream_t st);
+                              unsigned long long* best, int32_t* end, const LruSortScratch& sc, int num_sms,
+                              cudaStream_t st);
 cudaError_t launch_lru_count(const TreeState& s, const int32_t* nodes, int32_t n, const int32_t* cslot,
                              const int64_t* rank, const int32_t* end, int mode, uint32_t S, unsigned long long K,
                              unsigned long long* out, int num_sms, cudaStream_t st);

@@ -26,7 +26,7 @@
 //   lru_stamp_kernel       thread per node: stamp fully touched nodes, split partially touched edges
 //   lru_bfs_kernel         warp per frontier node: children, parent links, child slots, next frontier
 //   lru_size_kernel        subtree sizes, one level at a time from the deepest
-//   lru_sib_kernel         warp per parent: per child, the sizes of its siblings with smaller first tokens
+//   lru_pairs/bitonic/runs/scan/off_kernel  sibling offsets: the (parent, first token) pairs sorted, sizes scanned
 //   lru_rank_kernel        preorder ranks, one level at a time from the top
 //   lru_end_kernel         end(v), one level at a time from the deepest
 //   lru_count_kernel       token count of the nodes below a key (binary search steps)
@@ -194,35 +194,91 @@ __global__ void __launch_bounds__(kLruThreads) lru_size_kernel(const int32_t* __
   }
 }
 
-// Warp per parent of one level: for every child c, off[c] = the total size of c's siblings whose first token
-// is smaller (signed order).  Quadratic in the fan-out, read from the parent's table.
-__global__ void __launch_bounds__(kLruThreads) lru_sib_kernel(LruTree t, const int32_t* __restrict__ lvl, int32_t n,
-                                                              const int64_t* __restrict__ size, int64_t* off) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warps = (int64_t)gridDim.x * (kLruThreads / 32);
-  for (int64_t i = ((int64_t)blockIdx.x * kLruThreads + threadIdx.x) >> 5; i < n; i += warps) {
-    const int4 nd = t.node[lvl[i]];
-    const int32_t bits = tab_bits(nd.y);
-    if (bits == 0) continue;
-    const int32_t ns = 1 << bits;
-    for (int32_t a0 = 0; a0 < ns; a0 += 32) {
-      const int32_t a = a0 + lane;
-      const int4 ca = a < ns ? t.child[nd.x + a] : make_int4(0, 0, 0, 0);
-      if (!__any_sync(kFull, ca.y >= 1)) continue;
-      int64_t sum = 0;
-      for (int32_t b0 = 0; b0 < ns; b0 += 32) {
-        const int32_t bb = b0 + lane;
-        const int4 cb = bb < ns ? t.child[nd.x + bb] : make_int4(0, 0, 0, 0);
-        const int64_t sb = cb.y >= 1 ? size[cb.y] : 0;
-        for (int j = 0; j < 32; ++j) {
-          const int32_t tok = __shfl_sync(kFull, cb.x, j);
-          const int64_t sz = __shfl_sync(kFull, sb, j);
-          if (ca.y >= 1 && sz > 0 && tok < ca.x) sum += sz;
-        }
-      }
-      if (ca.y >= 1) off[ca.y] = sum;
+// Sibling offsets for the preorder ranks: off[c] = the total subtree size of c's siblings whose first token
+// is smaller (signed order).  All (parent, first token) pairs of the tree are sorted at once (a bitonic sort:
+// a pair per live non-root node, padded to a power of two with the largest key), so each parent's children
+// form one run in first-token order; off[c] is then an exclusive scan of the sizes in that order, less the
+// scan at the start of c's run.  O(n log^2 n) for any fan-out.
+__global__ void __launch_bounds__(kLruThreads) lru_pairs_kernel(LruTree t, const int32_t* __restrict__ nodes, int32_t n,
+                                                                int64_t n2, const int32_t* __restrict__ parent,
+                                                                const int32_t* __restrict__ cslot,
+                                                                unsigned long long* key, int32_t* val) {
+  const int64_t stride = (int64_t)gridDim.x * kLruThreads;
+  for (int64_t i = (int64_t)blockIdx.x * kLruThreads + threadIdx.x; i < n2; i += stride) {
+    if (i < n) {
+      const int32_t v = nodes[i];
+      const uint32_t tok = (uint32_t)t.child[cslot[v]].x ^ 0x80000000u;  // signed order as unsigned
+      key[i] = ((unsigned long long)(uint32_t)parent[v] << 32) | tok;
+      val[i] = v;
+    } else {
+      key[i] = ~0ull;
+      val[i] = -1;
     }
   }
+}
+
+// One compare-exchange step of the bitonic sort of (key, val) over n2 (a power of two) entries.
+__global__ void __launch_bounds__(kLruThreads) lru_bitonic_kernel(unsigned long long* key, int32_t* val, int64_t n2,
+                                                                  int64_t j, int64_t k) {
+  const int64_t stride = (int64_t)gridDim.x * kLruThreads;
+  for (int64_t i = (int64_t)blockIdx.x * kLruThreads + threadIdx.x; i < n2; i += stride) {
+    const int64_t l = i ^ j;
+    if (l <= i) continue;
+    const unsigned long long a = key[i], b = key[l];
+    if ((a > b) == ((i & k) == 0)) {
+      key[i] = b;
+      key[l] = a;
+      const int32_t va = val[i];
+      val[i] = val[l];
+      val[l] = va;
+    }
+  }
+}
+
+// For the sorted pairs [0, n): the first position of each parent's run (first[parent]) and the sizes in
+// sorted order (into scan, scanned next).
+__global__ void __launch_bounds__(kLruThreads) lru_runs_kernel(const unsigned long long* __restrict__ key,
+                                                               const int32_t* __restrict__ val, int32_t n,
+                                                               const int64_t* __restrict__ size, int32_t* first,
+                                                               int64_t* scan) {
+  const int64_t stride = (int64_t)gridDim.x * kLruThreads;
+  for (int64_t i = (int64_t)blockIdx.x * kLruThreads + threadIdx.x; i < n; i += stride) {
+    if (i == 0 || (key[i] >> 32) != (key[i - 1] >> 32)) first[(int32_t)(key[i] >> 32)] = (int32_t)i;
+    scan[i] = size[val[i]];
+  }
+}
+
+// Exclusive scan of scan[0, n) in place, one CTA: each thread sums a contiguous stretch, the CTA scans the
+// stretch sums, each thread rewrites its stretch.
+__global__ void __launch_bounds__(1024) lru_scan_kernel(int64_t* scan, int32_t n) {
+  __shared__ int64_t s_part[1024];
+  const int32_t per = (n + 1023) / 1024, a = min(n, (int32_t)threadIdx.x * per), b = min(n, a + per);
+  int64_t sum = 0;
+  for (int32_t i = a; i < b; ++i) sum += scan[i];
+  s_part[threadIdx.x] = sum;
+  __syncthreads();
+  for (int o = 1; o < 1024; o <<= 1) {  // inclusive scan of the stretch sums (Hillis-Steele)
+    const int64_t x = threadIdx.x >= (unsigned)o ? s_part[threadIdx.x - o] : 0;
+    __syncthreads();
+    s_part[threadIdx.x] += x;
+    __syncthreads();
+  }
+  int64_t run = s_part[threadIdx.x] - sum;
+  for (int32_t i = a; i < b; ++i) {
+    const int64_t x = scan[i];
+    scan[i] = run;
+    run += x;
+  }
+}
+
+// off[c] for every sorted pair: the scan at c less the scan at the start of its parent's run.
+__global__ void __launch_bounds__(kLruThreads) lru_off_kernel(const unsigned long long* __restrict__ key,
+                                                              const int32_t* __restrict__ val, int32_t n,
+                                                              const int32_t* __restrict__ first,
+                                                              const int64_t* __restrict__ scan, int64_t* off) {
+  const int64_t stride = (int64_t)gridDim.x * kLruThreads;
+  for (int64_t i = (int64_t)blockIdx.x * kLruThreads + threadIdx.x; i < n; i += stride)
+    off[val[i]] = scan[i] - scan[first[(int32_t)(key[i] >> 32)]];
 }
 
 // Preorder ranks of one level: rank[v] = rank[parent] + 1 + the sizes of v's earlier siblings.
@@ -402,7 +458,8 @@ cudaError_t launch_lru_bfs(const TreeState& s, const int32_t* front, int32_t n_f
 
 cudaError_t launch_lru_levels(const TreeState& s, const int32_t* order, const int32_t* lvl_begin, int32_t n_levels,
                               const int32_t* parent, const int32_t* cslot, int64_t* size, int64_t* off, int64_t* rank,
-                              unsigned long long* best, int32_t* end, int num_sms, cudaStream_t st) {
+                              unsigned long long* best, int32_t* end, const LruSortScratch& sc, int num_sms,
+                              cudaStream_t st) {
   const LruTree t = lru_tree(s, nullptr);
   // Sizes, from the deepest level up (level 0 is the root).
   for (int32_t l = n_levels - 1; l >= 1; --l) {
@@ -411,12 +468,27 @@ cudaError_t launch_lru_levels(const TreeState& s, const int32_t* order, const in
               (lru_size_kernel<<<grid_for(n, kLruThreads, num_sms), kLruThreads, 0, st>>>(order + lvl_begin[l], n,
                                                                                           parent, size)));
   }
-  // Sibling offsets (per parent level), then preorder ranks from the top.
-  for (int32_t l = 0; l + 1 < n_levels; ++l) {
-    const int32_t n = lvl_begin[l + 1] - lvl_begin[l];
+  // Sibling offsets (all parents at once, by a sort of the (parent, first token) pairs), then preorder ranks
+  // from the top.
+  const int32_t m = lvl_begin[n_levels] - 1;  // the live non-root nodes: order[1 .. m]
+  if (m > 0) {
+    int64_t n2 = 1;
+    while (n2 < m) n2 <<= 1;
     P2P_TIMED(K_LRU_ORDER, st,
-              (lru_sib_kernel<<<grid_for(n, kLruThreads / 32, num_sms), kLruThreads, 0, st>>>(t, order + lvl_begin[l],
-                                                                                              n, size, off)));
+              (lru_pairs_kernel<<<grid_for(n2, kLruThreads, num_sms), kLruThreads, 0, st>>>(
+                  t, order + 1, m, n2, parent, cslot, sc.key, sc.val)));
+    for (int64_t k = 2; k <= n2; k <<= 1)
+      for (int64_t j = k >> 1; j > 0; j >>= 1)
+        P2P_TIMED(K_LRU_ORDER, st,
+                  (lru_bitonic_kernel<<<grid_for(n2, kLruThreads, num_sms), kLruThreads, 0, st>>>(sc.key, sc.val, n2,
+                                                                                                  j, k)));
+    P2P_TIMED(K_LRU_ORDER, st,
+              (lru_runs_kernel<<<grid_for(m, kLruThreads, num_sms), kLruThreads, 0, st>>>(sc.key, sc.val, m, size,
+                                                                                         sc.first, sc.scan)));
+    P2P_TIMED(K_LRU_ORDER, st, (lru_scan_kernel<<<1, 1024, 0, st>>>(sc.scan, m)));
+    P2P_TIMED(K_LRU_ORDER, st,
+              (lru_off_kernel<<<grid_for(m, kLruThreads, num_sms), kLruThreads, 0, st>>>(sc.key, sc.val, m, sc.first,
+                                                                                        sc.scan, off)));
   }
   for (int32_t l = 1; l < n_levels; ++l) {
     const int32_t n = lvl_begin[l + 1] - lvl_begin[l];

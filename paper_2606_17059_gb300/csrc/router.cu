@@ -1710,11 +1710,20 @@ int p2p_lru_evict(p2p_router* r, int32_t tree, int64_t n_tokens, int64_t* n_evic
   DeviceGuard g(r);
   const TreeState& t = r->hs[(size_t)tree];
   const int64_t N = std::max<int32_t>(t.n_node, 1);
-  // Scratch, per node slot: order, parent, cslot, end, surv (int32); size, off, rank, best (64-bit); gone; and
-  // two counters.
-  const size_t bytes = (size_t)N * (5 * 4 + 4 * 8 + 1) + 64;
+  // Scratch, per node slot: order, parent, cslot, end, surv (int32); size, off, rank, best (64-bit); gone; two
+  // counters; then the sibling-offset sort (a power of two of entries at least N - 1: key, scan 64-bit; val;
+  // and first per node slot).
+  int64_t n2 = 1;
+  while (n2 < N - 1) n2 <<= 1;
+  const size_t main_bytes = ((size_t)N * (5 * 4 + 4 * 8 + 1) + 64 + 15) & ~(size_t)15;
+  const size_t bytes = main_bytes + (size_t)n2 * (8 + 8 + 4) + (size_t)N * 4;
   CK(ensure(r, r->lru_buf, bytes));
   char* base = static_cast<char*>(r->lru_buf.p);
+  p2p::LruSortScratch sc;
+  sc.key = reinterpret_cast<unsigned long long*>(base + main_bytes);
+  sc.scan = reinterpret_cast<int64_t*>(sc.key + n2);
+  sc.val = reinterpret_cast<int32_t*>(sc.scan + n2);
+  sc.first = sc.val + n2;
   int64_t* size = reinterpret_cast<int64_t*>(base);
   int64_t* off = size + N;
   int64_t* rank = off + N;
@@ -1744,9 +1753,13 @@ int p2p_lru_evict(p2p_router* r, int32_t tree, int64_t n_tokens, int64_t* n_evic
   }
   const int32_t n_levels = (int32_t)lvl.size() - 1, total = lvl.back();
   CK(p2p::launch_lru_init(order, total, size, off, rank, best, gone, r->num_sms, r->stream));
-  CK(p2p::launch_lru_levels(t, order, lvl.data(), n_levels, parent, cslot, size, off, rank, best, end, r->num_sms,
+  CK(p2p::launch_lru_levels(t, order, lvl.data(), n_levels, parent, cslot, size, off, rank, best, end, sc, r->num_sms,
                             r->stream));
-  r->launches += 1 + 4 * (n_levels - 1);
+  {
+    int64_t stages = 0, m = total - 1, k2 = 1;
+    for (int32_t lg = 0; k2 < m; ++lg, k2 <<= 1) stages += lg + 1;  // bitonic steps: L (L + 1) / 2 for n2 = 2^L
+    r->launches += 1 + 3 * (n_levels - 1) + (m > 0 ? 4 + stages : 0);
+  }
   auto count = [&](int mode, uint32_t S, unsigned long long K, unsigned long long& out) -> int {
     CK(p2p::launch_lru_count(t, order + 1, total - 1, cslot, rank, end, mode, S, K, ctr, r->num_sms, r->stream));
     r->launches += 1;

@@ -105,6 +105,35 @@ def test_random_operation_sequences(seed):
     assert m.cpu().numpy()[:, 1].tolist() == [o.match(s) for s in reqs]
 
 
+@pytest.mark.parametrize("seed", range(3))
+def test_wide_nodes_eviction_order(seed):
+    """Eviction order among many siblings: a root with ~250 children and a node with ~400, stamped at several
+    times (the sibling offsets of the preorder ranks come from a sort of all (parent, first token) pairs, so
+    the order must hold at any fan-out, negative first tokens included); every snapshot against the oracle."""
+    rng = random.Random(900 + seed)
+    r = g.Router(1)
+    g.p2p_lru_enable(r.handle, 0)
+    o = LRUTrie()
+    seqs = [[rng.randrange(-50, 5000)] + [rng.randrange(100) for _ in range(rng.randint(0, 3))] for _ in range(250)]
+    seqs += [[7, 7, 7] + [rng.randrange(-30, 2000)] + [rng.randrange(50) for _ in range(rng.randint(0, 2))]
+             for _ in range(400)]
+    _insert(r, 0, seqs, 1)
+    for s in seqs:
+        o.insert(s, 1)
+    t = 1
+    for n in (5, 40, 120, 300):
+        t += 1
+        reqs = [list(rng.choice(seqs))[: rng.randint(1, 5)] for _ in range(120)]
+        got = _access(r, 0, reqs, t)
+        assert got.tolist() == [o.access(s, t) for s in reqs]
+        evicted = g.p2p_lru_evict(r.handle, 0, n)
+        k = 0
+        while k < n and o.evict() is not None:
+            k += 1
+        assert evicted == k
+        assert same_snapshot(r.download(0), _oracle_export(o)), (seed, n)
+
+
 def test_workload_tree_made_lru_after_upload():
     """A generator tree (shared prompt prefixes, Zipf requests) made an LRU tree after its upload: accesses,
     inserts of new prompts, and evictions of a few tokens at a time (the oracle evicts one token per scan of its
