@@ -296,9 +296,10 @@ struct RouteAcc<true> {
       k2 = key;
     }
   }
-  __device__ __forceinline__ void warp_merge() {
+  // Merges the keys of lane groups of 2 * first lanes (the whole warp by default) into each of their lanes.
+  __device__ __forceinline__ void warp_merge(int first = 16) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
+    for (int o = first; o > 0; o >>= 1) {
       const unsigned long long o1 = __shfl_xor_sync(kFull, k1, o), o2 = __shfl_xor_sync(kFull, k2, o);
       const unsigned long long lo = k1 < o1 ? k1 : o1, hi = k1 < o1 ? o1 : k1, r2 = k2 < o2 ? o2 : k2;
       k1 = hi;
@@ -830,16 +831,108 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
   }
 }
 
-// Route decision from a match matrix with excluded peers (one warp per request): the best and the next-best
-// candidate by the route order of route_key, skipping trees whose staged load word carries kExcluded
-// (Section 3.2: a peer that pushes back; Section 3.3: a suspected-failed peer, and the next-best target a
-// request falls back to when forwarding times out), with RouteAcc<true>.  Match values below 0 count as 0.
-constexpr int kDecideUnroll = 8;  // columns a lane loads per stretch (a 256-tree row in one stretch)
+// Route decision from a match matrix with excluded peers: the best and the next-best candidate by the route
+// order of route_key, skipping trees whose staged load word carries kExcluded (Section 3.2: a peer that
+// pushes back; Section 3.3: a suspected-failed peer, and the next-best target a request falls back to when
+// forwarding times out).  Match values below 0 count as 0.
+//
+// Up to 256 trees (P a multiple of 4, the matrix on a 16-byte boundary) a row is read by 8 lanes, four rows
+// per warp at a time: lane j of a row's group takes columns 32i + 4j .. 32i + 4j + 3 (i < 8, one 16-byte load
+// each), so a group reads 128 contiguous bytes per load.  The route order of a column is its score
+// m - alpha * load, then its tie-break (lower load, then lower index), which is a fixed order of the columns:
+// with rank(p) = the number of columns p comes before on the tie-break, a unique 8-bit value, the order is
+// that of the 32-bit key (m - alpha * load + 2^22) * 256 + rank(p) whenever 0 <= m < 2^22 and
+// 0 <= alpha * load < 2^22 (the key then lies in [256, 2^31)).  A lane holds (2^22 - alpha * load) * 256 + rank
+// of each of its columns (INT_MIN for an excluded one, so its key stays negative), and a column costs one
+// shift-add and three min/max for the top two keys.  A warp's four rows take the 64-bit keys of RouteAcc
+// instead when one of their values is outside [0, 2^22), and every row does when a load term is 2^22 or more.
+// Other shapes take one warp per row with RouteAcc<true>.
+constexpr int kDecideUnroll = 8;        // columns a lane loads per stretch on the one-warp-per-row path
+constexpr int32_t kSmallKey = 1 << 22;  // bound on match values and load terms of the 32-bit keys
 __global__ void __launch_bounds__(256) decide_kernel(const int32_t* __restrict__ match, int64_t B, int32_t P,
                                                      const int32_t* __restrict__ load, int32_t alpha,
                                                      int32_t* __restrict__ out_peer, int32_t* __restrict__ out_next) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = (int64_t)gridDim.x * (blockDim.x / 32);
+  if (P <= 256 && P % 4 == 0 && (reinterpret_cast<uintptr_t>(match) & 15) == 0) {
+    __shared__ int32_t s_rank[256];   // tie-break rank of each column
+    __shared__ int16_t s_col[256];    // the column of each rank
+    for (int32_t p = threadIdx.x; p < P; p += blockDim.x) {
+      const int32_t lp = __ldg(load + p) & 0xFFFF;
+      int32_t r = 0;
+      for (int32_t q = 0; q < P; ++q) {
+        const int32_t lq = __ldg(load + q) & 0xFFFF;
+        r += lq > lp || (lq == lp && q > p);
+      }
+      s_rank[p] = r;
+      s_col[r] = (int16_t)p;
+    }
+    __syncthreads();
+    const int j = lane & 7;
+    int32_t base[32];
+    bool small = true;
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+      const int32_t p = 32 * (c >> 2) + 4 * j + (c & 3);
+      base[c] = INT_MIN;
+      if (p < P) {
+        const int32_t ldw = __ldg(load + p);
+        const long long term = (long long)alpha * (ldw & 0xFFFF);
+        if (!(ldw & kExcluded)) {
+          if (term < kSmallKey)
+            base[c] = (int32_t)(((kSmallKey - term) << 8) | s_rank[p]);
+          else
+            small = false;
+        }
+      }
+    }
+    small = __all_sync(kFull, small);  // every warp holds every column, so every warp agrees
+    const int64_t quads = (B + 3) / 4;
+    for (int64_t w = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; w < quads; w += warps) {
+      const int64_t b = 4 * w + (lane >> 3);
+      const bool row_ok = b < B;
+      const int4* r4 = reinterpret_cast<const int4*>(match + (row_ok ? b : 0) * P + 4 * j);
+      int4 v[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) v[i] = row_ok && 32 * i + 4 * j < P ? __ldg(r4 + 8 * i) : make_int4(0, 0, 0, 0);
+      uint32_t any = 0;  // OR of the values: below 2^22 (unsigned) iff every value is in [0, 2^22)
+#pragma unroll
+      for (int i = 0; i < 8; ++i) any |= (uint32_t)(v[i].x | v[i].y | v[i].z | v[i].w);
+      if (small && !__any_sync(kFull, any >= (uint32_t)kSmallKey)) {
+        int32_t k1 = 0, k2 = 0;
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const int4& x = v[c >> 2];
+          const int32_t m = (c & 3) == 0 ? x.x : (c & 3) == 1 ? x.y : (c & 3) == 2 ? x.z : x.w;
+          const int32_t key = (m << 8) + base[c];
+          k2 = max(k2, min(k1, key));
+          k1 = max(k1, key);
+        }
+#pragma unroll
+        for (int o = 4; o > 0; o >>= 1) {
+          const int32_t o1 = __shfl_xor_sync(kFull, k1, o), o2 = __shfl_xor_sync(kFull, k2, o);
+          k2 = max(min(k1, o1), max(k2, o2));
+          k1 = max(k1, o1);
+        }
+        if (j == 0 && row_ok) {
+          out_peer[b] = k1 > 0 ? s_col[k1 & 0xFF] : -1;
+          if (out_next) out_next[b] = k2 > 0 ? s_col[k2 & 0xFF] : -1;
+        }
+      } else {
+        RouteAcc<true> acc;
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const int32_t p = 32 * (c >> 2) + 4 * j + (c & 3);
+          const int4& x = v[c >> 2];
+          const int32_t m = (c & 3) == 0 ? x.x : (c & 3) == 1 ? x.y : (c & 3) == 2 ? x.z : x.w;
+          if (p < P) acc.add(max(m, 0), __ldg(load + p), p, alpha);
+        }
+        acc.warp_merge(4);
+        if (j == 0 && row_ok) acc.write(b, out_peer, out_next);
+      }
+    }
+    return;
+  }
   for (int64_t b = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5; b < B; b += warps) {
     const int32_t* row = match + b * P;
     RouteAcc<true> acc;

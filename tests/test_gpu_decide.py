@@ -29,10 +29,10 @@ def _decide(r, match, load, alpha, excluded):
     return peer.cpu().numpy(), nxt.cpu().numpy()
 
 
-@pytest.mark.parametrize("P", [1, 2, 7, 32, 45, 256])
+@pytest.mark.parametrize("P", [1, 2, 7, 32, 45, 252, 256, 260, 300])
 def test_random_matrices_and_masks(P):
     rng = np.random.default_rng(P)
-    B = 600 if P == 256 else 2000
+    B = 600 if P >= 252 else 2000
     r = g.Router(P)
     match = rng.integers(0, 40, size=(B, P), dtype=np.int32)  # many ties
     load = rng.integers(0, 6, size=P).astype(np.int32)
@@ -61,6 +61,48 @@ def test_negative_entries_count_as_zero(P):
             gp, gn = _decide(r, match, load, alpha, ex)
             op, on = oracle.decide(match, load, alpha, ex)
             assert np.array_equal(gp, op) and np.array_equal(gn, on), (P, alpha)
+
+
+@pytest.mark.parametrize("P", [8, 36])
+def test_batch_beyond_the_grid_and_matrix_off_a_16_byte_boundary(P):
+    """More rows than the launch has warps (each warp takes several rows, two at a time, with a ragged last
+    pair), once from a matrix on a 16-byte boundary and once from one 4 bytes past it."""
+    import torch
+    rng = np.random.default_rng(200 + P)
+    B = 25_001
+    r = g.Router(P)
+    match = rng.integers(0, 30, size=(B, P), dtype=np.int32)
+    load = rng.integers(0, 5, size=P).astype(np.int32)
+    ex = (rng.random(P) < 0.25).astype(np.uint8)
+    op, on = oracle.decide(match, load, 2, ex)
+    flat = torch.zeros(B * P + 4, dtype=torch.int32, device="cuda")
+    for shift in (0, 1):
+        view = flat[shift:shift + B * P].view(B, P)
+        view.copy_(torch.from_numpy(match))
+        peer, nxt = r.decide(view, load, 2, ex)
+        assert np.array_equal(peer.cpu().numpy(), op) and np.array_equal(nxt.cpu().numpy(), on), (P, shift)
+
+
+@pytest.mark.parametrize("alpha", [64, 65])
+def test_values_and_load_terms_at_the_edge_of_the_short_keys(alpha):
+    """Match values just below and at or above 2^22, negative ones, and loads up to 0xFFFF: with alpha = 64
+    every load term is below 2^22 (65,535 * 64 = 4,194,240), with alpha = 65 some are not.  Row groups that
+    hold an out-of-range value and those that do not share one launch."""
+    rng = np.random.default_rng(300 + alpha)
+    B, P = 4001, 64
+    r = g.Router(P)
+    match = rng.integers(0, 50, size=(B, P), dtype=np.int32)
+    edge = np.array([(1 << 22) - 1, 1 << 22, (1 << 22) + 1, np.iinfo(np.int32).max, -1], np.int32)
+    rows = rng.choice(B, 200, replace=False)
+    match[rows, rng.integers(0, P, 200)] = edge[rng.integers(0, len(edge), 200)]
+    match[rng.choice(B, 300, replace=False), :] += (1 << 22) - 60   # whole rows just below the bound
+    load = rng.integers(0, 4, size=P).astype(np.int32)
+    load[rng.choice(P, 8, replace=False)] = 0xFFFF
+    load[rng.choice(P, 4, replace=False)] = 0xFFFE
+    for ex in (None, (rng.random(P) < 0.2).astype(np.uint8)):
+        gp, gn = _decide(r, match, load, alpha, ex)
+        op, on = oracle.decide(match, load, alpha, ex)
+        assert np.array_equal(gp, op) and np.array_equal(gn, on), (alpha, ex is None)
 
 
 def test_decision_of_a_routed_batch():
