@@ -76,16 +76,16 @@ KERNEL_SOURCE = {
 # differs from the current source is not reported (the kernel changed since it was taken).
 TRAFFIC: dict = {
     "cfg4": {k: dict(v, profile="profiles/traffic_workload4.md") for k, v in {
-        "delta_kernel": {"bytes": 6722429107, "source": "0b558fa44276b221"},
-        "validate_kernel": {"bytes": 98813542, "source": "0b558fa44276b221"},
-        "compact_kernel": {"bytes": 10288611840, "source": "0b558fa44276b221"},
-        "compact_labels_kernel": {"bytes": 24294580224, "source": "0b558fa44276b221"},
-        "group_hash_kernel": {"bytes": 491260902, "source": "c540f29ec07fe042"},
-        "group_resolve32_kernel": {"bytes": 9457387801, "source": "c540f29ec07fe042"},
-        "group_ranges_kernel": {"bytes": 4005196, "source": "c540f29ec07fe042"},
-        "group_place_kernel": {"bytes": 8145356, "source": "c540f29ec07fe042"},
-        "lane_kernel<true>": {"bytes": 6160865945, "source": "78aca06860acc42f"},
-        "lane_kernel<false>": {"bytes": 17196897484, "source": "78aca06860acc42f"},
+        "delta_kernel": {"bytes": 6722955162, "source": "e2ef36bc7089a1f9"},
+        "validate_kernel": {"bytes": 99170202, "source": "e2ef36bc7089a1f9"},
+        "compact_kernel": {"bytes": 10286514944, "source": "e2ef36bc7089a1f9"},
+        "compact_labels_kernel": {"bytes": 24298933760, "source": "e2ef36bc7089a1f9"},
+        "group_hash_kernel": {"bytes": 491484160, "source": "5dbd6a2a3cb8351d"},
+        "group_resolve32_kernel": {"bytes": 9457201050, "source": "5dbd6a2a3cb8351d"},
+        "group_ranges_kernel": {"bytes": 4005018, "source": "5dbd6a2a3cb8351d"},
+        "group_place_kernel": {"bytes": 8143744, "source": "5dbd6a2a3cb8351d"},
+        "lane_kernel<true>": {"bytes": 6153706214, "source": "860a53f264d1bcdd"},
+        "lane_kernel<false>": {"bytes": 16302165555, "source": "860a53f264d1bcdd"},
     }.items()},
 }
 
