@@ -1059,6 +1059,8 @@ void p2p_router_destroy(p2p_router* r) {
   if (!r) return;
   DeviceGuard g(r);
   cudaStreamSynchronize(r->stream);
+  for (cudaStream_t s : {r->cp_in, r->cp_out, r->grp_stream})  // copies or a prepared grouping in flight
+    if (s) cudaStreamSynchronize(s);
   if (r->pool) {
     for (TreeState& t : r->hs) free_tree_arrays(r, t);
     for (TreeState& t : r->spare) free_tree_arrays(r, t);
