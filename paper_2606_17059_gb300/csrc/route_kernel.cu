@@ -849,7 +849,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
 // Other shapes take one warp per row with RouteAcc<true>.
 constexpr int kDecideUnroll = 8;        // columns a lane loads per stretch on the one-warp-per-row path
 constexpr int32_t kSmallKey = 1 << 22;  // bound on match values and load terms of the 32-bit keys
-__global__ void __launch_bounds__(256) decide_kernel(const int32_t* __restrict__ match, int64_t B, int32_t P,
+__global__ void __launch_bounds__(256, 2) decide_kernel(const int32_t* __restrict__ match, int64_t B, int32_t P,
                                                      const int32_t* __restrict__ load, int32_t alpha,
                                                      int32_t* __restrict__ out_peer, int32_t* __restrict__ out_next) {
   const int lane = threadIdx.x & 31;
@@ -1017,8 +1017,9 @@ cudaError_t launch_route(const TreeView* d_trees, int32_t P, const int32_t* toke
 cudaError_t launch_decide(const int32_t* match, int64_t B, int32_t P, const int32_t* d_load, int32_t alpha,
                           int32_t* out_peer, int32_t* out_next, int num_sms, cudaStream_t st) {
   if (B <= 0) return cudaSuccess;
+  // One wave of resident CTAs (the kernel's registers allow 2 per SM): every CTA ranks the columns once.
   const int64_t want = (B + 7) / 8;
-  const int grid = (int)std::min<int64_t>(want, (int64_t)std::max(num_sms, 1) * 8);
+  const int grid = (int)std::min<int64_t>(want, (int64_t)std::max(num_sms, 1) * 2);
   P2P_TIMED(K_DECIDE, st, (decide_kernel<<<grid, 256, 0, st>>>(match, B, P, d_load, alpha, out_peer, out_next)));
   return cudaGetLastError();
 }
