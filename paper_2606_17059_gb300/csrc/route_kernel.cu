@@ -619,9 +619,11 @@ __device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab,
 // calls it).  Lane state: tree p, the edge ce to walk at position pos (act), m = tokens matched so far,
 // known = tokens known to match without comparing, and for leaders the checkpoint slot ck (NULL: none)
 // with the deepest position climit it records.  A lane compares an edge's label itself when it leaves
-// within the first 8 tokens or the edge has at most kThreadSpan tokens left; longer compares are done by
-// the whole warp, once per distinct (label address, request position): the long prompt prefixes are
-// interned labels shared by many trees, so one compare serves every lane at that label.
+// within the first 8 tokens (16 for a follower) or the edge has at most kThreadSpan tokens left; longer
+// compares are done by the whole warp, once per distinct (label address, request position): the long
+// prompt prefixes are interned labels shared by many trees, so one compare serves every lane at that label.
+// (Followers resume past the shared prefix, where labels tend to end within a few tokens: 16 took the
+// follower pass of the scale workload from 5.0 to 4.8 ms; for leaders 16 was slower, 1.9 to 2.4 ms.)
 template <bool kLeader>
 __device__ __forceinline__ void lane_walks(const TreeView* __restrict__ trees, int32_t p, const int32_t* req,
                                            int32_t len, int32_t known, bool act, int4 ce, int32_t& pos, int32_t& m,
@@ -642,7 +644,7 @@ __device__ __forceinline__ void lane_walks(const TreeView* __restrict__ trees, i
         const int32_t from = max(1, known - pos);
         k = lim;
         if (from < lim) {
-          const int32_t first = min(lim, from + 8);
+          const int32_t first = min(lim, from + (kLeader ? 8 : 16));
           k = first_diff_1(lab, req + pos, from, first);
           if (k == first && first < lim) {
             if (lim - first <= kThreadSpan) {
