@@ -619,12 +619,14 @@ __device__ __forceinline__ int32_t first_diff_1(const int32_t* __restrict__ lab,
 // calls it).  Lane state: tree p, the edge ce to walk at position pos (act), m = tokens matched so far,
 // known = tokens known to match without comparing, and for leaders the checkpoint slot ck (NULL: none)
 // with the deepest position climit it records.  A lane compares an edge's label itself when it leaves
-// within the first 8 tokens (16 for a follower) or the edge has at most kThreadSpan tokens left; longer
-// compares are done by the whole warp, once per distinct (label address, request position): the long
-// prompt prefixes are interned labels shared by many trees, so one compare serves every lane at that label.
-// (Followers resume past the shared prefix, where labels tend to end within a few tokens: 16 took the
-// follower pass of the scale workload from 5.0 to 4.8 ms; for leaders 16 was slower, 1.9 to 2.4 ms.)
-template <bool kLeader>
+// within the first kFirst tokens or the edge has at most kThreadSpan tokens left; longer compares are done
+// by the whole warp, once per distinct (label address, request position): the long prompt prefixes are
+// interned labels shared by many trees, so one compare serves every lane at that label.  Leaders take
+// kFirst = 8.  Followers of a batch of requests shorter than a staging window on average take 16: they
+// resume past the shared prefix, where labels tend to end within a few tokens (the scale workload's follower
+// pass 5.0 -> 4.8 ms); followers of long requests take 8 (16 cost the long-context workload's followers a
+// round trip on most long edges, 0.20 -> 0.27 ms); for leaders 16 was slower (1.9 -> 2.4 ms).
+template <bool kLeader, int kFirst>
 __device__ __forceinline__ void lane_walks(const TreeView* __restrict__ trees, int32_t p, const int32_t* req,
                                            int32_t len, int32_t known, bool act, int4 ce, int32_t& pos, int32_t& m,
                                            int4* ck, int32_t climit, int lane, int32_t* err) {
@@ -644,7 +646,7 @@ __device__ __forceinline__ void lane_walks(const TreeView* __restrict__ trees, i
         const int32_t from = max(1, known - pos);
         k = lim;
         if (from < lim) {
-          const int32_t first = min(lim, from + (kLeader ? 8 : 16));
+          const int32_t first = min(lim, from + kFirst);
           k = first_diff_1(lab, req + pos, from, first);
           if (k == first && first < lim) {
             if (lim - first <= kThreadSpan) {
@@ -705,7 +707,7 @@ __device__ __forceinline__ int probe_first2(const int4& a, const int4& b, int32_
 //   T) if that is < c, else a walk resumed at the leader's checkpoint that does not compare f's first c
 //   tokens.  A lane takes kFollowIlp trees at a time (p, p + 32, ...): the leader's matches, the
 //   checkpoints and the first probe step of each are loaded before any of them is looked at.
-template <bool kLeader, bool kDecide>
+template <bool kLeader, bool kDecide, int kFirst = 8>
 __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
     const TreeView* __restrict__ trees, int32_t P, const int32_t* __restrict__ tokens, int64_t n_tokens,
     int64_t tok_base, const int64_t* __restrict__ offsets, const int32_t* __restrict__ list,
@@ -764,7 +766,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
           act = st.w > 0 && root_filter_has(trees[p].rfilter, tok0) &&
                 find_child_1(trees[p].child + st.y, tab_bits(st.z), tok0, ce);
         }
-        lane_walks<true>(trees, p, req, len, 0, act, ce, pos, m, ck, climit, lane, err);
+        lane_walks<true, kFirst>(trees, p, req, len, 0, act, ce, pos, m, ck, climit, lane, err);
         if (p < P) {
           out_match[frow + p] = m;
           acc.add(m, __ldg(load + p), p, alpha);
@@ -821,7 +823,7 @@ __global__ void __launch_bounds__(kFollowThreads, kFollowCtasPerSm) lane_kernel(
         }
 #pragma unroll
         for (int g = 0; g < kFollowIlp; ++g) {
-          lane_walks<false>(trees, pt[g], req, len, c, act[g], ce[g], pos[g], m[g], nullptr, -1, lane, err);
+          lane_walks<false, kFirst>(trees, pt[g], req, len, c, act[g], ce[g], pos[g], m[g], nullptr, -1, lane, err);
           if (pt[g] < P) {
             out_match[frow + pt[g]] = m[g];
             acc.add(m[g], __ldg(load + pt[g]), pt[g], alpha);
@@ -992,10 +994,18 @@ cudaError_t launch_passes(const TreeView* d_trees, int32_t P, const int32_t* tok
   }
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  P2P_TIMED(K_LANE_FOLLOWER, st,
-            (lane_kernel<false, kDecide><<<grid2, kFollowThreads, 0, st>>>(
-                d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
-                nullptr, g->ckpt, d_load, alpha, out_match, out_peer, d_err, nullptr, out_next)));
+  // The followers' first per-lane compare: 8 tokens for long requests, 16 otherwise (lane_walks).
+  if (n_tokens >= B * (int64_t)kSlotTokens) {
+    P2P_TIMED(K_LANE_FOLLOWER, st,
+              (lane_kernel<false, kDecide, 8><<<grid2, kFollowThreads, 0, st>>>(
+                  d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
+                  nullptr, g->ckpt, d_load, alpha, out_match, out_peer, d_err, nullptr, out_next)));
+  } else {
+    P2P_TIMED(K_LANE_FOLLOWER, st,
+              (lane_kernel<false, kDecide, 16><<<grid2, kFollowThreads, 0, st>>>(
+                  d_trees, P, tokens, n_tokens, tok_base, offsets, g->lists + B, g->counts + 1, g->lead, g->cpre, g->gid,
+                  nullptr, g->ckpt, d_load, alpha, out_match, out_peer, d_err, nullptr, out_next)));
+  }
   *launched += 1;
   return cudaGetLastError();
 }
