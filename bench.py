@@ -84,8 +84,8 @@ TRAFFIC: dict = {
         "group_resolve32_kernel": {"bytes": 9457201050, "source": "5dbd6a2a3cb8351d"},
         "group_ranges_kernel": {"bytes": 4005018, "source": "5dbd6a2a3cb8351d"},
         "group_place_kernel": {"bytes": 8143744, "source": "5dbd6a2a3cb8351d"},
-        "lane_kernel<true>": {"bytes": 6158302771, "source": "76e33428fba97445"},
-        "lane_kernel<false>": {"bytes": 16554845926, "source": "76e33428fba97445"},
+        "lane_kernel<true>": {"bytes": 6151677824, "source": "73d5d75a48fec1cc"},
+        "lane_kernel<false>": {"bytes": 16206268134, "source": "73d5d75a48fec1cc"},
     }.items()},
 }
 
